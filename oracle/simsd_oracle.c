@@ -1,0 +1,402 @@
+/*
+ * simsd_oracle.c -- plain fp64 CPU oracle for the SimSD verification step.
+ *
+ * TEST INFRASTRUCTURE ONLY.  This file is the slow, obviously-correct
+ * statement of what the verification step computes.  Only the tests, the
+ * smoke check and the CPU-baseline leg of the benchmark may load it; the
+ * product path never calls it, and it shares no code, header or constant
+ * with the CUDA library.
+ *
+ * Paper: "SimSD: Simple Speculative Decoding in Diffusion Language Models".
+ *   - Sec. 3.1 "Input Layout Prepare": prompt, data section D (B reference
+ *     tokens), mask section D~ (B prediction slots); D_k and D~_k are the
+ *     same response position.
+ *   - Sec. 3.1 "Temporal Attention Mask", Eq. (1): the four-case visibility
+ *     rule over response positions; prompt visible to every response
+ *     position; padding rows and columns zeroed.
+ *   - Sec. 3.1 "Position Encoding Alignment": D~_k reuses the RoPE index of
+ *     D_k.
+ *   - Sec. 3.2 "Target Model Verification": slot with tau = r holds the r-th
+ *     draft; acceptance along the draft order, longest prefix before the
+ *     first rejection; Eq. (2) with one-hot distributions (temperature 0)
+ *     reduces to "accept iff the target argmax equals the draft".
+ *   - Sec. 3.3 "Adaptation under Blockwise Decoding and KV Cache": the
+ *     prefix K/V is reused from the cache; only new positions are computed.
+ *
+ * Readings where the paper is silent (each one is listed in the design
+ * notes): slot k in [0,gamma) is D_k and slot gamma+k is D~_k; step-map
+ * value 0 marks a padding position; a step map that is not a partial
+ * permutation of 1..gamma makes the whole sequence padding; argmax ties go
+ * to the lowest index and NaN ranks above every number (first NaN wins);
+ * the accepted count excludes the correction token; the committed K/V of
+ * an accepted draft is its data-slot K/V, appended in tau order.
+ *
+ * Everything is computed in double precision, in the order the definitions
+ * state, with no blocking or fusion.  OpenMP only distributes independent
+ * output rows over threads; each row is computed by one thread in a fixed
+ * order, so results do not depend on the thread count.
+ */
+#include <math.h>
+#include <stdint.h>
+#include <stdlib.h>
+#include <string.h>
+#ifdef _OPENMP
+#include <omp.h>
+#endif
+
+/* error bits (the oracle's own copy of the documented meanings) */
+#define OR_ERR_STEP_MAP 1
+#define OR_ERR_PREFIX_LEN 2
+#define OR_ERR_PAGE 4
+#define OR_ERR_DRAFT 8
+#define OR_ERR_ACCEPT_LEN 32
+
+#define OR_SECT_D 0
+#define OR_SECT_DT 1
+#define OR_SECT_PAD 255
+
+/* ---------------------------------------------------------------------- */
+/* Sec. 3.1: step map -> per-slot temporal label, section and RoPE index.  */
+/* ---------------------------------------------------------------------- */
+
+/* Checks that step_map row b is a partial permutation of 1..gamma (0 marks
+ * padding).  Returns 1 when valid. */
+static int step_map_row_valid(const int32_t *mu, int gamma) {
+    for (int k = 0; k < gamma; ++k) {
+        if (mu[k] < 0 || mu[k] > gamma) return 0;
+        if (mu[k] == 0) continue;
+        for (int k2 = 0; k2 < k; ++k2)
+            if (mu[k2] == mu[k]) return 0;
+    }
+    return 1;
+}
+
+/* Per-slot labels for one sequence.  Slot k (k < gamma) is D_k, slot gamma+k
+ * is D~_k; both carry tau = mu_k (Sec. 3.1 "Temporal Attention Mask").  A
+ * zero entry or an invalid map marks the slot(s) as padding.  The RoPE index
+ * of both D_k and D~_k is the absolute position of D_k, i.e. n + k, where n is
+ * the cached prefix length (Sec. 3.1 "Position Encoding Alignment"). */
+static int labels_for_sequence(const int32_t *mu, int n, int gamma, int32_t *tau,
+                               uint8_t *sect, int32_t *rope) {
+    int ok = step_map_row_valid(mu, gamma);
+    for (int k = 0; k < gamma; ++k) {
+        int pad = (!ok) || mu[k] == 0;
+        tau[k] = pad ? 0 : mu[k];
+        tau[gamma + k] = tau[k];
+        sect[k] = pad ? OR_SECT_PAD : OR_SECT_D;
+        sect[gamma + k] = pad ? OR_SECT_PAD : OR_SECT_DT;
+        rope[k] = n + k;
+        rope[gamma + k] = n + k;
+    }
+    return ok ? 0 : OR_ERR_STEP_MAP;
+}
+
+/* Eq. (1), written case by case.  i is the attending (row) slot, j the
+ * attended (column) slot.  Padding rows and columns are zero (Sec. 3.1, the
+ * sentence after Eq. (1)). */
+static int eq1_visible(uint8_t si, int ti, uint8_t sj, int tj) {
+    if (si == OR_SECT_PAD || sj == OR_SECT_PAD) return 0;
+    if (si == OR_SECT_D && sj == OR_SECT_D && tj <= ti) return 1;   /* case 1 */
+    if (si == OR_SECT_D && sj == OR_SECT_DT && tj > ti) return 1;   /* case 2 */
+    if (si == OR_SECT_DT && sj == OR_SECT_D && tj < ti) return 1;   /* case 3 */
+    if (si == OR_SECT_DT && sj == OR_SECT_DT && tj >= ti) return 1; /* case 4 */
+    return 0;                                                       /* otherwise */
+}
+
+/* Builds tau/section/rope_pos and the response-block mask for every sequence.
+ *   step_map  [Bt][gamma] int32, or NULL for the identity map mu = (1..gamma)
+ *   prefix_len[Bt]
+ *   tau, rope_pos [Bt][2gamma] int32; section [Bt][2gamma] uint8
+ *   mask_bits [Bt][2gamma] uint64 (bit j of row i = A_ij), may be NULL
+ *   dense     [Bt][2gamma][2gamma] uint8, may be NULL
+ * Returns the OR of the error bits. */
+int oracle_build_mask(const int32_t *step_map, const int32_t *prefix_len, int Bt, int gamma,
+                      int32_t *tau, uint8_t *section, int32_t *rope_pos, uint64_t *mask_bits,
+                      uint8_t *dense) {
+    int S = 2 * gamma, err = 0;
+    int32_t *ident = (int32_t *)malloc(sizeof(int32_t) * (size_t)(gamma > 0 ? gamma : 1));
+    for (int k = 0; k < gamma; ++k) ident[k] = k + 1;
+    for (int b = 0; b < Bt; ++b) {
+        const int32_t *mu = step_map ? step_map + (size_t)b * gamma : ident;
+        int32_t *t = tau + (size_t)b * S;
+        uint8_t *s = section + (size_t)b * S;
+        err |= labels_for_sequence(mu, prefix_len[b], gamma, t, s, rope_pos + (size_t)b * S);
+        for (int i = 0; i < S; ++i) {
+            uint64_t bits = 0;
+            for (int j = 0; j < S; ++j) {
+                int v = eq1_visible(s[i], t[i], s[j], t[j]);
+                if (v) bits |= (uint64_t)1 << j;
+                if (dense) dense[((size_t)b * S + i) * S + j] = (uint8_t)v;
+            }
+            if (mask_bits) mask_bits[(size_t)b * S + i] = bits;
+        }
+    }
+    free(ident);
+    return err;
+}
+
+/* ---------------------------------------------------------------------- */
+/* Masked attention of the verification forward (Sec. 3.2, Sec. 3.3).     */
+/* ---------------------------------------------------------------------- */
+
+/* Widens one stored element to double.  dtype 0: IEEE binary32; dtype 1:
+ * bfloat16 (the upper 16 bits of a binary32). */
+static double load_elem(const void *base, size_t idx, int dtype) {
+    if (dtype == 0) return (double)((const float *)base)[idx];
+    uint32_t bits = (uint32_t)((const uint16_t *)base)[idx] << 16;
+    float f;
+    memcpy(&f, &bits, sizeof f);
+    return (double)f;
+}
+
+/* out[b][s][h][:] = sum_j softmax_j(scale * q.k_j) v_j over the keys the
+ * row may see: every cached prefix row of sequence b (the prompt / earlier
+ * blocks, visible to all response positions) read through the page table,
+ * plus each new slot t with A_st = 1 under Eq. (1).  Query head h reads KV
+ * head h / (Hq/Hkv).
+ *
+ * Layouts (row-major):
+ *   q, out  [Bt][2gamma][Hq][d]
+ *   k_new, v_new [Bt][2gamma][Hkv][d]
+ *   k_cache, v_cache [num_pages][Hkv][page_size][d]
+ *   block_table [Bt][max_pages]; prefix row p of sequence b lives in page
+ *   block_table[b][p / page_size] at offset p % page_size.
+ * A sequence whose prefix length is outside [0, max_pages*page_size], whose
+ * needed pages are outside [0, num_pages), or whose step map is invalid gets
+ * all-zero output rows and sets the matching error bit.  Padding rows are
+ * zero.  Returns the error bits. */
+int oracle_verify_attention(int dtype, const void *q, const void *k_new, const void *v_new,
+                            const void *k_cache, const void *v_cache, const int32_t *block_table,
+                            int max_pages, int page_size, int num_pages, const int32_t *prefix_len,
+                            const int32_t *step_map, int Bt, int gamma, int Hq, int Hkv, int d,
+                            double scale, double *out, int nthreads) {
+    const int S = 2 * gamma, g = Hq / Hkv;
+    int err = 0;
+    int32_t *tau = (int32_t *)malloc(sizeof(int32_t) * (size_t)Bt * S);
+    uint8_t *sect = (uint8_t *)malloc((size_t)Bt * S);
+    int32_t *rope = (int32_t *)malloc(sizeof(int32_t) * (size_t)Bt * S);
+    int32_t *nvalid = (int32_t *)malloc(sizeof(int32_t) * (size_t)Bt);
+    err |= oracle_build_mask(step_map, prefix_len, Bt, gamma, tau, sect, rope, NULL, NULL);
+
+    for (int b = 0; b < Bt; ++b) {
+        int n = prefix_len[b], ok = 1;
+        if (n < 0 || (long long)n > (long long)max_pages * page_size) {
+            err |= OR_ERR_PREFIX_LEN;
+            ok = 0;
+        } else {
+            int npages = (n + page_size - 1) / page_size;
+            for (int p = 0; p < npages; ++p) {
+                int pg = block_table[(size_t)b * max_pages + p];
+                if (pg < 0 || pg >= num_pages) {
+                    err |= OR_ERR_PAGE;
+                    ok = 0;
+                }
+            }
+        }
+        nvalid[b] = ok ? n : -1;
+    }
+
+    long long rows = (long long)Bt * S * Hq;
+#ifdef _OPENMP
+    if (nthreads > 0) omp_set_num_threads(nthreads);
+#else
+    (void)nthreads;
+#endif
+#pragma omp parallel for schedule(dynamic, 4)
+    for (long long row = 0; row < rows; ++row) {
+        int h = (int)(row % Hq);
+        int s = (int)((row / Hq) % S);
+        int b = (int)(row / ((long long)Hq * S));
+        int kvh = h / g;
+        double *o = out + (size_t)row * d;
+        for (int c = 0; c < d; ++c) o[c] = 0.0;
+        int n = nvalid[b];
+        uint8_t si = sect[(size_t)b * S + s];
+        if (n < 0 || si == OR_SECT_PAD) continue;
+
+        /* gather the visible keys: (source array, element offset) pairs */
+        int cap = n + S;
+        size_t *koff = (size_t *)malloc(sizeof(size_t) * (size_t)cap);
+        int *is_new = (int *)malloc(sizeof(int) * (size_t)cap);
+        double *score = (double *)malloc(sizeof(double) * (size_t)cap);
+        int cnt = 0;
+        for (int p = 0; p < n; ++p) {
+            int pg = block_table[(size_t)b * max_pages + p / page_size];
+            koff[cnt] = (((size_t)pg * Hkv + kvh) * page_size + (size_t)(p % page_size)) * d;
+            is_new[cnt] = 0;
+            ++cnt;
+        }
+        int ti = tau[(size_t)b * S + s];
+        for (int t = 0; t < S; ++t) {
+            if (!eq1_visible(si, ti, sect[(size_t)b * S + t], tau[(size_t)b * S + t])) continue;
+            koff[cnt] = (((size_t)b * S + t) * Hkv + kvh) * d;
+            is_new[cnt] = 1;
+            ++cnt;
+        }
+        size_t qoff = (size_t)row * d;
+        /* pass 1: scaled dot products and their maximum */
+        double m = -INFINITY;
+        for (int j = 0; j < cnt; ++j) {
+            const void *kb = is_new[j] ? k_new : k_cache;
+            double acc = 0.0;
+            for (int c = 0; c < d; ++c)
+                acc += load_elem(q, qoff + c, dtype) * load_elem(kb, koff[j] + c, dtype);
+            score[j] = acc * scale;
+            if (score[j] > m) m = score[j];
+        }
+        /* pass 2: normalised weights times values */
+        double z = 0.0;
+        for (int j = 0; j < cnt; ++j) {
+            score[j] = exp(score[j] - m);
+            z += score[j];
+        }
+        for (int j = 0; j < cnt; ++j) {
+            const void *vb = is_new[j] ? v_new : v_cache;
+            double w = score[j] / z;
+            for (int c = 0; c < d; ++c) o[c] += w * load_elem(vb, koff[j] + c, dtype);
+        }
+        free(koff);
+        free(is_new);
+        free(score);
+    }
+    free(tau);
+    free(sect);
+    free(rope);
+    free(nvalid);
+    return err;
+}
+
+/* ---------------------------------------------------------------------- */
+/* Greedy acceptance (Sec. 3.2, Eq. (2) at temperature 0).                 */
+/* ---------------------------------------------------------------------- */
+
+/* logits [Bt][gamma+1][vocab] fp32, row r scores the draft with tau = r+1
+ * (row gamma is only used when every draft is accepted).
+ * draft  [Bt][gamma] int32 in tau order.
+ * accepted_len[Bt] = number of leading drafts equal to the row argmax.
+ * out_tokens[Bt][gamma+1] = accepted drafts, then the target's token at the
+ * first rejected position (argmax of row a), then -1.
+ * row_argmax[Bt][gamma+1] may be NULL.  Returns the error bits. */
+int oracle_accept(const float *logits, const int32_t *draft, int Bt, int gamma, int vocab,
+                  int32_t *accepted_len, int32_t *out_tokens, int32_t *row_argmax) {
+    int err = 0;
+    int32_t *am = (int32_t *)malloc(sizeof(int32_t) * (size_t)(gamma + 1));
+    for (int b = 0; b < Bt; ++b) {
+        for (int r = 0; r <= gamma; ++r) {
+            const float *row = logits + ((size_t)b * (gamma + 1) + r) * vocab;
+            int best = 0;
+            double bv = (double)row[0];
+            for (int v = 1; v < vocab; ++v) {
+                double x = (double)row[v];
+                if (isnan(bv)) break;             /* the first NaN is the maximum */
+                if (isnan(x) || x > bv) {         /* strict '>': ties keep the lower index */
+                    best = v;
+                    bv = x;
+                }
+            }
+            am[r] = best;
+            if (row_argmax) row_argmax[(size_t)b * (gamma + 1) + r] = best;
+        }
+        int a = 0;
+        while (a < gamma) {
+            int dr = draft[(size_t)b * gamma + a];
+            if (dr < 0 || dr >= vocab) {
+                err |= OR_ERR_DRAFT;
+                break;
+            }
+            if (dr != am[a]) break;
+            ++a;
+        }
+        /* report every out-of-range draft, not only the first one reached */
+        for (int r = a; r < gamma; ++r) {
+            int dr = draft[(size_t)b * gamma + r];
+            if (dr < 0 || dr >= vocab) err |= OR_ERR_DRAFT;
+        }
+        accepted_len[b] = a;
+        int32_t *ot = out_tokens + (size_t)b * (gamma + 1);
+        for (int r = 0; r <= gamma; ++r) ot[r] = -1;
+        for (int r = 0; r < a; ++r) ot[r] = draft[(size_t)b * gamma + r];
+        ot[a] = am[a];
+    }
+    free(am);
+    return err;
+}
+
+/* ---------------------------------------------------------------------- */
+/* Commit of the accepted K/V to the paged cache (Sec. 3.2, Sec. 3.3).     */
+/* ---------------------------------------------------------------------- */
+
+/* For every layer l, sequence b, accepted draft r < a_b and KV head:
+ * copy the data-slot row whose tau is r+1 into cache row n_b + r, then set
+ * n_b += a_b.  Byte copies; elem_bytes is 2 or 4.
+ *   k_new, v_new  [L][Bt][2gamma][Hkv][d]
+ *   k_cache, v_cache [L][num_pages][Hkv][page_size][d]
+ * A destination page outside the table or the pool sets OR_ERR_PAGE and that
+ * row is skipped; a missing source slot sets OR_ERR_STEP_MAP and the row is
+ * skipped; a negative prefix or an accepted length outside [0,gamma] leaves
+ * the sequence untouched.  Returns the error bits. */
+int oracle_kv_commit(int elem_bytes, const void *k_new, const void *v_new, int L,
+                     const int32_t *step_map, const int32_t *accepted_len, void *k_cache,
+                     void *v_cache, const int32_t *block_table, int max_pages, int page_size,
+                     int num_pages, int32_t *prefix_len, int Bt, int gamma, int Hkv, int d) {
+    const int S = 2 * gamma;
+    int err = 0;
+    size_t row_bytes = (size_t)d * elem_bytes;
+    for (int b = 0; b < Bt; ++b) {
+        int n = prefix_len[b], a = accepted_len[b];
+        if (a < 0 || a > gamma) {
+            err |= OR_ERR_ACCEPT_LEN;
+            continue;
+        }
+        if (n < 0) {
+            err |= OR_ERR_PREFIX_LEN;
+            continue;
+        }
+        const int32_t *mu = step_map ? step_map + (size_t)b * gamma : NULL;
+        int valid_map = mu ? step_map_row_valid(mu, gamma) : 1;
+        for (int r = 0; r < a; ++r) {
+            int src = -1;
+            for (int k = 0; k < gamma; ++k) {
+                int tk = mu ? mu[k] : k + 1;
+                if (valid_map && tk == r + 1) src = k;
+            }
+            if (src < 0) {
+                err |= OR_ERR_STEP_MAP;
+                continue;
+            }
+            long long dst = (long long)n + r;
+            long long pidx = dst / page_size;
+            if (pidx >= max_pages) {
+                err |= OR_ERR_PAGE;
+                continue;
+            }
+            int pg = block_table[(size_t)b * max_pages + pidx];
+            if (pg < 0 || pg >= num_pages) {
+                err |= OR_ERR_PAGE;
+                continue;
+            }
+            int off = (int)(dst % page_size);
+            for (int l = 0; l < L; ++l) {
+                for (int kvh = 0; kvh < Hkv; ++kvh) {
+                    size_t s_el = ((((size_t)l * Bt + b) * S + src) * Hkv + kvh) * d;
+                    size_t d_el = ((((size_t)l * num_pages + pg) * Hkv + kvh) * page_size + off) * d;
+                    memcpy((char *)k_cache + d_el * elem_bytes, (const char *)k_new + s_el * elem_bytes,
+                           row_bytes);
+                    memcpy((char *)v_cache + d_el * elem_bytes, (const char *)v_new + s_el * elem_bytes,
+                           row_bytes);
+                }
+            }
+        }
+        prefix_len[b] = n + a;
+    }
+    return err;
+}
+
+/* Number of OpenMP threads the oracle uses by default. */
+int oracle_max_threads(void) {
+#ifdef _OPENMP
+    return omp_get_max_threads();
+#else
+    return 1;
+#endif
+}

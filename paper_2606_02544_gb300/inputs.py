@@ -1,0 +1,224 @@
+"""Seeded synthetic inputs for the SimSD verification step.
+
+This module only draws random tensors and lays them out; it contains none of
+the method's arithmetic (no mask, no attention, no acceptance, no commit).
+Both the CUDA path and the fp64 oracle are fed from it.
+
+The paper measures end-to-end decoding of SDAR models on GSM8K, TriviaQA,
+MBPP and MMLU (Sec. 4.1).  Neither the weights nor the datasets are used
+here: the verification forward is driven by synthetic tensors with the head
+shapes of SDAR-1.7B/4B/8B, the block lengths of the paper (B = gamma = 4, 8,
+plus 16 and 32 for the sweep) and draft agreement rates in the range of the
+paper's measured token-level acceptance (Table 2: 0.52 to 0.97).
+
+Recipe (one per workload, all values seeded):
+  * prefix lengths: fixed, or uniform integers in [lo, hi];
+  * paged cache: page size P (64), every sequence owns ceil((n_b + gamma)/P)
+    pages (room to commit gamma rows) drawn from one random permutation of the
+    page pool; unused block-table entries are -1;
+  * Q, K_new, V_new and the cache ~ N(0, std^2) (std 1 for the fp32 case,
+    1/sqrt(128) for the bf16 SDAR-shaped cases), one independent draw per
+    layer (seed + 1000*l);
+  * logits [Bt][gamma+1][V] ~ N(0, sigma^2) in fp32;
+  * drafts: with probability p the row's argmax (torch.argmax), otherwise a
+    uniform token in [0, V);
+  * step map: the identity (left-to-right) unless a random permutation is
+    requested.
+"""
+from __future__ import annotations
+
+import dataclasses
+import math
+from typing import Optional
+
+import numpy as np
+import torch
+
+
+@dataclasses.dataclass(frozen=True)
+class Workload:
+    name: str
+    dtype: str            # "f32" or "bf16": storage and compute type of Q/K/V/O
+    Bt: int               # sequences in the batch
+    Hq: int               # query heads
+    Hkv: int              # KV heads
+    d: int                # head dimension
+    gamma: int            # draft length = block length
+    prefix: tuple         # (lo, hi) inclusive; lo == hi for a fixed prefix
+    layers: int           # stacked attention layers (independent K/V per layer)
+    vocab: int
+    p_agree: float        # probability that a draft equals the row argmax
+    qkv_std: float
+    logit_std: float
+    seed: int
+    page_size: int = 64
+
+    @property
+    def S(self) -> int:
+        return 2 * self.gamma
+
+    @property
+    def g(self) -> int:
+        return self.Hq // self.Hkv
+
+    def describe(self) -> dict:
+        return dataclasses.asdict(self)
+
+
+_SD = 1.0 / math.sqrt(128.0)
+
+WORKLOADS = {
+    # tiny fp32 correctness case
+    "c1": Workload("c1_tiny_fp32", "f32", 1, 2, 1, 64, 4, (128, 128), 1, 1024, 0.7, 1.0, 1.0, 0),
+    # SDAR-1.7B-shaped verification layer
+    "c2": Workload("c2_sdar1.7b_layer", "bf16", 8, 16, 8, 128, 4, (512, 1024), 1, 151936, 0.6, _SD, 2.0, 1),
+    # SDAR-4B-shaped verification layer, paged cache P=64
+    "c3": Workload("c3_sdar4b_layer_paged64", "bf16", 32, 32, 8, 128, 8, (4096, 4096), 1, 151936, 0.5, _SD, 2.0, 2),
+    # SDAR-8B-shaped step over 36 stacked layers
+    "c4": Workload("c4_sdar8b_36layers", "bf16", 64, 32, 8, 128, 16, (2048, 8192), 36, 151936, 0.8, _SD, 2.0, 3),
+}
+
+
+def sweep_points():
+    """The SDAR-8B head-shape sweep: batch x prefix x gamma x agreement."""
+    pts = []
+    i = 0
+    for Bt in (1, 8, 32, 128):
+        for n in (512, 2048, 8192, 32768):
+            for gamma in (4, 8, 16, 32):
+                for p in (0.3, 0.6, 0.9):
+                    pts.append(Workload(f"c5_b{Bt}_n{n}_g{gamma}_p{p}", "bf16", Bt, 32, 8, 128, gamma,
+                                        (n, n), 1, 151936, p, _SD, 2.0, 4 + i))
+                    i += 1
+    return pts
+
+
+def torch_dtype(w: Workload):
+    return torch.float32 if w.dtype == "f32" else torch.bfloat16
+
+
+@dataclasses.dataclass
+class StepInputs:
+    """All tensors of one verification step (device or host)."""
+    w: Workload
+    prefix_len: torch.Tensor      # int32 [Bt]
+    block_table: torch.Tensor     # int32 [Bt][max_pages]
+    num_pages: int
+    step_map: torch.Tensor        # int32 [Bt][gamma]
+    q: torch.Tensor               # [L][Bt][S][Hq][d]
+    k_new: torch.Tensor           # [L][Bt][S][Hkv][d]
+    v_new: torch.Tensor           # [L][Bt][S][Hkv][d]
+    k_cache: torch.Tensor         # [L][num_pages][Hkv][P][d]
+    v_cache: torch.Tensor         # [L][num_pages][Hkv][P][d]
+    logits: torch.Tensor          # fp32 [Bt][gamma+1][V]
+    draft: torch.Tensor           # int32 [Bt][gamma]
+    row_valid: np.ndarray         # bool [num_pages][P]: row holds a prefix row
+
+
+def _cpu_gen(seed: int) -> torch.Generator:
+    return torch.Generator(device="cpu").manual_seed(int(seed))
+
+
+def _dev_gen(seed: int, device) -> torch.Generator:
+    return torch.Generator(device=device).manual_seed(int(seed))
+
+
+def make_metadata(w: Workload, seed: Optional[int] = None, prefix_override=None, random_step_map=False,
+                  spare_pages: int = 3):
+    """Prefix lengths, page table and step map (host tensors, int32)."""
+    seed = w.seed if seed is None else seed
+    gen = _cpu_gen(seed)
+    lo, hi = w.prefix
+    if prefix_override is not None:
+        n = torch.as_tensor(np.asarray(prefix_override, dtype=np.int32))
+    elif lo == hi:
+        n = torch.full((w.Bt,), lo, dtype=torch.int32)
+    else:
+        n = torch.randint(lo, hi + 1, (w.Bt,), generator=gen, dtype=torch.int64).to(torch.int32)
+    P = w.page_size
+    pages_b = [(int(x) + w.gamma + P - 1) // P for x in n.tolist()]
+    num_pages = sum(pages_b) + spare_pages
+    max_pages = max(max(pages_b), 1)
+    perm = torch.randperm(num_pages, generator=gen).to(torch.int32)
+    bt = torch.full((w.Bt, max_pages), -1, dtype=torch.int32)
+    pos = 0
+    for b, cnt in enumerate(pages_b):
+        bt[b, :cnt] = perm[pos:pos + cnt]
+        pos += cnt
+    if random_step_map:
+        sm = torch.stack([torch.randperm(w.gamma, generator=gen) + 1 for _ in range(w.Bt)]).to(torch.int32)
+    else:
+        sm = torch.arange(1, w.gamma + 1, dtype=torch.int32).repeat(w.Bt, 1)
+    # rows of the pool that hold a prefix row
+    row_valid = np.zeros((num_pages, P), dtype=bool)
+    bt_np = bt.numpy()
+    for b in range(w.Bt):
+        nb = int(n[b])
+        for p in range(pages_b[b]):
+            lo_r = p * P
+            cnt = min(max(nb - lo_r, 0), P)
+            row_valid[bt_np[b, p], :cnt] = True
+    return n, bt, num_pages, sm, row_valid
+
+
+def make_step_inputs(w: Workload, device="cpu", seed: Optional[int] = None, prefix_override=None,
+                     random_step_map=False, poison_unused_rows=False, layers: Optional[int] = None,
+                     qkv_std: Optional[float] = None, with_logits=True) -> StepInputs:
+    """Draws every tensor of one verification step for workload ``w``.
+
+    ``poison_unused_rows`` fills cache rows that hold no prefix row with NaN,
+    so that a kernel which reads past a sequence's prefix shows it.
+    """
+    seed = w.seed if seed is None else seed
+    L = w.layers if layers is None else layers
+    std = w.qkv_std if qkv_std is None else qkv_std
+    n, bt, num_pages, sm, row_valid = make_metadata(w, seed, prefix_override, random_step_map)
+    dt = torch_dtype(w)
+    S, P = w.S, w.page_size
+    qs, kns, vns, kcs, vcs = [], [], [], [], []
+    poison = None
+    if poison_unused_rows:
+        poison = torch.as_tensor(~row_valid, device=device).view(num_pages, 1, P, 1)
+    for l in range(L):
+        g = _dev_gen(seed + 1000 * l, device)
+        qs.append((torch.randn(w.Bt, S, w.Hq, w.d, generator=g, device=device) * std).to(dt))
+        kns.append((torch.randn(w.Bt, S, w.Hkv, w.d, generator=g, device=device) * std).to(dt))
+        vns.append((torch.randn(w.Bt, S, w.Hkv, w.d, generator=g, device=device) * std).to(dt))
+        kc = (torch.randn(num_pages, w.Hkv, P, w.d, generator=g, device=device) * std).to(dt)
+        vc = (torch.randn(num_pages, w.Hkv, P, w.d, generator=g, device=device) * std).to(dt)
+        if poison is not None:
+            kc = torch.where(poison, torch.full_like(kc, float("nan")), kc)
+            vc = torch.where(poison, torch.full_like(vc, float("nan")), vc)
+        kcs.append(kc)
+        vcs.append(vc)
+    q = torch.stack(qs)
+    k_new = torch.stack(kns)
+    v_new = torch.stack(vns)
+    k_cache = torch.stack(kcs)
+    v_cache = torch.stack(vcs)
+    del qs, kns, vns, kcs, vcs
+    if with_logits:
+        g = _dev_gen(seed + 7, device)
+        logits = torch.randn(w.Bt, w.gamma + 1, w.vocab, generator=g, device=device) * w.logit_std
+        cg = _cpu_gen(seed + 11)
+        agree = torch.rand(w.Bt, w.gamma, generator=cg) < w.p_agree
+        rnd = torch.randint(0, w.vocab, (w.Bt, w.gamma), generator=cg, dtype=torch.int64)
+        am = torch.argmax(logits[:, : w.gamma, :], dim=-1).cpu()
+        draft = torch.where(agree, am, rnd).to(torch.int32)
+    else:
+        logits = torch.zeros(w.Bt, w.gamma + 1, 1, device=device)
+        draft = torch.zeros(w.Bt, w.gamma, dtype=torch.int32)
+    dev = torch.device(device)
+    return StepInputs(w, n.to(dev), bt.to(dev), num_pages, sm.to(dev), q, k_new, v_new, k_cache, v_cache,
+                      logits, draft.to(dev), row_valid)
+
+
+def host_bits(t: torch.Tensor) -> np.ndarray:
+    """Host numpy view of a tensor's stored values: float32 as float32,
+    bfloat16 as its uint16 bit patterns (exact; no rounding)."""
+    t = t.detach().contiguous().cpu()
+    if t.dtype == torch.bfloat16:
+        return t.view(torch.int16).numpy().view(np.uint16)
+    if t.dtype == torch.float32:
+        return t.numpy()
+    return t.numpy()
