@@ -1,0 +1,196 @@
+/*
+ * simsd.h -- C ABI of libsimsd.so: the verification forward of SimSD
+ * speculative decoding for block-diffusion language models, on one GB300
+ * (sm_103a).
+ *
+ * Paper: "SimSD: Simple Speculative Decoding in Diffusion Language Models".
+ * One speculative step drafts gamma tokens, then the target verifies them in
+ * a single forward pass over a paired layout: a data section D holding the
+ * drafted (reference) tokens and a mask section D~ of prediction slots
+ * (Sec. 3.1 "Input Layout Prepare", Sec. 3.2 "Target Model Verification").
+ * A token-level temporal mask, Eq. (1), decides what each slot sees; the
+ * prefix (prompt and earlier blocks) is read from a KV cache (Sec. 3.3).
+ * The drafts are accepted along the draft order up to the first rejection
+ * (Sec. 3.2, Eq. (2)), and the accepted drafts' K/V are appended to the
+ * cache.
+ *
+ * Conventions shared by every call
+ *   - Slot layout of one sequence: S = 2*gamma slots; slot k in [0,gamma)
+ *     is the data slot D_k, slot gamma+k is the mask slot D~_k of the same
+ *     block position k.  Row r of the acceptance logits and entry r of the
+ *     draft array belong to the draft with temporal label tau = r+1.
+ *   - Every pointer is caller-owned device memory unless stated otherwise;
+ *     the library keeps no allocation of its own.  Arrays are dense,
+ *     row-major, 16-byte aligned.
+ *   - Every compute call is asynchronous on `stream` (a cudaStream_t passed
+ *     as void*; NULL = the legacy default stream) and never synchronises.
+ *   - Every call returns one of the SIMSD_* status codes.  Argument errors
+ *     are detected on the host before anything is launched.  Errors that
+ *     depend on device data (a bad step map, prefix length, page id, draft
+ *     id or accepted length) are OR-ed into the caller's int32 error word
+ *     (may be NULL) as SIMSD_EW_* bits, and the affected outputs are
+ *     defined below; read the word with simsd_check_error.
+ *   - dtype selects the storage and compute type of Q/K/V/O:
+ *     SIMSD_BF16 (tensor cores, fp32 accumulation and softmax) or
+ *     SIMSD_F32 (CUDA cores, fp32 throughout).
+ */
+#ifndef SIMSD_H_
+#define SIMSD_H_
+
+#include <stddef.h>
+#include <stdint.h>
+
+#if defined(__GNUC__)
+#define SIMSD_API __attribute__((visibility("default")))
+#else
+#define SIMSD_API
+#endif
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+/* status codes */
+#define SIMSD_OK 0
+#define SIMSD_ERR_INVALID_ARG 1 /* null pointer, bad size, misaligned pointer */
+#define SIMSD_ERR_UNSUPPORTED 2 /* dtype, head size or device not supported */
+#define SIMSD_ERR_CUDA 3        /* a CUDA call failed; see simsd_last_error() */
+#define SIMSD_ERR_DEVICE 4      /* simsd_check_error: the error word is non-zero */
+
+/* dtypes */
+#define SIMSD_F32 0
+#define SIMSD_BF16 1
+
+/* slot sections */
+#define SIMSD_SECT_DATA 0 /* D: reference (drafted) token */
+#define SIMSD_SECT_MASK 1 /* D~: prediction slot */
+#define SIMSD_SECT_PAD 255 /* padding: row outputs zero, column never visible */
+
+/* device error-word bits */
+#define SIMSD_EW_STEP_MAP 1u    /* step map is not a partial permutation of 1..gamma */
+#define SIMSD_EW_PREFIX_LEN 2u  /* prefix length < 0 or beyond the block table */
+#define SIMSD_EW_PAGE 4u        /* a needed page id is outside [0, num_pages) */
+#define SIMSD_EW_DRAFT 8u       /* a draft id is outside [0, vocab) */
+#define SIMSD_EW_TIMEOUT 16u    /* a bounded on-device wait expired */
+#define SIMSD_EW_ACCEPT_LEN 32u /* an accepted length is outside [0, gamma] */
+
+/*
+ * simsd_build_mask -- per-slot metadata of the verification input.
+ * Sec. 3.1 "Temporal Attention Mask" and Eq. (1); "Position Encoding
+ * Alignment" (RoPE copy); Sec. 3.2 (the slot of the r-th draft gets tau=r).
+ *
+ *   step_map   [Bt][gamma] int32, mu_k in 1..gamma (a permutation), 0 marks a
+ *              padding position; NULL means the identity mu_k = k+1.
+ *   prefix_len [Bt] int32, cached prefix length n_b.
+ *   tau        [Bt][2gamma] int32 out: tau of D_k and D~_k is mu_k (0 if pad).
+ *   section    [Bt][2gamma] uint8 out: SIMSD_SECT_DATA / _MASK / _PAD.
+ *   rope_pos   [Bt][2gamma] int32 out: n_b + k for both D_k and D~_k.
+ *   mask_bits  [Bt][2gamma] uint64 out or NULL: bit j of row i is A_ij of
+ *              Eq. (1) over the new slots (prefix columns are always visible).
+ *   1 <= gamma <= 32.  A step map row that is not a partial permutation sets
+ *   SIMSD_EW_STEP_MAP and turns every slot of that sequence into padding.
+ */
+SIMSD_API int simsd_build_mask(const int32_t* step_map, const int32_t* prefix_len, int Bt, int gamma,
+                     int32_t* tau, uint8_t* section, int32_t* rope_pos, uint64_t* mask_bits,
+                     int32_t* err_word, void* stream);
+
+/*
+ * simsd_verify_workspace_bytes -- bytes of scratch simsd_verify_attention
+ * needs for these sizes on the current device (0 when no split of the
+ * prefix is used).  max_pages*page_size bounds every prefix length.
+ */
+SIMSD_API size_t simsd_verify_workspace_bytes(int dtype, int Bt, int gamma, int Hq, int Hkv, int d, int max_pages,
+                                    int page_size);
+
+/*
+ * simsd_verify_attention -- the masked attention of the verification
+ * forward (Sec. 3.2 "Target Model Verification"; Sec. 3.3 KV cache; cost of
+ * the paired layout linear in the prefix, Eqs. (4)-(5)).
+ *
+ * For each sequence b, slot s and query head h (KV head h/(Hq/Hkv)):
+ *   out[b][s][h] = softmax_j(scale * q.k_j) v_j over the keys j that the
+ *   slot sees: all n_b cached prefix rows (visible to every response
+ *   position) and each new slot t with A_st = 1 under Eq. (1), evaluated on
+ *   the fly from tau/section.
+ *
+ *   q, out       [Bt][2gamma][Hq][d]   dtype
+ *   k_new, v_new [Bt][2gamma][Hkv][d]  dtype (K/V of the new slots)
+ *   k_cache, v_cache [num_pages][Hkv][page_size][d] dtype; prefix row p of
+ *                sequence b is row p % page_size of page
+ *                block_table[b][p / page_size].  Rows past n_b are never used.
+ *   block_table  [Bt][max_pages] int32; entries past the prefix are ignored.
+ *   tau, section [Bt][2gamma] from simsd_build_mask.
+ *   rope_pos     must be NULL: Q and K arrive already rotated (RoPE-copy
+ *                positions are applied by the caller).
+ *   softmax_scale 0 selects 1/sqrt(d).
+ *   workspace    scratch of simsd_verify_workspace_bytes() bytes (NULL if 0).
+ * Supported: SIMSD_BF16 with d = 128 and Hq/Hkv*2gamma <= 128 or
+ * 128 % (Hq/Hkv) == 0; SIMSD_F32 with d in {64, 128}; page_size a multiple
+ * of 64 or a divisor of 64 (>= 8).
+ * A sequence with a bad prefix length or page id gets all-zero output rows
+ * and sets SIMSD_EW_PREFIX_LEN / SIMSD_EW_PAGE; padding rows are zero.
+ */
+SIMSD_API int simsd_verify_attention(int dtype, const void* q, const void* k_new, const void* v_new, const void* k_cache,
+                           const void* v_cache, int num_pages, const int32_t* block_table, int max_pages,
+                           int page_size, const int32_t* prefix_len, const int32_t* tau, const uint8_t* section,
+                           const int32_t* rope_pos, int Bt, int gamma, int Hq, int Hkv, int d, float softmax_scale,
+                           void* out, void* workspace, size_t workspace_bytes, int32_t* err_word, void* stream);
+
+/*
+ * simsd_accept -- greedy longest-prefix acceptance (Sec. 3.2, Eq. (2) with
+ * temperature 0: accept the r-th draft iff it equals the target argmax).
+ *
+ *   logits      [Bt][gamma+1][vocab] fp32; row r scores the draft with
+ *               tau = r+1, row gamma gives the next token when every draft
+ *               is accepted.
+ *   draft       [Bt][gamma] int32, in tau order.
+ *   accepted_len[Bt] int32 out: a_b = leading drafts equal to their row argmax.
+ *   out_tokens  [Bt][gamma+1] int32 out: the a_b accepted drafts, the argmax of
+ *               row a_b (the target's token at the first rejected position),
+ *               then -1.
+ *   row_argmax  [Bt][gamma+1] int32 out or NULL.
+ * Argmax ties go to the lowest index; NaN ranks above every number (the
+ * first NaN wins); -0.0 equals +0.0.  A draft id outside [0, vocab) sets
+ * SIMSD_EW_DRAFT and never matches.  No scratch memory is used.
+ */
+SIMSD_API int simsd_accept(const float* logits, const int32_t* draft, int Bt, int gamma, int vocab, int32_t* accepted_len,
+                 int32_t* out_tokens, int32_t* row_argmax, int32_t* err_word, void* stream);
+
+/*
+ * simsd_kv_commit -- append the accepted drafts' K/V to the paged cache of
+ * every layer (Sec. 3.2: accepted tokens are committed; Sec. 3.3: the cache
+ * is reused by later steps).
+ *
+ * For each layer l, sequence b, r < accepted_len[b] and KV head: the
+ * data-slot row whose tau is r+1 is copied to cache row prefix_len[b] + r;
+ * then prefix_len[b] += accepted_len[b] (in place).
+ *   k_new, v_new [L][Bt][2gamma][Hkv][d] dtype
+ *   k_cache, v_cache [L][num_pages][Hkv][page_size][d] dtype
+ * A destination page outside the table or pool sets SIMSD_EW_PAGE and that
+ * row is skipped; a missing source slot sets SIMSD_EW_STEP_MAP and that row
+ * is skipped; a negative prefix length (SIMSD_EW_PREFIX_LEN) or an accepted
+ * length outside [0, gamma] (SIMSD_EW_ACCEPT_LEN) leaves the sequence
+ * untouched.
+ */
+SIMSD_API int simsd_kv_commit(int dtype, const void* k_new, const void* v_new, int L, const int32_t* tau,
+                    const uint8_t* section, const int32_t* accepted_len, void* k_cache, void* v_cache,
+                    int num_pages, const int32_t* block_table, int max_pages, int page_size, int32_t* prefix_len,
+                    int Bt, int gamma, int Hkv, int d, int32_t* err_word, void* stream);
+
+/*
+ * simsd_check_error -- synchronises `stream`, copies the device error word
+ * to *host_word (may be NULL) and returns SIMSD_ERR_DEVICE if it is
+ * non-zero, SIMSD_OK otherwise.  The only call that synchronises.
+ */
+SIMSD_API int simsd_check_error(const int32_t* err_word, int32_t* host_word, void* stream);
+
+/* Text of the last CUDA error seen by this thread (empty if none). */
+SIMSD_API const char* simsd_last_error(void);
+
+/* Library version: major*10000 + minor*100 + patch. */
+SIMSD_API int simsd_version(void);
+
+#ifdef __cplusplus
+}
+#endif
+#endif /* SIMSD_H_ */

@@ -1,0 +1,201 @@
+// accept.cu -- greedy longest-prefix acceptance (Sec. 3.2, Eq. (2) at
+// temperature 0: the r-th draft is accepted iff it equals the argmax of the
+// target's distribution at its verification slot).
+//
+// One thread-block cluster per sequence.  The CL CTAs of a cluster split the
+// vocabulary of all gamma+1 rows of that sequence; each CTA streams its
+// slice with 16-byte loads and reduces a 64-bit (value, index) key per row.
+// CTA 0 then gathers the CL partial keys per row through distributed shared
+// memory and walks the draft order.  No global scratch memory is used.
+#include <cooperative_groups.h>
+#include <cuda_runtime.h>
+
+#include "common.cuh"
+#include "kernels.h"
+
+namespace cg = cooperative_groups;
+
+namespace simsd {
+
+constexpr int kAcceptThreads = 512;
+constexpr int kAcceptUnroll = 4;
+constexpr int kMaxRows = 33;  // gamma + 1 <= 33
+
+// Total order used by the argmax: larger key = better.  NaN ranks above every
+// number, -0.0 equals +0.0, and among equal values the lower index wins
+// (the index is stored complemented in the low half).
+__device__ __forceinline__ unsigned long long argmax_key(float x, uint32_t idx) {
+  uint32_t u = __float_as_uint(x);
+  uint32_t k;
+  if (x != x) {
+    k = 0xFFFFFFFFu;
+  } else {
+    if (u == 0x80000000u) u = 0u;
+    k = (u & 0x80000000u) ? ~u : (u | 0x80000000u);
+  }
+  return (static_cast<unsigned long long>(k) << 32) | static_cast<unsigned long long>(~idx);
+}
+
+__device__ __forceinline__ float4 ld_stream_f4(const float* p) {
+  float4 v;
+  asm volatile("ld.global.nc.L1::no_allocate.v4.f32 {%0,%1,%2,%3}, [%4];"
+               : "=f"(v.x), "=f"(v.y), "=f"(v.z), "=f"(v.w)
+               : "l"(p));
+  return v;
+}
+
+template <int CL>
+__global__ void __launch_bounds__(kAcceptThreads) accept_kernel(const float* __restrict__ logits,
+                                                                const int32_t* __restrict__ draft, int gamma,
+                                                                int vocab, int vec4, int32_t* __restrict__ accepted_len,
+                                                                int32_t* __restrict__ out_tokens,
+                                                                int32_t* __restrict__ row_argmax, int32_t* err_word) {
+  __shared__ unsigned long long best[kMaxRows];
+  __shared__ int am[kMaxRows];
+  cg::cluster_group cluster = cg::this_cluster();
+  const int c = static_cast<int>(cluster.block_rank());
+  const int b = blockIdx.x / CL;
+  const int rows = gamma + 1;
+  const int tid = threadIdx.x;
+  for (int r = tid; r < rows; r += kAcceptThreads) best[r] = 0ull;
+  __syncthreads();
+
+  const float* base = logits + static_cast<size_t>(b) * rows * vocab;
+  int cur_row = -1;
+  unsigned long long cur = 0ull;
+  if (vec4) {
+    // this CTA owns float4 columns [c0, c1) of every row
+    const int V4 = vocab >> 2;
+    const int per = (V4 + CL - 1) / CL;
+    const int c0 = min(V4, c * per), c1 = min(V4, c0 + per);
+    const int w = c1 - c0;
+    const int total = rows * w;
+    for (int i0 = tid; i0 < total; i0 += kAcceptThreads * kAcceptUnroll) {
+      float4 v[kAcceptUnroll];
+#pragma unroll
+      for (int u = 0; u < kAcceptUnroll; ++u) {
+        const int idx = i0 + u * kAcceptThreads;
+        if (idx < total) {
+          const int r = idx / w, col = c0 + (idx - r * w);
+          v[u] = ld_stream_f4(base + static_cast<size_t>(r) * vocab + 4 * static_cast<size_t>(col));
+        }
+      }
+#pragma unroll
+      for (int u = 0; u < kAcceptUnroll; ++u) {
+        const int idx = i0 + u * kAcceptThreads;
+        if (idx < total) {
+          const int r = idx / w, col = c0 + (idx - r * w);
+          if (r != cur_row) {
+            if (cur_row >= 0) atomicMax(&best[cur_row], cur);
+            cur_row = r;
+            cur = 0ull;
+          }
+          const uint32_t e = 4u * static_cast<uint32_t>(col);
+          unsigned long long k0 = argmax_key(v[u].x, e), k1 = argmax_key(v[u].y, e + 1);
+          unsigned long long k2 = argmax_key(v[u].z, e + 2), k3 = argmax_key(v[u].w, e + 3);
+          k0 = k0 > k1 ? k0 : k1;
+          k2 = k2 > k3 ? k2 : k3;
+          k0 = k0 > k2 ? k0 : k2;
+          cur = cur > k0 ? cur : k0;
+        }
+      }
+    }
+  } else {
+    const int per = (vocab + CL - 1) / CL;
+    const int c0 = min(vocab, c * per), c1 = min(vocab, c0 + per);
+    const int w = c1 - c0;
+    const int total = rows * w;
+    for (int idx = tid; idx < total; idx += kAcceptThreads) {
+      const int r = idx / w, col = c0 + (idx - r * w);
+      if (r != cur_row) {
+        if (cur_row >= 0) atomicMax(&best[cur_row], cur);
+        cur_row = r;
+        cur = 0ull;
+      }
+      const unsigned long long k = argmax_key(__ldg(base + static_cast<size_t>(r) * vocab + col),
+                                              static_cast<uint32_t>(col));
+      cur = cur > k ? cur : k;
+    }
+  }
+  if (cur_row >= 0) atomicMax(&best[cur_row], cur);
+  __syncthreads();
+  cluster.sync();
+
+  if (c == 0) {
+    for (int r = tid; r < rows; r += kAcceptThreads) {
+      unsigned long long k = best[r];
+#pragma unroll 1
+      for (int peer = 1; peer < CL; ++peer) {
+        const unsigned long long* pb = cluster.map_shared_rank(best, peer);
+        const unsigned long long kp = pb[r];
+        k = k > kp ? k : kp;
+      }
+      const int idx = static_cast<int>(~static_cast<uint32_t>(k & 0xFFFFFFFFull));
+      am[r] = idx;
+      if (row_argmax) row_argmax[static_cast<size_t>(b) * rows + r] = idx;
+    }
+    __syncthreads();
+    if (tid < 32) {
+      // drafts in tau order; lane r checks draft r (gamma <= 32)
+      const int lane = tid;
+      int dr = 0;
+      bool in_range = true, match = false;
+      if (lane < gamma) {
+        dr = draft[static_cast<size_t>(b) * gamma + lane];
+        in_range = dr >= 0 && dr < vocab;
+        match = in_range && dr == am[lane];
+      }
+      const unsigned bad = __ballot_sync(0xffffffffu, !in_range);
+      const unsigned miss = __ballot_sync(0xffffffffu, lane < gamma && !match);
+      const int a = miss ? (__ffs(miss) - 1) : gamma;
+      if (lane == 0) {
+        if (bad) raise_error(err_word, SIMSD_EW_DRAFT);
+        accepted_len[b] = a;
+      }
+      int32_t* ot = out_tokens + static_cast<size_t>(b) * rows;
+      for (int r = lane; r < rows; r += 32) ot[r] = r < a ? draft[static_cast<size_t>(b) * gamma + r] : (r == a ? am[a] : -1);
+    }
+  }
+  cluster.sync();  // peers stay resident until CTA 0 has read their keys
+}
+
+template <int CL>
+static cudaError_t launch_accept_cl(const float* logits, const int32_t* draft, int Bt, int gamma, int vocab,
+                                    int32_t* accepted_len, int32_t* out_tokens, int32_t* row_argmax,
+                                    int32_t* err_word, cudaStream_t stream) {
+  auto kern = accept_kernel<CL>;
+  if (CL > 8) {
+    cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
+    if (e != cudaSuccess) return e;
+  }
+  const int vec4 = (vocab % 4 == 0) && ((reinterpret_cast<uintptr_t>(logits) & 15u) == 0);
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(static_cast<unsigned>(Bt) * CL);
+  cfg.blockDim = dim3(kAcceptThreads);
+  cfg.dynamicSmemBytes = 0;
+  cfg.stream = stream;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeClusterDimension;
+  attr[0].val.clusterDim.x = CL;
+  attr[0].val.clusterDim.y = 1;
+  attr[0].val.clusterDim.z = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, kern, logits, draft, gamma, vocab, vec4, accepted_len, out_tokens, row_argmax,
+                            err_word);
+}
+
+cudaError_t launch_accept(const float* logits, const int32_t* draft, int Bt, int gamma, int vocab,
+                          int32_t* accepted_len, int32_t* out_tokens, int32_t* row_argmax, int32_t* err_word,
+                          int num_sms, cudaStream_t stream) {
+  // enough CTAs to cover every SM a few times; smaller clusters for big batches
+  const int want = 4 * num_sms;
+  if (Bt * 8 < want) return launch_accept_cl<16>(logits, draft, Bt, gamma, vocab, accepted_len, out_tokens,
+                                                 row_argmax, err_word, stream);
+  if (Bt * 4 < want) return launch_accept_cl<8>(logits, draft, Bt, gamma, vocab, accepted_len, out_tokens,
+                                                row_argmax, err_word, stream);
+  return launch_accept_cl<4>(logits, draft, Bt, gamma, vocab, accepted_len, out_tokens, row_argmax, err_word,
+                             stream);
+}
+
+}  // namespace simsd

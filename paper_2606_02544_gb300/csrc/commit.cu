@@ -1,0 +1,105 @@
+// commit.cu -- append the accepted drafts' K/V to the paged cache (Sec. 3.2:
+// the accepted prefix is committed to the block; Sec. 3.3: later steps reuse
+// the cached K/V).  Row r < a_b of sequence b takes the data-slot K/V whose
+// temporal label is r+1 and lands in cache row n_b + r.
+#include <cuda_runtime.h>
+
+#include "common.cuh"
+#include "kernels.h"
+
+namespace simsd {
+
+constexpr int kCommitWarps = 8;
+
+// One warp per (layer, sequence, accepted row, KV head); each lane moves
+// 16-byte chunks of the K row and the V row.
+__global__ void __launch_bounds__(kCommitWarps * 32) kv_commit_copy_kernel(
+    const uint8_t* __restrict__ k_new, const uint8_t* __restrict__ v_new, int L, const int32_t* __restrict__ tau,
+    const uint8_t* __restrict__ section, const int32_t* __restrict__ accepted_len, uint8_t* __restrict__ k_cache,
+    uint8_t* __restrict__ v_cache, int num_pages, const int32_t* __restrict__ block_table, int max_pages,
+    int page_size, const int32_t* __restrict__ prefix_len, int Bt, int gamma, int Hkv, int row_bytes,
+    int32_t* err_word) {
+  const long long wid = (static_cast<long long>(blockIdx.x) * blockDim.x + threadIdx.x) >> 5;
+  const int lane = threadIdx.x & 31;
+  const long long total = static_cast<long long>(L) * Bt * gamma * Hkv;
+  if (wid >= total) return;
+  const int kvh = static_cast<int>(wid % Hkv);
+  const int r = static_cast<int>((wid / Hkv) % gamma);
+  const int b = static_cast<int>((wid / (static_cast<long long>(Hkv) * gamma)) % Bt);
+  const int l = static_cast<int>(wid / (static_cast<long long>(Hkv) * gamma * Bt));
+  const int a = accepted_len[b];
+  const int n = prefix_len[b];
+  if (a < 0 || a > gamma || n < 0 || r >= a) return;  // invalid sequences are reported by the advance kernel
+  const int S = 2 * gamma;
+  // source: the data slot whose label is r+1
+  const bool hit = lane < gamma && section[static_cast<size_t>(b) * S + lane] == kSectData &&
+                   tau[static_cast<size_t>(b) * S + lane] == r + 1;
+  const unsigned m = __ballot_sync(0xffffffffu, hit);
+  if (!m) {
+    if (lane == 0) raise_error(err_word, SIMSD_EW_STEP_MAP);
+    return;
+  }
+  const int src = __ffs(m) - 1;
+  const long long dst_row = static_cast<long long>(n) + r;
+  const long long pidx = dst_row / page_size;
+  if (pidx >= max_pages) {
+    if (lane == 0) raise_error(err_word, SIMSD_EW_PAGE);
+    return;
+  }
+  const int pg = block_table[static_cast<size_t>(b) * max_pages + pidx];
+  if (pg < 0 || pg >= num_pages) {
+    if (lane == 0) raise_error(err_word, SIMSD_EW_PAGE);
+    return;
+  }
+  const int off = static_cast<int>(dst_row % page_size);
+  const size_t s_row = ((static_cast<size_t>(l) * Bt + b) * S + src) * Hkv + kvh;
+  const size_t d_row = ((static_cast<size_t>(l) * num_pages + pg) * Hkv + kvh) * page_size + off;
+  const uint4* ks = reinterpret_cast<const uint4*>(k_new + s_row * row_bytes);
+  const uint4* vs = reinterpret_cast<const uint4*>(v_new + s_row * row_bytes);
+  uint4* kd = reinterpret_cast<uint4*>(k_cache + d_row * row_bytes);
+  uint4* vd = reinterpret_cast<uint4*>(v_cache + d_row * row_bytes);
+  const int chunks = row_bytes >> 4;
+  for (int c = lane; c < chunks; c += 32) {
+    kd[c] = ks[c];
+    vd[c] = vs[c];
+  }
+}
+
+// n_b += a_b once every copy that read n_b has finished (stream order).
+__global__ void kv_commit_advance_kernel(const int32_t* __restrict__ accepted_len, int32_t* __restrict__ prefix_len,
+                                         int Bt, int gamma, int32_t* err_word) {
+  const int b = blockIdx.x * blockDim.x + threadIdx.x;
+  if (b >= Bt) return;
+  const int a = accepted_len[b];
+  const int n = prefix_len[b];
+  if (a < 0 || a > gamma) {
+    raise_error(err_word, SIMSD_EW_ACCEPT_LEN);
+    return;
+  }
+  if (n < 0) {
+    raise_error(err_word, SIMSD_EW_PREFIX_LEN);
+    return;
+  }
+  prefix_len[b] = n + a;
+}
+
+cudaError_t launch_kv_commit(int elem_bytes, const void* k_new, const void* v_new, int L, const int32_t* tau,
+                             const uint8_t* section, const int32_t* accepted_len, void* k_cache, void* v_cache,
+                             int num_pages, const int32_t* block_table, int max_pages, int page_size,
+                             int32_t* prefix_len, int Bt, int gamma, int Hkv, int d, int32_t* err_word,
+                             cudaStream_t stream) {
+  const long long warps = static_cast<long long>(L) * Bt * gamma * Hkv;
+  const long long blocks = (warps + kCommitWarps - 1) / kCommitWarps;
+  if (blocks > 0) {
+    kv_commit_copy_kernel<<<static_cast<unsigned>(blocks), kCommitWarps * 32, 0, stream>>>(
+        static_cast<const uint8_t*>(k_new), static_cast<const uint8_t*>(v_new), L, tau, section, accepted_len,
+        static_cast<uint8_t*>(k_cache), static_cast<uint8_t*>(v_cache), num_pages, block_table, max_pages,
+        page_size, prefix_len, Bt, gamma, Hkv, d * elem_bytes, err_word);
+    cudaError_t e = cudaGetLastError();
+    if (e != cudaSuccess) return e;
+  }
+  kv_commit_advance_kernel<<<(Bt + 127) / 128, 128, 0, stream>>>(accepted_len, prefix_len, Bt, gamma, err_word);
+  return cudaGetLastError();
+}
+
+}  // namespace simsd

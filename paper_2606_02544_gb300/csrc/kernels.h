@@ -1,0 +1,65 @@
+// kernels.h -- internal launch functions behind the C ABI (not exported).
+#pragma once
+#include <cuda.h>
+#include <cuda_runtime.h>
+
+#include <cstddef>
+#include <cstdint>
+
+namespace simsd {
+
+cudaError_t launch_build_mask(const int32_t* step_map, const int32_t* prefix_len, int Bt, int gamma, int32_t* tau,
+                              uint8_t* section, int32_t* rope_pos, uint64_t* mask_bits, int32_t* err_word,
+                              cudaStream_t stream);
+
+cudaError_t launch_accept(const float* logits, const int32_t* draft, int Bt, int gamma, int vocab,
+                          int32_t* accepted_len, int32_t* out_tokens, int32_t* row_argmax, int32_t* err_word,
+                          int num_sms, cudaStream_t stream);
+
+cudaError_t launch_kv_commit(int elem_bytes, const void* k_new, const void* v_new, int L, const int32_t* tau,
+                             const uint8_t* section, const int32_t* accepted_len, void* k_cache, void* v_cache,
+                             int num_pages, const int32_t* block_table, int max_pages, int page_size,
+                             int32_t* prefix_len, int Bt, int gamma, int Hkv, int d, int32_t* err_word,
+                             cudaStream_t stream);
+
+struct AttnF32Args {
+  const float *q, *k_new, *v_new, *k_cache, *v_cache;
+  const int32_t *block_table, *prefix_len, *tau;
+  const uint8_t* section;
+  float* out;
+  int32_t* err_word;
+  int num_pages, max_pages, page_size, Bt, gamma, Hq, Hkv, d;
+  float scale;
+};
+cudaError_t launch_attention_f32(const AttnF32Args& a, cudaStream_t stream);
+
+// bf16 tensor-core path
+struct AttnTcPlan {
+  int nsplit;       // prefix splits per (sequence, KV head, row block)
+  int rb;           // row blocks of 128 query rows
+  int rows_blk;     // query rows per row block (<= 128)
+  int s_blk;        // slots per row block
+  size_t ws_bytes;  // workspace bytes for the split partials (0 if nsplit == 1)
+};
+// Returns false if the shape is not supported by the tensor-core kernel.
+bool plan_attention_tc(int Bt, int gamma, int Hq, int Hkv, int max_pages, int page_size, int num_sms,
+                       AttnTcPlan* plan);
+
+struct AttnTcArgs {
+  const void *q, *k_new, *v_new, *k_cache, *v_cache;
+  const int32_t *block_table, *prefix_len, *tau;
+  const uint8_t* section;
+  void* out;
+  void* workspace;
+  int32_t* err_word;
+  int num_pages, max_pages, page_size, Bt, gamma, Hq, Hkv;
+  float scale;
+};
+// The tensor-map encoder is the driver's cuTensorMapEncodeTiled.
+typedef CUresult (*EncodeTiledFn)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*, const cuuint64_t*,
+                                  const cuuint64_t*, const cuuint32_t*, const cuuint32_t*, CUtensorMapInterleave,
+                                  CUtensorMapSwizzle, CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
+cudaError_t launch_attention_tc(const AttnTcArgs& a, const AttnTcPlan& plan, EncodeTiledFn encode,
+                                cudaStream_t stream);
+
+}  // namespace simsd

@@ -1,0 +1,146 @@
+"""Python binding of libsimsd.so (argument marshalling only).
+
+Each function has the name of the C entry point it calls (include/simsd.h)
+and takes torch CUDA tensors; it reads shapes and data pointers, passes them
+with the current CUDA stream, and raises :class:`SimsdError` on a non-zero
+status.  Every step of the computation runs in the library's kernels; there
+is no fallback: if the library is missing or fails to load, the first call
+raises.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+import threading
+
+import torch
+
+_HERE = os.path.dirname(os.path.abspath(__file__))
+LIB_PATH = os.path.join(_HERE, "_build", "libsimsd.so")
+
+SIMSD_OK, SIMSD_ERR_INVALID_ARG, SIMSD_ERR_UNSUPPORTED, SIMSD_ERR_CUDA, SIMSD_ERR_DEVICE = 0, 1, 2, 3, 4
+SIMSD_F32, SIMSD_BF16 = 0, 1
+SECT_DATA, SECT_MASK, SECT_PAD = 0, 1, 255
+EW_STEP_MAP, EW_PREFIX_LEN, EW_PAGE, EW_DRAFT, EW_TIMEOUT, EW_ACCEPT_LEN = 1, 2, 4, 8, 16, 32
+
+EXPORTED = ("simsd_build_mask", "simsd_verify_workspace_bytes", "simsd_verify_attention", "simsd_accept",
+            "simsd_kv_commit", "simsd_check_error", "simsd_last_error", "simsd_version")
+
+
+class SimsdError(RuntimeError):
+    def __init__(self, status, where, detail=""):
+        super().__init__(f"{where} failed with status {status}: {detail}")
+        self.status = status
+
+
+_lib = None
+_lock = threading.Lock()
+
+
+def load_library(path: str = LIB_PATH):
+    """Loads libsimsd.so once; raises if it is missing (build it with
+    ``paper_2606_02544_gb300.build.build()``)."""
+    global _lib
+    with _lock:
+        if _lib is None:
+            if not os.path.exists(path):
+                raise RuntimeError(f"libsimsd.so not found at {path}; run paper_2606_02544_gb300.build.build()")
+            lib = ctypes.CDLL(path)
+            P, I, F, Z = ctypes.c_void_p, ctypes.c_int, ctypes.c_float, ctypes.c_size_t
+            lib.simsd_build_mask.argtypes = [P, P, I, I, P, P, P, P, P, P]
+            lib.simsd_verify_workspace_bytes.argtypes = [I, I, I, I, I, I, I, I]
+            lib.simsd_verify_workspace_bytes.restype = Z
+            lib.simsd_verify_attention.argtypes = [I, P, P, P, P, P, I, P, I, I, P, P, P, P, I, I, I, I, I, F, P,
+                                                   P, Z, P, P]
+            lib.simsd_accept.argtypes = [P, P, I, I, I, P, P, P, P, P]
+            lib.simsd_kv_commit.argtypes = [I, P, P, I, P, P, P, P, P, I, P, I, I, P, I, I, I, I, P, P]
+            lib.simsd_check_error.argtypes = [P, P, P]
+            lib.simsd_last_error.restype = ctypes.c_char_p
+            for name in ("simsd_build_mask", "simsd_verify_attention", "simsd_accept", "simsd_kv_commit",
+                         "simsd_check_error", "simsd_version"):
+                getattr(lib, name).restype = ctypes.c_int
+            _lib = lib
+    return _lib
+
+
+def _p(t):
+    return None if t is None else ctypes.c_void_p(t.data_ptr())
+
+
+def _stream(stream):
+    s = torch.cuda.current_stream() if stream is None else stream
+    return ctypes.c_void_p(s.cuda_stream)
+
+
+def _check(rc, where):
+    if rc != SIMSD_OK:
+        detail = load_library().simsd_last_error().decode(errors="replace")
+        raise SimsdError(rc, where, detail)
+
+
+def _dtype_code(t):
+    if t.dtype == torch.bfloat16:
+        return SIMSD_BF16
+    if t.dtype == torch.float32:
+        return SIMSD_F32
+    raise TypeError(f"unsupported dtype {t.dtype}")
+
+
+def simsd_version() -> int:
+    return load_library().simsd_version()
+
+
+def simsd_build_mask(step_map, prefix_len, gamma, tau, section, rope_pos, mask_bits=None, err_word=None,
+                     stream=None):
+    Bt = prefix_len.shape[0]
+    rc = load_library().simsd_build_mask(_p(step_map), _p(prefix_len), Bt, gamma, _p(tau), _p(section),
+                                         _p(rope_pos), _p(mask_bits), _p(err_word), _stream(stream))
+    _check(rc, "simsd_build_mask")
+
+
+def simsd_verify_workspace_bytes(dtype_code, Bt, gamma, Hq, Hkv, d, max_pages, page_size) -> int:
+    return int(load_library().simsd_verify_workspace_bytes(dtype_code, Bt, gamma, Hq, Hkv, d, max_pages, page_size))
+
+
+def simsd_verify_attention(q, k_new, v_new, k_cache, v_cache, block_table, prefix_len, tau, section, out,
+                           workspace=None, err_word=None, softmax_scale=0.0, rope_pos=None, stream=None):
+    """q/out [Bt][2g][Hq][d]; k_new/v_new [Bt][2g][Hkv][d];
+    k_cache/v_cache [num_pages][Hkv][P][d]; block_table [Bt][max_pages]."""
+    Bt, S, Hq, d = q.shape
+    Hkv = k_new.shape[2]
+    num_pages, _, P, _ = k_cache.shape
+    max_pages = block_table.shape[1]
+    ws_bytes = 0 if workspace is None else workspace.numel() * workspace.element_size()
+    rc = load_library().simsd_verify_attention(
+        _dtype_code(q), _p(q), _p(k_new), _p(v_new), _p(k_cache), _p(v_cache), num_pages, _p(block_table),
+        max_pages, P, _p(prefix_len), _p(tau), _p(section), _p(rope_pos), Bt, S // 2, Hq, Hkv, d,
+        float(softmax_scale), _p(out), _p(workspace), ws_bytes, _p(err_word), _stream(stream))
+    _check(rc, "simsd_verify_attention")
+
+
+def simsd_accept(logits, draft, accepted_len, out_tokens, row_argmax=None, err_word=None, stream=None):
+    Bt, rows, V = logits.shape
+    rc = load_library().simsd_accept(_p(logits), _p(draft), Bt, rows - 1, V, _p(accepted_len), _p(out_tokens),
+                                     _p(row_argmax), _p(err_word), _stream(stream))
+    _check(rc, "simsd_accept")
+
+
+def simsd_kv_commit(k_new, v_new, tau, section, accepted_len, k_cache, v_cache, block_table, prefix_len,
+                    err_word=None, stream=None):
+    """k_new/v_new [L][Bt][2g][Hkv][d]; k_cache/v_cache [L][num_pages][Hkv][P][d]."""
+    L, Bt, S, Hkv, d = k_new.shape
+    num_pages, P = k_cache.shape[1], k_cache.shape[3]
+    rc = load_library().simsd_kv_commit(
+        _dtype_code(k_new), _p(k_new), _p(v_new), L, _p(tau), _p(section), _p(accepted_len), _p(k_cache),
+        _p(v_cache), num_pages, _p(block_table), block_table.shape[1], P, _p(prefix_len), Bt, S // 2, Hkv, d,
+        _p(err_word), _stream(stream))
+    _check(rc, "simsd_kv_commit")
+
+
+def simsd_check_error(err_word, stream=None):
+    """Synchronises the stream; returns the device error word (int)."""
+    w = ctypes.c_int32(0)
+    rc = load_library().simsd_check_error(_p(err_word), ctypes.byref(w), _stream(stream))
+    if rc not in (SIMSD_OK, SIMSD_ERR_DEVICE):
+        _check(rc, "simsd_check_error")
+    return int(w.value)

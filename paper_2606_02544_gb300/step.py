@@ -1,0 +1,104 @@
+"""One verification step of SimSD through the C ABI.
+
+A step (Sec. 3.2, one target verification forward per speculative step):
+  1. simsd_build_mask      tau / section / RoPE-copy positions (Eq. (1))
+  2. simsd_verify_attention, once per layer (the masked attention)
+  3. simsd_accept          greedy longest-prefix acceptance (Eq. (2), T=0)
+  4. simsd_kv_commit       append the accepted drafts' K/V, advance n_b
+All four run on one stream and are captured into one CUDA graph, so the
+step needs no host round trip.  PyTorch only allocates the buffers.
+"""
+from __future__ import annotations
+
+import torch
+
+from . import simsd
+from .inputs import StepInputs
+
+
+class VerifyStep:
+    """Device buffers and the call sequence of one verification step.
+
+    ``restore_prefix`` copies the original prefix lengths back before each
+    step (a 4*Bt-byte device copy) so that repeated steps verify the same
+    block against the same prefix: the commit writes rows past the original
+    prefix, which the restored lengths never read.
+    """
+
+    def __init__(self, si: StepInputs, restore_prefix: bool = True):
+        w = si.w
+        dev = si.q.device
+        self.si = si
+        self.w = w
+        self.restore_prefix = restore_prefix
+        self.L = si.q.shape[0]
+        i32 = dict(dtype=torch.int32, device=dev)
+        self.n_orig = si.prefix_len.clone()
+        self.n = si.prefix_len.clone()
+        self.tau = torch.empty(w.Bt, w.S, **i32)
+        self.section = torch.empty(w.Bt, w.S, dtype=torch.uint8, device=dev)
+        self.rope_pos = torch.empty(w.Bt, w.S, **i32)
+        self.out = torch.empty_like(si.q)
+        dt = simsd.SIMSD_BF16 if si.q.dtype == torch.bfloat16 else simsd.SIMSD_F32
+        ws = simsd.simsd_verify_workspace_bytes(dt, w.Bt, w.gamma, w.Hq, w.Hkv, w.d, si.block_table.shape[1],
+                                                w.page_size)
+        self.workspace = torch.empty(max(ws, 16), dtype=torch.uint8, device=dev) if ws > 0 else None
+        self.accepted_len = torch.empty(w.Bt, **i32)
+        self.out_tokens = torch.empty(w.Bt, w.gamma + 1, **i32)
+        self.row_argmax = torch.empty(w.Bt, w.gamma + 1, **i32)
+        self.err = torch.zeros(1, **i32)
+        self.graph = None
+        self.attn_events = None
+
+    # ------------------------------------------------------------------
+    def run(self, attn_events=None):
+        """Issues the whole step on the current stream (eager or captured).
+        ``attn_events`` = (start, end) events recorded around the layers'
+        attention calls."""
+        si, w = self.si, self.w
+        if self.restore_prefix:
+            self.n.copy_(self.n_orig, non_blocking=True)
+        simsd.simsd_build_mask(si.step_map, self.n, w.gamma, self.tau, self.section, self.rope_pos,
+                               err_word=self.err)
+        if attn_events is not None:
+            attn_events[0].record()
+        for l in range(self.L):
+            simsd.simsd_verify_attention(si.q[l], si.k_new[l], si.v_new[l], si.k_cache[l], si.v_cache[l],
+                                         si.block_table, self.n, self.tau, self.section, self.out[l],
+                                         workspace=self.workspace, err_word=self.err)
+        if attn_events is not None:
+            attn_events[1].record()
+        simsd.simsd_accept(si.logits, si.draft, self.accepted_len, self.out_tokens, self.row_argmax,
+                           err_word=self.err)
+        simsd.simsd_kv_commit(si.k_new, si.v_new, self.tau, self.section, self.accepted_len, si.k_cache,
+                              si.v_cache, si.block_table, self.n, err_word=self.err)
+
+    def launches_per_step(self) -> int:
+        """Kernels of this library launched by one step."""
+        combine = 1 if self.workspace is not None else 0
+        return 1 + self.L * (1 + combine) + 1 + 2
+
+    def capture(self, time_attention: bool = True):
+        """Captures one step into a CUDA graph (with event-record nodes
+        around the attention layers when ``time_attention``)."""
+        if time_attention:
+            self.attn_events = (torch.cuda.Event(enable_timing=True, external=True),
+                                torch.cuda.Event(enable_timing=True, external=True))
+        s = torch.cuda.Stream()
+        s.wait_stream(torch.cuda.current_stream())
+        with torch.cuda.stream(s):
+            self.run()  # warm-up outside capture (lazy library setup)
+        torch.cuda.current_stream().wait_stream(s)
+        torch.cuda.synchronize()
+        g = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(g):
+            self.run(self.attn_events)
+        self.graph = g
+        return g
+
+    def replay(self):
+        self.graph.replay()
+
+    def verified_tokens(self) -> int:
+        """Accepted drafts plus the one target token per sequence."""
+        return int(self.accepted_len.sum().item()) + self.w.Bt

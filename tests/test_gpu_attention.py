@@ -1,0 +1,155 @@
+"""GPU parity of simsd_verify_attention against the fp64 oracle.
+
+fp32 path: max abs error <= 1e-5.  bf16 path: |gpu - oracle| <= 2e-2 +
+2e-2*|oracle| element-wise.  Shapes span several 64-key tiles with ragged
+tails, page-boundary prefixes, every page size the kernel takes, split and
+unsplit prefixes, row blocks, non-identity step maps, padding, poisoned
+unused cache rows, harder score distributions, and the error paths.
+"""
+import numpy as np
+import pytest
+import torch
+
+from paper_2606_02544_gb300 import inputs, simsd
+from tests._gpu import assert_attention_close, gpu_attention, oracle_attention
+
+pytestmark = pytest.mark.gpu
+
+
+def _w(dtype="bf16", Bt=3, Hq=16, Hkv=8, d=128, gamma=4, prefix=(0, 300), P=64, seed=0, std=None):
+    std = (1.0 if dtype == "f32" else 1 / np.sqrt(128)) if std is None else std
+    return inputs.Workload("t", dtype, Bt, Hq, Hkv, d, gamma, prefix, 1, 64, 0.5, std, 1.0, seed, P)
+
+
+def _check(si, seqs=None):
+    out, word, _ = gpu_attention(si)
+    want, werr = oracle_attention(si, seqs=seqs)
+    assert word == werr
+    got = out if seqs is None else out[torch.as_tensor(seqs, device=out.device)]
+    return assert_attention_close(got, want, si.w.dtype)
+
+
+def test_c1_tiny_fp32():
+    si = inputs.make_step_inputs(inputs.WORKLOADS["c1"], device="cuda")
+    _check(si)
+
+
+@pytest.mark.parametrize("d", [64, 128])
+def test_fp32_ragged_paged(d):
+    w = _w("f32", Bt=4, Hq=4, Hkv=2, d=d, gamma=3, P=16)
+    si = inputs.make_step_inputs(w, device="cuda", prefix_override=[0, 17, 64, 130], random_step_map=True,
+                                 poison_unused_rows=True)
+    _check(si)
+
+
+@pytest.mark.parametrize("gamma,Hq,Hkv", [(1, 8, 8), (4, 16, 8), (8, 32, 8), (16, 32, 8), (32, 32, 8),
+                                          (3, 6, 2), (5, 24, 8)])
+def test_bf16_shapes(gamma, Hq, Hkv):
+    # R = (Hq/Hkv)*2*gamma rows per KV head: 2 .. 256 (two row blocks)
+    w = _w(Bt=3, Hq=Hq, Hkv=Hkv, gamma=gamma, seed=gamma)
+    si = inputs.make_step_inputs(w, device="cuda", prefix_override=[0, 65, 200], random_step_map=True,
+                                 poison_unused_rows=True)
+    _check(si)
+
+
+@pytest.mark.parametrize("n", [0, 1, 63, 64, 65, 127, 128, 129, 1000])
+def test_bf16_page_edges(n):
+    w = _w(Bt=2, gamma=4)
+    si = inputs.make_step_inputs(w, device="cuda", prefix_override=[n, max(n - 1, 0)], poison_unused_rows=True)
+    _check(si)
+
+
+@pytest.mark.parametrize("P", [8, 16, 32, 64, 128, 256])
+def test_bf16_page_sizes(P):
+    w = _w(Bt=3, gamma=4, P=P, seed=P)
+    si = inputs.make_step_inputs(w, device="cuda", prefix_override=[5, 200, 333], random_step_map=True,
+                                 poison_unused_rows=True)
+    _check(si)
+
+
+@pytest.mark.parametrize("Bt", [1, 2, 9, 40, 130])
+def test_bf16_split_and_unsplit(Bt):
+    # small batches split the prefix (partials + combine); big ones do not
+    w = _w(Bt=Bt, Hq=32, Hkv=8, gamma=8, prefix=(1, 700), seed=Bt)
+    si = inputs.make_step_inputs(w, device="cuda", random_step_map=True, poison_unused_rows=True)
+    seqs = None if Bt <= 9 else list(range(0, Bt, max(1, Bt // 7)))
+    _check(si, seqs)
+
+
+@pytest.mark.parametrize("kind", ["unit_scores", "peaked", "growing"])
+def test_bf16_hard_score_distributions(kind):
+    # Q,K ~ N(0,1): scores ~ N(0,1) after the 1/sqrt(d) scale; "peaked": one
+    # key per row far above the rest; "growing": later keys score higher, so
+    # the running maximum rises many times (exercises the O rescale).
+    w = _w(Bt=3, Hq=32, Hkv=8, gamma=8, seed=11, std=1.0 if kind == "unit_scores" else None)
+    si = inputs.make_step_inputs(w, device="cuda", prefix_override=[300, 1000, 64 * 9 + 5], random_step_map=True)
+    if kind == "peaked":
+        q = si.q[0].float()
+        bt = si.block_table
+        for b in range(w.Bt):
+            j = (b * 37) % int(si.prefix_len[b])
+            pg, off = int(bt[b, j // w.page_size]), j % w.page_size
+            for kvh in range(w.Hkv):
+                qm = q[b, :, kvh * w.g:(kvh + 1) * w.g].mean((0, 1))
+                si.k_cache[0, pg, kvh, off] = (qm / qm.norm() * 40).to(torch.bfloat16)
+    if kind == "growing":
+        ramp = torch.linspace(0, 6, w.page_size, device="cuda")
+        qdir = si.q[0].float().mean((0, 1, 2))
+        qdir = qdir / qdir.norm()
+        order = torch.zeros(si.num_pages, device="cuda")
+        for b in range(w.Bt):
+            for p_i in range((int(si.prefix_len[b]) + w.page_size - 1) // w.page_size):
+                order[int(si.block_table[b, p_i])] = p_i
+        boost = (order[:, None] * 6 + ramp[None, :])  # [pages][P]
+        si.k_cache[0] = (si.k_cache[0].float() + boost[:, None, :, None] * qdir * 3).to(torch.bfloat16)
+    _check(si)
+
+
+def test_padding_slots_and_error_paths():
+    w = _w(Bt=4, gamma=4)
+    si = inputs.make_step_inputs(w, device="cuda", prefix_override=[10, 100, 70, 5])
+    sm = si.step_map.clone()
+    sm[0, 2] = 0                                  # padding slot in sequence 0
+    sm[3] = torch.tensor([1, 1, 2, 3], dtype=torch.int32)   # invalid map: all padding
+    si.step_map = sm
+    n = si.prefix_len.clone()
+    n[1] = si.block_table.shape[1] * w.page_size + 3         # beyond the block table
+    si.prefix_len = n
+    bt = si.block_table.clone()
+    bt[2, 1] = si.num_pages + 5                              # page id outside the pool
+    si.block_table = bt
+    out, word, _ = gpu_attention(si)
+    want, werr = oracle_attention(si)
+    assert word == werr and word & simsd.EW_PREFIX_LEN and word & simsd.EW_PAGE and word & simsd.EW_STEP_MAP
+    assert_attention_close(out, want, "bf16")
+    assert (out[1:4].float() == 0).all() and (out[0, [2, 6]].float() == 0).all()
+
+
+def test_deterministic():
+    w = _w(Bt=5, Hq=32, Hkv=8, gamma=8, prefix=(100, 900), seed=3)
+    si = inputs.make_step_inputs(w, device="cuda", random_step_map=True)
+    a, _, _ = gpu_attention(si)
+    b, _, _ = gpu_attention(si)
+    assert torch.equal(a, b)
+
+
+@pytest.mark.parametrize("name", ["c2", "c3"])
+def test_full_size_configs(name):
+    wl = inputs.WORKLOADS[name]
+    si = inputs.make_step_inputs(wl, device="cuda", poison_unused_rows=True)
+    seqs = None if name == "c2" else [0, 11, 31]
+    _check(si, seqs)
+
+
+def test_c4_sampled_layers():
+    # SDAR-8B shapes at full batch and prefix range; two of the 36 layers
+    # (each layer is one independent launch with the same configuration)
+    wl = inputs.WORKLOADS["c4"]
+    si = inputs.make_step_inputs(wl, device="cuda", layers=2)
+    n = si.prefix_len.cpu()
+    seqs = [int(torch.argmax(n)), int(torch.argmin(n)), 17]
+    for layer in (0, 1):
+        out, word, _ = gpu_attention(si, layer=layer)
+        want, werr = oracle_attention(si, layer=layer, seqs=seqs)
+        assert word == werr == 0
+        assert_attention_close(out[torch.as_tensor(seqs, device="cuda")], want, "bf16")

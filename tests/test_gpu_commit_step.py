@@ -1,0 +1,93 @@
+"""GPU parity of simsd_kv_commit (bit-exact cache and prefix lengths) and of
+the whole verification step, eager and captured in a CUDA graph."""
+import numpy as np
+import pytest
+import torch
+
+from oracle import simsd_oracle as orc
+from paper_2606_02544_gb300 import inputs, simsd
+from paper_2606_02544_gb300.step import VerifyStep
+from tests._gpu import assert_attention_close, gpu_mask, oracle_attention
+
+pytestmark = pytest.mark.gpu
+
+
+def _commit_case(dtype, L, gamma, P, n, seed):
+    w = inputs.Workload("c", dtype, len(n), 8, 4, 128 if dtype == "bf16" else 64, gamma, (0, 0), L, 16, 0.5,
+                        1.0, 1.0, seed, P)
+    return inputs.make_step_inputs(w, device="cuda", prefix_override=n, random_step_map=True, with_logits=False)
+
+
+@pytest.mark.parametrize("dtype,L,gamma,P", [("bf16", 3, 8, 64), ("bf16", 2, 32, 16), ("f32", 2, 4, 8),
+                                             ("bf16", 1, 1, 64)])
+def test_commit_bit_exact(dtype, L, gamma, P):
+    n = [0, 63, 64, 5, 200, 127]
+    si = _commit_case(dtype, L, gamma, P, n, seed=gamma + P)
+    rng = np.random.default_rng(gamma)
+    a = torch.as_tensor(rng.integers(0, gamma + 1, len(n)).astype(np.int32), device="cuda")
+    tau, sect, _, _, err = gpu_mask(si, mask_bits=False)
+    kc0, vc0 = si.k_cache.clone(), si.v_cache.clone()
+    nn = si.prefix_len.clone()
+    simsd.simsd_kv_commit(si.k_new, si.v_new, tau, sect, a, si.k_cache, si.v_cache, si.block_table, nn, err)
+    word = simsd.simsd_check_error(err)
+    rk, rv, rn, rerr = orc.kv_commit(inputs.host_bits(si.k_new), inputs.host_bits(si.v_new),
+                                     si.step_map.cpu().numpy(), a.cpu().numpy(), inputs.host_bits(kc0),
+                                     inputs.host_bits(vc0), si.block_table.cpu().numpy(),
+                                     si.prefix_len.cpu().numpy(), gamma)
+    assert word == rerr == 0
+    np.testing.assert_array_equal(nn.cpu().numpy(), rn)
+    np.testing.assert_array_equal(inputs.host_bits(si.k_cache), rk)
+    np.testing.assert_array_equal(inputs.host_bits(si.v_cache), rv)
+
+
+def test_commit_error_paths():
+    si = _commit_case("bf16", 2, 4, 16, [0, 14, 30, 7], seed=1)
+    sm = si.step_map.clone()
+    sm[3] = 0                                   # no source slot for sequence 3
+    si.step_map = sm
+    bt = si.block_table.clone()
+    bt[2, 30 // 16] = si.num_pages              # destination page outside the pool
+    si.block_table = bt
+    a = torch.tensor([2, 9, 3, 1], dtype=torch.int32, device="cuda")  # sequence 1: a > gamma
+    tau, sect, _, _, err = gpu_mask(si, mask_bits=False)
+    kc0, vc0 = si.k_cache.clone(), si.v_cache.clone()
+    nn = si.prefix_len.clone()
+    simsd.simsd_kv_commit(si.k_new, si.v_new, tau, sect, a, si.k_cache, si.v_cache, si.block_table, nn, err)
+    word = simsd.simsd_check_error(err)
+    rk, rv, rn, rerr = orc.kv_commit(inputs.host_bits(si.k_new), inputs.host_bits(si.v_new),
+                                     si.step_map.cpu().numpy(), a.cpu().numpy(), inputs.host_bits(kc0),
+                                     inputs.host_bits(vc0), si.block_table.cpu().numpy(),
+                                     si.prefix_len.cpu().numpy(), 4)
+    assert word == rerr and word & simsd.EW_PAGE and word & simsd.EW_ACCEPT_LEN and word & simsd.EW_STEP_MAP
+    np.testing.assert_array_equal(nn.cpu().numpy(), rn)
+    np.testing.assert_array_equal(inputs.host_bits(si.k_cache), rk)
+    np.testing.assert_array_equal(inputs.host_bits(si.v_cache), rv)
+
+
+@pytest.mark.parametrize("name", ["c1", "c2"])
+@pytest.mark.parametrize("graph", [False, True])
+def test_whole_step(name, graph):
+    wl = inputs.WORKLOADS[name]
+    si = inputs.make_step_inputs(wl, device="cuda")
+    want_out, werr = oracle_attention(si)
+    ra, rot, ram, aerr = orc.accept(si.logits.cpu().numpy(), si.draft.cpu().numpy(), wl.gamma)
+    kc0, vc0 = inputs.host_bits(si.k_cache), inputs.host_bits(si.v_cache)
+    st = VerifyStep(si, restore_prefix=True)
+    if graph:
+        st.capture()
+        for _ in range(3):
+            st.replay()
+    else:
+        st.run()
+        st.run()
+    word = simsd.simsd_check_error(st.err)
+    assert word == 0 and werr == 0 and aerr == 0
+    assert_attention_close(st.out[0], want_out, wl.dtype)
+    np.testing.assert_array_equal(st.accepted_len.cpu().numpy(), ra)
+    np.testing.assert_array_equal(st.out_tokens.cpu().numpy(), rot)
+    np.testing.assert_array_equal(st.n.cpu().numpy(), si.prefix_len.cpu().numpy() + ra)
+    rk, rv, rn, cerr = orc.kv_commit(inputs.host_bits(si.k_new), inputs.host_bits(si.v_new),
+                                     si.step_map.cpu().numpy(), ra, kc0, vc0, si.block_table.cpu().numpy(),
+                                     si.prefix_len.cpu().numpy(), wl.gamma)
+    np.testing.assert_array_equal(inputs.host_bits(si.k_cache), rk)
+    np.testing.assert_array_equal(inputs.host_bits(si.v_cache), rv)
