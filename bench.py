@@ -147,6 +147,13 @@ def _algorithmic_bytes(si):
     return attn, flops, accept
 
 
+def _flush_l2(buf):
+    """Evicts the step's data from L2: write a buffer twice the L2 size, then
+    read it back so the dirty lines are written out before the next step."""
+    buf.fill_(1)
+    buf.view(-1, 4096).amax(dim=1)
+
+
 # ----------------------------------------------------------------------------
 def run_gpu(args):
     import torch
@@ -185,7 +192,7 @@ def run_gpu(args):
     with torch.cuda.graph(graph, stream=stream):
         for m in range(M):
             if flush is not None:
-                flush.zero_()
+                _flush_l2(flush)
             e = ev[m]
             e[0].record()
             st.run(attn_events=(e[1], e[2]))
@@ -197,7 +204,7 @@ def run_gpu(args):
     g_acc = torch.cuda.CUDAGraph()
     with torch.cuda.graph(g_acc, stream=stream):
         if flush is not None:
-            flush.zero_()
+            _flush_l2(flush)
         acc_ev[0].record()
         simsd.simsd_accept(si.logits, si.draft, st.accepted_len, st.out_tokens, st.row_argmax, err_word=st.err)
         acc_ev[1].record()
@@ -284,7 +291,7 @@ def run_gpu(args):
                        "gamma": wl.gamma, "prefix": list(wl.prefix), "layers": st.L, "vocab": wl.vocab,
                        "page_size": wl.page_size, "p_agree": wl.p_agree, "seed": wl.seed,
                        "verified_tokens_per_step": tokens_per_step, "draft_tokens_per_step": wl.Bt * wl.gamma,
-                       "l2": "flushed (256 MB write) before every step" if need_flush else
+                       "l2": "flushed before every step (258 MB write + read)" if need_flush else
                        "inputs larger than L2 (no flush)",
                        "timing": f"CUDA graph of {M} steps; per-step CUDA events; max over ranks",
                        "parallelism": f"replicas x{world}"},

@@ -3,8 +3,10 @@
 // target's distribution at its verification slot).
 //
 // One thread-block cluster per sequence.  The CL CTAs of a cluster split the
-// vocabulary of all gamma+1 rows of that sequence; each CTA streams its
-// slice with 16-byte loads and reduces a 64-bit (value, index) key per row.
+// sequence's [gamma+1][vocab] block into contiguous spans; each thread
+// streams 16-byte loads (8 in flight), keeps a running (value, index) per
+// row with plain float compares, and folds it into a 64-bit key per row in
+// shared memory when its row changes.
 // CTA 0 then gathers the CL partial keys per row through distributed shared
 // memory and walks the draft order.  No global scratch memory is used.
 #include <cooperative_groups.h>
@@ -18,7 +20,7 @@ namespace cg = cooperative_groups;
 namespace simsd {
 
 constexpr int kAcceptThreads = 512;
-constexpr int kAcceptUnroll = 4;
+constexpr int kAcceptUnroll = 8;
 constexpr int kMaxRows = 33;  // gamma + 1 <= 33
 
 // Total order used by the argmax: larger key = better.  NaN ranks above every
@@ -44,6 +46,28 @@ __device__ __forceinline__ float4 ld_stream_f4(const float* p) {
   return v;
 }
 
+// Running argmax of one thread over the elements it visits in increasing
+// index order within one row: the strict '>' keeps the first of equal
+// values (and treats -0.0 as +0.0); NaNs are tracked apart (first one wins).
+struct RowBest {
+  float v;
+  uint32_t i;
+  uint32_t nan_i;
+  __device__ __forceinline__ void reset(uint32_t first) {
+    v = -INFINITY;
+    i = first;
+    nan_i = 0xFFFFFFFFu;
+  }
+  __device__ __forceinline__ void see(float x, uint32_t e) {
+    const bool gt = x > v;
+    v = gt ? x : v;
+    i = gt ? e : i;
+  }
+  __device__ __forceinline__ unsigned long long key() const {
+    return nan_i != 0xFFFFFFFFu ? argmax_key(__int_as_float(0x7fc00000), nan_i) : argmax_key(v, i);
+  }
+};
+
 template <int CL>
 __global__ void __launch_bounds__(kAcceptThreads) accept_kernel(const float* __restrict__ logits,
                                                                 const int32_t* __restrict__ draft, int gamma,
@@ -60,64 +84,71 @@ __global__ void __launch_bounds__(kAcceptThreads) accept_kernel(const float* __r
   for (int r = tid; r < rows; r += kAcceptThreads) best[r] = 0ull;
   __syncthreads();
 
+  // This CTA owns one contiguous span of the sequence's [rows][vocab] block
+  // (in 16-byte units when rows are 16-byte aligned).
   const float* base = logits + static_cast<size_t>(b) * rows * vocab;
-  int cur_row = -1;
-  unsigned long long cur = 0ull;
+  const int W = vec4 ? (vocab >> 2) : vocab;   // units per row
+  const long long F = static_cast<long long>(rows) * W;
+  const long long per = (F + CL - 1) / CL;
+  const long long f0 = min(F, c * per), f1 = min(F, f0 + per);
+  long long f = f0 + tid;
+  int row = static_cast<int>(f / W);
+  int col = static_cast<int>(f - static_cast<long long>(row) * W);
+  int cur = row;
+  RowBest rb;
+  rb.reset(vec4 ? 4u * col : static_cast<uint32_t>(col));
+  constexpr int kStride = kAcceptThreads;
   if (vec4) {
-    // this CTA owns float4 columns [c0, c1) of every row
-    const int V4 = vocab >> 2;
-    const int per = (V4 + CL - 1) / CL;
-    const int c0 = min(V4, c * per), c1 = min(V4, c0 + per);
-    const int w = c1 - c0;
-    const int total = rows * w;
-    for (int i0 = tid; i0 < total; i0 += kAcceptThreads * kAcceptUnroll) {
+    const float4* b4 = reinterpret_cast<const float4*>(base);
+    for (; f < f1; f += static_cast<long long>(kStride) * kAcceptUnroll) {
       float4 v[kAcceptUnroll];
 #pragma unroll
       for (int u = 0; u < kAcceptUnroll; ++u) {
-        const int idx = i0 + u * kAcceptThreads;
-        if (idx < total) {
-          const int r = idx / w, col = c0 + (idx - r * w);
-          v[u] = ld_stream_f4(base + static_cast<size_t>(r) * vocab + 4 * static_cast<size_t>(col));
-        }
+        const long long fu = f + static_cast<long long>(u) * kStride;
+        if (fu < f1) v[u] = ld_stream_f4(reinterpret_cast<const float*>(b4 + fu));
       }
 #pragma unroll
       for (int u = 0; u < kAcceptUnroll; ++u) {
-        const int idx = i0 + u * kAcceptThreads;
-        if (idx < total) {
-          const int r = idx / w, col = c0 + (idx - r * w);
-          if (r != cur_row) {
-            if (cur_row >= 0) atomicMax(&best[cur_row], cur);
-            cur_row = r;
-            cur = 0ull;
-          }
-          const uint32_t e = 4u * static_cast<uint32_t>(col);
-          unsigned long long k0 = argmax_key(v[u].x, e), k1 = argmax_key(v[u].y, e + 1);
-          unsigned long long k2 = argmax_key(v[u].z, e + 2), k3 = argmax_key(v[u].w, e + 3);
-          k0 = k0 > k1 ? k0 : k1;
-          k2 = k2 > k3 ? k2 : k3;
-          k0 = k0 > k2 ? k0 : k2;
-          cur = cur > k0 ? cur : k0;
+        if (f + static_cast<long long>(u) * kStride >= f1) break;
+        if (row != cur) {
+          atomicMax(&best[cur], rb.key());
+          cur = row;
+          rb.reset(4u * col);
+        }
+        const uint32_t e = 4u * static_cast<uint32_t>(col);
+        if (isnan(v[u].x) | isnan(v[u].y) | isnan(v[u].z) | isnan(v[u].w)) {
+          if (rb.nan_i == 0xFFFFFFFFu)
+            rb.nan_i = isnan(v[u].x) ? e : isnan(v[u].y) ? e + 1 : isnan(v[u].z) ? e + 2 : e + 3;
+        }
+        rb.see(v[u].x, e);
+        rb.see(v[u].y, e + 1);
+        rb.see(v[u].z, e + 2);
+        rb.see(v[u].w, e + 3);
+        col += kStride;
+        if (col >= W) {
+          row += col / W;
+          col %= W;
         }
       }
     }
   } else {
-    const int per = (vocab + CL - 1) / CL;
-    const int c0 = min(vocab, c * per), c1 = min(vocab, c0 + per);
-    const int w = c1 - c0;
-    const int total = rows * w;
-    for (int idx = tid; idx < total; idx += kAcceptThreads) {
-      const int r = idx / w, col = c0 + (idx - r * w);
-      if (r != cur_row) {
-        if (cur_row >= 0) atomicMax(&best[cur_row], cur);
-        cur_row = r;
-        cur = 0ull;
+    for (; f < f1; f += kStride) {
+      const float x = __ldg(base + f);
+      if (row != cur) {
+        atomicMax(&best[cur], rb.key());
+        cur = row;
+        rb.reset(col);
       }
-      const unsigned long long k = argmax_key(__ldg(base + static_cast<size_t>(r) * vocab + col),
-                                              static_cast<uint32_t>(col));
-      cur = cur > k ? cur : k;
+      if (isnan(x) && rb.nan_i == 0xFFFFFFFFu) rb.nan_i = col;
+      rb.see(x, static_cast<uint32_t>(col));
+      col += kStride;
+      if (col >= W) {
+        row += col / W;
+        col %= W;
+      }
     }
   }
-  if (cur_row >= 0) atomicMax(&best[cur_row], cur);
+  if (f0 + tid < f1) atomicMax(&best[cur], rb.key());
   __syncthreads();
   cluster.sync();
 

@@ -1,7 +1,9 @@
 // attention_f32.cu -- fp32 verification attention on CUDA cores (the paper's
-// own runs are fp32, Sec. 4.1).  One warp per query row; lanes split the
-// head dimension; online softmax over the visible keys: the paged prefix,
-// then the new slots admitted by Eq. (1).
+// own runs are fp32, Sec. 4.1).  One warp per query row.  Keys go in chunks
+// of 32: the paged prefix rows, then the new slots admitted by Eq. (1);
+// each lane scores one key of the chunk, the warp folds the chunk into a
+// running max / sum (online softmax) and accumulates V with lanes over the
+// head dimension.
 #include <cuda_runtime.h>
 
 #include "common.cuh"
@@ -13,9 +15,11 @@ constexpr int kF32Warps = 4;
 
 template <int DPL>  // head-dim elements per lane (d = 32 * DPL)
 __global__ void __launch_bounds__(kF32Warps * 32) attention_f32_kernel(AttnF32Args a) {
-  const int lane = threadIdx.x & 31;
+  __shared__ __align__(16) float q_s[kF32Warps][32 * DPL];
+  const int lane = threadIdx.x & 31, wib = threadIdx.x >> 5;
   const long long row = (static_cast<long long>(blockIdx.x) * blockDim.x + threadIdx.x) >> 5;
-  const int S = 2 * a.gamma, g = a.Hq / a.Hkv, d = 32 * DPL;
+  const int S = 2 * a.gamma, g = a.Hq / a.Hkv;
+  constexpr int d = 32 * DPL;
   const long long rows = static_cast<long long>(a.Bt) * S * a.Hq;
   if (row >= rows) return;
   const int h = static_cast<int>(row % a.Hq);
@@ -46,39 +50,84 @@ __global__ void __launch_bounds__(kF32Warps * 32) attention_f32_kernel(AttnF32Ar
     return;
   }
   const int ti = a.tau[static_cast<size_t>(b) * S + s];
-  float qv[DPL], acc[DPL];
 #pragma unroll
-  for (int c = 0; c < DPL; ++c) {
-    qv[c] = a.q[row * d + lane + 32 * c];
-    acc[c] = 0.f;
-  }
+  for (int c = 0; c < DPL; ++c) q_s[wib][lane + 32 * c] = a.q[row * d + lane + 32 * c];
+  __syncwarp();
+  float acc[DPL];
+#pragma unroll
+  for (int c = 0; c < DPL; ++c) acc[c] = 0.f;
   float m = -INFINITY, l = 0.f;
-  auto visit = [&](const float* kr, const float* vr) {
-    float dot = 0.f;
+  // keys 0..n-1 are the prefix rows, keys n..n+S-1 the new slots; lane j of
+  // each chunk of 32 scores key base+j, then the warp folds the chunk in
+  const int nkeys = n + S;
+  for (int base = 0; base < nkeys; base += 32) {
+    const int j = base + lane;
+    const float* kr = nullptr;
+    long long voff = -1;
+    bool from_cache = false;
+    if (j < n) {
+      const int pg = a.block_table[static_cast<size_t>(b) * a.max_pages + j / a.page_size];
+      voff = ((static_cast<long long>(pg) * a.Hkv + kvh) * a.page_size + (j % a.page_size)) * d;
+      kr = a.k_cache + voff;
+      from_cache = true;
+    } else if (j < nkeys) {
+      const int t = j - n;
+      const size_t st_i = static_cast<size_t>(b) * S + t;
+      if (temporal_visible(si, ti, a.section[st_i], a.tau[st_i])) {
+        voff = ((static_cast<long long>(b) * S + t) * a.Hkv + kvh) * d;
+        kr = a.k_new + voff;
+      }
+    }
+    float sc = -INFINITY;
+    if (kr) {
+      float dot = 0.f;
+      const float4* k4 = reinterpret_cast<const float4*>(kr);
+      const float4* q4 = reinterpret_cast<const float4*>(q_s[wib]);
+#pragma unroll 8
+      for (int c = 0; c < d / 4; ++c) {
+        const float4 kv = __ldg(k4 + c);
+        const float4 qv = q4[c];
+        dot = fmaf(qv.x, kv.x, dot);
+        dot = fmaf(qv.y, kv.y, dot);
+        dot = fmaf(qv.z, kv.z, dot);
+        dot = fmaf(qv.w, kv.w, dot);
+      }
+      sc = dot * a.scale;
+    }
+    float mc = sc;
 #pragma unroll
-    for (int c = 0; c < DPL; ++c) dot = fmaf(qv[c], kr[lane + 32 * c], dot);
-#pragma unroll
-    for (int off = 16; off > 0; off >>= 1) dot += __shfl_xor_sync(0xffffffffu, dot, off);
-    const float sc = dot * a.scale;
-    const float m_new = fmaxf(m, sc);
+    for (int off = 16; off > 0; off >>= 1) mc = fmaxf(mc, __shfl_xor_sync(0xffffffffu, mc, off));
+    const float m_new = fmaxf(m, mc);
+    if (m_new == -INFINITY) continue;  // nothing visible yet
     const float corr = expf(m - m_new);
-    const float pr = expf(sc - m_new);
-    l = l * corr + pr;
+    const float pr = kr ? expf(sc - m_new) : 0.f;
+    float ps = pr;
 #pragma unroll
-    for (int c = 0; c < DPL; ++c) acc[c] = fmaf(acc[c], corr, pr * vr[lane + 32 * c]);
+    for (int off = 16; off > 0; off >>= 1) ps += __shfl_xor_sync(0xffffffffu, ps, off);
+    l = l * corr + ps;
+#pragma unroll
+    for (int c = 0; c < DPL; ++c) acc[c] *= corr;
+    // P.V of the chunk, 8 keys at a time so that their V loads overlap
+    const float* vrow = kr ? (from_cache ? a.v_cache : a.v_new) + voff : a.v_new;
+#pragma unroll 1
+    for (int j0 = 0; j0 < 32; j0 += 8) {
+      float vv[8][DPL], pj[8];
+      bool use[8];
+#pragma unroll
+      for (int u = 0; u < 8; ++u) {
+        const float* vr = reinterpret_cast<const float*>(
+            __shfl_sync(0xffffffffu, reinterpret_cast<uintptr_t>(vrow), j0 + u));
+        pj[u] = __shfl_sync(0xffffffffu, pr, j0 + u);
+        use[u] = __shfl_sync(0xffffffffu, kr != nullptr, j0 + u);
+#pragma unroll
+        for (int c = 0; c < DPL; ++c) vv[u][c] = use[u] ? __ldg(vr + lane + 32 * c) : 0.f;
+      }
+#pragma unroll
+      for (int u = 0; u < 8; ++u)
+#pragma unroll
+        for (int c = 0; c < DPL; ++c) acc[c] = use[u] ? fmaf(pj[u], vv[u][c], acc[c]) : acc[c];
+    }
     m = m_new;
-  };
-  for (int p = 0; p < n; ++p) {
-    const int pg = a.block_table[static_cast<size_t>(b) * a.max_pages + p / a.page_size];
-    const size_t off = ((static_cast<size_t>(pg) * a.Hkv + kvh) * a.page_size + (p % a.page_size)) * d;
-    visit(a.k_cache + off, a.v_cache + off);
-  }
-  for (int t = 0; t < S; ++t) {
-    const uint8_t sj = a.section[static_cast<size_t>(b) * S + t];
-    const int tj = a.tau[static_cast<size_t>(b) * S + t];
-    if (!temporal_visible(si, ti, sj, tj)) continue;
-    const size_t off = ((static_cast<size_t>(b) * S + t) * a.Hkv + kvh) * d;
-    visit(a.k_new + off, a.v_new + off);
   }
   const float inv = l > 0.f ? 1.f / l : 0.f;
 #pragma unroll

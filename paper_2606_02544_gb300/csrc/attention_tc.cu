@@ -9,18 +9,22 @@
 // the page table with TMA), then one tile with the 2*gamma new slots, whose
 // Eq. (1) visibility is evaluated on the fly from (section, tau).
 //
-// Warp roles (192 threads):
-//   warps 0-3  softmax: thread i owns query row i (TMEM lane i).  Loads S,
-//              applies the mask, keeps the running max/sum in fp32, writes P
-//              (bf16) to TMEM, rescales O in TMEM when the max grows by more
-//              than 2^8, and writes the output.
-//   warp 4     TMA producer (one thread): Q once, then K/V tiles into a
+// Warp roles (320 threads):
+//   warps 0-3, 4-7  two softmax warpgroups.  Group w takes the unit's tiles
+//              w, w+2, w+4, ... with its own S, P and O in TMEM and its own
+//              running max / sum; thread i of a group owns query row i (TMEM
+//              lane i).  Two groups keep two tiles in flight through the
+//              softmax, so the shared-memory ring recycles twice as fast.
+//              At the end group 1 hands its (m, l, O) rows to group 0 through
+//              shared memory and group 0 writes the merged result.
+//   warp 8     TMA producer (one thread): Q once, then K/V tiles into a
 //              STAGES-deep shared-memory ring.
-//   warp 5     MMA issuer (one thread) and TMEM owner:
-//              S = Q K^T (SS MMA, 128x64x128), O += P V (TS MMA, P in TMEM,
-//              V MN-major in shared memory, 128x128x64).
-// TMEM (256 columns): S [0,64) fp32, P0 [64,96) and P1 [96,128) bf16 pairs,
-// O [128,256) fp32.
+//   warp 9     MMA issuer (one thread) and TMEM owner.  It polls both
+//              groups and issues whatever is ready: S_i = Q K_i^T (SS MMA,
+//              128x64x128) or O_w += P_i V_i (TS MMA, P in TMEM, V MN-major in
+//              shared memory, 128x128x64).
+// TMEM (512 columns): group w owns [256w, 256w+256): S [0,64) fp32, P in two
+// buffers [64,96) and [96,128) (bf16 pairs), O [128,256) fp32.
 //
 // Every mbarrier wait is bounded; a wait that expires sets SIMSD_EW_TIMEOUT
 // and makes the whole CTA stop, drain its async work and free its TMEM.
@@ -40,11 +44,13 @@ namespace {
 constexpr int kTile = 64;            // keys per tile
 constexpr int kD = 128;              // head dimension
 constexpr int kRows = 128;           // MMA M (query rows per CTA)
-constexpr int kThreads = 192;
-constexpr int kWarpProducer = 4;
-constexpr int kWarpMma = 5;
-constexpr uint32_t kTmemCols = 256;
-constexpr uint32_t kColS = 0, kColP0 = 64, kColO = 128;
+constexpr int kGroups = 2;           // softmax warpgroups
+constexpr int kThreads = 32 * (4 * kGroups + 2);
+constexpr int kWarpProducer = 4 * kGroups;
+constexpr int kWarpMma = 4 * kGroups + 1;
+constexpr uint32_t kTmemCols = 512;
+constexpr uint32_t kGroupCols = 256;
+constexpr uint32_t kColS = 0, kColP = 64, kColO = 128;
 constexpr int kQHalfBytes = kRows * 128;    // 128 rows x 64 bf16
 constexpr int kKvHalfBytes = kTile * 128;   // 64 rows x 64 bf16
 constexpr float kRescaleThreshold = 8.0f;   // log2 units: rescale when the max grows by > 2^8
@@ -68,20 +74,21 @@ struct alignas(1024) Smem {
   uint8_t kv[STAGES][4][kKvHalfBytes];      // [stage][K0, K1, V0, V1][key][64]
   uint64_t bar_q;
   uint64_t bar_k[STAGES], bar_v[STAGES], bar_empty[STAGES];
-  uint64_t bar_s_full, bar_s_free, bar_p[2], bar_o, bar_ofinal, bar_drain;
+  uint64_t bar_s_full[kGroups], bar_s_free[kGroups], bar_p[kGroups][2], bar_o[kGroups];
+  uint64_t bar_ofinal, bar_drain;
   uint32_t tmem_base;
   int abort_flag;
   int seq_bad;
   int b_sel;
   int32_t tau[64];
   uint8_t sect[64];
-  int32_t nval[256];
 };
 
 template <int STAGES>
 constexpr size_t smem_bytes() {
   return sizeof(Smem<STAGES>) + 1024;
 }
+static_assert(smem_bytes<6>() <= 232448, "shared memory budget of one CTA");
 
 template <int STAGES>
 __device__ __forceinline__ void signal_abort(Smem<STAGES>& sm, int32_t* err_word) {
@@ -90,7 +97,7 @@ __device__ __forceinline__ void signal_abort(Smem<STAGES>& sm, int32_t* err_word
 }
 
 template <int STAGES>
-__global__ void __launch_bounds__(kThreads, 2)
+__global__ void __launch_bounds__(kThreads, 1)
     attention_tc_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ CUtensorMap tm_kn,
                         const __grid_constant__ CUtensorMap tm_vn, const __grid_constant__ CUtensorMap tm_kc,
                         const __grid_constant__ CUtensorMap tm_vc, const __grid_constant__ TcParams p) {
@@ -114,16 +121,18 @@ __global__ void __launch_bounds__(kThreads, 2)
     sm.seq_bad = 0;
     sm.b_sel = rank;
   }
+  // prefix lengths, staged in the (still unused) K/V ring for the ranking
+  int32_t* nval = reinterpret_cast<int32_t*>(sm.kv[0][0]);
   const bool sort = p.Bt <= 256;
   if (sort)
-    for (int i = tid; i < p.Bt; i += kThreads) sm.nval[i] = p.prefix_len[i];
+    for (int i = tid; i < p.Bt; i += kThreads) nval[i] = p.prefix_len[i];
   __syncthreads();
   if (sort) {
     for (int i = tid; i < p.Bt; i += kThreads) {
-      const int ni = sm.nval[i];
+      const int ni = nval[i];
       int r = 0;
       for (int j = 0; j < p.Bt; ++j) {
-        const int nj = sm.nval[j];
+        const int nj = nval[j];
         r += (nj > ni) || (nj == ni && j < i);
       }
       if (r == rank) sm.b_sel = i;
@@ -159,11 +168,13 @@ __global__ void __launch_bounds__(kThreads, 2)
       mbar_init(smem_u32(&sm.bar_v[s]), 1);
       mbar_init(smem_u32(&sm.bar_empty[s]), 1);
     }
-    mbar_init(smem_u32(&sm.bar_s_full), 1);
-    mbar_init(smem_u32(&sm.bar_s_free), 4);
-    mbar_init(smem_u32(&sm.bar_p[0]), 4);
-    mbar_init(smem_u32(&sm.bar_p[1]), 4);
-    mbar_init(smem_u32(&sm.bar_o), 1);
+    for (int w = 0; w < kGroups; ++w) {
+      mbar_init(smem_u32(&sm.bar_s_full[w]), 1);
+      mbar_init(smem_u32(&sm.bar_s_free[w]), 4);
+      mbar_init(smem_u32(&sm.bar_p[w][0]), 4);
+      mbar_init(smem_u32(&sm.bar_p[w][1]), 4);
+      mbar_init(smem_u32(&sm.bar_o[w]), 1);
+    }
     mbar_init(smem_u32(&sm.bar_ofinal), 1);
     mbar_init(smem_u32(&sm.bar_drain), 1);
     fence_mbar_init();
@@ -257,48 +268,64 @@ __global__ void __launch_bounds__(kThreads, 2)
     __syncwarp();
   } else if (warp == kWarpMma) {
     // ----------------------------------------------------------- MMA issuer
+    // Tile i belongs to group w = i & 1 as its j = i >> 1-th tile.
+    //   QK_i needs K_i and S_w free (group w has read S of tile i-2), and,
+    //   because P_w is double-buffered, PV_{i-4} already issued.
+    //   PV_i needs P_i and V_i; PVs go in tile order.
     if (lane == 0 && ntiles > 0) {
       constexpr uint32_t kIdescQK = idesc_bf16_f32(kRows, kTile, 0, 0);
       constexpr uint32_t kIdescPV = idesc_bf16_f32(kRows, kD, 0, 1);
       bool ok = mbar_wait(smem_u32(&sm.bar_q), 0, abort_flag);
       tc_fence_after();
       const uint32_t q0 = smem_u32(sm.q[0]), q1 = smem_u32(sm.q[1]);
-      auto issue_qk = [&](int i) -> bool {
-        const int st = i % STAGES;
-        if (!mbar_wait(smem_u32(&sm.bar_k[st]), (i / STAGES) & 1, abort_flag)) return false;
-        if (i > 0 && !mbar_wait(smem_u32(&sm.bar_s_free), (i - 1) & 1, abort_flag)) return false;
-        tc_fence_after();
-        const uint32_t kb0 = smem_u32(sm.kv[st][0]), kb1 = smem_u32(sm.kv[st][1]);
+      int next_qk = 0, next_pv = 0;
+      unsigned long long t_idle = 0;
+      uint32_t spins = 0;
+      while (ok && next_pv < ntiles) {
+        bool progressed = false;
+        if (next_qk < ntiles && next_qk - 4 < next_pv) {
+          const int i = next_qk, w = i & 1, j = i >> 1, st = i % STAGES;
+          if (mbar_try_wait(smem_u32(&sm.bar_k[st]), (i / STAGES) & 1) &&
+              (j == 0 || mbar_try_wait(smem_u32(&sm.bar_s_free[w]), (j - 1) & 1))) {
+            tc_fence_after();
+            const uint32_t kb0 = smem_u32(sm.kv[st][0]), kb1 = smem_u32(sm.kv[st][1]);
+            const uint32_t d_s = tmem + w * kGroupCols + kColS;
 #pragma unroll
-        for (int kk = 0; kk < kD / 16; ++kk) {
-          const uint32_t qa = (kk < 4 ? q0 : q1) + (kk & 3) * 32;
-          const uint32_t ka = (kk < 4 ? kb0 : kb1) + (kk & 3) * 32;
-          tc_mma_ss(tmem + kColS, sdesc_sw128(qa, 16, 1024), sdesc_sw128(ka, 16, 1024), kIdescQK, kk > 0);
+            for (int kk = 0; kk < kD / 16; ++kk) {
+              const uint32_t qa = (kk < 4 ? q0 : q1) + (kk & 3) * 32;
+              const uint32_t ka = (kk < 4 ? kb0 : kb1) + (kk & 3) * 32;
+              tc_mma_ss(d_s, sdesc_sw128(qa, 16, 1024), sdesc_sw128(ka, 16, 1024), kIdescQK, kk > 0);
+            }
+            tc_commit(smem_u32(&sm.bar_s_full[w]));
+            ++next_qk;
+            progressed = true;
+          }
         }
-        tc_commit(smem_u32(&sm.bar_s_full));
-        return true;
-      };
-      if (ok) ok = issue_qk(0);
-      for (int i = 0; ok && i < ntiles; ++i) {
-        if (i + 1 < ntiles && !issue_qk(i + 1)) {
-          ok = false;
-          break;
-        }
-        const int st = i % STAGES, pb = i & 1;
-        if (!mbar_wait(smem_u32(&sm.bar_p[pb]), (i >> 1) & 1, abort_flag) ||
-            !mbar_wait(smem_u32(&sm.bar_v[st]), (i / STAGES) & 1, abort_flag)) {
-          ok = false;
-          break;
-        }
-        tc_fence_after();
-        const uint32_t vb = smem_u32(sm.kv[st][2]);
+        if (next_pv < next_qk) {
+          const int i = next_pv, w = i & 1, j = i >> 1, st = i % STAGES;
+          if (mbar_try_wait(smem_u32(&sm.bar_p[w][j & 1]), (j >> 1) & 1) &&
+              mbar_try_wait(smem_u32(&sm.bar_v[st]), (i / STAGES) & 1)) {
+            tc_fence_after();
+            const uint32_t vb = smem_u32(sm.kv[st][2]);
+            const uint32_t gbase = tmem + w * kGroupCols;
 #pragma unroll
-        for (int kk = 0; kk < kTile / 16; ++kk) {
-          tc_mma_ts(tmem + kColO, tmem + kColP0 + 32 * pb + 8 * kk, sdesc_sw128(vb + kk * 2048, kKvHalfBytes, 1024),
-                    kIdescPV, (i > 0 || kk > 0) ? 1u : 0u);
+            for (int kk = 0; kk < kTile / 16; ++kk) {
+              tc_mma_ts(gbase + kColO, gbase + kColP + 32 * (j & 1) + 8 * kk,
+                        sdesc_sw128(vb + kk * 2048, kKvHalfBytes, 1024), kIdescPV, (j > 0 || kk > 0) ? 1u : 0u);
+            }
+            tc_commit(smem_u32(&sm.bar_empty[st]));
+            tc_commit(smem_u32(&sm.bar_o[w]));
+            ++next_pv;
+            progressed = true;
+          }
         }
-        tc_commit(smem_u32(&sm.bar_empty[st]));
-        tc_commit(smem_u32(&sm.bar_o));
+        if (progressed) {
+          spins = 0;
+        } else if ((++spins & 63u) == 0) {
+          const unsigned long long now = globaltimer_ns();
+          if (spins == 64) t_idle = now;
+          if (*abort_flag || now - t_idle > kWaitLimitNs) ok = false;
+        }
       }
       if (!ok) signal_abort(sm, p.err_word);
       tc_commit(smem_u32(&sm.bar_ofinal));
@@ -309,7 +336,9 @@ __global__ void __launch_bounds__(kThreads, 2)
     __syncwarp();
   } else {
     // -------------------------------------------------------------- softmax
-    const int row = tid;
+    const int grp = warp >> 2;                 // 0 or 1
+    const int row = tid & (kRows - 1);         // TMEM lane / query row
+    const int wq = warp & 3;                   // lane quadrant of this warp
     const int s = rblk * p.s_blk + row / p.g;
     const int hl = row % p.g;
     const bool row_exists = row < p.rows_blk && s < p.S;
@@ -321,12 +350,13 @@ __global__ void __launch_bounds__(kThreads, 2)
       for (int t = 0; t < p.S; ++t)
         if (temporal_visible(si, ti, sm.sect[t], sm.tau[t])) vis |= 1ull << t;
     }
-    const uint32_t lane_tmem = tmem + (static_cast<uint32_t>(warp * 32) << 16);
+    const uint32_t lane_tmem = tmem + grp * kGroupCols + (static_cast<uint32_t>(wq * 32) << 16);
     float m_ref = -INFINITY, l_sum = 0.f;
     bool ok = true;
-    for (int i = 0; i < ntiles; ++i) {
-      const int t = t0 + i, st = i % STAGES, pb = i & 1;
-      if (!mbar_wait_warp(smem_u32(&sm.bar_s_full), i & 1, abort_flag)) {
+    int j = 0;
+    for (int i = grp; i < ntiles; i += kGroups, ++j) {
+      const int t = t0 + i, st = i % STAGES;
+      if (!mbar_wait_warp(smem_u32(&sm.bar_s_full[grp]), j & 1, abort_flag)) {
         ok = false;
         break;
       }
@@ -337,18 +367,32 @@ __global__ void __launch_bounds__(kThreads, 2)
       tmem_wait_ld();
       tc_fence_before();
       __syncwarp();
-      if (lane == 0) mbar_arrive(smem_u32(&sm.bar_s_free));
+      if (lane == 0) mbar_arrive(smem_u32(&sm.bar_s_free[grp]));
 
       const bool is_new = (t == T);
       const int valid = is_new ? p.S : min(kTile, n - t * kTile);
       float x[kTile];
-      float mx = -INFINITY;
 #pragma unroll
-      for (int c = 0; c < kTile; ++c) {
-        const float sv = __uint_as_float(c < 32 ? sa[c] : sb[c - 32]);
-        const bool see = active && c < valid && (!is_new || ((vis >> c) & 1ull));
-        x[c] = see ? sv * p.scale_log2 : -INFINITY;
-        mx = fmaxf(mx, x[c]);
+      for (int c = 0; c < kTile; ++c) x[c] = __uint_as_float(c < 32 ? sa[c] : sb[c - 32]);
+      if (is_new || valid < kTile) {
+        // partial prefix tile or the tile of new slots: hide what the row may not see
+#pragma unroll
+        for (int c = 0; c < kTile; ++c) {
+          const bool see = c < valid && (!is_new || ((vis >> c) & 1ull));
+          x[c] = see ? x[c] : -INFINITY;
+        }
+      }
+      // raw-score maximum (pairwise tree); scale_log2 > 0 commutes with max
+      float mx;
+      {
+        float r[kTile / 2];
+#pragma unroll
+        for (int c = 0; c < kTile / 2; ++c) r[c] = fmaxf(x[2 * c], x[2 * c + 1]);
+#pragma unroll
+        for (int w2 = kTile / 4; w2 >= 1; w2 >>= 1)
+#pragma unroll
+          for (int c = 0; c < w2; ++c) r[c] = fmaxf(r[c], r[c + w2]);
+        mx = active ? r[0] * p.scale_log2 : -INFINITY;
       }
       bool need = false;
       if (active && mx != -INFINITY) {
@@ -358,13 +402,14 @@ __global__ void __launch_bounds__(kThreads, 2)
           need = true;
       }
       if (__any_sync(0xffffffffu, need)) {
-        // O holds the tiles before i: wait for PV of tile i-1, then rescale
-        if (!mbar_wait_warp(smem_u32(&sm.bar_o), (i - 1) & 1, abort_flag)) {
+        // O_grp holds this group's earlier tiles: wait for the PV of its
+        // previous tile, then rescale
+        if (!mbar_wait_warp(smem_u32(&sm.bar_o[grp]), (j - 1) & 1, abort_flag)) {
           ok = false;
           break;
         }
         tc_fence_after();
-        const float f = need ? exp2f(m_ref - mx) : 1.0f;
+        const float f = need ? fast_exp2(m_ref - mx) : 1.0f;
         if (need) {
           l_sum *= f;
           m_ref = mx;
@@ -375,58 +420,65 @@ __global__ void __launch_bounds__(kThreads, 2)
           tmem_ld32(lane_tmem + kColO + 32 * ch, o);
           tmem_wait_ld();
 #pragma unroll
-          for (int j = 0; j < 32; ++j) o[j] = __float_as_uint(__uint_as_float(o[j]) * f);
+          for (int c = 0; c < 32; ++c) o[c] = __float_as_uint(__uint_as_float(o[c]) * f);
           tmem_st32(lane_tmem + kColO + 32 * ch, o);
         }
         tmem_wait_st();
       }
-      const float mref = (active && m_ref != -INFINITY) ? m_ref : 0.f;
+      // p = 2^(s*scale*log2e - m): one FFMA and one MUFU.EX2 per score.  Rows
+      // that are not active leave garbage in their own P/O rows only (MMA rows
+      // are independent) and write zeros at the end.
+      const float neg_m = (active && m_ref != -INFINITY) ? -m_ref : 0.f;
       uint32_t pk[32];
-      float lt = 0.f;
+      float ps[kTile / 2];
 #pragma unroll
       for (int c = 0; c < kTile / 2; ++c) {
-        const float p0 = exp2f(x[2 * c] - mref);
-        const float p1 = exp2f(x[2 * c + 1] - mref);
-        lt += p0 + p1;
+        const float p0 = fast_exp2(fmaf(x[2 * c], p.scale_log2, neg_m));
+        const float p1 = fast_exp2(fmaf(x[2 * c + 1], p.scale_log2, neg_m));
+        ps[c] = p0 + p1;
         pk[c] = pack_bf16x2(p0, p1);
       }
-      l_sum += lt;
-      tmem_st32(lane_tmem + kColP0 + 32 * pb, pk);
+#pragma unroll
+      for (int w2 = kTile / 4; w2 >= 1; w2 >>= 1)
+#pragma unroll
+        for (int c = 0; c < w2; ++c) ps[c] += ps[c + w2];
+      l_sum += ps[0];
+      tmem_st32(lane_tmem + kColP + 32 * (j & 1), pk);
       tmem_wait_st();
-      if (warp < 2 && (valid < kTile || is_new)) {
+      if (wq < 2 && (valid < kTile || is_new)) {
         // rows of V that no query may use are zeroed so that 0 * (stale or
         // non-finite data) cannot reach O
         if (!mbar_wait_warp(smem_u32(&sm.bar_v[st]), (i / STAGES) & 1, abort_flag)) {
           ok = false;
           break;
         }
-        const int kr = tid;
+        const int kr = row;
         const bool zero = kr >= valid || (is_new && sm.sect[kr] == kSectPad);
         if (zero) {
           const uint4 z = make_uint4(0u, 0u, 0u, 0u);
           uint4* r0 = reinterpret_cast<uint4*>(sm.kv[st][2] + kr * 128);
           uint4* r1 = reinterpret_cast<uint4*>(sm.kv[st][3] + kr * 128);
 #pragma unroll
-          for (int j = 0; j < 8; ++j) {
-            r0[j] = z;
-            r1[j] = z;
+          for (int c = 0; c < 8; ++c) {
+            r0[c] = z;
+            r1[c] = z;
           }
         }
         fence_proxy_async_smem();
       }
       tc_fence_before();
       __syncwarp();
-      if (lane == 0) mbar_arrive(smem_u32(&sm.bar_p[pb]));
+      if (lane == 0) mbar_arrive(smem_u32(&sm.bar_p[grp][j & 1]));
     }
     if (!ok && lane == 0) signal_abort(sm, p.err_word);
-    // ---- epilogue
+    // ---- epilogue: group 1 hands (m, l, O) to group 0, which merges
     const bool have_o = ok && ntiles > 0 && mbar_wait_warp(smem_u32(&sm.bar_ofinal), 0, abort_flag);
     if (have_o) tc_fence_after();
-    const int h = kvh * p.g + hl;
-    const bool live = have_o && active;
-    if (p.nsplit == 1) {
-      const float inv = (live && l_sum > 0.f) ? 1.0f / l_sum : 0.f;
-      __nv_bfloat16* orow = p.out + ((static_cast<size_t>(b) * p.S + s) * p.Hq + h) * kD;
+    const bool live = have_o && active && j > 0;   // this group saw at least one tile
+    // the ring is idle once every MMA has completed: reuse it for the hand-off
+    float* xo = reinterpret_cast<float*>(sm.kv[0][0]);          // [128 rows][132]
+    constexpr int kXStride = kD + 4;
+    if (grp == 1) {
 #pragma unroll 1
       for (int ch = 0; ch < kD / 32; ++ch) {
         uint32_t o[32];
@@ -434,44 +486,84 @@ __global__ void __launch_bounds__(kThreads, 2)
           tmem_ld32(lane_tmem + kColO + 32 * ch, o);
           tmem_wait_ld();
         }
-        if (row_exists) {
-          uint4 pkd[4];
-          uint32_t* w = reinterpret_cast<uint32_t*>(pkd);
+        float4* dst = reinterpret_cast<float4*>(xo + row * kXStride + 32 * ch);
 #pragma unroll
-          for (int j = 0; j < 16; ++j) {
-            const float a0 = live ? __uint_as_float(o[2 * j]) * inv : 0.f;
-            const float a1 = live ? __uint_as_float(o[2 * j + 1]) * inv : 0.f;
-            w[j] = pack_bf16x2(a0, a1);
-          }
-          uint4* dst = reinterpret_cast<uint4*>(orow + 32 * ch);
-#pragma unroll
-          for (int j = 0; j < 4; ++j) dst[j] = pkd[j];
-        }
+        for (int c = 0; c < 8; ++c)
+          dst[c] = live ? make_float4(__uint_as_float(o[4 * c]), __uint_as_float(o[4 * c + 1]),
+                                      __uint_as_float(o[4 * c + 2]), __uint_as_float(o[4 * c + 3]))
+                        : make_float4(0.f, 0.f, 0.f, 0.f);
       }
-    } else {
-      const size_t unit = ((static_cast<size_t>(b) * p.Hkv + kvh) * p.rb + rblk) * p.nsplit + split;
-      const size_t nunits = static_cast<size_t>(p.Bt) * p.Hkv * p.rb * p.nsplit;
-      float* wo = p.ws + (unit * p.rows_blk + row) * kD;
-      float* wml = p.ws + nunits * p.rows_blk * kD + (unit * p.rows_blk + row) * 2;
+      xo[row * kXStride + kD] = live ? m_ref : -INFINITY;
+      xo[row * kXStride + kD + 1] = live ? l_sum : 0.f;
+    }
+    asm volatile("bar.sync 1, %0;" ::"r"(4 * kGroups * 32) : "memory");
+    if (grp == 0) {
+      // merge the two groups' partial softmax states of this row
+      const float m1 = xo[row * kXStride + kD], l1 = xo[row * kXStride + kD + 1];
+      const float m0 = live ? m_ref : -INFINITY, l0 = live ? l_sum : 0.f;
+      const float M = fmaxf(m0, m1);
+      const float a0 = (M == -INFINITY || m0 == -INFINITY) ? 0.f : fast_exp2(m0 - M);
+      const float a1 = (M == -INFINITY || m1 == -INFINITY) ? 0.f : fast_exp2(m1 - M);
+      const float L = a0 * l0 + a1 * l1;
+      const bool any = active && have_o && L > 0.f;
+      const int h = kvh * p.g + hl;
+      if (p.nsplit == 1) {
+        const float inv = any ? 1.0f / L : 0.f;
+        __nv_bfloat16* orow = p.out + ((static_cast<size_t>(b) * p.S + s) * p.Hq + h) * kD;
 #pragma unroll 1
-      for (int ch = 0; ch < kD / 32; ++ch) {
-        uint32_t o[32];
-        if (have_o) {
-          tmem_ld32(lane_tmem + kColO + 32 * ch, o);
-          tmem_wait_ld();
+        for (int ch = 0; ch < kD / 32; ++ch) {
+          uint32_t o[32];
+          if (have_o) {
+            tmem_ld32(lane_tmem + kColO + 32 * ch, o);
+            tmem_wait_ld();
+          }
+          if (row_exists) {
+            const float* o1 = xo + row * kXStride + 32 * ch;
+            uint4 pkd[4];
+            uint32_t* wv = reinterpret_cast<uint32_t*>(pkd);
+#pragma unroll
+            for (int c = 0; c < 16; ++c) {
+              const float v0 = live ? __uint_as_float(o[2 * c]) : 0.f;
+              const float v1 = live ? __uint_as_float(o[2 * c + 1]) : 0.f;
+              const float r0 = any ? (a0 * v0 + a1 * o1[2 * c]) * inv : 0.f;
+              const float r1 = any ? (a0 * v1 + a1 * o1[2 * c + 1]) * inv : 0.f;
+              wv[c] = pack_bf16x2(r0, r1);
+            }
+            uint4* dst = reinterpret_cast<uint4*>(orow + 32 * ch);
+#pragma unroll
+            for (int c = 0; c < 4; ++c) dst[c] = pkd[c];
+          }
+        }
+      } else {
+        const size_t unit = ((static_cast<size_t>(b) * p.Hkv + kvh) * p.rb + rblk) * p.nsplit + split;
+        const size_t nunits = static_cast<size_t>(p.Bt) * p.Hkv * p.rb * p.nsplit;
+        float* wo = p.ws + (unit * p.rows_blk + row) * kD;
+        float* wml = p.ws + nunits * p.rows_blk * kD + (unit * p.rows_blk + row) * 2;
+#pragma unroll 1
+        for (int ch = 0; ch < kD / 32; ++ch) {
+          uint32_t o[32];
+          if (have_o) {
+            tmem_ld32(lane_tmem + kColO + 32 * ch, o);
+            tmem_wait_ld();
+          }
+          if (row < p.rows_blk) {
+            const float* o1 = xo + row * kXStride + 32 * ch;
+            float4* dst = reinterpret_cast<float4*>(wo + 32 * ch);
+#pragma unroll
+            for (int c = 0; c < 8; ++c) {
+              float4 v;
+              v.x = any ? a0 * (live ? __uint_as_float(o[4 * c]) : 0.f) + a1 * o1[4 * c] : 0.f;
+              v.y = any ? a0 * (live ? __uint_as_float(o[4 * c + 1]) : 0.f) + a1 * o1[4 * c + 1] : 0.f;
+              v.z = any ? a0 * (live ? __uint_as_float(o[4 * c + 2]) : 0.f) + a1 * o1[4 * c + 2] : 0.f;
+              v.w = any ? a0 * (live ? __uint_as_float(o[4 * c + 3]) : 0.f) + a1 * o1[4 * c + 3] : 0.f;
+              dst[c] = v;
+            }
+          }
         }
         if (row < p.rows_blk) {
-          float4* dst = reinterpret_cast<float4*>(wo + 32 * ch);
-#pragma unroll
-          for (int j = 0; j < 8; ++j)
-            dst[j] = live ? make_float4(__uint_as_float(o[4 * j]), __uint_as_float(o[4 * j + 1]),
-                                        __uint_as_float(o[4 * j + 2]), __uint_as_float(o[4 * j + 3]))
-                          : make_float4(0.f, 0.f, 0.f, 0.f);
+          wml[0] = any ? M : -INFINITY;
+          wml[1] = any ? L : 0.f;
         }
-      }
-      if (row < p.rows_blk) {
-        wml[0] = live ? m_ref : -INFINITY;
-        wml[1] = live ? l_sum : 0.f;
       }
     }
   }
@@ -530,7 +622,7 @@ __global__ void __launch_bounds__(128) combine_kernel(const TcParams p) {
   reinterpret_cast<uint2*>(orow)[lane] = v;
 }
 
-constexpr int kStages = 2;
+constexpr int kStages = 6;
 
 cudaError_t ensure_smem_attr() {
   static bool done = false;
@@ -586,7 +678,8 @@ bool plan_attention_tc(int Bt, int gamma, int Hq, int Hkv, int max_pages, int pa
   const long long max_tiles = (static_cast<long long>(max_pages) * page_size + kTile - 1) / kTile + 1;
   int ns = 1;
   if (units < slots) {
-    ns = static_cast<int>((slots + units - 1) / units);
+    // as many splits as keep every CTA in one wave
+    ns = static_cast<int>(std::max<long long>(1, slots / units));
     ns = static_cast<int>(std::min<long long>(ns, std::max<long long>(1, max_tiles / 2)));
     ns = std::min(ns, 64);
   }

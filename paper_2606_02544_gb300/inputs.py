@@ -175,28 +175,21 @@ def make_step_inputs(w: Workload, device="cpu", seed: Optional[int] = None, pref
     n, bt, num_pages, sm, row_valid = make_metadata(w, seed, prefix_override, random_step_map)
     dt = torch_dtype(w)
     S, P = w.S, w.page_size
-    qs, kns, vns, kcs, vcs = [], [], [], [], []
     poison = None
     if poison_unused_rows:
         poison = torch.as_tensor(~row_valid, device=device).view(num_pages, 1, P, 1)
+    q = torch.empty(L, w.Bt, S, w.Hq, w.d, dtype=dt, device=device)
+    k_new = torch.empty(L, w.Bt, S, w.Hkv, w.d, dtype=dt, device=device)
+    v_new = torch.empty_like(k_new)
+    k_cache = torch.empty(L, num_pages, w.Hkv, P, w.d, dtype=dt, device=device)
+    v_cache = torch.empty_like(k_cache)
     for l in range(L):
         g = _dev_gen(seed + 1000 * l, device)
-        qs.append((torch.randn(w.Bt, S, w.Hq, w.d, generator=g, device=device) * std).to(dt))
-        kns.append((torch.randn(w.Bt, S, w.Hkv, w.d, generator=g, device=device) * std).to(dt))
-        vns.append((torch.randn(w.Bt, S, w.Hkv, w.d, generator=g, device=device) * std).to(dt))
-        kc = (torch.randn(num_pages, w.Hkv, P, w.d, generator=g, device=device) * std).to(dt)
-        vc = (torch.randn(num_pages, w.Hkv, P, w.d, generator=g, device=device) * std).to(dt)
+        for dst in (q[l], k_new[l], v_new[l], k_cache[l], v_cache[l]):
+            dst.copy_(torch.randn(dst.shape, generator=g, device=device).mul_(std))
         if poison is not None:
-            kc = torch.where(poison, torch.full_like(kc, float("nan")), kc)
-            vc = torch.where(poison, torch.full_like(vc, float("nan")), vc)
-        kcs.append(kc)
-        vcs.append(vc)
-    q = torch.stack(qs)
-    k_new = torch.stack(kns)
-    v_new = torch.stack(vns)
-    k_cache = torch.stack(kcs)
-    v_cache = torch.stack(vcs)
-    del qs, kns, vns, kcs, vcs
+            k_cache[l].masked_fill_(poison, float("nan"))
+            v_cache[l].masked_fill_(poison, float("nan"))
     if with_logits:
         g = _dev_gen(seed + 7, device)
         logits = torch.randn(w.Bt, w.gamma + 1, w.vocab, generator=g, device=device) * w.logit_std
