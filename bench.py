@@ -265,7 +265,7 @@ def run_gpu(args):
     acc_launch_ms = statistics.median(acc_times)
     attn_gbs = attn_bytes / (attn_launch_ms * 1e-3) / 1e9
     acc_gbs = acc_bytes / (acc_launch_ms * 1e-3) / 1e9
-    attn_roof = {"kernel": "simsd_verify_attention (attention_tc + combine)", "bound": "hbm",
+    attn_roof = {"kernel": "simsd_verify_attention (attention_tc_kernel + combine_kernel when split)", "bound": "hbm",
                  "achieved": round(attn_gbs, 1), "peak": hbm_peak, "unit": "GB/s",
                  "frac": round(attn_gbs / hbm_peak, 4), "frac_of_8TBs": round(attn_gbs / 8000.0, 4),
                  "peak_source": peak_kind, "algorithmic_bytes_per_launch": int(attn_bytes),

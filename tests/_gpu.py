@@ -37,7 +37,7 @@ def gpu_attention(si, layer=0, mask=None, err=None):
     dt = simsd.SIMSD_BF16 if si.q.dtype == torch.bfloat16 else simsd.SIMSD_F32
     ws = simsd.simsd_verify_workspace_bytes(dt, w.Bt, w.gamma, w.Hq, w.Hkv, w.d, si.block_table.shape[1],
                                             w.page_size)
-    work = torch.empty(ws, dtype=torch.uint8, device=si.q.device) if ws else None
+    work = torch.zeros(ws, dtype=torch.uint8, device=si.q.device) if ws else None
     out = torch.full_like(si.q[layer], float("nan"))
     e = torch.zeros(1, dtype=torch.int32, device=si.q.device) if err is None else err
     simsd.simsd_verify_attention(si.q[layer], si.k_new[layer], si.v_new[layer], si.k_cache[layer],
