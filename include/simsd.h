@@ -137,6 +137,36 @@ SIMSD_API int simsd_verify_attention(int dtype, const void* q, const void* k_new
                            void* out, void* workspace, size_t workspace_bytes, int32_t* err_word, void* stream);
 
 /*
+ * simsd_verify_attention_noalloc -- simsd_verify_attention for callers that
+ * cannot allocate device memory.  The paper has no counterpart; this is a
+ * deployment convenience.
+ *
+ * Some callers cannot call cudaMalloc: a serving loop that is being captured
+ * into a CUDA graph (allocation is not allowed inside stream capture), or an
+ * engine that hands all device memory to its own pool at start-up and must
+ * not stall on the allocator (cudaMalloc may synchronise the device).  This
+ * entry point takes the same arguments minus the workspace: the scratch for
+ * the split partials comes from a 12 MiB array in device memory that the
+ * library owns (every GPU that loads libsimsd.so holds it until the process
+ * exits).  It allocates nothing and calls no allocating routine.
+ *   - The first call on each device looks up the array's device address
+ *     (cudaGetSymbolAddress); make that first call before any stream capture.
+ *   - Sizes whose scratch would exceed 12 MiB are rejected with
+ *     SIMSD_ERR_UNSUPPORTED (see simsd_last_error); use
+ *     simsd_verify_attention with a caller workspace for those.
+ *   - All calls share the one array: calls that overlap on the GPU (on
+ *     different streams, or different threads) race and give wrong results.
+ *     Nothing in the array has to start at zero; each call overwrites what it
+ *     reads.
+ */
+SIMSD_API int simsd_verify_attention_noalloc(int dtype, const void* q, const void* k_new, const void* v_new,
+                                             const void* k_cache, const void* v_cache, int num_pages,
+                                             const int32_t* block_table, int max_pages, int page_size,
+                                             const int32_t* prefix_len, const int32_t* tau, const uint8_t* section,
+                                             const int32_t* rope_pos, int Bt, int gamma, int Hq, int Hkv, int d,
+                                             float softmax_scale, void* out, int32_t* err_word, void* stream);
+
+/*
  * simsd_accept -- greedy longest-prefix acceptance (Sec. 3.2, Eq. (2) with
  * temperature 0: accept the r-th draft iff it equals the target argmax).
  *

@@ -212,6 +212,88 @@ int simsd_verify_attention(int dtype, const void* q, const void* k_new, const vo
   return e == cudaSuccess ? SIMSD_OK : cuda_fail(e, "attention_tc launch");
 }
 
+int simsd_verify_attention_noalloc(int dtype, const void* q, const void* k_new, const void* v_new,
+                                   const void* k_cache, const void* v_cache, int num_pages,
+                                   const int32_t* block_table, int max_pages, int page_size,
+                                   const int32_t* prefix_len, const int32_t* tau, const uint8_t* section,
+                                   const int32_t* rope_pos, int Bt, int gamma, int Hq, int Hkv, int d,
+                                   float softmax_scale, void* out, int32_t* err_word, void* stream) {
+  if (Bt < 0) return arg_fail("Bt < 0");
+  if (gamma < 1 || gamma > 32) return arg_fail("gamma must be in [1, 32]");
+  if (Hq <= 0 || Hkv <= 0 || Hq % Hkv != 0) return arg_fail("Hq must be a positive multiple of Hkv");
+  if (num_pages < 0 || max_pages < 0) return arg_fail("negative page count");
+  if (page_size < 8 || !((page_size % 64 == 0) || (64 % page_size == 0)))
+    return unsupported("page_size must be a multiple of 64 or a divisor of 64 (>= 8)");
+  if (rope_pos) return unsupported("rope_pos must be NULL (inputs arrive rotated)");
+  if (!(softmax_scale >= 0.f) || std::isinf(softmax_scale)) return arg_fail("softmax_scale");
+  if (Bt == 0) return SIMSD_OK;
+  if (!q || !k_new || !v_new || !prefix_len || !tau || !section || !out) return arg_fail("null pointer");
+  if (max_pages > 0 && (!block_table || !k_cache || !v_cache || num_pages == 0))
+    return arg_fail("null cache or block table");
+  if (!aligned16(q) || !aligned16(k_new) || !aligned16(v_new) || !aligned16(out) ||
+      (k_cache && !aligned16(k_cache)) || (v_cache && !aligned16(v_cache)))
+    return arg_fail("tensor pointers must be 16-byte aligned");
+  DeviceInfo info;
+  int rc = require_sm103(&info);
+  if (rc != SIMSD_OK) return rc;
+  if (dtype != SIMSD_BF16 && dtype != SIMSD_F32) return unsupported("dtype");
+  if (dtype == SIMSD_F32) {
+    // the fp32 path uses no scratch: same launch as simsd_verify_attention
+    return simsd_verify_attention(dtype, q, k_new, v_new, k_cache, v_cache, num_pages, block_table, max_pages,
+                                  page_size, prefix_len, tau, section, rope_pos, Bt, gamma, Hq, Hkv, d,
+                                  softmax_scale, out, nullptr, 0, err_word, stream);
+  }
+  if (d != 128) return unsupported("bf16 path needs d = 128");
+  if (static_cast<long long>(num_pages) * Hkv * page_size >= (1ll << 31))
+    return unsupported("page pool too large for 32-bit TMA row coordinates");
+  if (static_cast<long long>(Bt) * 2 * gamma * Hq >= (1ll << 31)) return unsupported("too many query rows");
+  simsd::AttnTcPlan plan;
+  if (!simsd::plan_attention_tc(Bt, gamma, Hq, Hkv, max_pages, page_size, info.num_sms, &plan))
+    return unsupported("query rows per KV head: need 2*gamma*Hq/Hkv <= 128 or 128 % (Hq/Hkv) == 0");
+  if (plan.ws_bytes > simsd::noalloc_scratch_capacity()) {
+    std::snprintf(g_last_error, sizeof(g_last_error),
+                  "unsupported: these sizes need %zu bytes of scratch, more than the %zu-byte static array; "
+                  "use simsd_verify_attention with a caller workspace",
+                  plan.ws_bytes, simsd::noalloc_scratch_capacity());
+    return SIMSD_ERR_UNSUPPORTED;
+  }
+  void* scratch = nullptr;
+  if (plan.ws_bytes > 0) {
+    cudaError_t e = simsd::noalloc_scratch_pointer(&scratch);
+    if (e != cudaSuccess) return cuda_fail(e, "cudaGetSymbolAddress of the static scratch");
+  }
+  simsd::EncodeTiledFn enc = encoder();
+  if (!enc) return cuda_fail(cudaErrorNotSupported, "cuTensorMapEncodeTiled entry point");
+  const float scale = softmax_scale > 0.f ? softmax_scale : 1.0f / std::sqrt(static_cast<float>(d));
+  simsd::AttnTcArgs a{};
+  a.q = q;
+  a.k_new = k_new;
+  a.v_new = v_new;
+  a.k_cache = k_cache ? k_cache : q;
+  a.v_cache = v_cache ? v_cache : q;
+  a.block_table = block_table;
+  a.prefix_len = prefix_len;
+  a.tau = tau;
+  a.section = section;
+  a.out = out;
+  a.workspace = scratch;
+  a.err_word = err_word;
+  a.num_pages = num_pages > 0 ? num_pages : 1;
+  a.max_pages = max_pages;
+  a.page_size = page_size;
+  a.Bt = Bt;
+  a.gamma = gamma;
+  a.Hq = Hq;
+  a.Hkv = Hkv;
+  a.scale = scale;
+  if (num_pages == 0) {
+    a.max_pages = 0;
+    a.num_pages = 0;
+  }
+  cudaError_t e = simsd::launch_attention_tc(a, plan, enc, as_stream(stream));
+  return e == cudaSuccess ? SIMSD_OK : cuda_fail(e, "attention_tc launch (static scratch)");
+}
+
 int simsd_accept(const float* logits, const int32_t* draft, int Bt, int gamma, int vocab, int32_t* accepted_len,
                  int32_t* out_tokens, int32_t* row_argmax, int32_t* err_word, void* stream) {
   if (Bt < 0) return arg_fail("Bt < 0");

@@ -33,10 +33,18 @@
 #include <cuda_runtime.h>
 
 #include <algorithm>
+#include <mutex>
 
 #include "common.cuh"
 #include "kernels.h"
 #include "ptx.cuh"
+
+// Scratch of simsd_verify_attention_noalloc: the split partials live in this
+// file-scope array instead of caller memory.  Every device that loads the
+// library holds it until the process exits.  Host code must not use the
+// symbol's address directly (on the host it is only a stand-in); it asks
+// the runtime for the device address once per device (below).
+static __device__ __align__(256) unsigned char g_noalloc_scratch[12u << 20];
 
 namespace simsd {
 namespace {
@@ -752,6 +760,28 @@ cudaError_t launch_attention_tc(const AttnTcArgs& a, const AttnTcPlan& pl, Encod
   const long long warps = static_cast<long long>(a.Bt) * a.Hkv * pl.rb * pl.rows_blk;
   combine_kernel<<<static_cast<unsigned>((warps + 3) / 4), 128, 0, stream>>>(p);
   return cudaGetLastError();
+}
+
+size_t noalloc_scratch_capacity() { return sizeof(g_noalloc_scratch); }
+
+cudaError_t noalloc_scratch_pointer(void** out) {
+  // Set-up, once per device and with that device current: the device
+  // address of the static scratch array.
+  static std::mutex mu;
+  static void* ptr[64] = {};
+  int dev = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) return e;
+  if (dev < 0 || dev >= 64) return cudaErrorInvalidDevice;
+  std::lock_guard<std::mutex> lk(mu);
+  if (!ptr[dev]) {
+    void* p = nullptr;
+    e = cudaGetSymbolAddress(&p, g_noalloc_scratch);
+    if (e != cudaSuccess) return e;
+    ptr[dev] = p;
+  }
+  *out = ptr[dev];
+  return cudaSuccess;
 }
 
 }  // namespace simsd

@@ -62,4 +62,8 @@ typedef CUresult (*EncodeTiledFn)(CUtensorMap*, CUtensorMapDataType, cuuint32_t,
 cudaError_t launch_attention_tc(const AttnTcArgs& a, const AttnTcPlan& plan, EncodeTiledFn encode,
                                 cudaStream_t stream);
 
+// Static device scratch of simsd_verify_attention_noalloc.
+size_t noalloc_scratch_capacity();
+cudaError_t noalloc_scratch_pointer(void** out);
+
 }  // namespace simsd

@@ -23,8 +23,9 @@ SIMSD_F32, SIMSD_BF16 = 0, 1
 SECT_DATA, SECT_MASK, SECT_PAD = 0, 1, 255
 EW_STEP_MAP, EW_PREFIX_LEN, EW_PAGE, EW_DRAFT, EW_TIMEOUT, EW_ACCEPT_LEN = 1, 2, 4, 8, 16, 32
 
-EXPORTED = ("simsd_build_mask", "simsd_verify_workspace_bytes", "simsd_verify_attention", "simsd_accept",
-            "simsd_kv_commit", "simsd_check_error", "simsd_last_error", "simsd_version")
+EXPORTED = ("simsd_build_mask", "simsd_verify_workspace_bytes", "simsd_verify_attention",
+            "simsd_verify_attention_noalloc", "simsd_accept", "simsd_kv_commit", "simsd_check_error",
+            "simsd_last_error", "simsd_version")
 
 
 class SimsdError(RuntimeError):
@@ -52,12 +53,14 @@ def load_library(path: str = LIB_PATH):
             lib.simsd_verify_workspace_bytes.restype = Z
             lib.simsd_verify_attention.argtypes = [I, P, P, P, P, P, I, P, I, I, P, P, P, P, I, I, I, I, I, F, P,
                                                    P, Z, P, P]
+            lib.simsd_verify_attention_noalloc.argtypes = [I, P, P, P, P, P, I, P, I, I, P, P, P, P, I, I, I, I, I,
+                                                           F, P, P, P]
             lib.simsd_accept.argtypes = [P, P, I, I, I, P, P, P, P, P]
             lib.simsd_kv_commit.argtypes = [I, P, P, I, P, P, P, P, P, I, P, I, I, P, I, I, I, I, P, P]
             lib.simsd_check_error.argtypes = [P, P, P]
             lib.simsd_last_error.restype = ctypes.c_char_p
-            for name in ("simsd_build_mask", "simsd_verify_attention", "simsd_accept", "simsd_kv_commit",
-                         "simsd_check_error", "simsd_version"):
+            for name in ("simsd_build_mask", "simsd_verify_attention", "simsd_verify_attention_noalloc",
+                         "simsd_accept", "simsd_kv_commit", "simsd_check_error", "simsd_version"):
                 getattr(lib, name).restype = ctypes.c_int
             _lib = lib
     return _lib
@@ -116,6 +119,21 @@ def simsd_verify_attention(q, k_new, v_new, k_cache, v_cache, block_table, prefi
         max_pages, P, _p(prefix_len), _p(tau), _p(section), _p(rope_pos), Bt, S // 2, Hq, Hkv, d,
         float(softmax_scale), _p(out), _p(workspace), ws_bytes, _p(err_word), _stream(stream))
     _check(rc, "simsd_verify_attention")
+
+
+def simsd_verify_attention_noalloc(q, k_new, v_new, k_cache, v_cache, block_table, prefix_len, tau, section, out,
+                                   err_word=None, softmax_scale=0.0, rope_pos=None, stream=None):
+    """simsd_verify_attention without a workspace: the library's static
+    device scratch is used instead (for callers that cannot allocate)."""
+    Bt, S, Hq, d = q.shape
+    Hkv = k_new.shape[2]
+    num_pages, _, P, _ = k_cache.shape
+    max_pages = block_table.shape[1]
+    rc = load_library().simsd_verify_attention_noalloc(
+        _dtype_code(q), _p(q), _p(k_new), _p(v_new), _p(k_cache), _p(v_cache), num_pages, _p(block_table),
+        max_pages, P, _p(prefix_len), _p(tau), _p(section), _p(rope_pos), Bt, S // 2, Hq, Hkv, d,
+        float(softmax_scale), _p(out), _p(err_word), _stream(stream))
+    _check(rc, "simsd_verify_attention_noalloc")
 
 
 def simsd_accept(logits, draft, accepted_len, out_tokens, row_argmax=None, err_word=None, stream=None):
