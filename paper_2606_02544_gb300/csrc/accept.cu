@@ -2,7 +2,7 @@
 // temperature 0: the r-th draft is accepted iff it equals the argmax of the
 // target's distribution at its verification slot).
 //
-// One thread-block cluster per sequence.  The CL CTAs of a cluster split the
+// One thread-block cluster per sequence.  The CTAs of a cluster split the
 // sequence's [gamma+1][vocab] block into contiguous spans; each thread
 // streams 16-byte loads (8 in flight), keeps a running (value, index) per
 // row with plain float compares, and folds it into a 64-bit key per row in
@@ -11,6 +11,8 @@
 // memory and walks the draft order.  No global scratch memory is used.
 #include <cooperative_groups.h>
 #include <cuda_runtime.h>
+
+#include <mutex>
 
 #include "common.cuh"
 #include "kernels.h"
@@ -68,7 +70,6 @@ struct RowBest {
   }
 };
 
-template <int CL>
 __global__ void __launch_bounds__(kAcceptThreads) accept_kernel(const float* __restrict__ logits,
                                                                 const int32_t* __restrict__ draft, int gamma,
                                                                 int vocab, int vec4, int32_t* __restrict__ accepted_len,
@@ -78,6 +79,7 @@ __global__ void __launch_bounds__(kAcceptThreads) accept_kernel(const float* __r
   __shared__ int am[kMaxRows];
   cg::cluster_group cluster = cg::this_cluster();
   const int c = static_cast<int>(cluster.block_rank());
+  const int CL = static_cast<int>(cluster.num_blocks());
   const int b = blockIdx.x / CL;
   const int rows = gamma + 1;
   const int tid = threadIdx.x;
@@ -190,14 +192,69 @@ __global__ void __launch_bounds__(kAcceptThreads) accept_kernel(const float* __r
   cluster.sync();  // peers stay resident until CTA 0 has read their keys
 }
 
-template <int CL>
-static cudaError_t launch_accept_cl(const float* logits, const int32_t* draft, int Bt, int gamma, int vocab,
-                                    int32_t* accepted_len, int32_t* out_tokens, int32_t* row_argmax,
-                                    int32_t* err_word, cudaStream_t stream) {
-  auto kern = accept_kernel<CL>;
-  if (CL > 8) {
-    cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
+namespace {
+
+constexpr int kMaxCluster = 16;
+
+// How many clusters of each size (1..16) the device keeps resident at once,
+// asked once per device from the occupancy calculator (clusters must fit in
+// one GPC, so this is less than SMs x CTAs per SM / size).
+struct ClusterCapacity {
+  bool ready = false;
+  int resident[kMaxCluster + 1] = {};
+};
+
+cudaError_t cluster_capacity(const ClusterCapacity** out) {
+  static std::mutex mu;
+  static ClusterCapacity cap[64];
+  int dev = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) return e;
+  if (dev < 0 || dev >= 64) return cudaErrorInvalidDevice;
+  std::lock_guard<std::mutex> lk(mu);
+  ClusterCapacity& c = cap[dev];
+  if (!c.ready) {
+    e = cudaFuncSetAttribute(accept_kernel, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
     if (e != cudaSuccess) return e;
+    for (int cl = 1; cl <= kMaxCluster; ++cl) {
+      cudaLaunchConfig_t cfg = {};
+      cfg.gridDim = dim3(static_cast<unsigned>(cl));
+      cfg.blockDim = dim3(kAcceptThreads);
+      cudaLaunchAttribute attr[1];
+      attr[0].id = cudaLaunchAttributeClusterDimension;
+      attr[0].val.clusterDim.x = static_cast<unsigned>(cl);
+      attr[0].val.clusterDim.y = 1;
+      attr[0].val.clusterDim.z = 1;
+      cfg.attrs = attr;
+      cfg.numAttrs = 1;
+      int n = 0;
+      e = cudaOccupancyMaxActiveClusters(&n, accept_kernel, &cfg);
+      if (e != cudaSuccess) return e;
+      c.resident[cl] = n;
+    }
+    c.ready = true;
+  }
+  *out = &c;
+  return cudaSuccess;
+}
+
+}  // namespace
+
+cudaError_t launch_accept(const float* logits, const int32_t* draft, int Bt, int gamma, int vocab,
+                          int32_t* accepted_len, int32_t* out_tokens, int32_t* row_argmax, int32_t* err_word,
+                          int num_sms, cudaStream_t stream) {
+  (void)num_sms;
+  const ClusterCapacity* cap = nullptr;
+  cudaError_t e = cluster_capacity(&cap);
+  if (e != cudaSuccess) return e;
+  // the largest cluster for which one cluster per sequence still fits in a
+  // single wave: more CTAs keep more loads in flight
+  int CL = 1;
+  for (int cl = kMaxCluster; cl >= 1; --cl) {
+    if (cap->resident[cl] >= Bt) {
+      CL = cl;
+      break;
+    }
   }
   const int vec4 = (vocab % 4 == 0) && ((reinterpret_cast<uintptr_t>(logits) & 15u) == 0);
   cudaLaunchConfig_t cfg = {};
@@ -207,26 +264,13 @@ static cudaError_t launch_accept_cl(const float* logits, const int32_t* draft, i
   cfg.stream = stream;
   cudaLaunchAttribute attr[1];
   attr[0].id = cudaLaunchAttributeClusterDimension;
-  attr[0].val.clusterDim.x = CL;
+  attr[0].val.clusterDim.x = static_cast<unsigned>(CL);
   attr[0].val.clusterDim.y = 1;
   attr[0].val.clusterDim.z = 1;
   cfg.attrs = attr;
   cfg.numAttrs = 1;
-  return cudaLaunchKernelEx(&cfg, kern, logits, draft, gamma, vocab, vec4, accepted_len, out_tokens, row_argmax,
-                            err_word);
-}
-
-cudaError_t launch_accept(const float* logits, const int32_t* draft, int Bt, int gamma, int vocab,
-                          int32_t* accepted_len, int32_t* out_tokens, int32_t* row_argmax, int32_t* err_word,
-                          int num_sms, cudaStream_t stream) {
-  // enough CTAs to cover every SM a few times; smaller clusters for big batches
-  const int want = 4 * num_sms;
-  if (Bt * 8 < want) return launch_accept_cl<16>(logits, draft, Bt, gamma, vocab, accepted_len, out_tokens,
-                                                 row_argmax, err_word, stream);
-  if (Bt * 4 < want) return launch_accept_cl<8>(logits, draft, Bt, gamma, vocab, accepted_len, out_tokens,
-                                                row_argmax, err_word, stream);
-  return launch_accept_cl<4>(logits, draft, Bt, gamma, vocab, accepted_len, out_tokens, row_argmax, err_word,
-                             stream);
+  return cudaLaunchKernelEx(&cfg, accept_kernel, logits, draft, gamma, vocab, vec4, accepted_len, out_tokens,
+                            row_argmax, err_word);
 }
 
 }  // namespace simsd

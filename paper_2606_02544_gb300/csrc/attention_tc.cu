@@ -9,22 +9,24 @@
 // the page table with TMA), then one tile with the 2*gamma new slots, whose
 // Eq. (1) visibility is evaluated on the fly from (section, tau).
 //
-// Warp roles (320 threads):
-//   warps 0-3, 4-7  two softmax warpgroups.  Group w takes the unit's tiles
-//              w, w+2, w+4, ... with its own S, P and O in TMEM and its own
-//              running max / sum; thread i of a group owns query row i (TMEM
-//              lane i).  Two groups keep two tiles in flight through the
-//              softmax, so the shared-memory ring recycles twice as fast.
-//              At the end group 1 hands its (m, l, O) rows to group 0 through
-//              shared memory and group 0 writes the merged result.
-//   warp 8     TMA producer (one thread): Q once, then K/V tiles into a
-//              STAGES-deep shared-memory ring.
-//   warp 9     MMA issuer (one thread) and TMEM owner.  It polls both
-//              groups and issues whatever is ready: S_i = Q K_i^T (SS MMA,
-//              128x64x128) or O_w += P_i V_i (TS MMA, P in TMEM, V MN-major in
-//              shared memory, 128x128x64).
-// TMEM (512 columns): group w owns [256w, 256w+256): S [0,64) fp32, P in two
-// buffers [64,96) and [96,128) (bf16 pairs), O [128,256) fp32.
+// Two CTAs share each SM (96 KB of shared memory, 256 TMEM columns and 192
+// threads apiece), so one CTA's set-up, first loads and epilogue overlap the
+// other's streaming, and the two rings together keep the same bytes in
+// flight as one large ring.
+//
+// Warp roles (192 threads):
+//   warps 0-3  softmax; thread i owns query row i (TMEM lane i).  They first
+//              move the Q tile from shared memory into TMEM, then per key
+//              tile read S, update the running max / sum, write P (bf16)
+//              over the first half of S and hand it to the MMA issuer.
+//   warp 4     TMA producer (one thread): Q, then K/V tiles into a 3-deep
+//              ring of 32 KB slots (Q uses the first slot once).
+//   warp 5     MMA issuer (one thread) and TMEM owner.  Per tile:
+//              S = Q K^T (TS MMA: Q in TMEM, K in shared memory) and, once P
+//              is written, O += P V (TS MMA: P in TMEM, V MN-major in shared
+//              memory).  The next S overwrites P, so it waits for that PV.
+// TMEM (256 columns): Q [0,64) as bf16 pairs, S [64,128) fp32 with P in its
+// first 32 columns, O [128,256) fp32.
 //
 // Every mbarrier wait is bounded; a wait that expires sets SIMSD_EW_TIMEOUT
 // and makes the whole CTA stop, drain its async work and free its TMEM.
@@ -52,15 +54,15 @@ namespace {
 constexpr int kTile = 64;            // keys per tile
 constexpr int kD = 128;              // head dimension
 constexpr int kRows = 128;           // MMA M (query rows per CTA)
-constexpr int kGroups = 2;           // softmax warpgroups
-constexpr int kThreads = 32 * (4 * kGroups + 2);
-constexpr int kWarpProducer = 4 * kGroups;
-constexpr int kWarpMma = 4 * kGroups + 1;
-constexpr uint32_t kTmemCols = 512;
-constexpr uint32_t kGroupCols = 256;
-constexpr uint32_t kColS = 0, kColP = 64, kColO = 128;
-constexpr int kQHalfBytes = kRows * 128;    // 128 rows x 64 bf16
-constexpr int kKvHalfBytes = kTile * 128;   // 64 rows x 64 bf16
+constexpr int kStages = 3;           // ring slots of one CTA
+constexpr int kThreads = 192;
+constexpr int kWarpProducer = 4;
+constexpr int kWarpMma = 5;
+constexpr uint32_t kTmemCols = 256;
+constexpr uint32_t kColQ = 0, kColS = 64, kColO = 128;
+constexpr int kHalfBytes = kTile * 128;     // 64 rows x 64 bf16 (one d-half of K or V)
+constexpr int kSlotBytes = 4 * kHalfBytes;  // K0 K1 V0 V1, or Q0 Q1 (16 KB each)
+constexpr int kPageCache = 512;             // page ids of one sequence kept in shared memory
 constexpr float kRescaleThreshold = 8.0f;   // log2 units: rescale when the max grows by > 2^8
 
 struct TcParams {
@@ -76,42 +78,38 @@ struct TcParams {
   float scale_log2;
 };
 
-template <int STAGES>
 struct alignas(1024) Smem {
-  uint8_t q[2][kQHalfBytes];                // [d half][row][64]
-  uint8_t kv[STAGES][4][kKvHalfBytes];      // [stage][K0, K1, V0, V1][key][64]
-  uint64_t bar_q;
-  uint64_t bar_k[STAGES], bar_v[STAGES], bar_empty[STAGES];
-  uint64_t bar_s_full[kGroups], bar_s_free[kGroups], bar_p[kGroups][2], bar_o[kGroups];
-  uint64_t bar_ofinal, bar_drain;
+  uint8_t ring[kStages][kSlotBytes];
+  uint64_t bar_k[kStages], bar_v[kStages], bar_empty[kStages];
+  uint64_t bar_qt, bar_s_full, bar_p, bar_pv, bar_drain;
   uint32_t tmem_base;
   int abort_flag;
   int seq_bad;
   int b_sel;
   int32_t tau[64];
   uint8_t sect[64];
+  int32_t pages[kPageCache];
 };
 
-template <int STAGES>
-constexpr size_t smem_bytes() {
-  return sizeof(Smem<STAGES>) + 1024;
-}
-static_assert(smem_bytes<6>() <= 232448, "shared memory budget of one CTA");
+constexpr size_t smem_bytes() { return sizeof(Smem) + 1024; }
+static_assert(2 * (smem_bytes() + 1024) <= 233472, "two CTAs per SM");
 
-template <int STAGES>
-__device__ __forceinline__ void signal_abort(Smem<STAGES>& sm, int32_t* err_word) {
+__device__ __forceinline__ void signal_abort(Smem& sm, int32_t* err_word) {
   raise_error(err_word, SIMSD_EW_TIMEOUT);
   *reinterpret_cast<volatile int*>(&sm.abort_flag) = 1;
 }
 
-template <int STAGES>
-__global__ void __launch_bounds__(kThreads, 1)
+// Row r of a 128-byte-swizzled tile: 16-byte chunk c sits at chunk c ^ (r & 7).
+__device__ __forceinline__ uint4 ld_sw128_chunk(const uint8_t* half, int r, int c) {
+  return *reinterpret_cast<const uint4*>(half + r * 128 + ((c ^ (r & 7)) << 4));
+}
+
+__global__ void __launch_bounds__(kThreads, 2)
     attention_tc_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ CUtensorMap tm_kn,
                         const __grid_constant__ CUtensorMap tm_vn, const __grid_constant__ CUtensorMap tm_kc,
                         const __grid_constant__ CUtensorMap tm_vc, const __grid_constant__ TcParams p) {
   extern __shared__ uint8_t smem_raw[];
-  Smem<STAGES>& sm =
-      *reinterpret_cast<Smem<STAGES>*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~static_cast<uintptr_t>(1023));
+  Smem& sm = *reinterpret_cast<Smem*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~static_cast<uintptr_t>(1023));
   volatile int* abort_flag = &sm.abort_flag;
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
 
@@ -129,11 +127,28 @@ __global__ void __launch_bounds__(kThreads, 1)
     sm.seq_bad = 0;
     sm.b_sel = rank;
   }
-  // prefix lengths, staged in the (still unused) K/V ring for the ranking
-  int32_t* nval = reinterpret_cast<int32_t*>(sm.kv[0][0]);
+  // prefix lengths, staged in the (still unused) ring for the ranking
+  int32_t* nval = reinterpret_cast<int32_t*>(sm.ring[0]);
   const bool sort = p.Bt <= 256;
   if (sort)
     for (int i = tid; i < p.Bt; i += kThreads) nval[i] = p.prefix_len[i];
+  if (tid == 0) {
+    for (int s = 0; s < kStages; ++s) {
+      mbar_init(smem_u32(&sm.bar_k[s]), 1);
+      mbar_init(smem_u32(&sm.bar_v[s]), 1);
+      mbar_init(smem_u32(&sm.bar_empty[s]), 1);
+    }
+    mbar_init(smem_u32(&sm.bar_qt), 1);
+    mbar_init(smem_u32(&sm.bar_s_full), 1);
+    mbar_init(smem_u32(&sm.bar_p), 4);
+    mbar_init(smem_u32(&sm.bar_pv), 1);
+    mbar_init(smem_u32(&sm.bar_drain), 1);
+    fence_mbar_init();
+  }
+  if (warp == kWarpMma) {
+    tmem_alloc(smem_u32(&sm.tmem_base), kTmemCols);
+    tmem_relinquish();
+  }
   __syncthreads();
   if (sort) {
     for (int i = tid; i < p.Bt; i += kThreads) {
@@ -145,6 +160,8 @@ __global__ void __launch_bounds__(kThreads, 1)
       }
       if (r == rank) sm.b_sel = i;
     }
+    // the staging area is overwritten by TMA later
+    fence_proxy_async_smem();
   }
   __syncthreads();
   const int b = sm.b_sel;
@@ -157,8 +174,10 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
   } else {
     const int npages = (n + p.page_size - 1) / p.page_size;
+    const int32_t* bt = p.block_table + static_cast<size_t>(b) * p.max_pages;
     for (int i = tid; i < npages; i += kThreads) {
-      const int pg = p.block_table[static_cast<size_t>(b) * p.max_pages + i];
+      const int pg = bt[i];
+      if (i < kPageCache) sm.pages[i] = pg;
       if (pg < 0 || pg >= p.num_pages) {
         sm.seq_bad = 1;
         raise_error(p.err_word, SIMSD_EW_PAGE);
@@ -168,28 +187,6 @@ __global__ void __launch_bounds__(kThreads, 1)
   for (int i = tid; i < p.S; i += kThreads) {
     sm.tau[i] = p.tau[static_cast<size_t>(b) * p.S + i];
     sm.sect[i] = p.section[static_cast<size_t>(b) * p.S + i];
-  }
-  if (tid == 0) {
-    mbar_init(smem_u32(&sm.bar_q), 1);
-    for (int s = 0; s < STAGES; ++s) {
-      mbar_init(smem_u32(&sm.bar_k[s]), 1);
-      mbar_init(smem_u32(&sm.bar_v[s]), 1);
-      mbar_init(smem_u32(&sm.bar_empty[s]), 1);
-    }
-    for (int w = 0; w < kGroups; ++w) {
-      mbar_init(smem_u32(&sm.bar_s_full[w]), 1);
-      mbar_init(smem_u32(&sm.bar_s_free[w]), 4);
-      mbar_init(smem_u32(&sm.bar_p[w][0]), 4);
-      mbar_init(smem_u32(&sm.bar_p[w][1]), 4);
-      mbar_init(smem_u32(&sm.bar_o[w]), 1);
-    }
-    mbar_init(smem_u32(&sm.bar_ofinal), 1);
-    mbar_init(smem_u32(&sm.bar_drain), 1);
-    fence_mbar_init();
-  }
-  if (warp == kWarpMma) {
-    tmem_alloc(smem_u32(&sm.tmem_base), kTmemCols);
-    tmem_relinquish();
   }
   tc_fence_before();
   __syncthreads();
@@ -205,36 +202,42 @@ __global__ void __launch_bounds__(kThreads, 1)
 
   if (warp == kWarpProducer) {
     // ------------------------------------------------------------ producer
+    // ring item 0 is Q, item i + 1 is the i-th key tile of this unit
     if (lane == 0 && ntiles > 0) {
       tma_prefetch_desc(&tm_q);
       tma_prefetch_desc(&tm_kc);
       tma_prefetch_desc(&tm_vc);
       const uint32_t q_bytes = 2u * static_cast<uint32_t>(p.g * p.s_blk) * 128u;
-      mbar_arrive_expect_tx(smem_u32(&sm.bar_q), q_bytes);
       const int qz = b * p.S + rblk * p.s_blk;
-      tma_load_3d(smem_u32(sm.q[0]), &tm_q, smem_u32(&sm.bar_q), 0, kvh * p.g, qz);
-      tma_load_3d(smem_u32(sm.q[1]), &tm_q, smem_u32(&sm.bar_q), 64, kvh * p.g, qz);
+      const uint32_t q0 = smem_u32(sm.ring[0]);
+      mbar_arrive_expect_tx(smem_u32(&sm.bar_k[0]), q_bytes);
+      tma_load_3d(q0, &tm_q, smem_u32(&sm.bar_k[0]), 0, kvh * p.g, qz);
+      tma_load_3d(q0 + 2 * kHalfBytes, &tm_q, smem_u32(&sm.bar_k[0]), 64, kvh * p.g, qz);
+      mbar_arrive(smem_u32(&sm.bar_v[0]));  // keeps the two barriers of slot 0 in step
       const int P = p.page_size;
-      int issued = 0;
+      const int32_t* bt = p.block_table + static_cast<size_t>(b) * p.max_pages;
+      int issued = 1;
       for (int i = 0; i < ntiles; ++i) {
-        const int t = t0 + i, st = i % STAGES;
-        if (i >= STAGES && !mbar_wait(smem_u32(&sm.bar_empty[st]), ((i / STAGES) - 1) & 1, abort_flag)) {
+        const int it = i + 1, st = it % kStages;
+        if (it >= kStages && !mbar_wait(smem_u32(&sm.bar_empty[st]), ((it / kStages) - 1) & 1, abort_flag)) {
           signal_abort(sm, p.err_word);
           break;
         }
+        const int t = t0 + i;
         const uint32_t bk = smem_u32(&sm.bar_k[st]), bv = smem_u32(&sm.bar_v[st]);
-        const uint32_t k0 = smem_u32(sm.kv[st][0]), k1 = smem_u32(sm.kv[st][1]);
-        const uint32_t v0 = smem_u32(sm.kv[st][2]), v1 = smem_u32(sm.kv[st][3]);
+        const uint32_t k0 = smem_u32(sm.ring[st]), k1 = k0 + kHalfBytes;
+        const uint32_t v0 = k0 + 2 * kHalfBytes, v1 = k0 + 3 * kHalfBytes;
         if (t < T) {
           const int key0 = t * kTile;
           const int valid = min(kTile, n - key0);
-          const int32_t* bt = p.block_table + static_cast<size_t>(b) * p.max_pages;
           if (P >= kTile) {
-            const int row = (bt[key0 / P] * p.Hkv + kvh) * P + (key0 % P);
-            mbar_arrive_expect_tx(bk, 2u * kKvHalfBytes);
+            const int pi = key0 / P;
+            const int pg = pi < kPageCache ? sm.pages[pi] : bt[pi];
+            const int row = (pg * p.Hkv + kvh) * P + (key0 % P);
+            mbar_arrive_expect_tx(bk, 2u * kHalfBytes);
             tma_load_2d(k0, &tm_kc, bk, 0, row);
             tma_load_2d(k1, &tm_kc, bk, 64, row);
-            mbar_arrive_expect_tx(bv, 2u * kKvHalfBytes);
+            mbar_arrive_expect_tx(bv, 2u * kHalfBytes);
             tma_load_2d(v0, &tm_vc, bv, 0, row);
             tma_load_2d(v1, &tm_vc, bv, 64, row);
           } else {
@@ -242,13 +245,17 @@ __global__ void __launch_bounds__(kThreads, 1)
             const uint32_t sub_bytes = static_cast<uint32_t>(P) * 128u;
             mbar_arrive_expect_tx(bk, 2u * nsub * sub_bytes);
             for (int sb = 0; sb < nsub; ++sb) {
-              const int row = (bt[(key0 + sb * P) / P] * p.Hkv + kvh) * P;
+              const int pi = (key0 + sb * P) / P;
+              const int pg = pi < kPageCache ? sm.pages[pi] : bt[pi];
+              const int row = (pg * p.Hkv + kvh) * P;
               tma_load_2d(k0 + sb * sub_bytes, &tm_kc, bk, 0, row);
               tma_load_2d(k1 + sb * sub_bytes, &tm_kc, bk, 64, row);
             }
             mbar_arrive_expect_tx(bv, 2u * nsub * sub_bytes);
             for (int sb = 0; sb < nsub; ++sb) {
-              const int row = (bt[(key0 + sb * P) / P] * p.Hkv + kvh) * P;
+              const int pi = (key0 + sb * P) / P;
+              const int pg = pi < kPageCache ? sm.pages[pi] : bt[pi];
+              const int row = (pg * p.Hkv + kvh) * P;
               tma_load_2d(v0 + sb * sub_bytes, &tm_vc, bv, 0, row);
               tma_load_2d(v1 + sb * sub_bytes, &tm_vc, bv, 64, row);
             }
@@ -266,77 +273,52 @@ __global__ void __launch_bounds__(kThreads, 1)
       }
       // Drain: every issued load must have landed before the CTA may exit.
       // In a normal run these phases completed long ago.
-      for (int i = max(0, issued - STAGES); i < issued; ++i) {
-        const int st = i % STAGES;
-        mbar_wait(smem_u32(&sm.bar_k[st]), (i / STAGES) & 1, nullptr);
-        mbar_wait(smem_u32(&sm.bar_v[st]), (i / STAGES) & 1, nullptr);
+      for (int it = max(0, issued - kStages); it < issued; ++it) {
+        const int st = it % kStages;
+        mbar_wait(smem_u32(&sm.bar_k[st]), (it / kStages) & 1, nullptr);
+        mbar_wait(smem_u32(&sm.bar_v[st]), (it / kStages) & 1, nullptr);
       }
-      mbar_wait(smem_u32(&sm.bar_q), 0, nullptr);
     }
     __syncwarp();
   } else if (warp == kWarpMma) {
     // ----------------------------------------------------------- MMA issuer
-    // Tile i belongs to group w = i & 1 as its j = i >> 1-th tile.
-    //   QK_i needs K_i and S_w free (group w has read S of tile i-2), and,
-    //   because P_w is double-buffered, PV_{i-4} already issued.
-    //   PV_i needs P_i and V_i; PVs go in tile order.
     if (lane == 0 && ntiles > 0) {
       constexpr uint32_t kIdescQK = idesc_bf16_f32(kRows, kTile, 0, 0);
       constexpr uint32_t kIdescPV = idesc_bf16_f32(kRows, kD, 0, 1);
-      bool ok = mbar_wait(smem_u32(&sm.bar_q), 0, abort_flag);
-      tc_fence_after();
-      const uint32_t q0 = smem_u32(sm.q[0]), q1 = smem_u32(sm.q[1]);
-      int next_qk = 0, next_pv = 0;
-      unsigned long long t_idle = 0;
-      uint32_t spins = 0;
-      while (ok && next_pv < ntiles) {
-        bool progressed = false;
-        if (next_qk < ntiles && next_qk - 4 < next_pv) {
-          const int i = next_qk, w = i & 1, j = i >> 1, st = i % STAGES;
-          if (mbar_try_wait(smem_u32(&sm.bar_k[st]), (i / STAGES) & 1) &&
-              (j == 0 || mbar_try_wait(smem_u32(&sm.bar_s_free[w]), (j - 1) & 1))) {
-            tc_fence_after();
-            const uint32_t kb0 = smem_u32(sm.kv[st][0]), kb1 = smem_u32(sm.kv[st][1]);
-            const uint32_t d_s = tmem + w * kGroupCols + kColS;
+      bool ok = mbar_wait(smem_u32(&sm.bar_qt), 0, abort_flag);
+      for (int i = 0; ok && i < ntiles; ++i) {
+        const int it = i + 1, st = it % kStages;
+        const uint32_t par = (it / kStages) & 1;
+        // S overwrites P of the previous tile; tcgen05.mma ops issued by one
+        // thread run in issue order, so that PV has read P before this S lands
+        if (!mbar_wait(smem_u32(&sm.bar_k[st]), par, abort_flag)) {
+          ok = false;
+          break;
+        }
+        tc_fence_after();
+        const uint32_t kb0 = smem_u32(sm.ring[st]), kb1 = kb0 + kHalfBytes;
 #pragma unroll
-            for (int kk = 0; kk < kD / 16; ++kk) {
-              const uint32_t qa = (kk < 4 ? q0 : q1) + (kk & 3) * 32;
-              const uint32_t ka = (kk < 4 ? kb0 : kb1) + (kk & 3) * 32;
-              tc_mma_ss(d_s, sdesc_sw128(qa, 16, 1024), sdesc_sw128(ka, 16, 1024), kIdescQK, kk > 0);
-            }
-            tc_commit(smem_u32(&sm.bar_s_full[w]));
-            ++next_qk;
-            progressed = true;
-          }
+        for (int kk = 0; kk < kD / 16; ++kk) {
+          const uint32_t ka = (kk < 4 ? kb0 : kb1) + (kk & 3) * 32;
+          tc_mma_ts(tmem + kColS, tmem + kColQ + 8 * kk, sdesc_sw128(ka, 16, 1024), kIdescQK, kk > 0);
         }
-        if (next_pv < next_qk) {
-          const int i = next_pv, w = i & 1, j = i >> 1, st = i % STAGES;
-          if (mbar_try_wait(smem_u32(&sm.bar_p[w][j & 1]), (j >> 1) & 1) &&
-              mbar_try_wait(smem_u32(&sm.bar_v[st]), (i / STAGES) & 1)) {
-            tc_fence_after();
-            const uint32_t vb = smem_u32(sm.kv[st][2]);
-            const uint32_t gbase = tmem + w * kGroupCols;
+        tc_commit(smem_u32(&sm.bar_s_full));
+        if (!mbar_wait(smem_u32(&sm.bar_p), i & 1, abort_flag) ||
+            !mbar_wait(smem_u32(&sm.bar_v[st]), par, abort_flag)) {
+          ok = false;
+          break;
+        }
+        tc_fence_after();
+        const uint32_t vb = kb0 + 2 * kHalfBytes;
 #pragma unroll
-            for (int kk = 0; kk < kTile / 16; ++kk) {
-              tc_mma_ts(gbase + kColO, gbase + kColP + 32 * (j & 1) + 8 * kk,
-                        sdesc_sw128(vb + kk * 2048, kKvHalfBytes, 1024), kIdescPV, (j > 0 || kk > 0) ? 1u : 0u);
-            }
-            tc_commit(smem_u32(&sm.bar_empty[st]));
-            tc_commit(smem_u32(&sm.bar_o[w]));
-            ++next_pv;
-            progressed = true;
-          }
+        for (int kk = 0; kk < kTile / 16; ++kk) {
+          tc_mma_ts(tmem + kColO, tmem + kColS + 8 * kk, sdesc_sw128(vb + kk * 2048, kHalfBytes, 1024),
+                    kIdescPV, (i > 0 || kk > 0) ? 1u : 0u);
         }
-        if (progressed) {
-          spins = 0;
-        } else if ((++spins & 63u) == 0) {
-          const unsigned long long now = globaltimer_ns();
-          if (spins == 64) t_idle = now;
-          if (*abort_flag || now - t_idle > kWaitLimitNs) ok = false;
-        }
+        tc_commit(smem_u32(&sm.bar_empty[st]));
+        tc_commit(smem_u32(&sm.bar_pv));
       }
       if (!ok) signal_abort(sm, p.err_word);
-      tc_commit(smem_u32(&sm.bar_ofinal));
       // every MMA issued by this thread has completed once this fires
       tc_commit(smem_u32(&sm.bar_drain));
       mbar_wait(smem_u32(&sm.bar_drain), 0, nullptr);
@@ -344,9 +326,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     __syncwarp();
   } else {
     // -------------------------------------------------------------- softmax
-    const int grp = warp >> 2;                 // 0 or 1
-    const int row = tid & (kRows - 1);         // TMEM lane / query row
-    const int wq = warp & 3;                   // lane quadrant of this warp
+    const int row = tid;                       // TMEM lane / query row
     const int s = rblk * p.s_blk + row / p.g;
     const int hl = row % p.g;
     const bool row_exists = row < p.rows_blk && s < p.S;
@@ -358,13 +338,42 @@ __global__ void __launch_bounds__(kThreads, 1)
       for (int t = 0; t < p.S; ++t)
         if (temporal_visible(si, ti, sm.sect[t], sm.tau[t])) vis |= 1ull << t;
     }
-    const uint32_t lane_tmem = tmem + grp * kGroupCols + (static_cast<uint32_t>(wq * 32) << 16);
+    const uint32_t lane_tmem = tmem + (static_cast<uint32_t>(warp * 32) << 16);
     float m_ref = -INFINITY, l_sum = 0.f;
     bool ok = true;
-    int j = 0;
-    for (int i = grp; i < ntiles; i += kGroups, ++j) {
-      const int t = t0 + i, st = i % STAGES;
-      if (!mbar_wait_warp(smem_u32(&sm.bar_s_full[grp]), j & 1, abort_flag)) {
+
+    // ---- Q: shared memory (ring slot 0) -> TMEM columns [0, 64)
+    if (ntiles > 0) {
+      ok = mbar_wait_warp(smem_u32(&sm.bar_k[0]), 0, abort_flag);
+      if (ok) {
+#pragma unroll 1
+        for (int h = 0; h < 2; ++h) {
+          const uint8_t* half = sm.ring[0] + h * 2 * kHalfBytes;
+          uint32_t qr[32];
+#pragma unroll
+          for (int c = 0; c < 8; ++c) {
+            const uint4 v = ld_sw128_chunk(half, row, c);
+            qr[4 * c] = v.x;
+            qr[4 * c + 1] = v.y;
+            qr[4 * c + 2] = v.z;
+            qr[4 * c + 3] = v.w;
+          }
+          tmem_st32(lane_tmem + kColQ + 32 * h, qr);
+        }
+        tmem_wait_st();
+      }
+      tc_fence_before();
+      asm volatile("bar.sync 1, 128;" ::: "memory");
+      if (tid == 0 && ok && !*abort_flag) {
+        mbar_arrive(smem_u32(&sm.bar_qt));
+        mbar_arrive(smem_u32(&sm.bar_empty[0]));
+      }
+    }
+
+    for (int i = 0; ok && i < ntiles; ++i) {
+      const int it = i + 1, st = it % kStages;
+      const int t = t0 + i;
+      if (!mbar_wait_warp(smem_u32(&sm.bar_s_full), i & 1, abort_flag)) {
         ok = false;
         break;
       }
@@ -373,9 +382,6 @@ __global__ void __launch_bounds__(kThreads, 1)
       tmem_ld32(lane_tmem + kColS, sa);
       tmem_ld32(lane_tmem + kColS + 32, sb);
       tmem_wait_ld();
-      tc_fence_before();
-      __syncwarp();
-      if (lane == 0) mbar_arrive(smem_u32(&sm.bar_s_free[grp]));
 
       const bool is_new = (t == T);
       const int valid = is_new ? p.S : min(kTile, n - t * kTile);
@@ -410,13 +416,8 @@ __global__ void __launch_bounds__(kThreads, 1)
           need = true;
       }
       if (__any_sync(0xffffffffu, need)) {
-        // O_grp holds this group's earlier tiles: wait for the PV of its
-        // previous tile, then rescale
-        if (!mbar_wait_warp(smem_u32(&sm.bar_o[grp]), (j - 1) & 1, abort_flag)) {
-          ok = false;
-          break;
-        }
-        tc_fence_after();
+        // O holds the earlier tiles; their PVs completed before this S was
+        // computed (the S MMA waited for the last one)
         const float f = need ? fast_exp2(m_ref - mx) : 1.0f;
         if (need) {
           l_sum *= f;
@@ -431,7 +432,6 @@ __global__ void __launch_bounds__(kThreads, 1)
           for (int c = 0; c < 32; ++c) o[c] = __float_as_uint(__uint_as_float(o[c]) * f);
           tmem_st32(lane_tmem + kColO + 32 * ch, o);
         }
-        tmem_wait_st();
       }
       // p = 2^(s*scale*log2e - m): one FFMA and one MUFU.EX2 per score.  Rows
       // that are not active leave garbage in their own P/O rows only (MMA rows
@@ -451,12 +451,12 @@ __global__ void __launch_bounds__(kThreads, 1)
 #pragma unroll
         for (int c = 0; c < w2; ++c) ps[c] += ps[c + w2];
       l_sum += ps[0];
-      tmem_st32(lane_tmem + kColP + 32 * (j & 1), pk);
+      tmem_st32(lane_tmem + kColS, pk);
       tmem_wait_st();
-      if (wq < 2 && (valid < kTile || is_new)) {
+      if (warp < 2 && (valid < kTile || is_new)) {
         // rows of V that no query may use are zeroed so that 0 * (stale or
         // non-finite data) cannot reach O
-        if (!mbar_wait_warp(smem_u32(&sm.bar_v[st]), (i / STAGES) & 1, abort_flag)) {
+        if (!mbar_wait_warp(smem_u32(&sm.bar_v[st]), (it / kStages) & 1, abort_flag)) {
           ok = false;
           break;
         }
@@ -464,8 +464,8 @@ __global__ void __launch_bounds__(kThreads, 1)
         const bool zero = kr >= valid || (is_new && sm.sect[kr] == kSectPad);
         if (zero) {
           const uint4 z = make_uint4(0u, 0u, 0u, 0u);
-          uint4* r0 = reinterpret_cast<uint4*>(sm.kv[st][2] + kr * 128);
-          uint4* r1 = reinterpret_cast<uint4*>(sm.kv[st][3] + kr * 128);
+          uint4* r0 = reinterpret_cast<uint4*>(sm.ring[st] + 2 * kHalfBytes + kr * 128);
+          uint4* r1 = reinterpret_cast<uint4*>(sm.ring[st] + 3 * kHalfBytes + kr * 128);
 #pragma unroll
           for (int c = 0; c < 8; ++c) {
             r0[c] = z;
@@ -476,17 +476,17 @@ __global__ void __launch_bounds__(kThreads, 1)
       }
       tc_fence_before();
       __syncwarp();
-      if (lane == 0) mbar_arrive(smem_u32(&sm.bar_p[grp][j & 1]));
+      if (lane == 0) mbar_arrive(smem_u32(&sm.bar_p));
     }
     if (!ok && lane == 0) signal_abort(sm, p.err_word);
-    // ---- epilogue: group 1 hands (m, l, O) to group 0, which merges
-    const bool have_o = ok && ntiles > 0 && mbar_wait_warp(smem_u32(&sm.bar_ofinal), 0, abort_flag);
+    // ---- epilogue: O of the last PV, scaled by 1/l
+    const bool have_o = ok && ntiles > 0 && mbar_wait_warp(smem_u32(&sm.bar_pv), (ntiles - 1) & 1, abort_flag);
     if (have_o) tc_fence_after();
-    const bool live = have_o && active && j > 0;   // this group saw at least one tile
-    // the ring is idle once every MMA has completed: reuse it for the hand-off
-    float* xo = reinterpret_cast<float*>(sm.kv[0][0]);          // [128 rows][132]
-    constexpr int kXStride = kD + 4;
-    if (grp == 1) {
+    const bool any = have_o && active && l_sum > 0.f;
+    const int h = kvh * p.g + hl;
+    if (p.nsplit == 1) {
+      const float inv = any ? 1.0f / l_sum : 0.f;
+      __nv_bfloat16* orow = p.out + ((static_cast<size_t>(b) * p.S + s) * p.Hq + h) * kD;
 #pragma unroll 1
       for (int ch = 0; ch < kD / 32; ++ch) {
         uint32_t o[32];
@@ -494,84 +494,44 @@ __global__ void __launch_bounds__(kThreads, 1)
           tmem_ld32(lane_tmem + kColO + 32 * ch, o);
           tmem_wait_ld();
         }
-        float4* dst = reinterpret_cast<float4*>(xo + row * kXStride + 32 * ch);
+        if (row_exists) {
+          uint4 pkd[4];
+          uint32_t* wv = reinterpret_cast<uint32_t*>(pkd);
 #pragma unroll
-        for (int c = 0; c < 8; ++c)
-          dst[c] = live ? make_float4(__uint_as_float(o[4 * c]), __uint_as_float(o[4 * c + 1]),
-                                      __uint_as_float(o[4 * c + 2]), __uint_as_float(o[4 * c + 3]))
-                        : make_float4(0.f, 0.f, 0.f, 0.f);
-      }
-      xo[row * kXStride + kD] = live ? m_ref : -INFINITY;
-      xo[row * kXStride + kD + 1] = live ? l_sum : 0.f;
-    }
-    asm volatile("bar.sync 1, %0;" ::"r"(4 * kGroups * 32) : "memory");
-    if (grp == 0) {
-      // merge the two groups' partial softmax states of this row
-      const float m1 = xo[row * kXStride + kD], l1 = xo[row * kXStride + kD + 1];
-      const float m0 = live ? m_ref : -INFINITY, l0 = live ? l_sum : 0.f;
-      const float M = fmaxf(m0, m1);
-      const float a0 = (M == -INFINITY || m0 == -INFINITY) ? 0.f : fast_exp2(m0 - M);
-      const float a1 = (M == -INFINITY || m1 == -INFINITY) ? 0.f : fast_exp2(m1 - M);
-      const float L = a0 * l0 + a1 * l1;
-      const bool any = active && have_o && L > 0.f;
-      const int h = kvh * p.g + hl;
-      if (p.nsplit == 1) {
-        const float inv = any ? 1.0f / L : 0.f;
-        __nv_bfloat16* orow = p.out + ((static_cast<size_t>(b) * p.S + s) * p.Hq + h) * kD;
-#pragma unroll 1
-        for (int ch = 0; ch < kD / 32; ++ch) {
-          uint32_t o[32];
-          if (have_o) {
-            tmem_ld32(lane_tmem + kColO + 32 * ch, o);
-            tmem_wait_ld();
+          for (int c = 0; c < 16; ++c) {
+            const float r0 = any ? __uint_as_float(o[2 * c]) * inv : 0.f;
+            const float r1 = any ? __uint_as_float(o[2 * c + 1]) * inv : 0.f;
+            wv[c] = pack_bf16x2(r0, r1);
           }
-          if (row_exists) {
-            const float* o1 = xo + row * kXStride + 32 * ch;
-            uint4 pkd[4];
-            uint32_t* wv = reinterpret_cast<uint32_t*>(pkd);
+          uint4* dst = reinterpret_cast<uint4*>(orow + 32 * ch);
 #pragma unroll
-            for (int c = 0; c < 16; ++c) {
-              const float v0 = live ? __uint_as_float(o[2 * c]) : 0.f;
-              const float v1 = live ? __uint_as_float(o[2 * c + 1]) : 0.f;
-              const float r0 = any ? (a0 * v0 + a1 * o1[2 * c]) * inv : 0.f;
-              const float r1 = any ? (a0 * v1 + a1 * o1[2 * c + 1]) * inv : 0.f;
-              wv[c] = pack_bf16x2(r0, r1);
-            }
-            uint4* dst = reinterpret_cast<uint4*>(orow + 32 * ch);
-#pragma unroll
-            for (int c = 0; c < 4; ++c) dst[c] = pkd[c];
-          }
+          for (int c = 0; c < 4; ++c) dst[c] = pkd[c];
         }
-      } else {
-        const size_t unit = ((static_cast<size_t>(b) * p.Hkv + kvh) * p.rb + rblk) * p.nsplit + split;
-        const size_t nunits = static_cast<size_t>(p.Bt) * p.Hkv * p.rb * p.nsplit;
-        float* wo = p.ws + (unit * p.rows_blk + row) * kD;
-        float* wml = p.ws + nunits * p.rows_blk * kD + (unit * p.rows_blk + row) * 2;
+      }
+    } else {
+      const size_t unit = ((static_cast<size_t>(b) * p.Hkv + kvh) * p.rb + rblk) * p.nsplit + split;
+      const size_t nunits = static_cast<size_t>(p.Bt) * p.Hkv * p.rb * p.nsplit;
+      float* wo = p.ws + (unit * p.rows_blk + row) * kD;
+      float* wml = p.ws + nunits * p.rows_blk * kD + (unit * p.rows_blk + row) * 2;
 #pragma unroll 1
-        for (int ch = 0; ch < kD / 32; ++ch) {
-          uint32_t o[32];
-          if (have_o) {
-            tmem_ld32(lane_tmem + kColO + 32 * ch, o);
-            tmem_wait_ld();
-          }
-          if (row < p.rows_blk) {
-            const float* o1 = xo + row * kXStride + 32 * ch;
-            float4* dst = reinterpret_cast<float4*>(wo + 32 * ch);
-#pragma unroll
-            for (int c = 0; c < 8; ++c) {
-              float4 v;
-              v.x = any ? a0 * (live ? __uint_as_float(o[4 * c]) : 0.f) + a1 * o1[4 * c] : 0.f;
-              v.y = any ? a0 * (live ? __uint_as_float(o[4 * c + 1]) : 0.f) + a1 * o1[4 * c + 1] : 0.f;
-              v.z = any ? a0 * (live ? __uint_as_float(o[4 * c + 2]) : 0.f) + a1 * o1[4 * c + 2] : 0.f;
-              v.w = any ? a0 * (live ? __uint_as_float(o[4 * c + 3]) : 0.f) + a1 * o1[4 * c + 3] : 0.f;
-              dst[c] = v;
-            }
-          }
+      for (int ch = 0; ch < kD / 32; ++ch) {
+        uint32_t o[32];
+        if (have_o) {
+          tmem_ld32(lane_tmem + kColO + 32 * ch, o);
+          tmem_wait_ld();
         }
         if (row < p.rows_blk) {
-          wml[0] = any ? M : -INFINITY;
-          wml[1] = any ? L : 0.f;
+          float4* dst = reinterpret_cast<float4*>(wo + 32 * ch);
+#pragma unroll
+          for (int c = 0; c < 8; ++c)
+            dst[c] = any ? make_float4(__uint_as_float(o[4 * c]), __uint_as_float(o[4 * c + 1]),
+                                       __uint_as_float(o[4 * c + 2]), __uint_as_float(o[4 * c + 3]))
+                         : make_float4(0.f, 0.f, 0.f, 0.f);
         }
+      }
+      if (row < p.rows_blk) {
+        wml[0] = any ? m_ref : -INFINITY;
+        wml[1] = any ? l_sum : 0.f;
       }
     }
   }
@@ -630,13 +590,14 @@ __global__ void __launch_bounds__(128) combine_kernel(const TcParams p) {
   reinterpret_cast<uint2*>(orow)[lane] = v;
 }
 
-constexpr int kStages = 6;
-
 cudaError_t ensure_smem_attr() {
   static bool done = false;
   if (done) return cudaSuccess;
-  cudaError_t e = cudaFuncSetAttribute(attention_tc_kernel<kStages>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                       static_cast<int>(smem_bytes<kStages>()));
+  cudaError_t e = cudaFuncSetAttribute(attention_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                       static_cast<int>(smem_bytes()));
+  if (e != cudaSuccess) return e;
+  e = cudaFuncSetAttribute(attention_tc_kernel, cudaFuncAttributePreferredSharedMemoryCarveout,
+                           cudaSharedmemCarveoutMaxShared);
   if (e == cudaSuccess) done = true;
   return e;
 }
@@ -646,8 +607,8 @@ int occupancy_per_sm() {
   if (occ < 0) {
     int o = 0;
     ensure_smem_attr();
-    if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&o, attention_tc_kernel<kStages>, kThreads,
-                                                      smem_bytes<kStages>()) != cudaSuccess ||
+    if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&o, attention_tc_kernel, kThreads, smem_bytes()) !=
+            cudaSuccess ||
         o < 1)
       o = 1;
     occ = o;
@@ -753,8 +714,7 @@ cudaError_t launch_attention_tc(const AttnTcArgs& a, const AttnTcPlan& pl, Encod
     if (e != cudaSuccess) return e;
   }
   const long long grid = static_cast<long long>(a.Bt) * pl.nsplit * a.Hkv * pl.rb;
-  attention_tc_kernel<kStages><<<static_cast<unsigned>(grid), kThreads, smem_bytes<kStages>(), stream>>>(
-      tq, tkn, tvn, tkc, tvc, p);
+  attention_tc_kernel<<<static_cast<unsigned>(grid), kThreads, smem_bytes(), stream>>>(tq, tkn, tvn, tkc, tvc, p);
   cudaError_t e = cudaGetLastError();
   if (e != cudaSuccess || pl.nsplit == 1) return e;
   const long long warps = static_cast<long long>(a.Bt) * a.Hkv * pl.rb * pl.rows_blk;
