@@ -15,7 +15,10 @@
  *     rule over response positions; prompt visible to every response
  *     position; padding rows and columns zeroed.
  *   - Sec. 3.1 "Position Encoding Alignment": D~_k reuses the RoPE index of
- *     D_k.
+ *     D_k; rotary position embedding as in Su et al. (RoFormer), in the
+ *     rotate-half layout of the Qwen-family SDAR models.  Sec. 4 ablation
+ *     (Table 4) "without aligned RoPE": mask slots take their physical
+ *     positions after the data section instead.
  *   - Sec. 3.2 "Target Model Verification": slot with tau = r holds the r-th
  *     draft; acceptance along the draft order, longest prefix before the
  *     first rejection; Eq. (2) with one-hot distributions (temperature 0)
@@ -149,6 +152,38 @@ static double load_elem(const void *base, size_t idx, int dtype) {
     return (double)f;
 }
 
+/* Rounds v to the stored type, nearest with ties to even, and stores it. */
+static void store_elem(void *base, size_t idx, int dtype, double v) {
+    if (dtype == 0) {
+        ((float *)base)[idx] = (float)v;
+        return;
+    }
+    double r = v;
+    if (v != 0.0 && isfinite(v)) {
+        int e;
+        double m = frexp(v, &e);       /* v = m 2^e, 0.5 <= |m| < 1 */
+        r = ldexp(nearbyint(ldexp(m, 8)), e - 8); /* 8 significant bits */
+    }
+    float f = (float)r;                /* exact: r has 8 significant bits */
+    uint32_t bits;
+    memcpy(&bits, &f, sizeof bits);
+    ((uint16_t *)base)[idx] = (uint16_t)(bits >> 16);
+}
+
+/* Rotary position embedding (Su et al., RoFormer) in the rotate-half layout:
+ * for i in [0, d/2) the pair (x_i, x_{i+d/2}) is rotated by the angle
+ * pos * theta^(-2i/d), i.e. x_i + j x_{i+d/2} is multiplied by e^{j angle}. */
+static void rope_rotate(double *x, int d, double pos, double theta) {
+    int half = d / 2;
+    for (int i = 0; i < half; ++i) {
+        double ang = pos * pow(theta, -2.0 * i / d);
+        double c = cos(ang), sn = sin(ang);
+        double a = x[i], b = x[i + half];
+        x[i] = a * c - b * sn;
+        x[i + half] = b * c + a * sn;
+    }
+}
+
 /* out[b][s][h][:] = sum_j softmax_j(scale * q.k_j) v_j over the keys the
  * row may see: every cached prefix row of sequence b (the prompt / earlier
  * blocks, visible to all response positions) read through the page table,
@@ -164,12 +199,18 @@ static double load_elem(const void *base, size_t idx, int dtype) {
  * A sequence whose prefix length is outside [0, max_pages*page_size], whose
  * needed pages are outside [0, num_pages), or whose step map is invalid gets
  * all-zero output rows and sets the matching error bit.  Padding rows are
- * zero.  Returns the error bits. */
+ * zero.
+ * rope_theta > 0: q and k_new hold values before the rotary embedding; each
+ * q row and each k_new row of slot t is rotated at the position of slot t
+ * first (the cached keys are stored rotated already).  rope_mode 1: the
+ * aligned RoPE copy of Sec. 3.1 (D_k and D~_k both at n + k); rope_mode 2:
+ * physical positions (slot t at n + t, the ablation of Table 4).
+ * Returns the error bits. */
 int oracle_verify_attention(int dtype, const void *q, const void *k_new, const void *v_new,
                             const void *k_cache, const void *v_cache, const int32_t *block_table,
                             int max_pages, int page_size, int num_pages, const int32_t *prefix_len,
                             const int32_t *step_map, int Bt, int gamma, int Hq, int Hkv, int d,
-                            double scale, double *out, int nthreads) {
+                            double scale, double rope_theta, int rope_mode, double *out, int nthreads) {
     const int S = 2 * gamma, g = Hq / Hkv;
     int err = 0;
     int32_t *tau = (int32_t *)malloc(sizeof(int32_t) * (size_t)Bt * S);
@@ -194,6 +235,28 @@ int oracle_verify_attention(int dtype, const void *q, const void *k_new, const v
             }
         }
         nvalid[b] = ok ? n : -1;
+    }
+
+    /* rotated copies of q and k_new when the inputs are not rotated yet */
+    double *qr = NULL, *kr = NULL;
+    if (rope_theta > 0.0) {
+        qr = (double *)malloc(sizeof(double) * (size_t)Bt * S * Hq * d);
+        kr = (double *)malloc(sizeof(double) * (size_t)Bt * S * Hkv * d);
+        for (int b = 0; b < Bt; ++b) {
+            for (int t = 0; t < S; ++t) {
+                double pos = rope_mode == 2 ? (double)prefix_len[b] + t : (double)rope[(size_t)b * S + t];
+                for (int h = 0; h < Hq; ++h) {
+                    size_t o = (((size_t)b * S + t) * Hq + h) * d;
+                    for (int c = 0; c < d; ++c) qr[o + c] = load_elem(q, o + c, dtype);
+                    rope_rotate(qr + o, d, pos, rope_theta);
+                }
+                for (int h = 0; h < Hkv; ++h) {
+                    size_t o = (((size_t)b * S + t) * Hkv + h) * d;
+                    for (int c = 0; c < d; ++c) kr[o + c] = load_elem(k_new, o + c, dtype);
+                    rope_rotate(kr + o, d, pos, rope_theta);
+                }
+            }
+        }
     }
 
     long long rows = (long long)Bt * S * Hq;
@@ -239,8 +302,11 @@ int oracle_verify_attention(int dtype, const void *q, const void *k_new, const v
         for (int j = 0; j < cnt; ++j) {
             const void *kb = is_new[j] ? k_new : k_cache;
             double acc = 0.0;
-            for (int c = 0; c < d; ++c)
-                acc += load_elem(q, qoff + c, dtype) * load_elem(kb, koff[j] + c, dtype);
+            for (int c = 0; c < d; ++c) {
+                double qv = qr ? qr[qoff + c] : load_elem(q, qoff + c, dtype);
+                double kv = (kr && is_new[j]) ? kr[koff[j] + c] : load_elem(kb, koff[j] + c, dtype);
+                acc += qv * kv;
+            }
             score[j] = acc * scale;
             if (score[j] > m) m = score[j];
         }
@@ -263,6 +329,8 @@ int oracle_verify_attention(int dtype, const void *q, const void *k_new, const v
     free(sect);
     free(rope);
     free(nvalid);
+    free(qr);
+    free(kr);
     return err;
 }
 
@@ -334,14 +402,21 @@ int oracle_accept(const float *logits, const int32_t *draft, int Bt, int gamma, 
  * A destination page outside the table or the pool sets OR_ERR_PAGE and that
  * row is skipped; a missing source slot sets OR_ERR_STEP_MAP and the row is
  * skipped; a negative prefix or an accepted length outside [0,gamma] leaves
- * the sequence untouched.  Returns the error bits. */
+ * the sequence untouched.
+ * rope_theta > 0: k_new holds keys before the rotary embedding; the copied
+ * key of data slot k is rotated at its position n_b + k (Sec. 3.1) and
+ * rounded to the stored type, so that the cache holds rotated keys.
+ * Returns the error bits. */
 int oracle_kv_commit(int elem_bytes, const void *k_new, const void *v_new, int L,
                      const int32_t *step_map, const int32_t *accepted_len, void *k_cache,
                      void *v_cache, const int32_t *block_table, int max_pages, int page_size,
-                     int num_pages, int32_t *prefix_len, int Bt, int gamma, int Hkv, int d) {
+                     int num_pages, int32_t *prefix_len, int Bt, int gamma, int Hkv, int d,
+                     double rope_theta) {
     const int S = 2 * gamma;
     int err = 0;
     size_t row_bytes = (size_t)d * elem_bytes;
+    int dtype = elem_bytes == 4 ? 0 : 1;
+    double *row = (double *)malloc(sizeof(double) * (size_t)(d > 0 ? d : 1));
     for (int b = 0; b < Bt; ++b) {
         int n = prefix_len[b], a = accepted_len[b];
         if (a < 0 || a > gamma) {
@@ -380,8 +455,14 @@ int oracle_kv_commit(int elem_bytes, const void *k_new, const void *v_new, int L
                 for (int kvh = 0; kvh < Hkv; ++kvh) {
                     size_t s_el = ((((size_t)l * Bt + b) * S + src) * Hkv + kvh) * d;
                     size_t d_el = ((((size_t)l * num_pages + pg) * Hkv + kvh) * page_size + off) * d;
-                    memcpy((char *)k_cache + d_el * elem_bytes, (const char *)k_new + s_el * elem_bytes,
-                           row_bytes);
+                    if (rope_theta > 0.0) {
+                        for (int c = 0; c < d; ++c) row[c] = load_elem(k_new, s_el + c, dtype);
+                        rope_rotate(row, d, (double)n + src, rope_theta);
+                        for (int c = 0; c < d; ++c) store_elem(k_cache, d_el + c, dtype, row[c]);
+                    } else {
+                        memcpy((char *)k_cache + d_el * elem_bytes, (const char *)k_new + s_el * elem_bytes,
+                               row_bytes);
+                    }
                     memcpy((char *)v_cache + d_el * elem_bytes, (const char *)v_new + s_el * elem_bytes,
                            row_bytes);
                 }
@@ -389,7 +470,14 @@ int oracle_kv_commit(int elem_bytes, const void *k_new, const void *v_new, int L
         }
         prefix_len[b] = n + a;
     }
+    free(row);
     return err;
+}
+
+/* Rotates rows of x [rows][d] in place at position pos (the oracle's RoPE,
+ * exported for its pins). */
+void oracle_rope_rotate(double *x, int rows, int d, double pos, double theta) {
+    for (int r = 0; r < rows; ++r) rope_rotate(x + (size_t)r * d, d, pos, theta);
 }
 
 /* Number of OpenMP threads the oracle uses by default. */

@@ -71,9 +71,12 @@ def _load():
             i = ctypes.c_int
             lib.oracle_build_mask.argtypes = [P, P, i, i, P, P, P, P, P]
             lib.oracle_verify_attention.argtypes = [i, P, P, P, P, P, P, i, i, i, P, P, i, i, i, i, i,
-                                                    ctypes.c_double, P, i]
+                                                    ctypes.c_double, ctypes.c_double, i, P, i]
             lib.oracle_accept.argtypes = [P, P, i, i, i, P, P, P]
-            lib.oracle_kv_commit.argtypes = [i, P, P, i, P, P, P, P, P, i, i, i, P, i, i, i, i]
+            lib.oracle_kv_commit.argtypes = [i, P, P, i, P, P, P, P, P, i, i, i, P, i, i, i, i,
+                                             ctypes.c_double]
+            lib.oracle_rope_rotate.argtypes = [P, i, i, ctypes.c_double, ctypes.c_double]
+            lib.oracle_rope_rotate.restype = None
             for f in (lib.oracle_build_mask, lib.oracle_verify_attention, lib.oracle_accept,
                       lib.oracle_kv_commit, lib.oracle_max_threads):
                 f.restype = ctypes.c_int
@@ -128,12 +131,15 @@ def _as_storage(x):
 
 
 def verify_attention(q, k_new, v_new, k_cache, v_cache, block_table, prefix_len, step_map,
-                     gamma: int, scale: float | None = None, threads: int = 0):
+                     gamma: int, scale: float | None = None, threads: int = 0, rope_theta: float = 0.0,
+                     rope_mode: int = 1):
     """Exact masked attention of the verification forward, in fp64.
 
     q [Bt][2g][Hq][d]; k_new, v_new [Bt][2g][Hkv][d];
     k_cache, v_cache [num_pages][Hkv][P][d]; block_table [Bt][max_pages];
-    all float32 or all bf16 bit patterns (uint16).  Returns (out float64
+    all float32 or all bf16 bit patterns (uint16).  rope_theta > 0: q and
+    k_new are rotated first (rope_mode 1: aligned RoPE copy of Sec. 3.1,
+    2: physical positions of the Table 4 ablation).  Returns (out float64
     [Bt][2g][Hq][d], error bits).
     """
     lib = _load()
@@ -160,8 +166,19 @@ def verify_attention(q, k_new, v_new, k_cache, v_cache, block_table, prefix_len,
     err = lib.oracle_verify_attention(dt, _ptr(q), _ptr(k_new), _ptr(v_new), _ptr(k_cache),
                                       _ptr(v_cache), _ptr(block_table), max_pages, P, num_pages,
                                       _ptr(prefix_len), _ptr(sm), Bt, gamma, Hq, Hkv, d,
-                                      float(scale), _ptr(out), int(threads))
+                                      float(scale), float(rope_theta), int(rope_mode), _ptr(out),
+                                      int(threads))
     return out, int(err)
+
+
+def rope_rotate(x, pos: float, theta: float):
+    """The oracle's rotary embedding of the rows of x [..., d] at one
+    position (rotate-half layout); returns a float64 copy."""
+    lib = _load()
+    a = np.array(x, dtype=np.float64, copy=True, order="C")
+    d = a.shape[-1]
+    lib.oracle_rope_rotate(_ptr(a), int(a.size // d), d, float(pos), float(theta))
+    return a
 
 
 def accept(logits, draft, gamma: int):
@@ -184,12 +201,13 @@ def accept(logits, draft, gamma: int):
 
 
 def kv_commit(k_new, v_new, step_map, accepted_len, k_cache, v_cache, block_table, prefix_len,
-              gamma: int):
+              gamma: int, rope_theta: float = 0.0):
     """Appends the accepted drafts' data-slot K/V to the paged cache.
 
     k_new, v_new [L][Bt][2g][Hkv][d]; k_cache, v_cache [L][num_pages][Hkv][P][d]
-    (float32 or bf16 bits as uint16).  Works on copies; returns (k_cache,
-    v_cache, prefix_len, error bits).
+    (float32 or bf16 bits as uint16).  rope_theta > 0: k_new is not rotated
+    yet and each committed key is rotated at its position n + k.  Works on
+    copies; returns (k_cache, v_cache, prefix_len, error bits).
     """
     lib = _load()
     k_new = np.ascontiguousarray(k_new)
@@ -205,5 +223,5 @@ def kv_commit(k_new, v_new, step_map, accepted_len, k_cache, v_cache, block_tabl
     sm = None if step_map is None else _c(step_map, np.int32)
     err = lib.oracle_kv_commit(k_new.dtype.itemsize, _ptr(k_new), _ptr(v_new), L, _ptr(sm), _ptr(a),
                                _ptr(kc), _ptr(vc), _ptr(block_table), block_table.shape[1], P,
-                               num_pages, _ptr(n), Bt, gamma, Hkv, d)
+                               num_pages, _ptr(n), Bt, gamma, Hkv, d, float(rope_theta))
     return kc, vc, n, int(err)
