@@ -169,7 +169,7 @@ def run_gpu(args):
     build.build()
     simsd.load_library()
     wl = inputs.WORKLOADS[args.workload]
-    si = inputs.make_step_inputs(wl, device="cuda")
+    si = inputs.make_step_inputs(wl, device="cuda", layers=args.layers)
     st = VerifyStep(si, restore_prefix=True)
     torch.cuda.synchronize()
 
@@ -464,6 +464,9 @@ def main():
     ap.add_argument("--workload", default=DEFAULT_WORKLOAD, choices=["c1", "c2", "c3", "c4"])
     ap.add_argument("--cpu-seconds", type=float, default=15.0)
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--layers", type=int, default=None,
+                    help="run only this many layers of the workload (a smaller case of the same per-layer "
+                         "kernels, for profiler captures)")
     args = ap.parse_args()
     if args.steps is None:
         args.steps = DEFAULT_STEPS[args.workload] if args.impl == "ours" else 10

@@ -56,6 +56,7 @@ constexpr int kD = 128;              // head dimension
 constexpr int kRows = 128;           // MMA M (query rows per CTA)
 constexpr int kStages = 3;           // ring slots of one CTA
 constexpr int kThreads = 192;
+constexpr int kCtasPerSm = 2;        // register (launch bounds) and shared-memory budget of one CTA
 constexpr int kWarpProducer = 4;
 constexpr int kWarpMma = 5;
 constexpr uint32_t kTmemCols = 256;
@@ -92,7 +93,7 @@ struct alignas(1024) Smem {
 };
 
 constexpr size_t smem_bytes() { return sizeof(Smem) + 1024; }
-static_assert(2 * (smem_bytes() + 1024) <= 233472, "two CTAs per SM");
+static_assert(kCtasPerSm * (smem_bytes() + 1024) <= 233472, "two CTAs per SM");
 
 __device__ __forceinline__ void signal_abort(Smem& sm, int32_t* err_word) {
   raise_error(err_word, SIMSD_EW_TIMEOUT);
@@ -104,7 +105,7 @@ __device__ __forceinline__ uint4 ld_sw128_chunk(const uint8_t* half, int r, int 
   return *reinterpret_cast<const uint4*>(half + r * 128 + ((c ^ (r & 7)) << 4));
 }
 
-__global__ void __launch_bounds__(kThreads, 2)
+__global__ void __launch_bounds__(kThreads, kCtasPerSm)
     attention_tc_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ CUtensorMap tm_kn,
                         const __grid_constant__ CUtensorMap tm_vn, const __grid_constant__ CUtensorMap tm_kc,
                         const __grid_constant__ CUtensorMap tm_vc, const __grid_constant__ TcParams p) {
@@ -602,20 +603,6 @@ cudaError_t ensure_smem_attr() {
   return e;
 }
 
-int occupancy_per_sm() {
-  static int occ = -1;
-  if (occ < 0) {
-    int o = 0;
-    ensure_smem_attr();
-    if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&o, attention_tc_kernel, kThreads, smem_bytes()) !=
-            cudaSuccess ||
-        o < 1)
-      o = 1;
-    occ = o;
-  }
-  return occ;
-}
-
 bool make_map(EncodeTiledFn encode, CUtensorMap* m, const void* base, int rank, const cuuint64_t* dims,
               const cuuint64_t* strides, const cuuint32_t* box) {
   cuuint32_t es[3] = {1, 1, 1};
@@ -641,9 +628,11 @@ bool plan_attention_tc(int Bt, int gamma, int Hq, int Hkv, int max_pages, int pa
   }
   pl.rows_blk = g * pl.s_blk;
   if (pl.rows_blk > kRows || g > 256 || pl.s_blk > 256) return false;
-  // split the prefix only when the units alone cannot fill the GPU
+  // split the prefix only when the units alone cannot fill the GPU (the
+  // occupancy calculator reports one CTA per SM for this kernel although two
+  // are resident, so the budget the kernel is built for is used instead)
   const long long units = static_cast<long long>(Bt) * Hkv * pl.rb;
-  const long long slots = static_cast<long long>(num_sms) * occupancy_per_sm();
+  const long long slots = static_cast<long long>(num_sms) * kCtasPerSm;
   const long long max_tiles = (static_cast<long long>(max_pages) * page_size + kTile - 1) / kTile + 1;
   int ns = 1;
   if (units < slots) {
