@@ -120,8 +120,17 @@ SIMSD_API size_t simsd_verify_workspace_bytes(int dtype, int Bt, int gamma, int 
  *                block_table[b][p / page_size].  Rows past n_b are never used.
  *   block_table  [Bt][max_pages] int32; entries past the prefix are ignored.
  *   tau, section [Bt][2gamma] from simsd_build_mask.
- *   rope_pos     must be NULL: Q and K arrive already rotated (RoPE-copy
- *                positions are applied by the caller).
+ *   rope_pos     NULL: q and k_new arrive rotated already.  Otherwise
+ *                [Bt][2gamma] int32 positions, normally the RoPE-copy
+ *                positions of simsd_build_mask (Sec. 3.1 "Position Encoding
+ *                Alignment": D~_k reuses n_b + k of D_k); any other positions
+ *                (e.g. the physical ones of the Table 4 ablation) may be
+ *                given.  Each q row of slot s and each k_new row of slot t
+ *                is then rotated at rope_pos[b][s] / rope_pos[b][t] before
+ *                use (rotary embedding of RoFormer, rotate-half layout: the
+ *                pair (x_i, x_{i+d/2}) turns by pos * rope_theta^(-2i/d));
+ *                cached keys must be stored rotated.  Positions in [0, 2^20).
+ *   rope_theta   RoPE base, > 0 when rope_pos is given (ignored otherwise).
  *   softmax_scale 0 selects 1/sqrt(d).
  *   workspace    scratch of simsd_verify_workspace_bytes() bytes (NULL if 0).
  * Supported: SIMSD_BF16 with d = 128 and Hq/Hkv*2gamma <= 128 or
@@ -133,8 +142,9 @@ SIMSD_API size_t simsd_verify_workspace_bytes(int dtype, int Bt, int gamma, int 
 SIMSD_API int simsd_verify_attention(int dtype, const void* q, const void* k_new, const void* v_new, const void* k_cache,
                            const void* v_cache, int num_pages, const int32_t* block_table, int max_pages,
                            int page_size, const int32_t* prefix_len, const int32_t* tau, const uint8_t* section,
-                           const int32_t* rope_pos, int Bt, int gamma, int Hq, int Hkv, int d, float softmax_scale,
-                           void* out, void* workspace, size_t workspace_bytes, int32_t* err_word, void* stream);
+                           const int32_t* rope_pos, float rope_theta, int Bt, int gamma, int Hq, int Hkv, int d,
+                           float softmax_scale, void* out, void* workspace, size_t workspace_bytes,
+                           int32_t* err_word, void* stream);
 
 /*
  * simsd_verify_attention_noalloc -- simsd_verify_attention for callers that
@@ -163,8 +173,9 @@ SIMSD_API int simsd_verify_attention_noalloc(int dtype, const void* q, const voi
                                              const void* k_cache, const void* v_cache, int num_pages,
                                              const int32_t* block_table, int max_pages, int page_size,
                                              const int32_t* prefix_len, const int32_t* tau, const uint8_t* section,
-                                             const int32_t* rope_pos, int Bt, int gamma, int Hq, int Hkv, int d,
-                                             float softmax_scale, void* out, int32_t* err_word, void* stream);
+                                             const int32_t* rope_pos, float rope_theta, int Bt, int gamma, int Hq,
+                                             int Hkv, int d, float softmax_scale, void* out, int32_t* err_word,
+                                             void* stream);
 
 /*
  * simsd_accept -- greedy longest-prefix acceptance (Sec. 3.2, Eq. (2) with
@@ -195,6 +206,11 @@ SIMSD_API int simsd_accept(const float* logits, const int32_t* draft, int Bt, in
  * data-slot row whose tau is r+1 is copied to cache row prefix_len[b] + r;
  * then prefix_len[b] += accepted_len[b] (in place).
  *   k_new, v_new [L][Bt][2gamma][Hkv][d] dtype
+ *   rope_pos     NULL: k_new is rotated already.  Otherwise [Bt][2gamma]
+ *                positions as for simsd_verify_attention: the copied key of
+ *                data slot k is rotated at rope_pos[b][k] (rope_theta > 0,
+ *                even d <= 128) and rounded to dtype, so that the cache
+ *                holds rotated keys; values are copied unchanged.
  *   k_cache, v_cache [L][num_pages][Hkv][page_size][d] dtype
  * A destination page outside the table or pool sets SIMSD_EW_PAGE and that
  * row is skipped; a missing source slot sets SIMSD_EW_STEP_MAP and that row
@@ -203,9 +219,10 @@ SIMSD_API int simsd_accept(const float* logits, const int32_t* draft, int Bt, in
  * untouched.
  */
 SIMSD_API int simsd_kv_commit(int dtype, const void* k_new, const void* v_new, int L, const int32_t* tau,
-                    const uint8_t* section, const int32_t* accepted_len, void* k_cache, void* v_cache,
-                    int num_pages, const int32_t* block_table, int max_pages, int page_size, int32_t* prefix_len,
-                    int Bt, int gamma, int Hkv, int d, int32_t* err_word, void* stream);
+                              const uint8_t* section, const int32_t* rope_pos, float rope_theta,
+                              const int32_t* accepted_len, void* k_cache, void* v_cache, int num_pages,
+                              const int32_t* block_table, int max_pages, int page_size, int32_t* prefix_len, int Bt,
+                              int gamma, int Hkv, int d, int32_t* err_word, void* stream);
 
 /*
  * simsd_check_error -- synchronises `stream`, copies the device error word

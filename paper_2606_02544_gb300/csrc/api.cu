@@ -85,7 +85,138 @@ simsd::EncodeTiledFn encoder() {
 
 cudaStream_t as_stream(void* s) { return static_cast<cudaStream_t>(s); }
 
+// Shared body of the two attention entry points.  static_scratch: the
+// split partials go to the library's static array instead of the caller's
+// workspace.
+int verify_attention_impl(int dtype, const void* q, const void* k_new, const void* v_new, const void* k_cache,
+                          const void* v_cache, int num_pages, const int32_t* block_table, int max_pages,
+                          int page_size, const int32_t* prefix_len, const int32_t* tau, const uint8_t* section,
+                          const int32_t* rope_pos, float rope_theta, int Bt, int gamma, int Hq, int Hkv, int d,
+                          float softmax_scale, void* out, void* workspace, size_t workspace_bytes,
+                          bool static_scratch, int32_t* err_word, void* stream) {
+  if (Bt < 0) return arg_fail("Bt < 0");
+  if (gamma < 1 || gamma > 32) return arg_fail("gamma must be in [1, 32]");
+  if (Hq <= 0 || Hkv <= 0 || Hq % Hkv != 0) return arg_fail("Hq must be a positive multiple of Hkv");
+  if (num_pages < 0 || max_pages < 0) return arg_fail("negative page count");
+  if (page_size < 8 || !((page_size % 64 == 0) || (64 % page_size == 0)))
+    return unsupported("page_size must be a multiple of 64 or a divisor of 64 (>= 8)");
+  if (rope_pos && (!(rope_theta > 0.f) || std::isinf(rope_theta)))
+    return arg_fail("rope_theta must be positive and finite when rope_pos is given");
+  if (!(softmax_scale >= 0.f) || std::isinf(softmax_scale)) return arg_fail("softmax_scale");
+  if (Bt == 0) return SIMSD_OK;
+  if (!q || !k_new || !v_new || !prefix_len || !tau || !section || !out) return arg_fail("null pointer");
+  if (max_pages > 0 && (!block_table || !k_cache || !v_cache || num_pages == 0))
+    return arg_fail("null cache or block table");
+  if (!aligned16(q) || !aligned16(k_new) || !aligned16(v_new) || !aligned16(out) ||
+      (k_cache && !aligned16(k_cache)) || (v_cache && !aligned16(v_cache)))
+    return arg_fail("tensor pointers must be 16-byte aligned");
+  DeviceInfo info;
+  int rc = require_sm103(&info);
+  if (rc != SIMSD_OK) return rc;
+  const float scale = softmax_scale > 0.f ? softmax_scale : 1.0f / std::sqrt(static_cast<float>(d));
+  cudaStream_t s = as_stream(stream);
+  if (dtype == SIMSD_F32) {
+    // the fp32 path uses no scratch
+    if (d != 64 && d != 128) return unsupported("fp32 path needs d in {64, 128}");
+    simsd::AttnF32Args a{};
+    a.q = static_cast<const float*>(q);
+    a.k_new = static_cast<const float*>(k_new);
+    a.v_new = static_cast<const float*>(v_new);
+    a.k_cache = static_cast<const float*>(k_cache);
+    a.v_cache = static_cast<const float*>(v_cache);
+    a.block_table = block_table;
+    a.prefix_len = prefix_len;
+    a.tau = tau;
+    a.section = section;
+    a.rope_pos = rope_pos;
+    if (rope_pos) a.rope = simsd::make_rope_table(rope_theta, d);
+    a.out = static_cast<float*>(out);
+    a.err_word = err_word;
+    a.num_pages = num_pages;
+    a.max_pages = max_pages;
+    a.page_size = page_size;
+    a.Bt = Bt;
+    a.gamma = gamma;
+    a.Hq = Hq;
+    a.Hkv = Hkv;
+    a.d = d;
+    a.scale = scale;
+    cudaError_t e = simsd::launch_attention_f32(a, s);
+    return e == cudaSuccess ? SIMSD_OK : cuda_fail(e, "attention_f32 launch");
+  }
+  if (dtype != SIMSD_BF16) return unsupported("dtype");
+  if (d != 128) return unsupported("bf16 path needs d = 128");
+  if (static_cast<long long>(num_pages) * Hkv * page_size >= (1ll << 31))
+    return unsupported("page pool too large for 32-bit TMA row coordinates");
+  if (static_cast<long long>(Bt) * 2 * gamma * Hq >= (1ll << 31)) return unsupported("too many query rows");
+  simsd::AttnTcPlan plan;
+  if (!simsd::plan_attention_tc(Bt, gamma, Hq, Hkv, max_pages, page_size, info.num_sms, &plan))
+    return unsupported("query rows per KV head: need 2*gamma*Hq/Hkv <= 128 or 128 % (Hq/Hkv) == 0");
+  if (static_scratch) {
+    if (plan.ws_bytes > simsd::noalloc_scratch_capacity()) {
+      std::snprintf(g_last_error, sizeof(g_last_error),
+                    "unsupported: these sizes need %zu bytes of scratch, more than the %zu-byte static array; "
+                    "use simsd_verify_attention with a caller workspace",
+                    plan.ws_bytes, simsd::noalloc_scratch_capacity());
+      return SIMSD_ERR_UNSUPPORTED;
+    }
+    workspace = nullptr;
+    if (plan.ws_bytes > 0) {
+      cudaError_t e = simsd::noalloc_scratch_pointer(&workspace);
+      if (e != cudaSuccess) return cuda_fail(e, "cudaGetSymbolAddress of the static scratch");
+    }
+  } else if (plan.ws_bytes > 0 && (!workspace || workspace_bytes < plan.ws_bytes || !aligned16(workspace))) {
+    return arg_fail("workspace smaller than simsd_verify_workspace_bytes()");
+  }
+  simsd::EncodeTiledFn enc = encoder();
+  if (!enc) return cuda_fail(cudaErrorNotSupported, "cuTensorMapEncodeTiled entry point");
+  simsd::AttnTcArgs a{};
+  a.q = q;
+  a.k_new = k_new;
+  a.v_new = v_new;
+  // a pool with no pages is still described by a valid (never read) map
+  a.k_cache = k_cache ? k_cache : q;
+  a.v_cache = v_cache ? v_cache : q;
+  a.block_table = block_table;
+  a.prefix_len = prefix_len;
+  a.tau = tau;
+  a.section = section;
+  a.rope_pos = rope_pos;
+  if (rope_pos) a.rope = simsd::make_rope_table(rope_theta, d);
+  a.out = out;
+  a.workspace = workspace;
+  a.err_word = err_word;
+  a.num_pages = num_pages > 0 ? num_pages : 1;
+  a.max_pages = max_pages;
+  a.page_size = page_size;
+  a.Bt = Bt;
+  a.gamma = gamma;
+  a.Hq = Hq;
+  a.Hkv = Hkv;
+  a.scale = scale;
+  if (num_pages == 0) {
+    a.max_pages = 0;
+    a.num_pages = 0;
+  }
+  cudaError_t e = simsd::launch_attention_tc(a, plan, enc, s);
+  return e == cudaSuccess ? SIMSD_OK : cuda_fail(e, "attention_tc launch");
+}
+
 }  // namespace
+
+namespace simsd {
+
+RopeTable make_rope_table(double theta, int d) {
+  RopeTable t{};
+  for (int i = 0; i < d / 2 && i < 64; ++i) {
+    const double f = std::pow(theta, -2.0 * i / d);
+    const float hi = static_cast<float>(f);
+    t.f[i] = make_float2(hi, static_cast<float>(f - static_cast<double>(hi)));
+  }
+  return t;
+}
+
+}  // namespace simsd
 
 extern "C" {
 
@@ -122,176 +253,23 @@ size_t simsd_verify_workspace_bytes(int dtype, int Bt, int gamma, int Hq, int Hk
 int simsd_verify_attention(int dtype, const void* q, const void* k_new, const void* v_new, const void* k_cache,
                            const void* v_cache, int num_pages, const int32_t* block_table, int max_pages,
                            int page_size, const int32_t* prefix_len, const int32_t* tau, const uint8_t* section,
-                           const int32_t* rope_pos, int Bt, int gamma, int Hq, int Hkv, int d, float softmax_scale,
-                           void* out, void* workspace, size_t workspace_bytes, int32_t* err_word, void* stream) {
-  if (Bt < 0) return arg_fail("Bt < 0");
-  if (gamma < 1 || gamma > 32) return arg_fail("gamma must be in [1, 32]");
-  if (Hq <= 0 || Hkv <= 0 || Hq % Hkv != 0) return arg_fail("Hq must be a positive multiple of Hkv");
-  if (num_pages < 0 || max_pages < 0) return arg_fail("negative page count");
-  if (page_size < 8 || !((page_size % 64 == 0) || (64 % page_size == 0)))
-    return unsupported("page_size must be a multiple of 64 or a divisor of 64 (>= 8)");
-  if (rope_pos) return unsupported("rope_pos must be NULL (inputs arrive rotated)");
-  if (!(softmax_scale >= 0.f) || std::isinf(softmax_scale)) return arg_fail("softmax_scale");
-  if (Bt == 0) return SIMSD_OK;
-  if (!q || !k_new || !v_new || !prefix_len || !tau || !section || !out) return arg_fail("null pointer");
-  if (max_pages > 0 && (!block_table || !k_cache || !v_cache || num_pages == 0))
-    return arg_fail("null cache or block table");
-  if (!aligned16(q) || !aligned16(k_new) || !aligned16(v_new) || !aligned16(out) ||
-      (k_cache && !aligned16(k_cache)) || (v_cache && !aligned16(v_cache)))
-    return arg_fail("tensor pointers must be 16-byte aligned");
-  DeviceInfo info;
-  int rc = require_sm103(&info);
-  if (rc != SIMSD_OK) return rc;
-  const float scale = softmax_scale > 0.f ? softmax_scale : 1.0f / std::sqrt(static_cast<float>(d));
-  cudaStream_t s = as_stream(stream);
-  if (dtype == SIMSD_F32) {
-    if (d != 64 && d != 128) return unsupported("fp32 path needs d in {64, 128}");
-    simsd::AttnF32Args a{};
-    a.q = static_cast<const float*>(q);
-    a.k_new = static_cast<const float*>(k_new);
-    a.v_new = static_cast<const float*>(v_new);
-    a.k_cache = static_cast<const float*>(k_cache);
-    a.v_cache = static_cast<const float*>(v_cache);
-    a.block_table = block_table;
-    a.prefix_len = prefix_len;
-    a.tau = tau;
-    a.section = section;
-    a.out = static_cast<float*>(out);
-    a.err_word = err_word;
-    a.num_pages = num_pages;
-    a.max_pages = max_pages;
-    a.page_size = page_size;
-    a.Bt = Bt;
-    a.gamma = gamma;
-    a.Hq = Hq;
-    a.Hkv = Hkv;
-    a.d = d;
-    a.scale = scale;
-    cudaError_t e = simsd::launch_attention_f32(a, s);
-    return e == cudaSuccess ? SIMSD_OK : cuda_fail(e, "attention_f32 launch");
-  }
-  if (dtype != SIMSD_BF16) return unsupported("dtype");
-  if (d != 128) return unsupported("bf16 path needs d = 128");
-  if (static_cast<long long>(num_pages) * Hkv * page_size >= (1ll << 31))
-    return unsupported("page pool too large for 32-bit TMA row coordinates");
-  if (static_cast<long long>(Bt) * 2 * gamma * Hq >= (1ll << 31)) return unsupported("too many query rows");
-  simsd::AttnTcPlan plan;
-  if (!simsd::plan_attention_tc(Bt, gamma, Hq, Hkv, max_pages, page_size, info.num_sms, &plan))
-    return unsupported("query rows per KV head: need 2*gamma*Hq/Hkv <= 128 or 128 % (Hq/Hkv) == 0");
-  if (plan.ws_bytes > 0 && (!workspace || workspace_bytes < plan.ws_bytes || !aligned16(workspace)))
-    return arg_fail("workspace smaller than simsd_verify_workspace_bytes()");
-  simsd::EncodeTiledFn enc = encoder();
-  if (!enc) return cuda_fail(cudaErrorNotSupported, "cuTensorMapEncodeTiled entry point");
-  simsd::AttnTcArgs a{};
-  a.q = q;
-  a.k_new = k_new;
-  a.v_new = v_new;
-  // a pool with no pages is still described by a valid (never read) map
-  a.k_cache = k_cache ? k_cache : q;
-  a.v_cache = v_cache ? v_cache : q;
-  a.block_table = block_table;
-  a.prefix_len = prefix_len;
-  a.tau = tau;
-  a.section = section;
-  a.out = out;
-  a.workspace = workspace;
-  a.err_word = err_word;
-  a.num_pages = num_pages > 0 ? num_pages : 1;
-  a.max_pages = max_pages;
-  a.page_size = page_size;
-  a.Bt = Bt;
-  a.gamma = gamma;
-  a.Hq = Hq;
-  a.Hkv = Hkv;
-  a.scale = scale;
-  if (num_pages == 0) {
-    a.max_pages = 0;
-    a.num_pages = 0;
-  }
-  cudaError_t e = simsd::launch_attention_tc(a, plan, enc, s);
-  return e == cudaSuccess ? SIMSD_OK : cuda_fail(e, "attention_tc launch");
+                           const int32_t* rope_pos, float rope_theta, int Bt, int gamma, int Hq, int Hkv, int d,
+                           float softmax_scale, void* out, void* workspace, size_t workspace_bytes,
+                           int32_t* err_word, void* stream) {
+  return verify_attention_impl(dtype, q, k_new, v_new, k_cache, v_cache, num_pages, block_table, max_pages,
+                               page_size, prefix_len, tau, section, rope_pos, rope_theta, Bt, gamma, Hq, Hkv, d,
+                               softmax_scale, out, workspace, workspace_bytes, false, err_word, stream);
 }
 
 int simsd_verify_attention_noalloc(int dtype, const void* q, const void* k_new, const void* v_new,
                                    const void* k_cache, const void* v_cache, int num_pages,
                                    const int32_t* block_table, int max_pages, int page_size,
                                    const int32_t* prefix_len, const int32_t* tau, const uint8_t* section,
-                                   const int32_t* rope_pos, int Bt, int gamma, int Hq, int Hkv, int d,
-                                   float softmax_scale, void* out, int32_t* err_word, void* stream) {
-  if (Bt < 0) return arg_fail("Bt < 0");
-  if (gamma < 1 || gamma > 32) return arg_fail("gamma must be in [1, 32]");
-  if (Hq <= 0 || Hkv <= 0 || Hq % Hkv != 0) return arg_fail("Hq must be a positive multiple of Hkv");
-  if (num_pages < 0 || max_pages < 0) return arg_fail("negative page count");
-  if (page_size < 8 || !((page_size % 64 == 0) || (64 % page_size == 0)))
-    return unsupported("page_size must be a multiple of 64 or a divisor of 64 (>= 8)");
-  if (rope_pos) return unsupported("rope_pos must be NULL (inputs arrive rotated)");
-  if (!(softmax_scale >= 0.f) || std::isinf(softmax_scale)) return arg_fail("softmax_scale");
-  if (Bt == 0) return SIMSD_OK;
-  if (!q || !k_new || !v_new || !prefix_len || !tau || !section || !out) return arg_fail("null pointer");
-  if (max_pages > 0 && (!block_table || !k_cache || !v_cache || num_pages == 0))
-    return arg_fail("null cache or block table");
-  if (!aligned16(q) || !aligned16(k_new) || !aligned16(v_new) || !aligned16(out) ||
-      (k_cache && !aligned16(k_cache)) || (v_cache && !aligned16(v_cache)))
-    return arg_fail("tensor pointers must be 16-byte aligned");
-  DeviceInfo info;
-  int rc = require_sm103(&info);
-  if (rc != SIMSD_OK) return rc;
-  if (dtype != SIMSD_BF16 && dtype != SIMSD_F32) return unsupported("dtype");
-  if (dtype == SIMSD_F32) {
-    // the fp32 path uses no scratch: same launch as simsd_verify_attention
-    return simsd_verify_attention(dtype, q, k_new, v_new, k_cache, v_cache, num_pages, block_table, max_pages,
-                                  page_size, prefix_len, tau, section, rope_pos, Bt, gamma, Hq, Hkv, d,
-                                  softmax_scale, out, nullptr, 0, err_word, stream);
-  }
-  if (d != 128) return unsupported("bf16 path needs d = 128");
-  if (static_cast<long long>(num_pages) * Hkv * page_size >= (1ll << 31))
-    return unsupported("page pool too large for 32-bit TMA row coordinates");
-  if (static_cast<long long>(Bt) * 2 * gamma * Hq >= (1ll << 31)) return unsupported("too many query rows");
-  simsd::AttnTcPlan plan;
-  if (!simsd::plan_attention_tc(Bt, gamma, Hq, Hkv, max_pages, page_size, info.num_sms, &plan))
-    return unsupported("query rows per KV head: need 2*gamma*Hq/Hkv <= 128 or 128 % (Hq/Hkv) == 0");
-  if (plan.ws_bytes > simsd::noalloc_scratch_capacity()) {
-    std::snprintf(g_last_error, sizeof(g_last_error),
-                  "unsupported: these sizes need %zu bytes of scratch, more than the %zu-byte static array; "
-                  "use simsd_verify_attention with a caller workspace",
-                  plan.ws_bytes, simsd::noalloc_scratch_capacity());
-    return SIMSD_ERR_UNSUPPORTED;
-  }
-  void* scratch = nullptr;
-  if (plan.ws_bytes > 0) {
-    cudaError_t e = simsd::noalloc_scratch_pointer(&scratch);
-    if (e != cudaSuccess) return cuda_fail(e, "cudaGetSymbolAddress of the static scratch");
-  }
-  simsd::EncodeTiledFn enc = encoder();
-  if (!enc) return cuda_fail(cudaErrorNotSupported, "cuTensorMapEncodeTiled entry point");
-  const float scale = softmax_scale > 0.f ? softmax_scale : 1.0f / std::sqrt(static_cast<float>(d));
-  simsd::AttnTcArgs a{};
-  a.q = q;
-  a.k_new = k_new;
-  a.v_new = v_new;
-  a.k_cache = k_cache ? k_cache : q;
-  a.v_cache = v_cache ? v_cache : q;
-  a.block_table = block_table;
-  a.prefix_len = prefix_len;
-  a.tau = tau;
-  a.section = section;
-  a.out = out;
-  a.workspace = scratch;
-  a.err_word = err_word;
-  a.num_pages = num_pages > 0 ? num_pages : 1;
-  a.max_pages = max_pages;
-  a.page_size = page_size;
-  a.Bt = Bt;
-  a.gamma = gamma;
-  a.Hq = Hq;
-  a.Hkv = Hkv;
-  a.scale = scale;
-  if (num_pages == 0) {
-    a.max_pages = 0;
-    a.num_pages = 0;
-  }
-  cudaError_t e = simsd::launch_attention_tc(a, plan, enc, as_stream(stream));
-  return e == cudaSuccess ? SIMSD_OK : cuda_fail(e, "attention_tc launch (static scratch)");
+                                   const int32_t* rope_pos, float rope_theta, int Bt, int gamma, int Hq, int Hkv,
+                                   int d, float softmax_scale, void* out, int32_t* err_word, void* stream) {
+  return verify_attention_impl(dtype, q, k_new, v_new, k_cache, v_cache, num_pages, block_table, max_pages,
+                               page_size, prefix_len, tau, section, rope_pos, rope_theta, Bt, gamma, Hq, Hkv, d,
+                               softmax_scale, out, nullptr, 0, true, err_word, stream);
 }
 
 int simsd_accept(const float* logits, const int32_t* draft, int Bt, int gamma, int vocab, int32_t* accepted_len,
@@ -310,15 +288,18 @@ int simsd_accept(const float* logits, const int32_t* draft, int Bt, int gamma, i
 }
 
 int simsd_kv_commit(int dtype, const void* k_new, const void* v_new, int L, const int32_t* tau,
-                    const uint8_t* section, const int32_t* accepted_len, void* k_cache, void* v_cache, int num_pages,
-                    const int32_t* block_table, int max_pages, int page_size, int32_t* prefix_len, int Bt, int gamma,
-                    int Hkv, int d, int32_t* err_word, void* stream) {
+                    const uint8_t* section, const int32_t* rope_pos, float rope_theta, const int32_t* accepted_len,
+                    void* k_cache, void* v_cache, int num_pages, const int32_t* block_table, int max_pages,
+                    int page_size, int32_t* prefix_len, int Bt, int gamma, int Hkv, int d, int32_t* err_word,
+                    void* stream) {
   if (Bt < 0 || L < 0) return arg_fail("Bt < 0 or L < 0");
   if (gamma < 1 || gamma > 32) return arg_fail("gamma must be in [1, 32]");
   if (Hkv <= 0 || page_size <= 0 || num_pages < 0 || max_pages < 0) return arg_fail("sizes");
   if (dtype != SIMSD_F32 && dtype != SIMSD_BF16) return unsupported("dtype");
   const int eb = dtype == SIMSD_F32 ? 4 : 2;
   if (d <= 0 || (d * eb) % 16 != 0) return arg_fail("d * element size must be a multiple of 16 bytes");
+  if (rope_pos && (!(rope_theta > 0.f) || std::isinf(rope_theta) || d > 128 || d % 2 != 0))
+    return arg_fail("rope needs a positive finite rope_theta and an even d <= 128");
   if (Bt == 0) return SIMSD_OK;
   if (!tau || !section || !accepted_len || !prefix_len) return arg_fail("null pointer");
   if (L > 0 && (!k_new || !v_new || !k_cache || !v_cache || !block_table)) return arg_fail("null pointer");
@@ -328,9 +309,10 @@ int simsd_kv_commit(int dtype, const void* k_new, const void* v_new, int L, cons
   DeviceInfo info;
   int rc = require_sm103(&info);
   if (rc != SIMSD_OK) return rc;
+  const simsd::RopeTable table = rope_pos ? simsd::make_rope_table(rope_theta, d) : simsd::RopeTable{};
   cudaError_t e = simsd::launch_kv_commit(eb, k_new, v_new, L, tau, section, accepted_len, k_cache, v_cache,
                                           num_pages, block_table, max_pages, page_size, prefix_len, Bt, gamma, Hkv,
-                                          d, err_word, as_stream(stream));
+                                          d, rope_pos, table, err_word, as_stream(stream));
   return e == cudaSuccess ? SIMSD_OK : cuda_fail(e, "kv_commit launch");
 }
 

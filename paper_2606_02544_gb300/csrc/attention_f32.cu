@@ -3,7 +3,9 @@
 // of 32: the paged prefix rows, then the new slots admitted by Eq. (1);
 // each lane scores one key of the chunk, the warp folds the chunk into a
 // running max / sum (online softmax) and accumulates V with lanes over the
-// head dimension.
+// head dimension.  When the inputs are not rotated yet (Sec. 3.1 RoPE copy),
+// the query row is rotated once in shared memory and each new key on the
+// fly while it is scored; cached keys are stored rotated.
 #include <cuda_runtime.h>
 
 #include "common.cuh"
@@ -14,7 +16,7 @@ namespace simsd {
 constexpr int kF32Warps = 4;
 
 template <int DPL>  // head-dim elements per lane (d = 32 * DPL)
-__global__ void __launch_bounds__(kF32Warps * 32) attention_f32_kernel(AttnF32Args a) {
+__global__ void __launch_bounds__(kF32Warps * 32) attention_f32_kernel(const __grid_constant__ AttnF32Args a) {
   __shared__ __align__(16) float q_s[kF32Warps][32 * DPL];
   const int lane = threadIdx.x & 31, wib = threadIdx.x >> 5;
   const long long row = (static_cast<long long>(blockIdx.x) * blockDim.x + threadIdx.x) >> 5;
@@ -53,6 +55,16 @@ __global__ void __launch_bounds__(kF32Warps * 32) attention_f32_kernel(AttnF32Ar
 #pragma unroll
   for (int c = 0; c < DPL; ++c) q_s[wib][lane + 32 * c] = a.q[row * d + lane + 32 * c];
   __syncwarp();
+  if (a.rope_pos) {
+    const int pos = a.rope_pos[static_cast<size_t>(b) * S + s];
+#pragma unroll
+    for (int i = lane; i < d / 2; i += 32) {
+      float sn, cs;
+      rope_sincos(pos, a.rope.f[i], &sn, &cs);
+      rope_pair(q_s[wib][i], q_s[wib][i + d / 2], sn, cs);
+    }
+    __syncwarp();
+  }
   float acc[DPL];
 #pragma unroll
   for (int c = 0; c < DPL; ++c) acc[c] = 0.f;
@@ -83,14 +95,35 @@ __global__ void __launch_bounds__(kF32Warps * 32) attention_f32_kernel(AttnF32Ar
       float dot = 0.f;
       const float4* k4 = reinterpret_cast<const float4*>(kr);
       const float4* q4 = reinterpret_cast<const float4*>(q_s[wib]);
+      if (!from_cache && a.rope_pos) {
+        // new key: rotate each (i, i + d/2) pair at its slot's position
+        const int pos = a.rope_pos[static_cast<size_t>(b) * S + (j - n)];
+        constexpr int hc = d / 8;  // float4 chunks per half
+#pragma unroll 2
+        for (int c = 0; c < hc; ++c) {
+          const float4 kl = __ldg(k4 + c), kh = __ldg(k4 + c + hc);
+          const float4 ql = q4[c], qh = q4[c + hc];
+          float kx[4] = {kl.x, kl.y, kl.z, kl.w}, ky[4] = {kh.x, kh.y, kh.z, kh.w};
+          const float qx[4] = {ql.x, ql.y, ql.z, ql.w}, qy[4] = {qh.x, qh.y, qh.z, qh.w};
+#pragma unroll
+          for (int e = 0; e < 4; ++e) {
+            float sn, cs;
+            rope_sincos(pos, a.rope.f[4 * c + e], &sn, &cs);
+            rope_pair(kx[e], ky[e], sn, cs);
+            dot = fmaf(qx[e], kx[e], dot);
+            dot = fmaf(qy[e], ky[e], dot);
+          }
+        }
+      } else {
 #pragma unroll 8
-      for (int c = 0; c < d / 4; ++c) {
-        const float4 kv = __ldg(k4 + c);
-        const float4 qv = q4[c];
-        dot = fmaf(qv.x, kv.x, dot);
-        dot = fmaf(qv.y, kv.y, dot);
-        dot = fmaf(qv.z, kv.z, dot);
-        dot = fmaf(qv.w, kv.w, dot);
+        for (int c = 0; c < d / 4; ++c) {
+          const float4 kv = __ldg(k4 + c);
+          const float4 qv = q4[c];
+          dot = fmaf(qv.x, kv.x, dot);
+          dot = fmaf(qv.y, kv.y, dot);
+          dot = fmaf(qv.z, kv.z, dot);
+          dot = fmaf(qv.w, kv.w, dot);
+        }
       }
       sc = dot * a.scale;
     }

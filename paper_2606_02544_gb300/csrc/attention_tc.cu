@@ -5,9 +5,12 @@
 // Work unit: (sequence b, KV head, row block, prefix split).  The query rows
 // of one unit are the g = Hq/Hkv heads x 2*gamma slots that share the KV
 // head ("GQA packing"), up to 128 rows, so QK^T and PV are M = 128 MMAs.
-// Keys stream in tiles of 64: first the cached prefix pages (read through
-// the page table with TMA), then one tile with the 2*gamma new slots, whose
-// Eq. (1) visibility is evaluated on the fly from (section, tau).
+// Keys stream in tiles of 64: first one tile with the 2*gamma new slots, whose
+// Eq. (1) visibility is evaluated on the fly from (section, tau), then the
+// cached prefix pages (read through the page table with TMA).  When the
+// inputs are not rotated yet (Sec. 3.1 RoPE copy), the softmax warps rotate
+// Q while moving it into TMEM and rotate the new keys in shared memory before
+// the first S is computed; cached keys are stored rotated.
 //
 // Two CTAs share each SM (96 KB of shared memory, 256 TMEM columns and 192
 // threads apiece), so one CTA's set-up, first loads and epilogue overlap the
@@ -71,12 +74,14 @@ struct TcParams {
   const int32_t* prefix_len;
   const int32_t* tau;
   const uint8_t* section;
+  const int32_t* rope_pos;  // [Bt][2*gamma] or null (inputs rotated already)
   __nv_bfloat16* out;
   float* ws;  // partials: O [units*nsplit][rows_blk][128] then (m, l) [units*nsplit][rows_blk][2]
   int32_t* err_word;
   int max_pages, page_size, num_pages;
   int Bt, gamma, S, Hq, Hkv, g, rb, rows_blk, s_blk, nsplit;
   float scale_log2;
+  RopeTable rope;
 };
 
 struct alignas(1024) Smem {
@@ -196,7 +201,7 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm)
 
   const bool seq_bad = sm.seq_bad != 0;
   const int T = seq_bad ? 0 : (n + kTile - 1) / kTile;  // prefix tiles
-  const int T_all = seq_bad ? 0 : T + 1;                 // + the tile of new slots
+  const int T_all = seq_bad ? 0 : T + 1;                 // tile 0: new slots, tiles 1..T: prefix
   const int t0 = static_cast<int>(static_cast<long long>(split) * T_all / p.nsplit);
   const int t1 = static_cast<int>(static_cast<long long>(split + 1) * T_all / p.nsplit);
   const int ntiles = t1 - t0;
@@ -228,8 +233,8 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm)
         const uint32_t bk = smem_u32(&sm.bar_k[st]), bv = smem_u32(&sm.bar_v[st]);
         const uint32_t k0 = smem_u32(sm.ring[st]), k1 = k0 + kHalfBytes;
         const uint32_t v0 = k0 + 2 * kHalfBytes, v1 = k0 + 3 * kHalfBytes;
-        if (t < T) {
-          const int key0 = t * kTile;
+        if (t > 0) {
+          const int key0 = (t - 1) * kTile;
           const int valid = min(kTile, n - key0);
           if (P >= kTile) {
             const int pi = key0 / P;
@@ -346,7 +351,33 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm)
     // ---- Q: shared memory (ring slot 0) -> TMEM columns [0, 64)
     if (ntiles > 0) {
       ok = mbar_wait_warp(smem_u32(&sm.bar_k[0]), 0, abort_flag);
-      if (ok) {
+      if (ok && p.rope_pos) {
+        // rotate this row's query at its slot's position on the way
+        const int pos = p.rope_pos[static_cast<size_t>(b) * p.S + (s < p.S ? s : 0)];
+        const uint8_t* h0 = sm.ring[0];
+        const uint8_t* h1 = sm.ring[0] + 2 * kHalfBytes;
+        uint32_t q0r[32], q1r[32];
+#pragma unroll
+        for (int c = 0; c < 8; ++c) {
+          const uint4 va = ld_sw128_chunk(h0, row, c), vb = ld_sw128_chunk(h1, row, c);
+          const uint32_t wa[4] = {va.x, va.y, va.z, va.w}, wb[4] = {vb.x, vb.y, vb.z, vb.w};
+#pragma unroll
+          for (int w = 0; w < 4; ++w) {
+            float x0 = __uint_as_float(wa[w] << 16), x1 = __uint_as_float(wa[w] & 0xffff0000u);
+            float y0 = __uint_as_float(wb[w] << 16), y1 = __uint_as_float(wb[w] & 0xffff0000u);
+            float sn, cs;
+            rope_sincos(pos, p.rope.f[8 * c + 2 * w], &sn, &cs);
+            rope_pair(x0, y0, sn, cs);
+            rope_sincos(pos, p.rope.f[8 * c + 2 * w + 1], &sn, &cs);
+            rope_pair(x1, y1, sn, cs);
+            q0r[4 * c + w] = pack_bf16x2(x0, x1);
+            q1r[4 * c + w] = pack_bf16x2(y0, y1);
+          }
+        }
+        tmem_st32(lane_tmem + kColQ, q0r);
+        tmem_st32(lane_tmem + kColQ + 32, q1r);
+        tmem_wait_st();
+      } else if (ok) {
 #pragma unroll 1
         for (int h = 0; h < 2; ++h) {
           const uint8_t* half = sm.ring[0] + h * 2 * kHalfBytes;
@@ -362,6 +393,39 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm)
           tmem_st32(lane_tmem + kColQ + 32 * h, qr);
         }
         tmem_wait_st();
+      }
+      if (ok && p.rope_pos && t0 == 0) {
+        // the new keys (ring item 1, the unit's first tile) are rotated in
+        // place before the first S = Q K^T reads them
+        constexpr int st1 = 1 % kStages;
+        ok = mbar_wait_warp(smem_u32(&sm.bar_k[st1]), 0, abort_flag);
+        if (ok) {
+          uint8_t* h0 = sm.ring[st1];
+          uint8_t* h1 = sm.ring[st1] + kHalfBytes;
+          for (int task = tid; task < p.S * 8; task += 128) {
+            const int r = task >> 3, c = task & 7;
+            const int pos = p.rope_pos[static_cast<size_t>(b) * p.S + r];
+            uint4* pa = reinterpret_cast<uint4*>(h0 + r * 128 + ((c ^ (r & 7)) << 4));
+            uint4* pb = reinterpret_cast<uint4*>(h1 + r * 128 + ((c ^ (r & 7)) << 4));
+            const uint4 va = *pa, vb = *pb;
+            uint32_t wa[4] = {va.x, va.y, va.z, va.w}, wb[4] = {vb.x, vb.y, vb.z, vb.w};
+#pragma unroll
+            for (int w = 0; w < 4; ++w) {
+              float x0 = __uint_as_float(wa[w] << 16), x1 = __uint_as_float(wa[w] & 0xffff0000u);
+              float y0 = __uint_as_float(wb[w] << 16), y1 = __uint_as_float(wb[w] & 0xffff0000u);
+              float sn, cs;
+              rope_sincos(pos, p.rope.f[8 * c + 2 * w], &sn, &cs);
+              rope_pair(x0, y0, sn, cs);
+              rope_sincos(pos, p.rope.f[8 * c + 2 * w + 1], &sn, &cs);
+              rope_pair(x1, y1, sn, cs);
+              wa[w] = pack_bf16x2(x0, x1);
+              wb[w] = pack_bf16x2(y0, y1);
+            }
+            *pa = make_uint4(wa[0], wa[1], wa[2], wa[3]);
+            *pb = make_uint4(wb[0], wb[1], wb[2], wb[3]);
+          }
+          fence_proxy_async_smem();
+        }
       }
       tc_fence_before();
       asm volatile("bar.sync 1, 128;" ::: "memory");
@@ -384,8 +448,8 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm)
       tmem_ld32(lane_tmem + kColS + 32, sb);
       tmem_wait_ld();
 
-      const bool is_new = (t == T);
-      const int valid = is_new ? p.S : min(kTile, n - t * kTile);
+      const bool is_new = (t == 0);
+      const int valid = is_new ? p.S : min(kTile, n - (t - 1) * kTile);
       float x[kTile];
 #pragma unroll
       for (int c = 0; c < kTile; ++c) x[c] = __uint_as_float(c < 32 ? sa[c] : sb[c - 32]);
@@ -680,6 +744,8 @@ cudaError_t launch_attention_tc(const AttnTcArgs& a, const AttnTcPlan& pl, Encod
   p.prefix_len = a.prefix_len;
   p.tau = a.tau;
   p.section = a.section;
+  p.rope_pos = a.rope_pos;
+  p.rope = a.rope;
   p.out = static_cast<__nv_bfloat16*>(a.out);
   p.ws = static_cast<float*>(a.workspace);
   p.err_word = a.err_word;

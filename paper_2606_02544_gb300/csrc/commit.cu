@@ -1,7 +1,10 @@
 // commit.cu -- append the accepted drafts' K/V to the paged cache (Sec. 3.2:
 // the accepted prefix is committed to the block; Sec. 3.3: later steps reuse
 // the cached K/V).  Row r < a_b of sequence b takes the data-slot K/V whose
-// temporal label is r+1 and lands in cache row n_b + r.
+// temporal label is r+1 and lands in cache row n_b + r.  When the new keys
+// are not rotated yet, each committed key is rotated at its slot's RoPE
+// position (Sec. 3.1) so that the cache holds rotated keys.
+#include <cuda_bf16.h>
 #include <cuda_runtime.h>
 
 #include "common.cuh"
@@ -12,13 +15,19 @@ namespace simsd {
 constexpr int kCommitWarps = 8;
 
 // One warp per (layer, sequence, accepted row, KV head); each lane moves
-// 16-byte chunks of the K row and the V row.
+// 16-byte chunks of the K row and the V row (or, with RoPE, rotates pairs
+// of the K row).
+struct CommitRope {
+  const int32_t* pos;  // [Bt][2*gamma] or null
+  RopeTable table;
+};
+
 __global__ void __launch_bounds__(kCommitWarps * 32) kv_commit_copy_kernel(
     const uint8_t* __restrict__ k_new, const uint8_t* __restrict__ v_new, int L, const int32_t* __restrict__ tau,
     const uint8_t* __restrict__ section, const int32_t* __restrict__ accepted_len, uint8_t* __restrict__ k_cache,
     uint8_t* __restrict__ v_cache, int num_pages, const int32_t* __restrict__ block_table, int max_pages,
     int page_size, const int32_t* __restrict__ prefix_len, int Bt, int gamma, int Hkv, int row_bytes,
-    int32_t* err_word) {
+    int elem_bytes, const __grid_constant__ CommitRope rope, int32_t* err_word) {
   const long long wid = (static_cast<long long>(blockIdx.x) * blockDim.x + threadIdx.x) >> 5;
   const int lane = threadIdx.x & 31;
   const long long total = static_cast<long long>(L) * Bt * gamma * Hkv;
@@ -59,9 +68,34 @@ __global__ void __launch_bounds__(kCommitWarps * 32) kv_commit_copy_kernel(
   uint4* kd = reinterpret_cast<uint4*>(k_cache + d_row * row_bytes);
   uint4* vd = reinterpret_cast<uint4*>(v_cache + d_row * row_bytes);
   const int chunks = row_bytes >> 4;
-  for (int c = lane; c < chunks; c += 32) {
-    kd[c] = ks[c];
-    vd[c] = vs[c];
+  if (rope.pos) {
+    const int pos = rope.pos[static_cast<size_t>(b) * S + src];
+    const int d = row_bytes / elem_bytes, half = d / 2;
+    for (int i = lane; i < half; i += 32) {
+      float sn, cs;
+      rope_sincos(pos, rope.table.f[i], &sn, &cs);
+      if (elem_bytes == 4) {
+        const float* kf = reinterpret_cast<const float*>(ks);
+        float* kdf = reinterpret_cast<float*>(kd);
+        float x = kf[i], y = kf[i + half];
+        rope_pair(x, y, sn, cs);
+        kdf[i] = x;
+        kdf[i + half] = y;
+      } else {
+        const __nv_bfloat16* kb = reinterpret_cast<const __nv_bfloat16*>(ks);
+        __nv_bfloat16* kdb = reinterpret_cast<__nv_bfloat16*>(kd);
+        float x = __bfloat162float(kb[i]), y = __bfloat162float(kb[i + half]);
+        rope_pair(x, y, sn, cs);
+        kdb[i] = __float2bfloat16_rn(x);
+        kdb[i + half] = __float2bfloat16_rn(y);
+      }
+    }
+    for (int c = lane; c < chunks; c += 32) vd[c] = vs[c];
+  } else {
+    for (int c = lane; c < chunks; c += 32) {
+      kd[c] = ks[c];
+      vd[c] = vs[c];
+    }
   }
 }
 
@@ -86,15 +120,16 @@ __global__ void kv_commit_advance_kernel(const int32_t* __restrict__ accepted_le
 cudaError_t launch_kv_commit(int elem_bytes, const void* k_new, const void* v_new, int L, const int32_t* tau,
                              const uint8_t* section, const int32_t* accepted_len, void* k_cache, void* v_cache,
                              int num_pages, const int32_t* block_table, int max_pages, int page_size,
-                             int32_t* prefix_len, int Bt, int gamma, int Hkv, int d, int32_t* err_word,
-                             cudaStream_t stream) {
+                             int32_t* prefix_len, int Bt, int gamma, int Hkv, int d, const int32_t* rope_pos,
+                             const RopeTable& rope_table, int32_t* err_word, cudaStream_t stream) {
   const long long warps = static_cast<long long>(L) * Bt * gamma * Hkv;
   const long long blocks = (warps + kCommitWarps - 1) / kCommitWarps;
   if (blocks > 0) {
     kv_commit_copy_kernel<<<static_cast<unsigned>(blocks), kCommitWarps * 32, 0, stream>>>(
         static_cast<const uint8_t*>(k_new), static_cast<const uint8_t*>(v_new), L, tau, section, accepted_len,
         static_cast<uint8_t*>(k_cache), static_cast<uint8_t*>(v_cache), num_pages, block_table, max_pages,
-        page_size, prefix_len, Bt, gamma, Hkv, d * elem_bytes, err_word);
+        page_size, prefix_len, Bt, gamma, Hkv, d * elem_bytes, elem_bytes, CommitRope{rope_pos, rope_table},
+        err_word);
     cudaError_t e = cudaGetLastError();
     if (e != cudaSuccess) return e;
   }

@@ -1,5 +1,7 @@
 // common.cuh -- constants and small device helpers shared by the kernels.
 #pragma once
+#include <cuda_runtime.h>
+
 #include <cstdint>
 
 #include "../../include/simsd.h"
@@ -23,6 +25,39 @@ __host__ __device__ __forceinline__ bool temporal_visible(uint8_t si, int ti, ui
   if (si == kSectPad || sj == kSectPad) return false;
   const int bias = (si == kSectData) ? 1 : 0;
   return (sj == kSectData) == (tj < ti + bias);
+}
+
+// ---- rotary position embedding (Su et al., RoFormer), rotate-half layout:
+// for i < d/2 the pair (x_i, x_{i+d/2}) turns by the angle pos * theta^(-2i/d).
+// The per-pair frequencies theta^(-2i/d) come in a RopeTable (kernels.h).
+
+// sin and cos of pos * f for 0 <= pos < 2^24.  The product is kept in
+// float-float (the rounding error of p * hi comes back exactly from an FMA)
+// and reduced to [-pi, pi] by Cody-Waite subtraction of k * 2pi, with 2pi
+// split into three floats of which the first has 8 significant bits, so the
+// first subtraction is exact; the reduced angle is good to ~2e-7 rad up to
+// pos = 2^20.
+__device__ __forceinline__ void rope_sincos(int pos, float2 f, float* sn, float* cs) {
+  constexpr float kTwoPiA = 6.28125f;
+  constexpr float kTwoPiB = 1.9353071693331003e-03f;
+  constexpr float kTwoPiC = 1.0253131677018246e-11f;
+  constexpr float kInvTwoPi = 0.15915493667125702f;
+  const float p = static_cast<float>(pos);
+  const float a = p * f.x;
+  const float b = fmaf(p, f.y, fmaf(p, f.x, -a));
+  const float k = rintf(a * kInvTwoPi);
+  float r = fmaf(-k, kTwoPiA, a);
+  r = fmaf(-k, kTwoPiB, r);
+  r = fmaf(-k, kTwoPiC, r);
+  sincosf(r + b, sn, cs);
+}
+
+// Rotates one pair in place.
+__device__ __forceinline__ void rope_pair(float& x, float& y, float sn, float cs) {
+  const float x2 = x * cs - y * sn;
+  const float y2 = fmaf(x, sn, y * cs);
+  x = x2;
+  y = y2;
 }
 
 }  // namespace simsd

@@ -8,6 +8,13 @@
 
 namespace simsd {
 
+// Rotary embedding frequencies theta^(-2i/d), i < d/2 <= 64, each as an
+// unevaluated sum f.x + f.y of two floats (rounded from double).
+struct RopeTable {
+  float2 f[64];
+};
+RopeTable make_rope_table(double theta, int d);
+
 cudaError_t launch_build_mask(const int32_t* step_map, const int32_t* prefix_len, int Bt, int gamma, int32_t* tau,
                               uint8_t* section, int32_t* rope_pos, uint64_t* mask_bits, int32_t* err_word,
                               cudaStream_t stream);
@@ -19,13 +26,15 @@ cudaError_t launch_accept(const float* logits, const int32_t* draft, int Bt, int
 cudaError_t launch_kv_commit(int elem_bytes, const void* k_new, const void* v_new, int L, const int32_t* tau,
                              const uint8_t* section, const int32_t* accepted_len, void* k_cache, void* v_cache,
                              int num_pages, const int32_t* block_table, int max_pages, int page_size,
-                             int32_t* prefix_len, int Bt, int gamma, int Hkv, int d, int32_t* err_word,
-                             cudaStream_t stream);
+                             int32_t* prefix_len, int Bt, int gamma, int Hkv, int d, const int32_t* rope_pos,
+                             const RopeTable& rope, int32_t* err_word, cudaStream_t stream);
 
 struct AttnF32Args {
   const float *q, *k_new, *v_new, *k_cache, *v_cache;
   const int32_t *block_table, *prefix_len, *tau;
   const uint8_t* section;
+  const int32_t* rope_pos;  // null: inputs rotated already
+  RopeTable rope;
   float* out;
   int32_t* err_word;
   int num_pages, max_pages, page_size, Bt, gamma, Hq, Hkv, d;
@@ -49,6 +58,8 @@ struct AttnTcArgs {
   const void *q, *k_new, *v_new, *k_cache, *v_cache;
   const int32_t *block_table, *prefix_len, *tau;
   const uint8_t* section;
+  const int32_t* rope_pos;  // null: inputs rotated already
+  RopeTable rope;
   void* out;
   void* workspace;
   int32_t* err_word;

@@ -51,12 +51,12 @@ def load_library(path: str = LIB_PATH):
             lib.simsd_build_mask.argtypes = [P, P, I, I, P, P, P, P, P, P]
             lib.simsd_verify_workspace_bytes.argtypes = [I, I, I, I, I, I, I, I]
             lib.simsd_verify_workspace_bytes.restype = Z
-            lib.simsd_verify_attention.argtypes = [I, P, P, P, P, P, I, P, I, I, P, P, P, P, I, I, I, I, I, F, P,
-                                                   P, Z, P, P]
-            lib.simsd_verify_attention_noalloc.argtypes = [I, P, P, P, P, P, I, P, I, I, P, P, P, P, I, I, I, I, I,
-                                                           F, P, P, P]
+            lib.simsd_verify_attention.argtypes = [I, P, P, P, P, P, I, P, I, I, P, P, P, P, F, I, I, I, I, I, F,
+                                                   P, P, Z, P, P]
+            lib.simsd_verify_attention_noalloc.argtypes = [I, P, P, P, P, P, I, P, I, I, P, P, P, P, F, I, I, I, I,
+                                                           I, F, P, P, P]
             lib.simsd_accept.argtypes = [P, P, I, I, I, P, P, P, P, P]
-            lib.simsd_kv_commit.argtypes = [I, P, P, I, P, P, P, P, P, I, P, I, I, P, I, I, I, I, P, P]
+            lib.simsd_kv_commit.argtypes = [I, P, P, I, P, P, P, F, P, P, P, I, P, I, I, P, I, I, I, I, P, P]
             lib.simsd_check_error.argtypes = [P, P, P]
             lib.simsd_last_error.restype = ctypes.c_char_p
             for name in ("simsd_build_mask", "simsd_verify_attention", "simsd_verify_attention_noalloc",
@@ -106,9 +106,11 @@ def simsd_verify_workspace_bytes(dtype_code, Bt, gamma, Hq, Hkv, d, max_pages, p
 
 
 def simsd_verify_attention(q, k_new, v_new, k_cache, v_cache, block_table, prefix_len, tau, section, out,
-                           workspace=None, err_word=None, softmax_scale=0.0, rope_pos=None, stream=None):
+                           workspace=None, err_word=None, softmax_scale=0.0, rope_pos=None, rope_theta=0.0,
+                           stream=None):
     """q/out [Bt][2g][Hq][d]; k_new/v_new [Bt][2g][Hkv][d];
-    k_cache/v_cache [num_pages][Hkv][P][d]; block_table [Bt][max_pages]."""
+    k_cache/v_cache [num_pages][Hkv][P][d]; block_table [Bt][max_pages].
+    rope_pos [Bt][2g] (with rope_theta > 0): q and k_new are rotated first."""
     Bt, S, Hq, d = q.shape
     Hkv = k_new.shape[2]
     num_pages, _, P, _ = k_cache.shape
@@ -116,13 +118,13 @@ def simsd_verify_attention(q, k_new, v_new, k_cache, v_cache, block_table, prefi
     ws_bytes = 0 if workspace is None else workspace.numel() * workspace.element_size()
     rc = load_library().simsd_verify_attention(
         _dtype_code(q), _p(q), _p(k_new), _p(v_new), _p(k_cache), _p(v_cache), num_pages, _p(block_table),
-        max_pages, P, _p(prefix_len), _p(tau), _p(section), _p(rope_pos), Bt, S // 2, Hq, Hkv, d,
-        float(softmax_scale), _p(out), _p(workspace), ws_bytes, _p(err_word), _stream(stream))
+        max_pages, P, _p(prefix_len), _p(tau), _p(section), _p(rope_pos), float(rope_theta), Bt, S // 2, Hq, Hkv,
+        d, float(softmax_scale), _p(out), _p(workspace), ws_bytes, _p(err_word), _stream(stream))
     _check(rc, "simsd_verify_attention")
 
 
 def simsd_verify_attention_noalloc(q, k_new, v_new, k_cache, v_cache, block_table, prefix_len, tau, section, out,
-                                   err_word=None, softmax_scale=0.0, rope_pos=None, stream=None):
+                                   err_word=None, softmax_scale=0.0, rope_pos=None, rope_theta=0.0, stream=None):
     """simsd_verify_attention without a workspace: the library's static
     device scratch is used instead (for callers that cannot allocate)."""
     Bt, S, Hq, d = q.shape
@@ -131,8 +133,8 @@ def simsd_verify_attention_noalloc(q, k_new, v_new, k_cache, v_cache, block_tabl
     max_pages = block_table.shape[1]
     rc = load_library().simsd_verify_attention_noalloc(
         _dtype_code(q), _p(q), _p(k_new), _p(v_new), _p(k_cache), _p(v_cache), num_pages, _p(block_table),
-        max_pages, P, _p(prefix_len), _p(tau), _p(section), _p(rope_pos), Bt, S // 2, Hq, Hkv, d,
-        float(softmax_scale), _p(out), _p(err_word), _stream(stream))
+        max_pages, P, _p(prefix_len), _p(tau), _p(section), _p(rope_pos), float(rope_theta), Bt, S // 2, Hq, Hkv,
+        d, float(softmax_scale), _p(out), _p(err_word), _stream(stream))
     _check(rc, "simsd_verify_attention_noalloc")
 
 
@@ -144,12 +146,14 @@ def simsd_accept(logits, draft, accepted_len, out_tokens, row_argmax=None, err_w
 
 
 def simsd_kv_commit(k_new, v_new, tau, section, accepted_len, k_cache, v_cache, block_table, prefix_len,
-                    err_word=None, stream=None):
-    """k_new/v_new [L][Bt][2g][Hkv][d]; k_cache/v_cache [L][num_pages][Hkv][P][d]."""
+                    err_word=None, rope_pos=None, rope_theta=0.0, stream=None):
+    """k_new/v_new [L][Bt][2g][Hkv][d]; k_cache/v_cache [L][num_pages][Hkv][P][d].
+    rope_pos [Bt][2g] (with rope_theta > 0): committed keys are rotated."""
     L, Bt, S, Hkv, d = k_new.shape
     num_pages, P = k_cache.shape[1], k_cache.shape[3]
     rc = load_library().simsd_kv_commit(
-        _dtype_code(k_new), _p(k_new), _p(v_new), L, _p(tau), _p(section), _p(accepted_len), _p(k_cache),
+        _dtype_code(k_new), _p(k_new), _p(v_new), L, _p(tau), _p(section), _p(rope_pos), float(rope_theta),
+        _p(accepted_len), _p(k_cache),
         _p(v_cache), num_pages, _p(block_table), block_table.shape[1], P, _p(prefix_len), Bt, S // 2, Hkv, d,
         _p(err_word), _stream(stream))
     _check(rc, "simsd_kv_commit")

@@ -2,7 +2,9 @@
 
 A step (Sec. 3.2, one target verification forward per speculative step):
   1. simsd_build_mask      tau / section / RoPE-copy positions (Eq. (1))
-  2. simsd_verify_attention, once per layer (the masked attention)
+  2. simsd_verify_attention, once per layer (the masked attention; with
+     ``rope_theta`` the un-rotated q / k_new are rotated at the RoPE-copy
+     positions inside the kernel, Sec. 3.1)
   3. simsd_accept          greedy longest-prefix acceptance (Eq. (2), T=0)
   4. simsd_kv_commit       append the accepted drafts' K/V, advance n_b
 All four run on one stream and are captured into one CUDA graph, so the
@@ -25,8 +27,9 @@ class VerifyStep:
     prefix, which the restored lengths never read.
     """
 
-    def __init__(self, si: StepInputs, restore_prefix: bool = True):
+    def __init__(self, si: StepInputs, restore_prefix: bool = True, rope_theta: float = 0.0):
         w = si.w
+        self.rope_theta = float(rope_theta)
         dev = si.q.device
         self.si = si
         self.w = w
@@ -60,18 +63,21 @@ class VerifyStep:
             self.n.copy_(self.n_orig, non_blocking=True)
         simsd.simsd_build_mask(si.step_map, self.n, w.gamma, self.tau, self.section, self.rope_pos,
                                err_word=self.err)
+        rope = self.rope_pos if self.rope_theta > 0 else None
         if attn_events is not None:
             attn_events[0].record()
         for l in range(self.L):
             simsd.simsd_verify_attention(si.q[l], si.k_new[l], si.v_new[l], si.k_cache[l], si.v_cache[l],
                                          si.block_table, self.n, self.tau, self.section, self.out[l],
-                                         workspace=self.workspace, err_word=self.err)
+                                         workspace=self.workspace, err_word=self.err, rope_pos=rope,
+                                         rope_theta=self.rope_theta)
         if attn_events is not None:
             attn_events[1].record()
         simsd.simsd_accept(si.logits, si.draft, self.accepted_len, self.out_tokens, self.row_argmax,
                            err_word=self.err)
         simsd.simsd_kv_commit(si.k_new, si.v_new, self.tau, self.section, self.accepted_len, si.k_cache,
-                              si.v_cache, si.block_table, self.n, err_word=self.err)
+                              si.v_cache, si.block_table, self.n, err_word=self.err, rope_pos=rope,
+                              rope_theta=self.rope_theta)
 
     def launches_per_step(self) -> int:
         """Kernels of this library launched by one step."""

@@ -27,7 +27,7 @@ def gpu_mask(si, mask_bits=True):
     return tau, sect, rope, bits, err
 
 
-def gpu_attention(si, layer=0, mask=None, err=None):
+def gpu_attention(si, layer=0, mask=None, err=None, rope_pos=None, rope_theta=0.0):
     w = si.w
     if mask is None:
         tau, sect, _, _, merr = gpu_mask(si, mask_bits=False)
@@ -42,21 +42,25 @@ def gpu_attention(si, layer=0, mask=None, err=None):
     e = torch.zeros(1, dtype=torch.int32, device=si.q.device) if err is None else err
     simsd.simsd_verify_attention(si.q[layer], si.k_new[layer], si.v_new[layer], si.k_cache[layer],
                                  si.v_cache[layer], si.block_table, si.prefix_len, tau, sect, out,
-                                 workspace=work, err_word=e)
+                                 workspace=work, err_word=e, rope_pos=rope_pos, rope_theta=rope_theta)
     word = simsd.simsd_check_error(e)
     if merr is not None:
         word |= simsd.simsd_check_error(merr)
     return out, word, ws
 
 
-def oracle_attention(si, layer=0, seqs=None):
+def oracle_attention(si, layer=0, seqs=None, rope_theta=0.0, rope_mode=1):
     """Oracle attention for all sequences, or for the listed ones only (a
-    sub-batch with its own compact page pool)."""
+    sub-batch with its own compact page pool).  rope_theta > 0: q and k_new
+    are rotated by the oracle first (rope_mode 1: RoPE copy, 2: physical
+    positions)."""
+    rope = dict(rope_theta=rope_theta, rope_mode=rope_mode)
     if seqs is None:
         return orc.verify_attention(
             inputs.host_bits(si.q[layer]), inputs.host_bits(si.k_new[layer]), inputs.host_bits(si.v_new[layer]),
             inputs.host_bits(si.k_cache[layer]), inputs.host_bits(si.v_cache[layer]),
-            si.block_table.cpu().numpy(), si.prefix_len.cpu().numpy(), si.step_map.cpu().numpy(), si.w.gamma)
+            si.block_table.cpu().numpy(), si.prefix_len.cpu().numpy(), si.step_map.cpu().numpy(), si.w.gamma,
+            **rope)
     idx = torch.as_tensor(seqs, device=si.q.device)
     bt = si.block_table[idx].cpu()
     n = si.prefix_len[idx].cpu()
@@ -79,7 +83,7 @@ def oracle_attention(si, layer=0, seqs=None):
     return orc.verify_attention(
         inputs.host_bits(si.q[layer][idx]), inputs.host_bits(si.k_new[layer][idx]),
         inputs.host_bits(si.v_new[layer][idx]), inputs.host_bits(kc), inputs.host_bits(vc), new_bt.numpy(),
-        n.numpy(), si.step_map[idx].cpu().numpy(), si.w.gamma)
+        n.numpy(), si.step_map[idx].cpu().numpy(), si.w.gamma, **rope)
 
 
 def assert_attention_close(got, want, dtype):

@@ -43,13 +43,18 @@ def test_host_validation_without_gpu(lib):
     # gamma outside [1, 32]
     assert lib.simsd_build_mask(None, one, 1, 0, one, one, one, None, None, None) == 1
     assert lib.simsd_build_mask(None, one, 1, 33, one, one, one, None, None, None) == 1
-    # rope_pos must be NULL (inputs arrive rotated)
-    rc = lib.simsd_verify_attention(1, one, one, one, one, one, 4, one, 1, 64, one, one, one, one, 1, 4, 8, 8, 128,
-                                    ctypes.c_float(0.0), one, None, 0, None, None)
-    assert rc == 2
+    F = ctypes.c_float
+    # rope_pos given without a positive, finite rope_theta
+    for theta in (0.0, -1.0, float("inf"), float("nan")):
+        rc = lib.simsd_verify_attention(1, one, one, one, one, one, 4, one, 1, 64, one, one, one, one, F(theta), 1, 4,
+                                        8, 8, 128, F(0.0), one, None, 0, None, None)
+        assert rc == 1
+        rc = lib.simsd_kv_commit(1, one, one, 1, one, one, one, F(theta), one, one, one, 4, one, 1, 64, one, 1, 4,
+                                 8, 128, None, None)
+        assert rc == 1
     # Hq not a multiple of Hkv
-    rc = lib.simsd_verify_attention(1, one, one, one, one, one, 4, one, 1, 64, one, one, one, None, 1, 4, 6, 4, 128,
-                                    ctypes.c_float(0.0), one, None, 0, None, None)
+    rc = lib.simsd_verify_attention(1, one, one, one, one, one, 4, one, 1, 64, one, one, one, None, F(0.0), 1, 4, 6,
+                                    4, 128, F(0.0), one, None, 0, None, None)
     assert rc == 1
     # vocab out of range
     assert lib.simsd_accept(one, one, 1, 4, 0, one, one, None, None, None) == 1
