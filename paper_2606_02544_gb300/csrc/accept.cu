@@ -22,7 +22,6 @@ namespace cg = cooperative_groups;
 namespace simsd {
 
 constexpr int kAcceptThreads = 512;
-constexpr int kAcceptUnroll = 8;
 constexpr int kMaxRows = 33;  // gamma + 1 <= 33
 
 // Total order used by the argmax: larger key = better.  NaN ranks above every
@@ -70,6 +69,9 @@ struct RowBest {
   }
 };
 
+// UNROLL 16-byte loads are in flight per thread: 8 in general, 16 when the
+// grid leaves SMs idle (then each CTA has the SM to itself).
+template <int UNROLL>
 __global__ void __launch_bounds__(kAcceptThreads) accept_kernel(const float* __restrict__ logits,
                                                                 const int32_t* __restrict__ draft, int gamma,
                                                                 int vocab, int vec4, int32_t* __restrict__ accepted_len,
@@ -77,6 +79,8 @@ __global__ void __launch_bounds__(kAcceptThreads) accept_kernel(const float* __r
                                                                 int32_t* __restrict__ row_argmax, int32_t* err_word) {
   __shared__ unsigned long long best[kMaxRows];
   __shared__ int am[kMaxRows];
+  pdl_wait();
+  pdl_launch_next();
   cg::cluster_group cluster = cg::this_cluster();
   const int c = static_cast<int>(cluster.block_rank());
   const int CL = static_cast<int>(cluster.num_blocks());
@@ -102,15 +106,15 @@ __global__ void __launch_bounds__(kAcceptThreads) accept_kernel(const float* __r
   constexpr int kStride = kAcceptThreads;
   if (vec4) {
     const float4* b4 = reinterpret_cast<const float4*>(base);
-    for (; f < f1; f += static_cast<long long>(kStride) * kAcceptUnroll) {
-      float4 v[kAcceptUnroll];
+    for (; f < f1; f += static_cast<long long>(kStride) * UNROLL) {
+      float4 v[UNROLL];
 #pragma unroll
-      for (int u = 0; u < kAcceptUnroll; ++u) {
+      for (int u = 0; u < UNROLL; ++u) {
         const long long fu = f + static_cast<long long>(u) * kStride;
         if (fu < f1) v[u] = ld_stream_f4(reinterpret_cast<const float*>(b4 + fu));
       }
 #pragma unroll
-      for (int u = 0; u < kAcceptUnroll; ++u) {
+      for (int u = 0; u < UNROLL; ++u) {
         if (f + static_cast<long long>(u) * kStride >= f1) break;
         if (row != cur) {
           atomicMax(&best[cur], rb.key());
@@ -204,6 +208,7 @@ struct ClusterCapacity {
   int resident[kMaxCluster + 1] = {};
 };
 
+template <int UNROLL>
 cudaError_t cluster_capacity(const ClusterCapacity** out) {
   static std::mutex mu;
   static ClusterCapacity cap[64];
@@ -214,7 +219,7 @@ cudaError_t cluster_capacity(const ClusterCapacity** out) {
   std::lock_guard<std::mutex> lk(mu);
   ClusterCapacity& c = cap[dev];
   if (!c.ready) {
-    e = cudaFuncSetAttribute(accept_kernel, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
+    e = cudaFuncSetAttribute(accept_kernel<UNROLL>, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
     if (e != cudaSuccess) return e;
     for (int cl = 1; cl <= kMaxCluster; ++cl) {
       cudaLaunchConfig_t cfg = {};
@@ -228,7 +233,7 @@ cudaError_t cluster_capacity(const ClusterCapacity** out) {
       cfg.attrs = attr;
       cfg.numAttrs = 1;
       int n = 0;
-      e = cudaOccupancyMaxActiveClusters(&n, accept_kernel, &cfg);
+      e = cudaOccupancyMaxActiveClusters(&n, accept_kernel<UNROLL>, &cfg);
       if (e != cudaSuccess) return e;
       c.resident[cl] = n;
     }
@@ -243,9 +248,19 @@ cudaError_t cluster_capacity(const ClusterCapacity** out) {
 cudaError_t launch_accept(const float* logits, const int32_t* draft, int Bt, int gamma, int vocab,
                           int32_t* accepted_len, int32_t* out_tokens, int32_t* row_argmax, int32_t* err_word,
                           int num_sms, cudaStream_t stream) {
-  (void)num_sms;
+  const int vec4 = (vocab % 4 == 0) && ((reinterpret_cast<uintptr_t>(logits) & 15u) == 0);
   const ClusterCapacity* cap = nullptr;
-  cudaError_t e = cluster_capacity(&cap);
+  // few sequences: the largest clusters still leave SMs idle, so each CTA
+  // keeps twice as many loads in flight
+  if (Bt * kMaxCluster <= num_sms) {
+    cudaError_t e = cluster_capacity<16>(&cap);
+    if (e != cudaSuccess) return e;
+    if (cap->resident[kMaxCluster] >= Bt)
+      return launch_overlapped(accept_kernel<16>, dim3(static_cast<unsigned>(Bt) * kMaxCluster),
+                               dim3(kAcceptThreads), 0, stream, static_cast<unsigned>(kMaxCluster), logits, draft,
+                               gamma, vocab, vec4, accepted_len, out_tokens, row_argmax, err_word);
+  }
+  cudaError_t e = cluster_capacity<8>(&cap);
   if (e != cudaSuccess) return e;
   // the largest cluster for which one cluster per sequence still fits in a
   // single wave: more CTAs keep more loads in flight
@@ -256,21 +271,9 @@ cudaError_t launch_accept(const float* logits, const int32_t* draft, int Bt, int
       break;
     }
   }
-  const int vec4 = (vocab % 4 == 0) && ((reinterpret_cast<uintptr_t>(logits) & 15u) == 0);
-  cudaLaunchConfig_t cfg = {};
-  cfg.gridDim = dim3(static_cast<unsigned>(Bt) * CL);
-  cfg.blockDim = dim3(kAcceptThreads);
-  cfg.dynamicSmemBytes = 0;
-  cfg.stream = stream;
-  cudaLaunchAttribute attr[1];
-  attr[0].id = cudaLaunchAttributeClusterDimension;
-  attr[0].val.clusterDim.x = static_cast<unsigned>(CL);
-  attr[0].val.clusterDim.y = 1;
-  attr[0].val.clusterDim.z = 1;
-  cfg.attrs = attr;
-  cfg.numAttrs = 1;
-  return cudaLaunchKernelEx(&cfg, accept_kernel, logits, draft, gamma, vocab, vec4, accepted_len, out_tokens,
-                            row_argmax, err_word);
+  return launch_overlapped(accept_kernel<8>, dim3(static_cast<unsigned>(Bt) * CL), dim3(kAcceptThreads), 0, stream,
+                           static_cast<unsigned>(CL), logits, draft, gamma, vocab, vec4, accepted_len, out_tokens,
+                           row_argmax, err_word);
 }
 
 }  // namespace simsd

@@ -18,6 +18,8 @@ constexpr int kF32Warps = 4;
 template <int DPL>  // head-dim elements per lane (d = 32 * DPL)
 __global__ void __launch_bounds__(kF32Warps * 32) attention_f32_kernel(const __grid_constant__ AttnF32Args a) {
   __shared__ __align__(16) float q_s[kF32Warps][32 * DPL];
+  pdl_wait();
+  pdl_launch_next();
   const int lane = threadIdx.x & 31, wib = threadIdx.x >> 5;
   const long long row = (static_cast<long long>(blockIdx.x) * blockDim.x + threadIdx.x) >> 5;
   const int S = 2 * a.gamma, g = a.Hq / a.Hkv;
@@ -170,11 +172,8 @@ __global__ void __launch_bounds__(kF32Warps * 32) attention_f32_kernel(const __g
 cudaError_t launch_attention_f32(const AttnF32Args& a, cudaStream_t stream) {
   const long long rows = static_cast<long long>(a.Bt) * 2 * a.gamma * a.Hq;
   const unsigned blocks = static_cast<unsigned>((rows + kF32Warps - 1) / kF32Warps);
-  if (a.d == 64)
-    attention_f32_kernel<2><<<blocks, kF32Warps * 32, 0, stream>>>(a);
-  else
-    attention_f32_kernel<4><<<blocks, kF32Warps * 32, 0, stream>>>(a);
-  return cudaGetLastError();
+  if (a.d == 64) return launch_overlapped(attention_f32_kernel<2>, dim3(blocks), dim3(kF32Warps * 32), 0, stream, 1, a);
+  return launch_overlapped(attention_f32_kernel<4>, dim3(blocks), dim3(kF32Warps * 32), 0, stream, 1, a);
 }
 
 }  // namespace simsd

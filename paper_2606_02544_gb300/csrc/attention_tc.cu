@@ -133,11 +133,6 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm)
     sm.seq_bad = 0;
     sm.b_sel = rank;
   }
-  // prefix lengths, staged in the (still unused) ring for the ranking
-  int32_t* nval = reinterpret_cast<int32_t*>(sm.ring[0]);
-  const bool sort = p.Bt <= 256;
-  if (sort)
-    for (int i = tid; i < p.Bt; i += kThreads) nval[i] = p.prefix_len[i];
   if (tid == 0) {
     for (int s = 0; s < kStages; ++s) {
       mbar_init(smem_u32(&sm.bar_k[s]), 1);
@@ -155,6 +150,15 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm)
     tmem_alloc(smem_u32(&sm.tmem_base), kTmemCols);
     tmem_relinquish();
   }
+  // the set-up above touches no global memory; from here on the previous
+  // kernel's results are needed
+  pdl_wait();
+  pdl_launch_next();
+  // prefix lengths, staged in the (still unused) ring for the ranking
+  int32_t* nval = reinterpret_cast<int32_t*>(sm.ring[0]);
+  const bool sort = p.Bt <= 256;
+  if (sort)
+    for (int i = tid; i < p.Bt; i += kThreads) nval[i] = p.prefix_len[i];
   __syncthreads();
   if (sort) {
     for (int i = tid; i < p.Bt; i += kThreads) {
@@ -173,6 +177,88 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm)
   const int b = sm.b_sel;
   const int n = p.prefix_len[b];
   const bool n_bad = n < 0 || static_cast<long long>(n) > static_cast<long long>(p.max_pages) * p.page_size;
+  const int32_t* bt = p.block_table + static_cast<size_t>(b) * p.max_pages;
+
+  // ---- TMA issue of ring items (producer thread only): item 0 is Q, item
+  // i + 1 is the i-th key tile of this unit (tile 0: new slots, 1..T: prefix)
+  auto issue_q = [&]() {
+    const uint32_t q_bytes = 2u * static_cast<uint32_t>(p.g * p.s_blk) * 128u;
+    const int qz = b * p.S + rblk * p.s_blk;
+    const uint32_t q0 = smem_u32(sm.ring[0]);
+    mbar_arrive_expect_tx(smem_u32(&sm.bar_k[0]), q_bytes);
+    tma_load_3d(q0, &tm_q, smem_u32(&sm.bar_k[0]), 0, kvh * p.g, qz);
+    tma_load_3d(q0 + 2 * kHalfBytes, &tm_q, smem_u32(&sm.bar_k[0]), 64, kvh * p.g, qz);
+    mbar_arrive(smem_u32(&sm.bar_v[0]));  // keeps the two barriers of slot 0 in step
+  };
+  auto issue_tile = [&](int it, int t) {
+    const int P = p.page_size;
+    const int st = it % kStages;
+    const uint32_t bk = smem_u32(&sm.bar_k[st]), bv = smem_u32(&sm.bar_v[st]);
+    const uint32_t k0 = smem_u32(sm.ring[st]), k1 = k0 + kHalfBytes;
+    const uint32_t v0 = k0 + 2 * kHalfBytes, v1 = k0 + 3 * kHalfBytes;
+    if (t > 0) {
+      const int key0 = (t - 1) * kTile;
+      const int valid = min(kTile, n - key0);
+      if (P >= kTile) {
+        const int pi = key0 / P;
+        const int pg = pi < kPageCache ? sm.pages[pi] : bt[pi];
+        const int row = (pg * p.Hkv + kvh) * P + (key0 % P);
+        mbar_arrive_expect_tx(bk, 2u * kHalfBytes);
+        tma_load_2d(k0, &tm_kc, bk, 0, row);
+        tma_load_2d(k1, &tm_kc, bk, 64, row);
+        mbar_arrive_expect_tx(bv, 2u * kHalfBytes);
+        tma_load_2d(v0, &tm_vc, bv, 0, row);
+        tma_load_2d(v1, &tm_vc, bv, 64, row);
+      } else {
+        const int nsub = (valid + P - 1) / P;
+        const uint32_t sub_bytes = static_cast<uint32_t>(P) * 128u;
+        mbar_arrive_expect_tx(bk, 2u * nsub * sub_bytes);
+        for (int sb = 0; sb < nsub; ++sb) {
+          const int pi = (key0 + sb * P) / P;
+          const int pg = pi < kPageCache ? sm.pages[pi] : bt[pi];
+          const int row = (pg * p.Hkv + kvh) * P;
+          tma_load_2d(k0 + sb * sub_bytes, &tm_kc, bk, 0, row);
+          tma_load_2d(k1 + sb * sub_bytes, &tm_kc, bk, 64, row);
+        }
+        mbar_arrive_expect_tx(bv, 2u * nsub * sub_bytes);
+        for (int sb = 0; sb < nsub; ++sb) {
+          const int pi = (key0 + sb * P) / P;
+          const int pg = pi < kPageCache ? sm.pages[pi] : bt[pi];
+          const int row = (pg * p.Hkv + kvh) * P;
+          tma_load_2d(v0 + sb * sub_bytes, &tm_vc, bv, 0, row);
+          tma_load_2d(v1 + sb * sub_bytes, &tm_vc, bv, 64, row);
+        }
+      }
+    } else {
+      const uint32_t new_bytes = static_cast<uint32_t>(p.S) * 128u;
+      mbar_arrive_expect_tx(bk, 2u * new_bytes);
+      tma_load_3d(k0, &tm_kn, bk, 0, kvh, b * p.S);
+      tma_load_3d(k1, &tm_kn, bk, 64, kvh, b * p.S);
+      mbar_arrive_expect_tx(bv, 2u * new_bytes);
+      tma_load_3d(v0, &tm_vn, bv, 0, kvh, b * p.S);
+      tma_load_3d(v1, &tm_vn, bv, 64, kvh, b * p.S);
+    }
+  };
+  // Q and the tile of new slots need no page id: they are issued before the
+  // page table is checked.  If the check fails they are drained unused.
+  int early = 0;
+  if (warp == kWarpProducer && lane == 0) {
+    tma_prefetch_desc(&tm_q);
+    tma_prefetch_desc(&tm_kc);
+    tma_prefetch_desc(&tm_vc);
+    if (!n_bad) {
+      issue_q();
+      early = 1;
+      const int tg = (n + kTile - 1) / kTile + 1;  // tiles of a valid sequence
+      const int t0g = static_cast<int>(static_cast<long long>(split) * tg / p.nsplit);
+      const int t1g = static_cast<int>(static_cast<long long>(split + 1) * tg / p.nsplit);
+      if (t0g == 0 && t1g > 0) {
+        issue_tile(1, 0);
+        early = 2;
+      }
+    }
+  }
+
   if (n_bad) {
     if (tid == 0) {
       sm.seq_bad = 1;
@@ -180,7 +266,6 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm)
     }
   } else {
     const int npages = (n + p.page_size - 1) / p.page_size;
-    const int32_t* bt = p.block_table + static_cast<size_t>(b) * p.max_pages;
     for (int i = tid; i < npages; i += kThreads) {
       const int pg = bt[i];
       if (i < kPageCache) sm.pages[i] = pg;
@@ -208,74 +293,19 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm)
 
   if (warp == kWarpProducer) {
     // ------------------------------------------------------------ producer
-    // ring item 0 is Q, item i + 1 is the i-th key tile of this unit
-    if (lane == 0 && ntiles > 0) {
-      tma_prefetch_desc(&tm_q);
-      tma_prefetch_desc(&tm_kc);
-      tma_prefetch_desc(&tm_vc);
-      const uint32_t q_bytes = 2u * static_cast<uint32_t>(p.g * p.s_blk) * 128u;
-      const int qz = b * p.S + rblk * p.s_blk;
-      const uint32_t q0 = smem_u32(sm.ring[0]);
-      mbar_arrive_expect_tx(smem_u32(&sm.bar_k[0]), q_bytes);
-      tma_load_3d(q0, &tm_q, smem_u32(&sm.bar_k[0]), 0, kvh * p.g, qz);
-      tma_load_3d(q0 + 2 * kHalfBytes, &tm_q, smem_u32(&sm.bar_k[0]), 64, kvh * p.g, qz);
-      mbar_arrive(smem_u32(&sm.bar_v[0]));  // keeps the two barriers of slot 0 in step
-      const int P = p.page_size;
-      const int32_t* bt = p.block_table + static_cast<size_t>(b) * p.max_pages;
-      int issued = 1;
-      for (int i = 0; i < ntiles; ++i) {
-        const int it = i + 1, st = it % kStages;
-        if (it >= kStages && !mbar_wait(smem_u32(&sm.bar_empty[st]), ((it / kStages) - 1) & 1, abort_flag)) {
-          signal_abort(sm, p.err_word);
-          break;
-        }
-        const int t = t0 + i;
-        const uint32_t bk = smem_u32(&sm.bar_k[st]), bv = smem_u32(&sm.bar_v[st]);
-        const uint32_t k0 = smem_u32(sm.ring[st]), k1 = k0 + kHalfBytes;
-        const uint32_t v0 = k0 + 2 * kHalfBytes, v1 = k0 + 3 * kHalfBytes;
-        if (t > 0) {
-          const int key0 = (t - 1) * kTile;
-          const int valid = min(kTile, n - key0);
-          if (P >= kTile) {
-            const int pi = key0 / P;
-            const int pg = pi < kPageCache ? sm.pages[pi] : bt[pi];
-            const int row = (pg * p.Hkv + kvh) * P + (key0 % P);
-            mbar_arrive_expect_tx(bk, 2u * kHalfBytes);
-            tma_load_2d(k0, &tm_kc, bk, 0, row);
-            tma_load_2d(k1, &tm_kc, bk, 64, row);
-            mbar_arrive_expect_tx(bv, 2u * kHalfBytes);
-            tma_load_2d(v0, &tm_vc, bv, 0, row);
-            tma_load_2d(v1, &tm_vc, bv, 64, row);
-          } else {
-            const int nsub = (valid + P - 1) / P;
-            const uint32_t sub_bytes = static_cast<uint32_t>(P) * 128u;
-            mbar_arrive_expect_tx(bk, 2u * nsub * sub_bytes);
-            for (int sb = 0; sb < nsub; ++sb) {
-              const int pi = (key0 + sb * P) / P;
-              const int pg = pi < kPageCache ? sm.pages[pi] : bt[pi];
-              const int row = (pg * p.Hkv + kvh) * P;
-              tma_load_2d(k0 + sb * sub_bytes, &tm_kc, bk, 0, row);
-              tma_load_2d(k1 + sb * sub_bytes, &tm_kc, bk, 64, row);
-            }
-            mbar_arrive_expect_tx(bv, 2u * nsub * sub_bytes);
-            for (int sb = 0; sb < nsub; ++sb) {
-              const int pi = (key0 + sb * P) / P;
-              const int pg = pi < kPageCache ? sm.pages[pi] : bt[pi];
-              const int row = (pg * p.Hkv + kvh) * P;
-              tma_load_2d(v0 + sb * sub_bytes, &tm_vc, bv, 0, row);
-              tma_load_2d(v1 + sb * sub_bytes, &tm_vc, bv, 64, row);
-            }
+    if (lane == 0) {
+      int issued = early;
+      if (ntiles > 0) {
+        // a valid sequence: Q (and the tile of new slots) went out already
+        for (int i = issued - 1; i < ntiles; ++i) {
+          const int it = i + 1, st = it % kStages;
+          if (it >= kStages && !mbar_wait(smem_u32(&sm.bar_empty[st]), ((it / kStages) - 1) & 1, abort_flag)) {
+            signal_abort(sm, p.err_word);
+            break;
           }
-        } else {
-          const uint32_t new_bytes = static_cast<uint32_t>(p.S) * 128u;
-          mbar_arrive_expect_tx(bk, 2u * new_bytes);
-          tma_load_3d(k0, &tm_kn, bk, 0, kvh, b * p.S);
-          tma_load_3d(k1, &tm_kn, bk, 64, kvh, b * p.S);
-          mbar_arrive_expect_tx(bv, 2u * new_bytes);
-          tma_load_3d(v0, &tm_vn, bv, 0, kvh, b * p.S);
-          tma_load_3d(v1, &tm_vn, bv, 64, kvh, b * p.S);
+          issue_tile(it, t0 + i);
+          ++issued;
         }
-        ++issued;
       }
       // Drain: every issued load must have landed before the CTA may exit.
       // In a normal run these phases completed long ago.
@@ -611,7 +641,9 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm)
 
 // Merges the prefix splits of every (sequence, KV head, row block):
 // O = sum_i 2^(m_i - M) O_i / sum_i 2^(m_i - M) l_i.  One warp per row.
-__global__ void __launch_bounds__(128) combine_kernel(const TcParams p) {
+__global__ void __launch_bounds__(128) combine_kernel(const __grid_constant__ TcParams p) {
+  pdl_wait();
+  pdl_launch_next();
   const int lane = threadIdx.x & 31;
   const long long wid = (static_cast<long long>(blockIdx.x) * blockDim.x + threadIdx.x) >> 5;
   const long long units = static_cast<long long>(p.Bt) * p.Hkv * p.rb;
@@ -769,12 +801,11 @@ cudaError_t launch_attention_tc(const AttnTcArgs& a, const AttnTcPlan& pl, Encod
     if (e != cudaSuccess) return e;
   }
   const long long grid = static_cast<long long>(a.Bt) * pl.nsplit * a.Hkv * pl.rb;
-  attention_tc_kernel<<<static_cast<unsigned>(grid), kThreads, smem_bytes(), stream>>>(tq, tkn, tvn, tkc, tvc, p);
-  cudaError_t e = cudaGetLastError();
+  cudaError_t e = launch_overlapped(attention_tc_kernel, dim3(static_cast<unsigned>(grid)), dim3(kThreads),
+                                    smem_bytes(), stream, 1, tq, tkn, tvn, tkc, tvc, p);
   if (e != cudaSuccess || pl.nsplit == 1) return e;
   const long long warps = static_cast<long long>(a.Bt) * a.Hkv * pl.rb * pl.rows_blk;
-  combine_kernel<<<static_cast<unsigned>((warps + 3) / 4), 128, 0, stream>>>(p);
-  return cudaGetLastError();
+  return launch_overlapped(combine_kernel, dim3(static_cast<unsigned>((warps + 3) / 4)), dim3(128), 0, stream, 1, p);
 }
 
 size_t noalloc_scratch_capacity() { return sizeof(g_noalloc_scratch); }

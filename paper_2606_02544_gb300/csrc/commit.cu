@@ -28,6 +28,8 @@ __global__ void __launch_bounds__(kCommitWarps * 32) kv_commit_copy_kernel(
     uint8_t* __restrict__ v_cache, int num_pages, const int32_t* __restrict__ block_table, int max_pages,
     int page_size, const int32_t* __restrict__ prefix_len, int Bt, int gamma, int Hkv, int row_bytes,
     int elem_bytes, const __grid_constant__ CommitRope rope, int32_t* err_word) {
+  pdl_wait();
+  pdl_launch_next();
   const long long wid = (static_cast<long long>(blockIdx.x) * blockDim.x + threadIdx.x) >> 5;
   const int lane = threadIdx.x & 31;
   const long long total = static_cast<long long>(L) * Bt * gamma * Hkv;
@@ -102,6 +104,8 @@ __global__ void __launch_bounds__(kCommitWarps * 32) kv_commit_copy_kernel(
 // n_b += a_b once every copy that read n_b has finished (stream order).
 __global__ void kv_commit_advance_kernel(const int32_t* __restrict__ accepted_len, int32_t* __restrict__ prefix_len,
                                          int Bt, int gamma, int32_t* err_word) {
+  pdl_wait();
+  pdl_launch_next();
   const int b = blockIdx.x * blockDim.x + threadIdx.x;
   if (b >= Bt) return;
   const int a = accepted_len[b];
@@ -125,16 +129,16 @@ cudaError_t launch_kv_commit(int elem_bytes, const void* k_new, const void* v_ne
   const long long warps = static_cast<long long>(L) * Bt * gamma * Hkv;
   const long long blocks = (warps + kCommitWarps - 1) / kCommitWarps;
   if (blocks > 0) {
-    kv_commit_copy_kernel<<<static_cast<unsigned>(blocks), kCommitWarps * 32, 0, stream>>>(
+    cudaError_t e = launch_overlapped(
+        kv_commit_copy_kernel, dim3(static_cast<unsigned>(blocks)), dim3(kCommitWarps * 32), 0, stream, 1,
         static_cast<const uint8_t*>(k_new), static_cast<const uint8_t*>(v_new), L, tau, section, accepted_len,
         static_cast<uint8_t*>(k_cache), static_cast<uint8_t*>(v_cache), num_pages, block_table, max_pages,
         page_size, prefix_len, Bt, gamma, Hkv, d * elem_bytes, elem_bytes, CommitRope{rope_pos, rope_table},
         err_word);
-    cudaError_t e = cudaGetLastError();
     if (e != cudaSuccess) return e;
   }
-  kv_commit_advance_kernel<<<(Bt + 127) / 128, 128, 0, stream>>>(accepted_len, prefix_len, Bt, gamma, err_word);
-  return cudaGetLastError();
+  return launch_overlapped(kv_commit_advance_kernel, dim3((Bt + 127) / 128), dim3(128), 0, stream, 1, accepted_len,
+                           prefix_len, Bt, gamma, err_word);
 }
 
 }  // namespace simsd

@@ -3,6 +3,7 @@
 #include <cuda_runtime.h>
 
 #include <cstdint>
+#include <utility>
 
 #include "../../include/simsd.h"
 
@@ -25,6 +26,42 @@ __host__ __device__ __forceinline__ bool temporal_visible(uint8_t si, int ti, ui
   if (si == kSectPad || sj == kSectPad) return false;
   const int bias = (si == kSectData) ? 1 : 0;
   return (sj == kSectData) == (tj < ti + bias);
+}
+
+// ---- programmatic dependent launch.  Every kernel of the library is
+// launched so that it may start (set-up only) while the previous kernel on
+// the stream finishes: it calls pdl_wait() before it reads or writes any
+// memory that earlier work may touch, and pdl_launch_next() to let the next
+// kernel start its own set-up early.  The wait returns once the previous
+// grid has completed and its memory operations are visible.
+__device__ __forceinline__ void pdl_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+__device__ __forceinline__ void pdl_launch_next() { asm volatile("griddepcontrol.launch_dependents;" ::: "memory"); }
+
+// Host side: launches kern with the attribute that allows the overlap above
+// (and a cluster dimension when cluster > 1).
+template <typename... KArgs, typename... Args>
+inline cudaError_t launch_overlapped(void (*kern)(KArgs...), dim3 grid, dim3 block, size_t smem, cudaStream_t stream,
+                                     unsigned cluster, Args&&... args) {
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = grid;
+  cfg.blockDim = block;
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = stream;
+  cudaLaunchAttribute attr[2];
+  unsigned na = 0;
+  attr[na].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[na].val.programmaticStreamSerializationAllowed = 1;
+  ++na;
+  if (cluster > 1) {
+    attr[na].id = cudaLaunchAttributeClusterDimension;
+    attr[na].val.clusterDim.x = cluster;
+    attr[na].val.clusterDim.y = 1;
+    attr[na].val.clusterDim.z = 1;
+    ++na;
+  }
+  cfg.attrs = attr;
+  cfg.numAttrs = na;
+  return cudaLaunchKernelEx(&cfg, kern, std::forward<Args>(args)...);
 }
 
 // ---- rotary position embedding (Su et al., RoFormer), rotate-half layout:

@@ -19,6 +19,8 @@ __global__ void __launch_bounds__(64) build_mask_kernel(const int32_t* __restric
   __shared__ int s_tau[64];
   __shared__ uint8_t s_sect[64];
   const int b = blockIdx.x, i = threadIdx.x, S = 2 * gamma;
+  pdl_wait();
+  pdl_launch_next();
   if (i == 0) map_ok = 1;
   if (i < gamma) mu[i] = step_map ? step_map[static_cast<size_t>(b) * gamma + i] : i + 1;
   __syncthreads();
@@ -57,9 +59,8 @@ __global__ void __launch_bounds__(64) build_mask_kernel(const int32_t* __restric
 cudaError_t launch_build_mask(const int32_t* step_map, const int32_t* prefix_len, int Bt, int gamma, int32_t* tau,
                               uint8_t* section, int32_t* rope_pos, uint64_t* mask_bits, int32_t* err_word,
                               cudaStream_t stream) {
-  build_mask_kernel<<<Bt, 64, 0, stream>>>(step_map, prefix_len, gamma, tau, section, rope_pos,
-                                           reinterpret_cast<unsigned long long*>(mask_bits), err_word);
-  return cudaGetLastError();
+  return launch_overlapped(build_mask_kernel, dim3(Bt), dim3(64), 0, stream, 1, step_map, prefix_len, gamma, tau,
+                           section, rope_pos, reinterpret_cast<unsigned long long*>(mask_bits), err_word);
 }
 
 }  // namespace simsd
