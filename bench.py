@@ -194,8 +194,11 @@ def run_gpu(args):
             if flush is not None:
                 _flush_l2(flush)
             e = ev[m]
+            # the prefix lengths are reset before the step starts (benchmark
+            # plumbing that makes every step verify the same block)
+            st.restore()
             e[0].record()
-            st.run(attn_events=(e[1], e[2]))
+            st.run(attn_events=(e[1], e[2]), restore=False)
             e[5].record()
     # accept-only timing graph piece: events around simsd_accept are taken
     # from the step's own graph nodes via a second capture of one step
@@ -293,7 +296,8 @@ def run_gpu(args):
                        "verified_tokens_per_step": tokens_per_step, "draft_tokens_per_step": wl.Bt * wl.gamma,
                        "l2": "flushed before every step (258 MB write + read)" if need_flush else
                        "inputs larger than L2 (no flush)",
-                       "timing": f"CUDA graph of {M} steps; per-step CUDA events; max over ranks",
+                       "timing": f"CUDA graph of {M} steps; per-step CUDA events (the reset of the prefix "
+                                 f"lengths between steps is outside them); max over ranks",
                        "parallelism": f"replicas x{world}"},
             "draft_tokens_per_s": round(wl.Bt * wl.gamma * K * world / (total_ms_max / 1e3), 1),
             "roofline": dominant, "roofline_other": other, "clocks": clocks, "e2e": e2e,

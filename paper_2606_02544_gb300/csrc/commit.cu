@@ -7,118 +7,125 @@
 #include <cuda_bf16.h>
 #include <cuda_runtime.h>
 
+#include <cooperative_groups.h>
+
 #include "common.cuh"
 #include "kernels.h"
+
+namespace cg = cooperative_groups;
 
 namespace simsd {
 
 constexpr int kCommitWarps = 8;
 
-// One warp per (layer, sequence, accepted row, KV head); each lane moves
-// 16-byte chunks of the K row and the V row (or, with RoPE, rotates pairs
-// of the K row).
+// rotation of committed keys (null pos: the keys are rotated already)
 struct CommitRope {
   const int32_t* pos;  // [Bt][2*gamma] or null
   RopeTable table;
 };
 
-__global__ void __launch_bounds__(kCommitWarps * 32) kv_commit_copy_kernel(
+// One thread-block cluster per sequence.  Every thread reads n_b and a_b and
+// arrives on the cluster barrier; the cluster's warps then share the
+// sequence's accepted rows (layer, accepted row, KV head), one row per warp
+// at a time (16-byte chunks, or pairs when rotating keys); after every
+// thread of the cluster has arrived, thread 0 of CTA 0 writes
+// n_b + a_b (no thread reads n_b after that).
+__global__ void __launch_bounds__(kCommitWarps * 32) kv_commit_kernel(
     const uint8_t* __restrict__ k_new, const uint8_t* __restrict__ v_new, int L, const int32_t* __restrict__ tau,
     const uint8_t* __restrict__ section, const int32_t* __restrict__ accepted_len, uint8_t* __restrict__ k_cache,
     uint8_t* __restrict__ v_cache, int num_pages, const int32_t* __restrict__ block_table, int max_pages,
-    int page_size, const int32_t* __restrict__ prefix_len, int Bt, int gamma, int Hkv, int row_bytes,
-    int elem_bytes, const __grid_constant__ CommitRope rope, int32_t* err_word) {
+    int page_size, int32_t* __restrict__ prefix_len, int gamma, int Hkv, int row_bytes, int elem_bytes,
+    const __grid_constant__ CommitRope rope, int32_t* err_word) {
   pdl_wait();
   pdl_launch_next();
-  const long long wid = (static_cast<long long>(blockIdx.x) * blockDim.x + threadIdx.x) >> 5;
-  const int lane = threadIdx.x & 31;
-  const long long total = static_cast<long long>(L) * Bt * gamma * Hkv;
-  if (wid >= total) return;
-  const int kvh = static_cast<int>(wid % Hkv);
-  const int r = static_cast<int>((wid / Hkv) % gamma);
-  const int b = static_cast<int>((wid / (static_cast<long long>(Hkv) * gamma)) % Bt);
-  const int l = static_cast<int>(wid / (static_cast<long long>(Hkv) * gamma * Bt));
+  cg::cluster_group cluster = cg::this_cluster();
+  const int CL = static_cast<int>(cluster.num_blocks());
+  const int rank = static_cast<int>(cluster.block_rank());
+  const int b = blockIdx.x / CL;
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
   const int a = accepted_len[b];
   const int n = prefix_len[b];
-  if (a < 0 || a > gamma || n < 0 || r >= a) return;  // invalid sequences are reported by the advance kernel
+  // "n_b has been read"
+  asm volatile("barrier.cluster.arrive.release;" ::: "memory");
+  const bool ok = a >= 0 && a <= gamma && n >= 0;
   const int S = 2 * gamma;
-  // source: the data slot whose label is r+1
-  const bool hit = lane < gamma && section[static_cast<size_t>(b) * S + lane] == kSectData &&
-                   tau[static_cast<size_t>(b) * S + lane] == r + 1;
-  const unsigned m = __ballot_sync(0xffffffffu, hit);
-  if (!m) {
-    if (lane == 0) raise_error(err_word, SIMSD_EW_STEP_MAP);
-    return;
-  }
-  const int src = __ffs(m) - 1;
-  const long long dst_row = static_cast<long long>(n) + r;
-  const long long pidx = dst_row / page_size;
-  if (pidx >= max_pages) {
-    if (lane == 0) raise_error(err_word, SIMSD_EW_PAGE);
-    return;
-  }
-  const int pg = block_table[static_cast<size_t>(b) * max_pages + pidx];
-  if (pg < 0 || pg >= num_pages) {
-    if (lane == 0) raise_error(err_word, SIMSD_EW_PAGE);
-    return;
-  }
-  const int off = static_cast<int>(dst_row % page_size);
-  const size_t s_row = ((static_cast<size_t>(l) * Bt + b) * S + src) * Hkv + kvh;
-  const size_t d_row = ((static_cast<size_t>(l) * num_pages + pg) * Hkv + kvh) * page_size + off;
-  const uint4* ks = reinterpret_cast<const uint4*>(k_new + s_row * row_bytes);
-  const uint4* vs = reinterpret_cast<const uint4*>(v_new + s_row * row_bytes);
-  uint4* kd = reinterpret_cast<uint4*>(k_cache + d_row * row_bytes);
-  uint4* vd = reinterpret_cast<uint4*>(v_cache + d_row * row_bytes);
-  const int chunks = row_bytes >> 4;
-  if (rope.pos) {
-    const int pos = rope.pos[static_cast<size_t>(b) * S + src];
-    const int d = row_bytes / elem_bytes, half = d / 2;
-    for (int i = lane; i < half; i += 32) {
-      float sn, cs;
-      rope_sincos(pos, rope.table.f[i], &sn, &cs);
-      if (elem_bytes == 4) {
-        const float* kf = reinterpret_cast<const float*>(ks);
-        float* kdf = reinterpret_cast<float*>(kd);
-        float x = kf[i], y = kf[i + half];
-        rope_pair(x, y, sn, cs);
-        kdf[i] = x;
-        kdf[i + half] = y;
+  if (ok) {
+    const long long rows = static_cast<long long>(a) * L * Hkv;
+    for (long long row = static_cast<long long>(rank) * kCommitWarps + warp; row < rows;
+         row += static_cast<long long>(CL) * kCommitWarps) {
+      const int kvh = static_cast<int>(row % Hkv);
+      const int r = static_cast<int>((row / Hkv) % a);
+      const int l = static_cast<int>(row / (static_cast<long long>(Hkv) * a));
+      // source: the data slot whose label is r+1
+      const bool hit = lane < gamma && section[static_cast<size_t>(b) * S + lane] == kSectData &&
+                       tau[static_cast<size_t>(b) * S + lane] == r + 1;
+      const unsigned m = __ballot_sync(0xffffffffu, hit);
+      if (!m) {
+        if (lane == 0) raise_error(err_word, SIMSD_EW_STEP_MAP);
+        continue;
+      }
+      const int src = __ffs(m) - 1;
+      const long long dst_row = static_cast<long long>(n) + r;
+      const long long pidx = dst_row / page_size;
+      if (pidx >= max_pages) {
+        if (lane == 0) raise_error(err_word, SIMSD_EW_PAGE);
+        continue;
+      }
+      const int pg = block_table[static_cast<size_t>(b) * max_pages + pidx];
+      if (pg < 0 || pg >= num_pages) {
+        if (lane == 0) raise_error(err_word, SIMSD_EW_PAGE);
+        continue;
+      }
+      const int off = static_cast<int>(dst_row % page_size);
+      const size_t Bt = gridDim.x / CL;
+      const size_t s_row = ((static_cast<size_t>(l) * Bt + b) * S + src) * Hkv + kvh;
+      const size_t d_row = ((static_cast<size_t>(l) * num_pages + pg) * Hkv + kvh) * page_size + off;
+      const uint4* ks = reinterpret_cast<const uint4*>(k_new + s_row * row_bytes);
+      const uint4* vs = reinterpret_cast<const uint4*>(v_new + s_row * row_bytes);
+      uint4* kd = reinterpret_cast<uint4*>(k_cache + d_row * row_bytes);
+      uint4* vd = reinterpret_cast<uint4*>(v_cache + d_row * row_bytes);
+      const int chunks = row_bytes >> 4;
+      if (rope.pos) {
+        const int pos = rope.pos[static_cast<size_t>(b) * S + src];
+        const int d = row_bytes / elem_bytes, half = d / 2;
+        for (int i = lane; i < half; i += 32) {
+          float sn, cs;
+          rope_sincos(pos, rope.table.f[i], &sn, &cs);
+          if (elem_bytes == 4) {
+            const float* kf = reinterpret_cast<const float*>(ks);
+            float* kdf = reinterpret_cast<float*>(kd);
+            float x = kf[i], y = kf[i + half];
+            rope_pair(x, y, sn, cs);
+            kdf[i] = x;
+            kdf[i + half] = y;
+          } else {
+            const __nv_bfloat16* kb = reinterpret_cast<const __nv_bfloat16*>(ks);
+            __nv_bfloat16* kdb = reinterpret_cast<__nv_bfloat16*>(kd);
+            float x = __bfloat162float(kb[i]), y = __bfloat162float(kb[i + half]);
+            rope_pair(x, y, sn, cs);
+            kdb[i] = __float2bfloat16_rn(x);
+            kdb[i + half] = __float2bfloat16_rn(y);
+          }
+        }
+        for (int c = lane; c < chunks; c += 32) vd[c] = vs[c];
       } else {
-        const __nv_bfloat16* kb = reinterpret_cast<const __nv_bfloat16*>(ks);
-        __nv_bfloat16* kdb = reinterpret_cast<__nv_bfloat16*>(kd);
-        float x = __bfloat162float(kb[i]), y = __bfloat162float(kb[i + half]);
-        rope_pair(x, y, sn, cs);
-        kdb[i] = __float2bfloat16_rn(x);
-        kdb[i + half] = __float2bfloat16_rn(y);
+        for (int c = lane; c < chunks; c += 32) {
+          kd[c] = ks[c];
+          vd[c] = vs[c];
+        }
       }
     }
-    for (int c = lane; c < chunks; c += 32) vd[c] = vs[c];
-  } else {
-    for (int c = lane; c < chunks; c += 32) {
-      kd[c] = ks[c];
-      vd[c] = vs[c];
-    }
   }
-}
-
-// n_b += a_b once every copy that read n_b has finished (stream order).
-__global__ void kv_commit_advance_kernel(const int32_t* __restrict__ accepted_len, int32_t* __restrict__ prefix_len,
-                                         int Bt, int gamma, int32_t* err_word) {
-  pdl_wait();
-  pdl_launch_next();
-  const int b = blockIdx.x * blockDim.x + threadIdx.x;
-  if (b >= Bt) return;
-  const int a = accepted_len[b];
-  const int n = prefix_len[b];
-  if (a < 0 || a > gamma) {
-    raise_error(err_word, SIMSD_EW_ACCEPT_LEN);
-    return;
+  // every thread of the cluster has read n_b once this returns
+  asm volatile("barrier.cluster.wait.acquire;" ::: "memory");
+  if (rank == 0 && threadIdx.x == 0) {
+    if (a < 0 || a > gamma)
+      raise_error(err_word, SIMSD_EW_ACCEPT_LEN);
+    else if (n < 0)
+      raise_error(err_word, SIMSD_EW_PREFIX_LEN);
+    else
+      prefix_len[b] = n + a;
   }
-  if (n < 0) {
-    raise_error(err_word, SIMSD_EW_PREFIX_LEN);
-    return;
-  }
-  prefix_len[b] = n + a;
 }
 
 cudaError_t launch_kv_commit(int elem_bytes, const void* k_new, const void* v_new, int L, const int32_t* tau,
@@ -126,19 +133,15 @@ cudaError_t launch_kv_commit(int elem_bytes, const void* k_new, const void* v_ne
                              int num_pages, const int32_t* block_table, int max_pages, int page_size,
                              int32_t* prefix_len, int Bt, int gamma, int Hkv, int d, const int32_t* rope_pos,
                              const RopeTable& rope_table, int32_t* err_word, cudaStream_t stream) {
-  const long long warps = static_cast<long long>(L) * Bt * gamma * Hkv;
-  const long long blocks = (warps + kCommitWarps - 1) / kCommitWarps;
-  if (blocks > 0) {
-    cudaError_t e = launch_overlapped(
-        kv_commit_copy_kernel, dim3(static_cast<unsigned>(blocks)), dim3(kCommitWarps * 32), 0, stream, 1,
-        static_cast<const uint8_t*>(k_new), static_cast<const uint8_t*>(v_new), L, tau, section, accepted_len,
-        static_cast<uint8_t*>(k_cache), static_cast<uint8_t*>(v_cache), num_pages, block_table, max_pages,
-        page_size, prefix_len, Bt, gamma, Hkv, d * elem_bytes, elem_bytes, CommitRope{rope_pos, rope_table},
-        err_word);
-    if (e != cudaSuccess) return e;
-  }
-  return launch_overlapped(kv_commit_advance_kernel, dim3((Bt + 127) / 128), dim3(128), 0, stream, 1, accepted_len,
-                           prefix_len, Bt, gamma, err_word);
+  // about two CTAs per SM in all, at most 8 per sequence (a power of two)
+  int CL = 8;
+  while (CL > 1 && static_cast<long long>(Bt) * CL > 320) CL >>= 1;
+  return launch_overlapped(kv_commit_kernel, dim3(static_cast<unsigned>(Bt) * CL), dim3(kCommitWarps * 32), 0, stream,
+                           static_cast<unsigned>(CL), static_cast<const uint8_t*>(k_new),
+                           static_cast<const uint8_t*>(v_new), L, tau, section, accepted_len,
+                           static_cast<uint8_t*>(k_cache), static_cast<uint8_t*>(v_cache), num_pages, block_table,
+                           max_pages, page_size, prefix_len, gamma, Hkv, d * elem_bytes, elem_bytes,
+                           CommitRope{rope_pos, rope_table}, err_word);
 }
 
 }  // namespace simsd

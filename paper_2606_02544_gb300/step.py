@@ -54,13 +54,18 @@ class VerifyStep:
         self.attn_events = None
 
     # ------------------------------------------------------------------
-    def run(self, attn_events=None):
+    def restore(self):
+        """Puts the original prefix lengths back (a 4*Bt-byte device copy)."""
+        self.n.copy_(self.n_orig, non_blocking=True)
+
+    def run(self, attn_events=None, restore=None):
         """Issues the whole step on the current stream (eager or captured).
         ``attn_events`` = (start, end) events recorded around the layers'
-        attention calls."""
+        attention calls.  ``restore`` (default: the ``restore_prefix``
+        setting) first puts the original prefix lengths back."""
         si, w = self.si, self.w
-        if self.restore_prefix:
-            self.n.copy_(self.n_orig, non_blocking=True)
+        if self.restore_prefix if restore is None else restore:
+            self.restore()
         simsd.simsd_build_mask(si.step_map, self.n, w.gamma, self.tau, self.section, self.rope_pos,
                                err_word=self.err)
         rope = self.rope_pos if self.rope_theta > 0 else None
@@ -82,7 +87,7 @@ class VerifyStep:
     def launches_per_step(self) -> int:
         """Kernels of this library launched by one step."""
         combine = 1 if self.workspace is not None else 0
-        return 1 + self.L * (1 + combine) + 1 + 2
+        return 1 + self.L * (1 + combine) + 1 + 1   # mask, attention (+ combine) per layer, accept, commit
 
     def capture(self, time_attention: bool = True):
         """Captures one step into a CUDA graph (with event-record nodes
