@@ -391,6 +391,108 @@ int oracle_accept(const float *logits, const int32_t *draft, int Bt, int gamma, 
 }
 
 /* ---------------------------------------------------------------------- */
+/* Stochastic acceptance (Sec. 3.2, Eq. (2)).                              */
+/* ---------------------------------------------------------------------- */
+
+/* Softmax of logits/temperature over one row, in double. */
+static void softmax_row(const float *x, int vocab, double inv_t, double *p) {
+    double m = -INFINITY;
+    for (int v = 0; v < vocab; ++v) {
+        double z = (double)x[v] * inv_t;
+        if (z > m) m = z;
+    }
+    double sum = 0.0;
+    for (int v = 0; v < vocab; ++v) {
+        p[v] = exp((double)x[v] * inv_t - m);
+        sum += p[v];
+    }
+    for (int v = 0; v < vocab; ++v) p[v] /= sum;
+}
+
+/* Inverse-CDF draw from the unnormalised weights w[0..vocab): the smallest
+ * v with w[0] + ... + w[v] > u * sum(w).  *margin = distance of u * sum(w)
+ * to the nearest cumulative boundary, relative to sum(w). */
+static int sample_index(const double *w, int vocab, double u, double *margin) {
+    double total = 0.0;
+    for (int v = 0; v < vocab; ++v) total += w[v];
+    double t = u * total, c = 0.0;
+    int pick = vocab - 1;
+    double lo = 0.0, hi = total;
+    for (int v = 0; v < vocab; ++v) {
+        double c2 = c + w[v];
+        if (c2 > t && w[v] > 0.0) {
+            pick = v;
+            lo = c;
+            hi = c2;
+            break;
+        }
+        c = c2;
+    }
+    if (margin) *margin = total > 0.0 ? fmin(t - lo, hi - t) / total : 0.0;
+    return pick;
+}
+
+/* target_logits [Bt][gamma+1][vocab], draft_logits [Bt][gamma][vocab]
+ * (float32); p = softmax(logits / temperature).  For r = 0..gamma-1 the
+ * draft x_r (tau order) is accepted iff u_accept[b][r] < alpha_r =
+ * min(1, p_theta^(r)(x_r) / p_phi^(r)(x_r)) (Eq. (2)), stopping at the first
+ * rejection a.  The token at the first rejected position is drawn from the
+ * residual max(0, p_theta^(a) - p_phi^(a)) renormalised (the
+ * rejection-sampling correction that keeps the target distribution, Sec.
+ * 3.2); when every draft is accepted it is drawn from p_theta^(gamma).  The
+ * draw uses u_sample[b]: the smallest v whose cumulative weight exceeds
+ * u_sample * total.  A draft id outside [0, vocab) sets OR_ERR_DRAFT and is
+ * rejected (alpha 0).
+ * Outputs: accepted_len[Bt], out_tokens[Bt][gamma+1] (accepted drafts, the
+ * drawn token, then -1), alpha[Bt][gamma] (may be NULL; rows past the first
+ * rejection are computed too), margin[Bt] (may be NULL: distance of the
+ * draw's threshold to the nearest cumulative boundary, relative to the
+ * total weight).  Returns the error bits. */
+int oracle_accept_sampled(const float *target_logits, const float *draft_logits, const int32_t *draft,
+                          const float *u_accept, const float *u_sample, double temperature, int Bt, int gamma,
+                          int vocab, int32_t *accepted_len, int32_t *out_tokens, double *alpha, double *margin) {
+    int err = 0;
+    double inv_t = 1.0 / temperature;
+    double *pt = (double *)malloc(sizeof(double) * (size_t)vocab);
+    double *pd = (double *)malloc(sizeof(double) * (size_t)vocab);
+    for (int b = 0; b < Bt; ++b) {
+        int a = gamma;
+        for (int r = 0; r < gamma; ++r) {
+            int x = draft[(size_t)b * gamma + r];
+            double al = 0.0;
+            if (x < 0 || x >= vocab) {
+                err |= OR_ERR_DRAFT;
+            } else {
+                softmax_row(target_logits + ((size_t)b * (gamma + 1) + r) * vocab, vocab, inv_t, pt);
+                softmax_row(draft_logits + ((size_t)b * gamma + r) * vocab, vocab, inv_t, pd);
+                al = pd[x] > 0.0 ? fmin(1.0, pt[x] / pd[x]) : 1.0;
+            }
+            if (alpha) alpha[(size_t)b * gamma + r] = al;
+            if (a == gamma && !((double)u_accept[(size_t)b * gamma + r] < al)) a = r;
+        }
+        accepted_len[b] = a;
+        int32_t *ot = out_tokens + (size_t)b * (gamma + 1);
+        for (int r = 0; r <= gamma; ++r) ot[r] = r < a ? draft[(size_t)b * gamma + r] : -1;
+        softmax_row(target_logits + ((size_t)b * (gamma + 1) + a) * vocab, vocab, inv_t, pt);
+        if (a < gamma) {
+            softmax_row(draft_logits + ((size_t)b * gamma + a) * vocab, vocab, inv_t, pd);
+            double total = 0.0;
+            for (int v = 0; v < vocab; ++v) {
+                pd[v] = fmax(0.0, pt[v] - pd[v]);
+                total += pd[v];
+            }
+            /* an empty residual (p_theta = p_phi) cannot reject; fall back to p_theta */
+            ot[a] = sample_index(total > 0.0 ? pd : pt, vocab, (double)u_sample[b], margin ? margin + b : NULL);
+        } else {
+            ot[a] = sample_index(pt, vocab, (double)u_sample[b], margin ? margin + b : NULL);
+        }
+    }
+    free(pt);
+    free(pd);
+    return err;
+}
+
+/* ---------------------------------------------------------------------- */
 /* Commit of the accepted K/V to the paged cache (Sec. 3.2, Sec. 3.3).     */
 /* ---------------------------------------------------------------------- */
 

@@ -75,6 +75,8 @@ def _load():
             lib.oracle_accept.argtypes = [P, P, i, i, i, P, P, P]
             lib.oracle_kv_commit.argtypes = [i, P, P, i, P, P, P, P, P, i, i, i, P, i, i, i, i,
                                              ctypes.c_double]
+            lib.oracle_accept_sampled.argtypes = [P, P, P, P, P, ctypes.c_double, i, i, i, P, P, P, P]
+            lib.oracle_accept_sampled.restype = ctypes.c_int
             lib.oracle_rope_rotate.argtypes = [P, i, i, ctypes.c_double, ctypes.c_double]
             lib.oracle_rope_rotate.restype = None
             for f in (lib.oracle_build_mask, lib.oracle_verify_attention, lib.oracle_accept,
@@ -198,6 +200,34 @@ def accept(logits, draft, gamma: int):
     am = np.zeros((Bt, gamma + 1), np.int32)
     err = lib.oracle_accept(_ptr(logits), _ptr(draft), Bt, gamma, V, _ptr(a), _ptr(ot), _ptr(am))
     return a, ot, am, int(err)
+
+
+def accept_sampled(target_logits, draft_logits, draft, u_accept, u_sample, gamma: int, temperature: float = 1.0):
+    """Stochastic acceptance, Eq. (2): accept draft r iff u_accept[r] <
+    min(1, p_theta(x_r) / p_phi(x_r)); at the first rejection draw from the
+    residual max(0, p_theta - p_phi), after full acceptance from
+    p_theta^(gamma), by inverse CDF with u_sample.
+
+    target_logits float32 [Bt][gamma+1][V]; draft_logits float32
+    [Bt][gamma][V]; draft int32 [Bt][gamma]; u_accept float32 [Bt][gamma];
+    u_sample float32 [Bt].  Returns (accepted_len, out_tokens, alpha
+    [Bt][gamma] float64, margin [Bt] float64, error bits).
+    """
+    lib = _load()
+    tl = _c(target_logits, np.float32)
+    Bt, rows, V = tl.shape
+    assert rows == gamma + 1
+    dl = _c(draft_logits, np.float32).reshape(Bt, gamma, V)
+    dr = _c(draft, np.int32).reshape(Bt, gamma)
+    ua = _c(u_accept, np.float32).reshape(Bt, gamma)
+    us = _c(u_sample, np.float32).reshape(Bt)
+    a = np.zeros(Bt, np.int32)
+    ot = np.zeros((Bt, gamma + 1), np.int32)
+    al = np.zeros((Bt, gamma), np.float64)
+    mg = np.zeros(Bt, np.float64)
+    err = lib.oracle_accept_sampled(_ptr(tl), _ptr(dl), _ptr(dr), _ptr(ua), _ptr(us), float(temperature), Bt, gamma,
+                                    V, _ptr(a), _ptr(ot), _ptr(al), _ptr(mg))
+    return a, ot, al, mg, int(err)
 
 
 def kv_commit(k_new, v_new, step_map, accepted_len, k_cache, v_cache, block_table, prefix_len,
