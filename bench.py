@@ -33,7 +33,6 @@ UNIT = "tokens/s"
 DEFAULT_WORKLOAD = "c2"
 DEFAULT_STEPS = {"c1": 2000, "c2": 2000, "c3": 400, "c4": 60}
 UNROLL = {"c1": 50, "c2": 50, "c3": 20, "c4": 1}
-L2_BYTES = 129 * 1024 * 1024
 
 
 def _dist_env():
@@ -131,34 +130,12 @@ class ClockSampler:
                 "reasons": sorted(reasons)}
 
 
-def _algorithmic_bytes(si):
-    """Bytes the verification attention must move per layer (read-once):
-    the prefix K/V, Q, K_new/V_new and O; plus the acceptance logits."""
-    w = si.w
-    eb = 4 if w.dtype == "f32" else 2
-    n = si.prefix_len.double().sum().item()
-    kv = n * w.Hkv * w.d * 2 * eb
-    q_o = 2 * w.Bt * w.S * w.Hq * w.d * eb
-    new = 2 * w.Bt * w.S * w.Hkv * w.d * eb
-    meta = w.Bt * (4 + 4 * si.block_table.shape[1] + 5 * w.S)
-    attn = kv + q_o + new + meta
-    flops = 4.0 * w.d * w.Hq * w.S * (n + w.Bt * w.gamma)
-    accept = w.Bt * (w.gamma + 1) * w.vocab * 4.0
-    return attn, flops, accept
-
-
-def _flush_l2(buf):
-    """Evicts the step's data from L2: write a buffer twice the L2 size, then
-    read it back so the dirty lines are written out before the next step."""
-    buf.fill_(1)
-    buf.view(-1, 4096).amax(dim=1)
-
-
 # ----------------------------------------------------------------------------
 def run_gpu(args):
     import torch
 
     from paper_2606_02544_gb300 import build, inputs, simsd
+    from paper_2606_02544_gb300.measure import L2_BYTES, algorithmic_bytes, flush_l2
     from paper_2606_02544_gb300.step import VerifyStep
 
     rank, world, local = _dist_env()
@@ -173,7 +150,7 @@ def run_gpu(args):
     st = VerifyStep(si, restore_prefix=True)
     torch.cuda.synchronize()
 
-    attn_bytes, attn_flops, acc_bytes = _algorithmic_bytes(si)
+    attn_bytes, attn_flops, acc_bytes = algorithmic_bytes(si)
     step_bytes = attn_bytes * st.L + acc_bytes
     need_flush = step_bytes < 4 * L2_BYTES
     flush = torch.empty(2 * L2_BYTES, dtype=torch.uint8, device="cuda") if need_flush else None
@@ -192,7 +169,7 @@ def run_gpu(args):
     with torch.cuda.graph(graph, stream=stream):
         for m in range(M):
             if flush is not None:
-                _flush_l2(flush)
+                flush_l2(flush)
             e = ev[m]
             # the prefix lengths are reset before the step starts (benchmark
             # plumbing that makes every step verify the same block)
@@ -207,7 +184,7 @@ def run_gpu(args):
     g_acc = torch.cuda.CUDAGraph()
     with torch.cuda.graph(g_acc, stream=stream):
         if flush is not None:
-            _flush_l2(flush)
+            flush_l2(flush)
         acc_ev[0].record()
         simsd.simsd_accept(si.logits, si.draft, st.accepted_len, st.out_tokens, st.row_argmax, err_word=st.err)
         acc_ev[1].record()

@@ -640,11 +640,14 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm)
 }
 
 // Merges the prefix splits of every (sequence, KV head, row block):
-// O = sum_i 2^(m_i - M) O_i / sum_i 2^(m_i - M) l_i.  One warp per row.
+// O = sum_i 2^(m_i - M) O_i / sum_i 2^(m_i - M) l_i.  One warp per row; the
+// lanes take the splits' (m, l) in parallel, then sum the partial O rows with
+// lanes over the head dimension (independent loads, several in flight).
 __global__ void __launch_bounds__(128) combine_kernel(const __grid_constant__ TcParams p) {
   pdl_wait();
   pdl_launch_next();
   const int lane = threadIdx.x & 31;
+  const unsigned full = 0xffffffffu;
   const long long wid = (static_cast<long long>(blockIdx.x) * blockDim.x + threadIdx.x) >> 5;
   const long long units = static_cast<long long>(p.Bt) * p.Hkv * p.rb;
   if (wid >= units * p.rows_blk) return;
@@ -658,27 +661,42 @@ __global__ void __launch_bounds__(128) combine_kernel(const __grid_constant__ Tc
   const int h = kvh * p.g + row % p.g;
   const size_t nunits = static_cast<size_t>(units) * p.nsplit;
   const float* wml = p.ws + nunits * p.rows_blk * kD;
+  const size_t e0 = static_cast<size_t>(u) * p.nsplit;
   float M = -INFINITY;
-  for (int i = 0; i < p.nsplit; ++i) {
-    const size_t e = (static_cast<size_t>(u) * p.nsplit + i) * p.rows_blk + row;
+  for (int i = lane; i < p.nsplit; i += 32) {
+    const size_t e = (e0 + i) * p.rows_blk + row;
     if (wml[2 * e + 1] > 0.f) M = fmaxf(M, wml[2 * e]);
   }
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) M = fmaxf(M, __shfl_xor_sync(full, M, o));
   float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
   float L = 0.f;
   if (M != -INFINITY) {
-    for (int i = 0; i < p.nsplit; ++i) {
-      const size_t e = (static_cast<size_t>(u) * p.nsplit + i) * p.rows_blk + row;
-      const float li = wml[2 * e + 1];
-      if (!(li > 0.f)) continue;
-      const float w = exp2f(wml[2 * e] - M);
-      L += w * li;
-      const float4 o = reinterpret_cast<const float4*>(p.ws + e * kD)[lane];
-      acc.x += w * o.x;
-      acc.y += w * o.y;
-      acc.z += w * o.z;
-      acc.w += w * o.w;
+    for (int c0 = 0; c0 < p.nsplit; c0 += 32) {
+      // lane j holds the weight of split c0 + j
+      float wj = 0.f;
+      if (c0 + lane < p.nsplit) {
+        const size_t e = (e0 + c0 + lane) * p.rows_blk + row;
+        const float lj = wml[2 * e + 1];
+        if (lj > 0.f) {
+          wj = exp2f(wml[2 * e] - M);
+          L = fmaf(wj, lj, L);
+        }
+      }
+      const int cnt = min(32, p.nsplit - c0);
+#pragma unroll 4
+      for (int j = 0; j < cnt; ++j) {
+        const float w = __shfl_sync(full, wj, j);
+        const float4 o = reinterpret_cast<const float4*>(p.ws + ((e0 + c0 + j) * p.rows_blk + row) * kD)[lane];
+        acc.x = fmaf(w, o.x, acc.x);
+        acc.y = fmaf(w, o.y, acc.y);
+        acc.z = fmaf(w, o.z, acc.z);
+        acc.w = fmaf(w, o.w, acc.w);
+      }
     }
   }
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) L += __shfl_xor_sync(full, L, o);
   const float inv = L > 0.f ? 1.f / L : 0.f;
   __nv_bfloat16* orow = p.out + ((static_cast<size_t>(b) * p.S + s) * p.Hq + h) * kD;
   uint2 v;

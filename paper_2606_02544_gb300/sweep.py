@@ -1,0 +1,118 @@
+"""The SDAR-8B head-shape sweep: verified tokens/s and the attention's share
+of the HBM copy peak at every point of batch x prefix x draft length x draft
+agreement (32 query / 8 KV heads, d 128, bf16, one layer, V 151936).
+
+    python -m paper_2606_02544_gb300.sweep [--out table.md] [--steps 10]
+        [--batch 1,8,32,128] [--prefix 512,2048,8192,32768]
+        [--gamma 4,8,16,32] [--agree 0.3,0.6,0.9]
+
+One JSON line per point on stdout.  Each point captures its step (mask,
+attention, acceptance, commit; the prefix lengths reset before every step)
+in a CUDA graph and times every step with CUDA events; attention is timed
+by events inside the same graph.  When a step's bytes are below 4x the L2
+size, L2 is flushed before every step.
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import os
+import statistics
+
+import torch
+
+from . import build, inputs, simsd
+from .measure import L2_BYTES, algorithmic_bytes, flush_l2
+from .step import VerifyStep
+
+_HERE = os.path.dirname(os.path.abspath(__file__))
+
+
+def _hbm_peak():
+    try:
+        with open(os.path.join(_HERE, "..", "MEASURED_PEAKS.json")) as f:
+            d = json.load(f)
+        return float(d["hbm_gbs"]), "measured"
+    except Exception:
+        return 6800.0, "fallback"
+
+
+def run_point(w: inputs.Workload, steps: int, peak: float) -> dict:
+    si = inputs.make_step_inputs(w, device="cuda")
+    st = VerifyStep(si, restore_prefix=True)
+    attn_bytes, attn_flops, acc_bytes = algorithmic_bytes(si)
+    need_flush = attn_bytes + acc_bytes < 4 * L2_BYTES
+    flush = torch.empty(2 * L2_BYTES, dtype=torch.uint8, device="cuda") if need_flush else None
+    ev = [[torch.cuda.Event(enable_timing=True, external=True) for _ in range(4)] for _ in range(steps)]
+    stream = torch.cuda.Stream()
+    stream.wait_stream(torch.cuda.current_stream())
+    with torch.cuda.stream(stream):
+        st.run()
+    torch.cuda.synchronize()
+    g = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(g, stream=stream):
+        for e in ev:
+            if flush is not None:
+                flush_l2(flush)
+            st.restore()
+            e[0].record()
+            st.run(attn_events=(e[1], e[2]), restore=False)
+            e[3].record()
+    for _ in range(2):
+        g.replay()
+    torch.cuda.synchronize()
+    step_ms, attn_ms = [], []
+    for _ in range(2):
+        g.replay()
+        torch.cuda.synchronize()
+        step_ms += [e[0].elapsed_time(e[3]) for e in ev]
+        attn_ms += [e[1].elapsed_time(e[2]) for e in ev]
+    assert simsd.simsd_check_error(st.err) == 0
+    tokens = st.verified_tokens()
+    t_step = statistics.median(step_ms)
+    t_attn = statistics.median(attn_ms)
+    gbs = attn_bytes / (t_attn * 1e-3) / 1e9
+    row = {"Bt": w.Bt, "prefix": w.prefix[0], "gamma": w.gamma, "p_agree": w.p_agree,
+           "verified_tokens_per_step": tokens, "tokens_per_s": round(tokens / (t_step * 1e-3), 1),
+           "step_us": round(t_step * 1e3, 2), "attention_us": round(t_attn * 1e3, 2),
+           "attention_gbs": round(gbs, 1), "attention_frac": round(gbs / peak, 4),
+           "attention_tflops": round(attn_flops / (t_attn * 1e-3) / 1e12, 1),
+           "l2": "flushed" if need_flush else "larger than L2"}
+    del g, st, si, flush
+    torch.cuda.empty_cache()
+    return row
+
+
+def main(argv=None):
+    ap = argparse.ArgumentParser(description=__doc__.split("\n\n")[0])
+    ap.add_argument("--out", default=None, help="also write a markdown table here")
+    ap.add_argument("--steps", type=int, default=10)
+    ap.add_argument("--batch", default="1,8,32,128")
+    ap.add_argument("--prefix", default="512,2048,8192,32768")
+    ap.add_argument("--gamma", default="4,8,16,32")
+    ap.add_argument("--agree", default="0.3,0.6,0.9")
+    args = ap.parse_args(argv)
+    sel = lambda s, cast: {cast(x) for x in s.split(",")}
+    bts, ns, gs, ps = sel(args.batch, int), sel(args.prefix, int), sel(args.gamma, int), sel(args.agree, float)
+    build.build()
+    simsd.load_library()
+    peak, kind = _hbm_peak()
+    rows = []
+    for w in inputs.sweep_points():
+        if w.Bt in bts and w.prefix[0] in ns and w.gamma in gs and w.p_agree in ps:
+            row = run_point(w, args.steps, peak)
+            row["peak_gbs"], row["peak_source"] = peak, kind
+            print(json.dumps(row), flush=True)
+            rows.append(row)
+    if args.out:
+        with open(args.out, "w") as f:
+            f.write("| Bt | prefix | gamma | p | tokens/s | step us | attention us | attention GB/s | "
+                    f"of {peak:.0f} GB/s |\n|---|---|---|---|---|---|---|---|---|\n")
+            for r in rows:
+                f.write(f"| {r['Bt']} | {r['prefix']} | {r['gamma']} | {r['p_agree']} | {r['tokens_per_s']:.0f} | "
+                        f"{r['step_us']:.1f} | {r['attention_us']:.1f} | {r['attention_gbs']:.0f} | "
+                        f"{100 * r['attention_frac']:.1f}% |\n")
+
+
+if __name__ == "__main__":
+    main()
