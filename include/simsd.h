@@ -198,6 +198,37 @@ SIMSD_API int simsd_accept(const float* logits, const int32_t* draft, int Bt, in
                  int32_t* out_tokens, int32_t* row_argmax, int32_t* err_word, void* stream);
 
 /*
+ * simsd_accept_sampled -- stochastic acceptance (Sec. 3.2, Eq. (2)): with
+ * p = softmax(logits / temperature), the r-th draft x_r is accepted iff
+ * u_accept[b][r] < alpha_r = min(1, p_theta^(r)(x_r) / p_phi^(r)(x_r)),
+ * along the draft order up to the first rejection.  The token at the first
+ * rejected position a is drawn from the residual max(0, p_theta^(a) -
+ * p_phi^(a)) renormalised (the rejection-sampling correction that keeps the
+ * target distribution; p_theta^(a) itself if the residual is empty to float
+ * precision); when every draft is accepted it is drawn from p_theta of row
+ * gamma.  The draw is an inverse CDF: the smallest token whose cumulative
+ * weight exceeds u_sample[b] times the total.
+ *
+ *   target_logits [Bt][gamma+1][vocab] fp32 (rows in tau order, as for
+ *                 simsd_accept)
+ *   draft_logits  [Bt][gamma][vocab] fp32: the draft model's logits that x_r
+ *                 was drawn from
+ *   draft         [Bt][gamma] int32, in tau order
+ *   u_accept      [Bt][gamma] fp32 uniform draws in [0, 1)
+ *   u_sample      [Bt] fp32 uniform draws in [0, 1)
+ *   temperature   > 0
+ *   accepted_len  [Bt] int32 out; out_tokens [Bt][gamma+1] int32 out: the
+ *                 accepted drafts, the drawn token, then -1.
+ * Probabilities are formed in fp32 from one pass over the logits (row a is
+ * read once more); a draft id outside [0, vocab) sets SIMSD_EW_DRAFT and is
+ * rejected.  No scratch memory is used.
+ */
+SIMSD_API int simsd_accept_sampled(const float* target_logits, const float* draft_logits, const int32_t* draft,
+                                   const float* u_accept, const float* u_sample, float temperature, int Bt, int gamma,
+                                   int vocab, int32_t* accepted_len, int32_t* out_tokens, int32_t* err_word,
+                                   void* stream);
+
+/*
  * simsd_kv_commit -- append the accepted drafts' K/V to the paged cache of
  * every layer (Sec. 3.2: accepted tokens are committed; Sec. 3.3: the cache
  * is reused by later steps).

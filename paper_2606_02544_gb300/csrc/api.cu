@@ -287,6 +287,25 @@ int simsd_accept(const float* logits, const int32_t* draft, int Bt, int gamma, i
   return e == cudaSuccess ? SIMSD_OK : cuda_fail(e, "accept launch");
 }
 
+int simsd_accept_sampled(const float* target_logits, const float* draft_logits, const int32_t* draft,
+                         const float* u_accept, const float* u_sample, float temperature, int Bt, int gamma,
+                         int vocab, int32_t* accepted_len, int32_t* out_tokens, int32_t* err_word, void* stream) {
+  if (Bt < 0) return arg_fail("Bt < 0");
+  if (gamma < 1 || gamma > 32) return arg_fail("gamma must be in [1, 32]");
+  if (vocab < 1 || vocab > (1 << 28)) return arg_fail("vocab must be in [1, 2^28]");
+  if (!(temperature > 0.f) || std::isinf(temperature)) return arg_fail("temperature must be positive and finite");
+  if (Bt == 0) return SIMSD_OK;
+  if (!target_logits || !draft_logits || !draft || !u_accept || !u_sample || !accepted_len || !out_tokens)
+    return arg_fail("null pointer");
+  DeviceInfo info;
+  int rc = require_sm103(&info);
+  if (rc != SIMSD_OK) return rc;
+  cudaError_t e = simsd::launch_accept_sampled(target_logits, draft_logits, draft, u_accept, u_sample, temperature,
+                                               Bt, gamma, vocab, accepted_len, out_tokens, err_word,
+                                               as_stream(stream));
+  return e == cudaSuccess ? SIMSD_OK : cuda_fail(e, "accept_sampled launch");
+}
+
 int simsd_kv_commit(int dtype, const void* k_new, const void* v_new, int L, const int32_t* tau,
                     const uint8_t* section, const int32_t* rope_pos, float rope_theta, const int32_t* accepted_len,
                     void* k_cache, void* v_cache, int num_pages, const int32_t* block_table, int max_pages,

@@ -23,6 +23,11 @@ cudaError_t launch_accept(const float* logits, const int32_t* draft, int Bt, int
                           int32_t* accepted_len, int32_t* out_tokens, int32_t* row_argmax, int32_t* err_word,
                           int num_sms, cudaStream_t stream);
 
+cudaError_t launch_accept_sampled(const float* target_logits, const float* draft_logits, const int32_t* draft,
+                                  const float* u_accept, const float* u_sample, float temperature, int Bt,
+                                  int gamma, int vocab, int32_t* accepted_len, int32_t* out_tokens,
+                                  int32_t* err_word, cudaStream_t stream);
+
 cudaError_t launch_kv_commit(int elem_bytes, const void* k_new, const void* v_new, int L, const int32_t* tau,
                              const uint8_t* section, const int32_t* accepted_len, void* k_cache, void* v_cache,
                              int num_pages, const int32_t* block_table, int max_pages, int page_size,

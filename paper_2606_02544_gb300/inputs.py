@@ -23,7 +23,12 @@ Recipe (one per workload, all values seeded):
   * drafts: with probability p the row's argmax (torch.argmax), otherwise a
     uniform token in [0, V);
   * step map: the identity (left-to-right) unless a random permutation is
-    requested.
+    requested;
+  * stochastic acceptance: target logits ~ N(0, sigma^2); the draft model's
+    logits are the target's plus N(0, (eta sigma)^2) noise (eta sets how
+    often drafts are accepted); each draft is drawn from the draft model's
+    softmax(logits / T) by the Gumbel-max rule (argmax of logits / T plus
+    Gumbel noise); u_accept and u_sample ~ U[0, 1).
 """
 from __future__ import annotations
 
@@ -204,6 +209,34 @@ def make_step_inputs(w: Workload, device="cpu", seed: Optional[int] = None, pref
     dev = torch.device(device)
     return StepInputs(w, n.to(dev), bt.to(dev), num_pages, sm.to(dev), q, k_new, v_new, k_cache, v_cache,
                       logits, draft.to(dev), row_valid)
+
+
+@dataclasses.dataclass
+class SampledInputs:
+    target_logits: torch.Tensor   # fp32 [Bt][gamma+1][V]
+    draft_logits: torch.Tensor    # fp32 [Bt][gamma][V]
+    draft: torch.Tensor           # int32 [Bt][gamma]
+    u_accept: torch.Tensor        # fp32 [Bt][gamma]
+    u_sample: torch.Tensor        # fp32 [Bt]
+    temperature: float
+
+
+def make_sampled_inputs(Bt: int, gamma: int, vocab: int, seed: int, logit_std: float = 2.0, eta: float = 0.5,
+                        temperature: float = 1.0, device="cpu") -> SampledInputs:
+    """Inputs of the stochastic acceptance; drawn on the CPU so that they
+    do not depend on the device."""
+    g = _cpu_gen(seed)
+    tl = torch.randn(Bt, gamma + 1, vocab, generator=g) * logit_std
+    dl = tl[:, :gamma] + torch.randn(Bt, gamma, vocab, generator=g) * (eta * logit_std)
+    # Gumbel-max: argmax(l / T + G), G = -log(-log U), U ~ U(0, 1)
+    uu = torch.rand(Bt, gamma, vocab, generator=g, dtype=torch.float64).clamp_(1e-300, 1.0 - 1e-16)
+    draft = torch.argmax(dl.double() / temperature - torch.log(-torch.log(uu)), dim=-1).to(torch.int32)
+    del uu
+    ua = torch.rand(Bt, gamma, generator=g)
+    us = torch.rand(Bt, generator=g)
+    dev = torch.device(device)
+    return SampledInputs(tl.contiguous().to(dev), dl.contiguous().to(dev), draft.to(dev), ua.to(dev), us.to(dev),
+                         float(temperature))
 
 
 def host_bits(t: torch.Tensor) -> np.ndarray:

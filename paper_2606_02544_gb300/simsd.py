@@ -24,7 +24,8 @@ SECT_DATA, SECT_MASK, SECT_PAD = 0, 1, 255
 EW_STEP_MAP, EW_PREFIX_LEN, EW_PAGE, EW_DRAFT, EW_TIMEOUT, EW_ACCEPT_LEN = 1, 2, 4, 8, 16, 32
 
 EXPORTED = ("simsd_build_mask", "simsd_verify_workspace_bytes", "simsd_verify_attention",
-            "simsd_verify_attention_noalloc", "simsd_accept", "simsd_kv_commit", "simsd_check_error",
+            "simsd_verify_attention_noalloc", "simsd_accept", "simsd_accept_sampled", "simsd_kv_commit",
+            "simsd_check_error",
             "simsd_last_error", "simsd_version")
 
 
@@ -56,11 +57,13 @@ def load_library(path: str = LIB_PATH):
             lib.simsd_verify_attention_noalloc.argtypes = [I, P, P, P, P, P, I, P, I, I, P, P, P, P, F, I, I, I, I,
                                                            I, F, P, P, P]
             lib.simsd_accept.argtypes = [P, P, I, I, I, P, P, P, P, P]
+            lib.simsd_accept_sampled.argtypes = [P, P, P, P, P, F, I, I, I, P, P, P, P]
             lib.simsd_kv_commit.argtypes = [I, P, P, I, P, P, P, F, P, P, P, I, P, I, I, P, I, I, I, I, P, P]
             lib.simsd_check_error.argtypes = [P, P, P]
             lib.simsd_last_error.restype = ctypes.c_char_p
             for name in ("simsd_build_mask", "simsd_verify_attention", "simsd_verify_attention_noalloc",
-                         "simsd_accept", "simsd_kv_commit", "simsd_check_error", "simsd_version"):
+                         "simsd_accept", "simsd_accept_sampled", "simsd_kv_commit", "simsd_check_error",
+                         "simsd_version"):
                 getattr(lib, name).restype = ctypes.c_int
             _lib = lib
     return _lib
@@ -143,6 +146,17 @@ def simsd_accept(logits, draft, accepted_len, out_tokens, row_argmax=None, err_w
     rc = load_library().simsd_accept(_p(logits), _p(draft), Bt, rows - 1, V, _p(accepted_len), _p(out_tokens),
                                      _p(row_argmax), _p(err_word), _stream(stream))
     _check(rc, "simsd_accept")
+
+
+def simsd_accept_sampled(target_logits, draft_logits, draft, u_accept, u_sample, accepted_len, out_tokens,
+                         temperature=1.0, err_word=None, stream=None):
+    """target_logits [Bt][g+1][V], draft_logits [Bt][g][V] fp32; draft [Bt][g];
+    u_accept [Bt][g], u_sample [Bt] fp32 uniform draws."""
+    Bt, rows, V = target_logits.shape
+    rc = load_library().simsd_accept_sampled(_p(target_logits), _p(draft_logits), _p(draft), _p(u_accept),
+                                             _p(u_sample), float(temperature), Bt, rows - 1, V, _p(accepted_len),
+                                             _p(out_tokens), _p(err_word), _stream(stream))
+    _check(rc, "simsd_accept_sampled")
 
 
 def simsd_kv_commit(k_new, v_new, tau, section, accepted_len, k_cache, v_cache, block_table, prefix_len,

@@ -58,6 +58,12 @@ def test_host_validation_without_gpu(lib):
     assert rc == 1
     # vocab out of range
     assert lib.simsd_accept(one, one, 1, 4, 0, one, one, None, None, None) == 1
+    # stochastic acceptance: temperature must be positive and finite, gamma in [1, 32]
+    for t, g, v in ((0.0, 4, 10), (-1.0, 4, 10), (float("inf"), 4, 10), (float("nan"), 4, 10), (1.0, 0, 10),
+                    (1.0, 33, 10), (1.0, 4, 0)):
+        assert lib.simsd_accept_sampled(one, one, one, one, one, F(t), 1, g, v, one, one, None, None) == 1
+    assert lib.simsd_accept_sampled(one, None, one, one, one, F(1.0), 1, 4, 10, one, one, None, None) == 1
+    assert lib.simsd_accept_sampled(None, None, None, None, None, F(1.0), 0, 4, 10, None, None, None, None) == 0
     # empty batches are no-ops that touch nothing
     assert lib.simsd_accept(None, None, 0, 4, 10, None, None, None, None, None) == 0
     assert lib.simsd_check_error(None, None, None) == 1
