@@ -216,7 +216,7 @@ SIMSD_API int simsd_accept(const float* logits, const int32_t* draft, int Bt, in
  *   draft         [Bt][gamma] int32, in tau order
  *   u_accept      [Bt][gamma] fp32 uniform draws in [0, 1)
  *   u_sample      [Bt] fp32 uniform draws in [0, 1)
- *   temperature   > 0
+ *   temperature   > 0;  vocab in [1, 2^24]
  *   accepted_len  [Bt] int32 out; out_tokens [Bt][gamma+1] int32 out: the
  *                 accepted drafts, the drawn token, then -1.
  * Probabilities are formed in fp32 from one pass over the logits (row a is

@@ -7,22 +7,24 @@
 //
 // One thread-block cluster per sequence.  Phase 1: the sequence's gamma+1
 // target rows and gamma draft rows are laid end to end, each row padded to a
-// multiple of 32 units (a unit is 4 or 1 floats), and the CTAs take
-// contiguous spans of warp-aligned units, so the 32 lanes of a warp are always
-// on the same row.  Each lane keeps the running maximum m of z = x*log2(e)/T
-// and s = sum 2^(z - m) of the row it is on; when the warp moves to the next
-// row it merges its lanes by shuffles and stores the pair in a per-warp slot
+// multiple of 32 units (a unit is 4 floats, or 1 when rows are not 16-byte
+// aligned), and the CTAs take contiguous spans of warp-aligned units, so the
+// 32 lanes of a warp are always on the same row.  Each lane keeps the running
+// maximum m of z = x*log2(e)/T and s = sum 2^(z - m) of its row; when the warp
+// moves to the next row it merges its lanes by shuffles into a per-warp slot
 // (no atomics).  CTA 0 merges the warps' and the CTAs' pairs (distributed
-// shared memory), forms alpha_r from the drafts' own logits and the accepted
-// length a, and broadcasts a.  Phase 2: each CTA takes a column range of row
-// a and each thread a contiguous run of it; the thread sums the weights of
-// its run.  CTA 0 forms the threshold u_sample * total and names the CTA
-// whose range holds it; that CTA scans its threads' sums, and the one thread
-// whose run holds the threshold walks it.  Row a is read a second time (2 of
-// the 2*gamma+1 rows); no global scratch memory is used.
+// shared memory), forms alpha_r from the drafts' own logits (fetched at the
+// start, while phase 1 streams) and the accepted length a, and broadcasts a.
+// Phase 2: each CTA takes a range of row a and each warp a contiguous part
+// of that, and sums the weights of its part (coalesced, 16-byte loads).  CTA
+// 0 forms the threshold u_sample * total and names the CTA whose range holds
+// it; in that CTA the warp whose part holds it walks the part in order, 32
+// units a step, with a warp scan.  Row a is read a second time (2 of the
+// 2*gamma+1 rows); no global scratch memory is used.
 #include <cooperative_groups.h>
 #include <cuda_runtime.h>
 
+#include <cfloat>
 #include <mutex>
 
 #include "common.cuh"
@@ -37,23 +39,31 @@ constexpr int kSampThreads = 512;
 constexpr int kSampWarps = kSampThreads / 32;
 constexpr int kSampUnroll = 8;
 constexpr int kSampMaxRows = 65;  // 2*gamma+1 <= 65
+constexpr int kSampMaxCluster = 16;
 constexpr float kLog2e = 1.4426950408889634f;
+// The running maximum starts at -FLT_MAX rather than -inf: 2^(z - m) is then
+// 0 for z = -inf (a masked logit) without a special case, and merging two
+// empty pairs gives an empty pair (s = 0).
+constexpr float kEmpty = -FLT_MAX;
 // A residual whose total is at most this is empty: p_theta and p_phi agree
 // to fp32 precision (each probability carries a relative error of a few
-// units of 2^-24, the row sums about 1e-6), so what is left is rounding.
+// units of 2^-22, the row sums about 1e-6), so what is left is rounding.
 constexpr float kResidFloor = 1.0f / 65536.0f;
 
+// 2^x by the PTX approximation (relative error about 2^-22; results below
+// 2^-126 flush to 0, far below any weight that matters in a row whose
+// largest weight is 1).
+__device__ __forceinline__ float ex2(float x) {
+  float y;
+  asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
+  return y;
+}
+
 // Merges two (m, s) pairs of a base-2 log-sum-exp: s = s1 2^(m1 - M) +
-// s2 2^(m2 - M), M = max; m = -inf stands for an empty set.
+// s2 2^(m2 - M), M = max(m1, m2).
 __device__ __forceinline__ void ms_merge(float& m, float& s, float m2, float s2) {
-  if (m2 == -INFINITY) return;
-  if (m == -INFINITY) {
-    m = m2;
-    s = s2;
-    return;
-  }
   const float M = fmaxf(m, m2);
-  s = s * exp2f(m - M) + s2 * exp2f(m2 - M);
+  s = s * ex2(m - M) + s2 * ex2(m2 - M);
   m = M;
 }
 
@@ -65,6 +75,13 @@ __device__ __forceinline__ float4 ld_stream_f4(const float* p) {
   return v;
 }
 
+__device__ __forceinline__ void cp_async4(void* smem, const void* gmem) {
+  const unsigned sa = static_cast<unsigned>(__cvta_generic_to_shared(smem));
+  asm volatile("cp.async.ca.shared.global [%0], [%1], 4;" ::"r"(sa), "l"(gmem) : "memory");
+}
+
+__device__ __forceinline__ void cp_async_wait_all() { asm volatile("cp.async.wait_all;" ::: "memory"); }
+
 // Row `row` of the combined row space: target rows 0..gamma, then draft rows.
 __device__ __forceinline__ const float* row_ptr(const float* tgt, const float* drf, int b, int gamma, int vocab,
                                                 int row) {
@@ -72,20 +89,30 @@ __device__ __forceinline__ const float* row_ptr(const float* tgt, const float* d
                       : drf + (static_cast<size_t>(b) * gamma + (row - gamma - 1)) * vocab;
 }
 
+template <bool VEC>
+__device__ __forceinline__ float4 load_unit(const float* rp, int col) {
+  if constexpr (VEC) {
+    return ld_stream_f4(rp + 4 * col);
+  } else {
+    return make_float4(__ldg(rp + col), -INFINITY, -INFINITY, -INFINITY);
+  }
+}
+
+template <bool VEC>
 __global__ void __launch_bounds__(kSampThreads, 2) accept_sampled_kernel(
     const float* __restrict__ tgt, const float* __restrict__ drf, const int32_t* __restrict__ draft,
     const float* __restrict__ u_accept, const float* __restrict__ u_sample, float zscale, int gamma, int vocab,
-    int vec4, int32_t* __restrict__ accepted_len, int32_t* __restrict__ out_tokens, int32_t* err_word) {
+    int32_t* __restrict__ accepted_len, int32_t* __restrict__ out_tokens, int32_t* err_word) {
   __shared__ float2 part[kSampWarps][kSampMaxRows];  // per warp (m, s) of each row
   __shared__ float2 cta_ms[kSampMaxRows];            // this CTA's (m, s) of each row
   __shared__ float row_m[kSampMaxRows], row_s[kSampMaxRows];
-  __shared__ float tsum[kSampThreads];               // phase 2: each thread's run total
   __shared__ float warp_tot[kSampWarps];
+  __shared__ float zt_sh[32], zd_sh[32], ua_sh[32];  // CTA 0: the drafts' logits and u_accept
+  __shared__ float us_sh;                            // CTA 0: u_sample
   __shared__ int a_sh;
   __shared__ float w_cta;          // this CTA's weight of row a
   __shared__ float w_off, w_thr;   // the owner's offset and threshold (-1 elsewhere), set by CTA 0
   __shared__ int w_state;          // 1: the total weight was positive (set by CTA 0)
-  __shared__ int pick_t, last_t;   // phase 2 owner thread
   pdl_wait();
   pdl_launch_next();
   cg::cluster_group cluster = cg::this_cluster();
@@ -96,21 +123,38 @@ __global__ void __launch_bounds__(kSampThreads, 2) accept_sampled_kernel(
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   const unsigned full = 0xffffffffu;
   for (int i = tid; i < kSampWarps * kSampMaxRows; i += kSampThreads)
-    part[i / kSampMaxRows][i % kSampMaxRows] = make_float2(-INFINITY, 0.f);
+    part[i / kSampMaxRows][i % kSampMaxRows] = make_float2(kEmpty, 0.f);
+  // CTA 0, warp 0: the drafts, their two logits and the uniforms, fetched now
+  // so that their latency hides behind phase 1
+  bool bad = false;
+  if (c == 0 && warp == 0) {
+    if (lane < gamma) {
+      const int x = draft[static_cast<size_t>(b) * gamma + lane];
+      ua_sh[lane] = u_accept[static_cast<size_t>(b) * gamma + lane];
+      bad = x < 0 || x >= vocab;
+      if (!bad) {
+        cp_async4(&zt_sh[lane], tgt + (static_cast<size_t>(b) * (gamma + 1) + lane) * vocab + x);
+        cp_async4(&zd_sh[lane], drf + (static_cast<size_t>(b) * gamma + lane) * vocab + x);
+      }
+    }
+    if (lane == 31) us_sh = u_sample[b];
+  }
   __syncthreads();
 
   // ---- phase 1: per-row (m, s) over this CTA's span of warp-aligned units
   {
-    const int W = vec4 ? (vocab >> 2) : vocab;  // units per row
-    const int Wp = (W + 31) & ~31;              // padded: a warp never straddles two rows
-    const long long G = static_cast<long long>(rows) * (Wp >> 5);  // groups of 32 units
-    const long long per = (G + CL - 1) / CL;
-    const long long f0 = 32 * min(G, c * per), f1 = 32 * min(G, c * per + per);
-    long long f = f0 + tid;
-    int row = static_cast<int>(f / Wp);
-    int col = static_cast<int>(f - static_cast<long long>(row) * Wp);
+    const int W = VEC ? (vocab >> 2) : vocab;  // units per row
+    const int Wp = (W + 31) & ~31;             // padded: a warp never straddles two rows
+    const int G = rows * (Wp >> 5);            // groups of 32 units
+    const int per = (G + CL - 1) / CL;
+    const int f0 = 32 * min(G, c * per), f1 = 32 * min(G, c * per + per);
+    constexpr int kStep = kSampThreads;
+    int f = f0 + tid;
+    int row = f / Wp;
+    int col = f - row * Wp;
+    const float* rp = row_ptr(tgt, drf, b, gamma, vocab, min(row, rows - 1));
     int cur = row;
-    float m = -INFINITY, s = 0.f;
+    float m = kEmpty, s = 0.f;
     // merges the warp's lanes (all on row `cur`) into its slot
     auto flush = [&]() {
 #pragma unroll
@@ -124,29 +168,38 @@ __global__ void __launch_bounds__(kSampThreads, 2) accept_sampled_kernel(
         part[warp][cur] = p;
       }
     };
-    // f, f0, f1 and Wp are multiples of 32 at the warp's first lane, so every
-    // test below is the same for the 32 lanes of a warp
-    for (; f < f1; f += static_cast<long long>(kSampThreads) * kSampUnroll) {
+    auto advance = [&](int by) {
+      col += by;
+      if (col >= Wp) {
+        do {
+          col -= Wp;
+          ++row;
+        } while (col >= Wp);
+        rp = row_ptr(tgt, drf, b, gamma, vocab, min(row, rows - 1));
+      }
+    };
+    // f0, f1, Wp and the f and col of a warp's first lane are multiples of
+    // 32, so every test below is the same for the 32 lanes of a warp
+    for (; f < f1; f += kStep * kSampUnroll) {
       float4 v[kSampUnroll];
       int vr[kSampUnroll];
+      if (f - lane + kStep * (kSampUnroll - 1) < f1 && col - lane + kStep * (kSampUnroll - 1) + 31 < W) {
+        // the common case: every unit valid, on one row, inside the row
 #pragma unroll
-      for (int u = 0; u < kSampUnroll; ++u) {
-        vr[u] = -1;
-        if (f + static_cast<long long>(u) * kSampThreads < f1) {
+        for (int u = 0; u < kSampUnroll; ++u) {
+          v[u] = load_unit<VEC>(rp, col + u * kStep);
           vr[u] = row;
-          v[u] = make_float4(-INFINITY, -INFINITY, -INFINITY, -INFINITY);
-          if (col < W) {
-            const float* rp = row_ptr(tgt, drf, b, gamma, vocab, row);
-            if (vec4)
-              v[u] = ld_stream_f4(rp + 4 * col);
-            else
-              v[u].x = __ldg(rp + col);
-          }
         }
-        col += kSampThreads;
-        if (col >= Wp) {
-          row += col / Wp;
-          col %= Wp;
+        advance(kStep * kSampUnroll);
+      } else {
+#pragma unroll
+        for (int u = 0; u < kSampUnroll; ++u) {
+          vr[u] = -1;
+          if (f + u * kStep < f1) {
+            vr[u] = row;
+            v[u] = col < W ? load_unit<VEC>(rp, col) : make_float4(-INFINITY, -INFINITY, -INFINITY, -INFINITY);
+          }
+          advance(kStep);
         }
       }
 #pragma unroll
@@ -155,26 +208,25 @@ __global__ void __launch_bounds__(kSampThreads, 2) accept_sampled_kernel(
         if (vr[u] != cur) {
           flush();
           cur = vr[u];
-          m = -INFINITY;
+          m = kEmpty;
           s = 0.f;
         }
-        const float z0 = v[u].x * zscale, z1 = v[u].y * zscale, z2 = v[u].z * zscale, z3 = v[u].w * zscale;
-        const float mz = fmaxf(fmaxf(z0, z1), fmaxf(z2, z3));
+        const float mz = fmaxf(fmaxf(v[u].x, v[u].y), fmaxf(v[u].z, v[u].w)) * zscale;
         if (mz > m) {
-          s = (m == -INFINITY) ? 0.f : s * exp2f(m - mz);
+          s *= ex2(m - mz);
           m = mz;
         }
-        // a logit of -inf has weight 0: while m is still -inf the exponent
-        // is taken against 0, so that -inf - -inf never occurs
-        const float mr = m == -INFINITY ? 0.f : m;
-        s += exp2f(z0 - mr) + exp2f(z1 - mr) + exp2f(z2 - mr) + exp2f(z3 - mr);
+        const float nm = -m;
+        s += ex2(fmaf(v[u].x, zscale, nm)) + ex2(fmaf(v[u].y, zscale, nm)) + ex2(fmaf(v[u].z, zscale, nm)) +
+             ex2(fmaf(v[u].w, zscale, nm));
       }
     }
     if (f0 + 32 * warp < f1) flush();
   }
   __syncthreads();
   for (int r = tid; r < rows; r += kSampThreads) {
-    float m = -INFINITY, s = 0.f;
+    float m = kEmpty, s = 0.f;
+#pragma unroll
     for (int w = 0; w < kSampWarps; ++w) ms_merge(m, s, part[w][r].x, part[w][r].y);
     cta_ms[r] = make_float2(m, s);
   }
@@ -182,123 +234,133 @@ __global__ void __launch_bounds__(kSampThreads, 2) accept_sampled_kernel(
 
   // ---- CTA 0: merge the CTAs, alpha_r, accepted length
   if (c == 0) {
-    for (int r = tid; r < rows; r += kSampThreads) {
-      float m = -INFINITY, s = 0.f;
-      for (int peer = 0; peer < CL; ++peer) {
-        const float2 v = *cluster.map_shared_rank(&cta_ms[r], peer);
-        ms_merge(m, s, v.x, v.y);
+    // warp w merges rows w, w+16, ...; lane p reads CTA p's pair
+    constexpr int kRowsPerWarp = (kSampMaxRows + kSampWarps - 1) / kSampWarps;
+    float2 pv[kRowsPerWarp];
+#pragma unroll
+    for (int j = 0; j < kRowsPerWarp; ++j) {
+      const int r = warp + kSampWarps * j;
+      pv[j] = (r < rows && lane < CL) ? *cluster.map_shared_rank(&cta_ms[r], lane) : make_float2(kEmpty, 0.f);
+    }
+#pragma unroll
+    for (int j = 0; j < kRowsPerWarp; ++j) {
+      const int r = warp + kSampWarps * j;
+      if (r < rows) {  // the same for the whole warp
+        float m = pv[j].x, s = pv[j].y;
+#pragma unroll
+        for (int o = 16; o > 0; o >>= 1) {
+          const float m2 = __shfl_xor_sync(full, m, o), s2 = __shfl_xor_sync(full, s, o);
+          ms_merge(m, s, m2, s2);
+        }
+        if (lane == 0) {
+          row_m[r] = m;
+          row_s[r] = s;
+        }
       }
-      row_m[r] = m;
-      row_s[r] = s;
     }
     __syncthreads();
     if (warp == 0) {
-      bool acc = false, bad = false;
-      if (lane < gamma) {
-        const int x = draft[static_cast<size_t>(b) * gamma + lane];
-        if (x < 0 || x >= vocab) {
-          bad = true;
-        } else {
-          // log2 of p_theta(x) / p_phi(x)
-          const float zt = __ldg(tgt + (static_cast<size_t>(b) * (gamma + 1) + lane) * vocab + x) * zscale;
-          const float zd = __ldg(drf + (static_cast<size_t>(b) * gamma + lane) * vocab + x) * zscale;
-          const int rd = gamma + 1 + lane;
-          const float lr = (zt - row_m[lane] - log2f(row_s[lane])) - (zd - row_m[rd] - log2f(row_s[rd]));
-          const float alpha = lr >= 0.f ? 1.f : exp2f(lr);
-          acc = u_accept[static_cast<size_t>(b) * gamma + lane] < alpha;
-        }
+      cp_async_wait_all();
+      __syncwarp();
+      bool acc = false;
+      if (lane < gamma && !bad) {
+        // log2 of p_theta(x) / p_phi(x)
+        const int rd = gamma + 1 + lane;
+        const float lr = (zt_sh[lane] * zscale - row_m[lane] - log2f(row_s[lane])) -
+                         (zd_sh[lane] * zscale - row_m[rd] - log2f(row_s[rd]));
+        const float alpha = lr >= 0.f ? 1.f : exp2f(lr);
+        acc = ua_sh[lane] < alpha;
       }
       const unsigned rej = __ballot_sync(full, lane < gamma && !acc);
       if (__any_sync(full, bad) && lane == 0) raise_error(err_word, SIMSD_EW_DRAFT);
       const int a = rej ? __ffs(rej) - 1 : gamma;
-      if (lane == 0) {
-        accepted_len[b] = a;
-        for (int peer = 0; peer < CL; ++peer) *cluster.map_shared_rank(&a_sh, peer) = a;
-      }
+      if (lane == 0) accepted_len[b] = a;
       int32_t* ot = out_tokens + static_cast<size_t>(b) * (gamma + 1);
       for (int r = lane; r <= gamma; r += 32)
         if (r != a) ot[r] = r < a ? draft[static_cast<size_t>(b) * gamma + r] : -1;
-      // the merged (m, s) of the rows phase 2 needs, for every CTA
-      if (lane < 2) {
-        const int rr = lane == 0 ? a : gamma + 1 + a;
-        if (lane == 0 || a < gamma)
-          for (int peer = 0; peer < CL; ++peer) {
-            *cluster.map_shared_rank(&row_m[rr], peer) = row_m[rr];
-            *cluster.map_shared_rank(&row_s[rr], peer) = row_s[rr];
-          }
+      // a and the merged (m, s) of the rows phase 2 needs, to every CTA
+      if (lane < CL) {
+        const int rd = gamma + 1 + a;
+        *cluster.map_shared_rank(&a_sh, lane) = a;
+        *cluster.map_shared_rank(&row_m[a], lane) = row_m[a];
+        *cluster.map_shared_rank(&row_s[a], lane) = row_s[a];
+        if (a < gamma) {
+          *cluster.map_shared_rank(&row_m[rd], lane) = row_m[rd];
+          *cluster.map_shared_rank(&row_s[rd], lane) = row_s[rd];
+        }
       }
     }
   }
   cluster.sync();
 
-  // ---- phase 2: weights of row a; CTA c takes a column range, each thread a
-  // contiguous run of it
+  // ---- phase 2: weights of row a.  CTA c takes a range of units of the
+  // row, warp w a contiguous part of that, and the lanes stride through it.
   const int a = a_sh;
   bool resid = a < gamma;
   const float* trow = tgt + (static_cast<size_t>(b) * (gamma + 1) + a) * vocab;
-  const float* drow = a < gamma ? drf + (static_cast<size_t>(b) * gamma + a) * vocab : nullptr;
-  const float mt = row_m[a], it = 1.f / row_s[a];
-  const float md = a < gamma ? row_m[gamma + 1 + a] : 0.f, id = a < gamma ? 1.f / row_s[gamma + 1 + a] : 0.f;
-  const int per = (vocab + CL - 1) / CL;
-  const int v0 = min(vocab, c * per), v1 = min(vocab, v0 + per);
-  const int q = (v1 - v0 + kSampThreads - 1) / kSampThreads;
-  const int r0 = min(v1, v0 + tid * q), r1 = min(v1, r0 + q);
-  auto weight = [&](int v) -> float {
-    const float pt = exp2f(__ldg(trow + v) * zscale - mt) * it;
-    if (!resid) return pt;
-    const float pd = exp2f(__ldg(drow + v) * zscale - md) * id;
-    return fmaxf(0.f, pt - pd);
+  const float* drow = a < gamma ? drf + (static_cast<size_t>(b) * gamma + a) * vocab : trow;
+  const float nmt = -row_m[a], it = 1.f / row_s[a];
+  const float nmd = a < gamma ? -row_m[gamma + 1 + a] : 0.f, id = a < gamma ? 1.f / row_s[gamma + 1 + a] : 0.f;
+  const int W = VEC ? (vocab >> 2) : vocab;
+  const int per_c = (W + CL - 1) / CL;
+  const int c0 = min(W, c * per_c), c1 = min(W, c0 + per_c);
+  const int per_w = (c1 - c0 + kSampWarps - 1) / kSampWarps;
+  const int w0 = min(c1, c0 + warp * per_w), w1 = min(c1, w0 + per_w);
+  // the four weights of a unit (the scalar layout has one column per unit)
+  auto weights = [&](int unit) -> float4 {
+    const float4 xt = load_unit<VEC>(trow, unit);
+    float4 w = make_float4(ex2(fmaf(xt.x, zscale, nmt)) * it, ex2(fmaf(xt.y, zscale, nmt)) * it,
+                           ex2(fmaf(xt.z, zscale, nmt)) * it, ex2(fmaf(xt.w, zscale, nmt)) * it);
+    if (resid) {
+      const float4 xd = load_unit<VEC>(drow, unit);
+      w.x = fmaxf(0.f, w.x - ex2(fmaf(xd.x, zscale, nmd)) * id);
+      w.y = fmaxf(0.f, w.y - ex2(fmaf(xd.y, zscale, nmd)) * id);
+      w.z = fmaxf(0.f, w.z - ex2(fmaf(xd.z, zscale, nmd)) * id);
+      w.w = fmaxf(0.f, w.w - ex2(fmaf(xd.w, zscale, nmd)) * id);
+    }
+    return w;
   };
   // an empty residual (p_theta = p_phi to fp32 precision) cannot reject:
   // the draw then falls back to p_theta (second pass)
-  float ts = 0.f;
   for (int pass = 0; pass < 2; ++pass) {
-    ts = 0.f;
+    float ws = 0.f;
 #pragma unroll 4
-    for (int v = r0; v < r1; ++v) ts += weight(v);
-    float ws = ts;
+    for (int u = w0 + lane; u < w1; u += 32) {
+      const float4 w = weights(u);
+      ws += (w.x + w.y) + (w.z + w.w);
+    }
 #pragma unroll
     for (int o = 16; o > 0; o >>= 1) ws += __shfl_xor_sync(full, ws, o);
     if (lane == 0) warp_tot[warp] = ws;
     __syncthreads();
     if (tid == 0) {
       float t = 0.f;
+#pragma unroll
       for (int w = 0; w < kSampWarps; ++w) t += warp_tot[w];
       w_cta = t;
     }
     cluster.sync();
-    if (c == 0 && tid == 0) {
-      // the threshold and the CTA whose range holds it: the first with
-      // positive weight whose range ends past it, else (rounding) the last
-      // with positive weight
-      float wc[16];
-      float total = 0.f;
-      for (int peer = 0; peer < CL; ++peer) {
-        wc[peer] = *cluster.map_shared_rank(&w_cta, peer);
-        total += wc[peer];
+    if (c == 0 && warp == 0) {
+      // lane p holds CTA p's weight; the threshold and the CTA whose range
+      // holds it: the first with positive weight whose range ends past it,
+      // else (rounding) the last with positive weight
+      const float wc = lane < CL ? *cluster.map_shared_rank(&w_cta, lane) : 0.f;
+      float incl = wc;
+#pragma unroll
+      for (int o = 1; o < 32; o <<= 1) {
+        const float y = __shfl_up_sync(full, incl, o);
+        if (lane >= o) incl += y;
       }
-      const float thr = u_sample[b] * total;
-      int owner = -1, last = -1;
-      float off = 0.f, own_off = 0.f, last_off = 0.f;
-      for (int peer = 0; peer < CL; ++peer) {
-        if (wc[peer] > 0.f) {
-          if (owner < 0 && thr < off + wc[peer]) {
-            owner = peer;
-            own_off = off;
-          }
-          last = peer;
-          last_off = off;
-        }
-        off += wc[peer];
-      }
-      if (owner < 0) {
-        owner = last;
-        own_off = last_off;
-      }
-      for (int peer = 0; peer < CL; ++peer) {
-        *cluster.map_shared_rank(&w_state, peer) = total > (resid ? kResidFloor : 0.f) ? 1 : 0;
-        *cluster.map_shared_rank(&w_thr, peer) = peer == owner ? thr : -1.f;
-        *cluster.map_shared_rank(&w_off, peer) = own_off;
+      const float total = __shfl_sync(full, incl, 31);
+      const float thr = us_sh * total;
+      const unsigned hold = __ballot_sync(full, wc > 0.f && thr < incl);
+      const unsigned pos = __ballot_sync(full, wc > 0.f);
+      const int owner = hold ? __ffs(hold) - 1 : (pos ? 31 - __clz(pos) : -1);
+      const float own_off = __shfl_sync(full, incl - wc, owner < 0 ? 0 : owner);
+      if (lane < CL) {
+        *cluster.map_shared_rank(&w_state, lane) = total > (resid ? kResidFloor : 0.f) ? 1 : 0;
+        *cluster.map_shared_rank(&w_thr, lane) = lane == owner ? thr : -1.f;
+        *cluster.map_shared_rank(&w_off, lane) = own_off;
       }
     }
     cluster.sync();
@@ -309,44 +371,71 @@ __global__ void __launch_bounds__(kSampThreads, 2) accept_sampled_kernel(
   if (!w_state && c == 0 && tid == 0) out_tokens[static_cast<size_t>(b) * (gamma + 1) + a] = -1;
   const float thr = w_thr;
   if (thr >= 0.f) {
-    // exclusive prefix of the threads' run totals, in thread order
-    if (tid == 0) {
-      pick_t = 0x7fffffff;
-      last_t = -1;
-    }
-    float x = ts;
-#pragma unroll
-    for (int o = 1; o < 32; o <<= 1) {
-      const float y = __shfl_up_sync(full, x, o);
-      if (lane >= o) x += y;
-    }
-    if (lane == 31) warp_tot[warp] = x;
-    __syncthreads();
-    float lo = w_off + x - ts;
-    for (int w = 0; w < warp; ++w) lo += warp_tot[w];
-    // the first thread of positive weight whose run ends past the threshold,
-    // else (rounding) the last thread of positive weight
-    if (ts > 0.f) {
-      if (thr < lo + ts) atomicMin(&pick_t, tid);
-      atomicMax(&last_t, tid);
-    }
-    __syncthreads();
-    const int owner_t = pick_t != 0x7fffffff ? pick_t : last_t;
-    if (tid == owner_t) {
-      int tok = -1, last_pos = -1;
-      float cum = lo;
-      for (int v = r0; v < r1; ++v) {
-        const float w = weight(v);
-        if (w > 0.f) {
-          last_pos = v;
-          if (cum + w > thr) {
-            tok = v;
-            break;
-          }
+    // the warp whose part holds the threshold: the first of positive weight
+    // whose part ends past it, else (rounding) the last of positive weight
+    float lo = w_off;
+    int owner_w = -1, last_w = -1;
+    float last_lo = lo;
+    for (int w = 0; w < kSampWarps; ++w) {
+      const float t = warp_tot[w];
+      if (t > 0.f) {
+        if (owner_w < 0 && thr < lo + t) {
+          owner_w = w;
+          break;
         }
-        cum += w;
+        last_w = w;
+        last_lo = lo;
       }
-      out_tokens[static_cast<size_t>(b) * (gamma + 1) + a] = tok >= 0 ? tok : last_pos;
+      lo += t;
+    }
+    if (owner_w < 0) {
+      owner_w = last_w;
+      lo = last_lo;
+    }
+    if (warp == owner_w) {
+      // walk the part in order, 32 units a step: lane sums, a warp scan, and
+      // the first lane whose cumulative weight passes the threshold
+      float base = lo;
+      int tok = -1, last_pos = -1;
+      for (int k0 = w0; k0 < w1 && tok < 0; k0 += 32 * 4) {
+        float4 wv[4];
+#pragma unroll
+        for (int j = 0; j < 4; ++j) {
+          const int u = k0 + 32 * j + lane;
+          wv[j] = u < w1 ? weights(u) : make_float4(0.f, 0.f, 0.f, 0.f);
+        }
+#pragma unroll
+        for (int j = 0; j < 4; ++j) {
+          if (tok >= 0) break;
+          const int u = k0 + 32 * j + lane;
+          const float w4[4] = {wv[j].x, wv[j].y, wv[j].z, wv[j].w};
+          const float ls = (w4[0] + w4[1]) + (w4[2] + w4[3]);
+          float incl = ls;
+#pragma unroll
+          for (int o = 1; o < 32; o <<= 1) {
+            const float y = __shfl_up_sync(full, incl, o);
+            if (lane >= o) incl += y;
+          }
+          // this lane's first column passing the threshold, and its last
+          // column of positive weight
+          int hit_col = -1, pos_col = -1;
+          float cum = base + incl - ls;
+#pragma unroll
+          for (int e = 0; e < 4; ++e) {
+            if (w4[e] > 0.f) {
+              if (hit_col < 0 && cum + w4[e] > thr) hit_col = VEC ? 4 * u + e : u;
+              pos_col = VEC ? 4 * u + e : u;
+            }
+            cum += w4[e];
+          }
+          const unsigned hit = __ballot_sync(full, hit_col >= 0);
+          const unsigned pos = __ballot_sync(full, pos_col >= 0);
+          if (hit) tok = __shfl_sync(full, hit_col, __ffs(hit) - 1);
+          if (pos) last_pos = __shfl_sync(full, pos_col, 31 - __clz(pos));
+          base += __shfl_sync(full, incl, 31);
+        }
+      }
+      if (lane == 0) out_tokens[static_cast<size_t>(b) * (gamma + 1) + a] = tok >= 0 ? tok : last_pos;
     }
   }
   cluster.sync();  // peers stay resident until every remote access is done
@@ -354,7 +443,7 @@ __global__ void __launch_bounds__(kSampThreads, 2) accept_sampled_kernel(
 
 struct SampCapacity {
   bool ready = false;
-  int resident[17] = {};
+  int resident[kSampMaxCluster + 1] = {};
 };
 
 cudaError_t samp_capacity(const SampCapacity** out) {
@@ -367,9 +456,11 @@ cudaError_t samp_capacity(const SampCapacity** out) {
   std::lock_guard<std::mutex> lk(mu);
   SampCapacity& cp = cap[dev];
   if (!cp.ready) {
-    e = cudaFuncSetAttribute(accept_sampled_kernel, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
+    e = cudaFuncSetAttribute(accept_sampled_kernel<true>, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
     if (e != cudaSuccess) return e;
-    for (int cl = 1; cl <= 16; ++cl) {
+    e = cudaFuncSetAttribute(accept_sampled_kernel<false>, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
+    if (e != cudaSuccess) return e;
+    for (int cl = 1; cl <= kSampMaxCluster; ++cl) {
       cudaLaunchConfig_t cfg = {};
       cfg.gridDim = dim3(static_cast<unsigned>(cl));
       cfg.blockDim = dim3(kSampThreads);
@@ -380,10 +471,12 @@ cudaError_t samp_capacity(const SampCapacity** out) {
       attr[0].val.clusterDim.z = 1;
       cfg.attrs = attr;
       cfg.numAttrs = 1;
-      int n = 0;
-      e = cudaOccupancyMaxActiveClusters(&n, accept_sampled_kernel, &cfg);
+      int n = 0, n2 = 0;
+      e = cudaOccupancyMaxActiveClusters(&n, accept_sampled_kernel<true>, &cfg);
       if (e != cudaSuccess) return e;
-      cp.resident[cl] = n;
+      e = cudaOccupancyMaxActiveClusters(&n2, accept_sampled_kernel<false>, &cfg);
+      if (e != cudaSuccess) return e;
+      cp.resident[cl] = n < n2 ? n : n2;
     }
     cp.ready = true;
   }
@@ -400,17 +493,24 @@ cudaError_t launch_accept_sampled(const float* target_logits, const float* draft
   const SampCapacity* cap = nullptr;
   cudaError_t e = samp_capacity(&cap);
   if (e != cudaSuccess) return e;
+  // the largest cluster with which the whole batch is resident at once
   int CL = 1;
-  for (int cl = 16; cl >= 1; cl >>= 1)
+  for (int cl = kSampMaxCluster; cl >= 1; cl >>= 1)
     if (cap->resident[cl] >= Bt) {
       CL = cl;
       break;
     }
-  const int vec4 = (vocab % 4 == 0) && ((reinterpret_cast<uintptr_t>(target_logits) & 15u) == 0) &&
-                   ((reinterpret_cast<uintptr_t>(draft_logits) & 15u) == 0);
-  return launch_overlapped(accept_sampled_kernel, dim3(static_cast<unsigned>(Bt) * CL), dim3(kSampThreads), 0,
-                           stream, static_cast<unsigned>(CL), target_logits, draft_logits, draft, u_accept, u_sample,
-                           kLog2e / temperature, gamma, vocab, vec4, accepted_len, out_tokens, err_word);
+  const bool vec4 = (vocab % 4 == 0) && ((reinterpret_cast<uintptr_t>(target_logits) & 15u) == 0) &&
+                    ((reinterpret_cast<uintptr_t>(draft_logits) & 15u) == 0);
+  const dim3 grid(static_cast<unsigned>(Bt) * CL);
+  const float zscale = kLog2e / temperature;
+  if (vec4)
+    return launch_overlapped(accept_sampled_kernel<true>, grid, dim3(kSampThreads), 0, stream,
+                             static_cast<unsigned>(CL), target_logits, draft_logits, draft, u_accept, u_sample,
+                             zscale, gamma, vocab, accepted_len, out_tokens, err_word);
+  return launch_overlapped(accept_sampled_kernel<false>, grid, dim3(kSampThreads), 0, stream,
+                           static_cast<unsigned>(CL), target_logits, draft_logits, draft, u_accept, u_sample, zscale,
+                           gamma, vocab, accepted_len, out_tokens, err_word);
 }
 
 }  // namespace simsd

@@ -292,7 +292,7 @@ int simsd_accept_sampled(const float* target_logits, const float* draft_logits, 
                          int vocab, int32_t* accepted_len, int32_t* out_tokens, int32_t* err_word, void* stream) {
   if (Bt < 0) return arg_fail("Bt < 0");
   if (gamma < 1 || gamma > 32) return arg_fail("gamma must be in [1, 32]");
-  if (vocab < 1 || vocab > (1 << 28)) return arg_fail("vocab must be in [1, 2^28]");
+  if (vocab < 1 || vocab > (1 << 24)) return arg_fail("vocab must be in [1, 2^24]");
   if (!(temperature > 0.f) || std::isinf(temperature)) return arg_fail("temperature must be positive and finite");
   if (Bt == 0) return SIMSD_OK;
   if (!target_logits || !draft_logits || !draft || !u_accept || !u_sample || !accepted_len || !out_tokens)
