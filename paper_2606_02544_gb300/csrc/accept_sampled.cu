@@ -9,17 +9,17 @@
 // target rows and gamma draft rows are laid end to end, each row padded to a
 // multiple of 32 units (a unit is 4 floats, or 1 when rows are not 16-byte
 // aligned), and the CTAs take contiguous spans of warp-aligned units, so the
-// 32 lanes of a warp are always on the same row.  Each lane keeps the running
-// maximum m of z = x*log2(e)/T and s = sum 2^(z - m) of its row; when the warp
-// moves to the next row it merges its lanes by shuffles into a per-warp slot
-// (no atomics).  CTA 0 merges the warps' and the CTAs' pairs (distributed
+// 32 lanes of a warp are always on the same row.  Each lane keeps the running maximum m of
+// z = x*log2(e)/T and s = sum 2^(z - m) of its row; when the warp moves to
+// the next row it merges its lanes by shuffles into a per-warp slot (no
+// atomics).  CTA 0 merges the warps' and the CTAs' pairs (distributed
 // shared memory), forms alpha_r from the drafts' own logits (fetched at the
 // start, while phase 1 streams) and the accepted length a, and broadcasts a.
 // Phase 2: each CTA takes a range of row a and each warp a contiguous part
-// of that, and sums the weights of its part (coalesced, 16-byte loads).  CTA
-// 0 forms the threshold u_sample * total and names the CTA whose range holds
-// it; in that CTA the warp whose part holds it walks the part in order, 32
-// units a step, with a warp scan.  Row a is read a second time (2 of the
+// of that, which it sums in coalesced steps of 32 units, keeping the sums of
+// up to 64 macro-steps.  CTA 0 forms the threshold u_sample * total and names
+// the CTA whose range holds it; there the warp whose part holds it finds the
+// macro-step by a scan of the kept sums and walks only that one.  Row a is read a second time (2 of the
 // 2*gamma+1 rows); no global scratch memory is used.
 #include <cooperative_groups.h>
 #include <cuda_runtime.h>
@@ -37,9 +37,9 @@ namespace {
 
 constexpr int kSampThreads = 512;
 constexpr int kSampWarps = kSampThreads / 32;
-constexpr int kSampUnroll = 8;
 constexpr int kSampMaxRows = 65;  // 2*gamma+1 <= 65
 constexpr int kSampMaxCluster = 16;
+constexpr int kSampMacros = 64;  // phase 2: macro-steps kept per warp
 constexpr float kLog2e = 1.4426950408889634f;
 // The running maximum starts at -FLT_MAX rather than -inf: 2^(z - m) is then
 // 0 for z = -inf (a masked logit) without a special case, and merging two
@@ -89,6 +89,16 @@ __device__ __forceinline__ const float* row_ptr(const float* tgt, const float* d
                       : drf + (static_cast<size_t>(b) * gamma + (row - gamma - 1)) * vocab;
 }
 
+// the same through L1 (phase 2 re-reads a thread's lines)
+template <bool VEC>
+__device__ __forceinline__ float4 load_unit_cached(const float* rp, int col) {
+  if constexpr (VEC) {
+    return __ldg(reinterpret_cast<const float4*>(rp) + col);
+  } else {
+    return make_float4(__ldg(rp + col), -INFINITY, -INFINITY, -INFINITY);
+  }
+}
+
 template <bool VEC>
 __device__ __forceinline__ float4 load_unit(const float* rp, int col) {
   if constexpr (VEC) {
@@ -98,8 +108,12 @@ __device__ __forceinline__ float4 load_unit(const float* rp, int col) {
   }
 }
 
-template <bool VEC>
-__global__ void __launch_bounds__(kSampThreads, 2) accept_sampled_kernel(
+// Units in flight per thread in phase 1: UNROLL 8 with two CTAs per SM;
+// UNROLL 16 when the grid has at most one CTA per SM (small batches), where
+// the CTA's bytes in flight set its bandwidth: two batches of 8, one loading
+// while the other is summed.
+template <bool VEC, int UNROLL>
+__global__ void __launch_bounds__(kSampThreads, UNROLL == 8 ? 2 : 1) accept_sampled_kernel(
     const float* __restrict__ tgt, const float* __restrict__ drf, const int32_t* __restrict__ draft,
     const float* __restrict__ u_accept, const float* __restrict__ u_sample, float zscale, int gamma, int vocab,
     int32_t* __restrict__ accepted_len, int32_t* __restrict__ out_tokens, int32_t* err_word) {
@@ -113,6 +127,7 @@ __global__ void __launch_bounds__(kSampThreads, 2) accept_sampled_kernel(
   __shared__ float w_cta;          // this CTA's weight of row a
   __shared__ float w_off, w_thr;   // the owner's offset and threshold (-1 elsewhere), set by CTA 0
   __shared__ int w_state;          // 1: the total weight was positive (set by CTA 0)
+  __shared__ float mac[kSampWarps][kSampMacros];     // phase 2: weight of each macro-step
   pdl_wait();
   pdl_launch_next();
   cg::cluster_group cluster = cg::this_cluster();
@@ -178,22 +193,22 @@ __global__ void __launch_bounds__(kSampThreads, 2) accept_sampled_kernel(
         rp = row_ptr(tgt, drf, b, gamma, vocab, min(row, rows - 1));
       }
     };
-    // f0, f1, Wp and the f and col of a warp's first lane are multiples of
-    // 32, so every test below is the same for the 32 lanes of a warp
-    for (; f < f1; f += kStep * kSampUnroll) {
-      float4 v[kSampUnroll];
-      int vr[kSampUnroll];
-      if (f - lane + kStep * (kSampUnroll - 1) < f1 && col - lane + kStep * (kSampUnroll - 1) + 31 < W) {
+    // Loads of H units.  f0, f1, Wp and the f and col of a warp's first lane
+    // are multiples of 32, so every test here is the same for the 32 lanes
+    // of a warp.  vr[u] is the unit's row, -1 past the span.
+    constexpr int H = UNROLL == 16 ? 8 : UNROLL;
+    auto fetch = [&](float4(&v)[H], int(&vr)[H]) {
+      if (f - lane + kStep * (H - 1) < f1 && col - lane + kStep * (H - 1) + 31 < W) {
         // the common case: every unit valid, on one row, inside the row
 #pragma unroll
-        for (int u = 0; u < kSampUnroll; ++u) {
+        for (int u = 0; u < H; ++u) {
           v[u] = load_unit<VEC>(rp, col + u * kStep);
           vr[u] = row;
         }
-        advance(kStep * kSampUnroll);
+        advance(kStep * H);
       } else {
 #pragma unroll
-        for (int u = 0; u < kSampUnroll; ++u) {
+        for (int u = 0; u < H; ++u) {
           vr[u] = -1;
           if (f + u * kStep < f1) {
             vr[u] = row;
@@ -202,8 +217,11 @@ __global__ void __launch_bounds__(kSampThreads, 2) accept_sampled_kernel(
           advance(kStep);
         }
       }
+      f += kStep * H;
+    };
+    auto consume = [&](const float4(&v)[H], const int(&vr)[H]) {
 #pragma unroll
-      for (int u = 0; u < kSampUnroll; ++u) {
+      for (int u = 0; u < H; ++u) {
         if (vr[u] < 0) break;
         if (vr[u] != cur) {
           flush();
@@ -219,6 +237,28 @@ __global__ void __launch_bounds__(kSampThreads, 2) accept_sampled_kernel(
         const float nm = -m;
         s += ex2(fmaf(v[u].x, zscale, nm)) + ex2(fmaf(v[u].y, zscale, nm)) + ex2(fmaf(v[u].z, zscale, nm)) +
              ex2(fmaf(v[u].w, zscale, nm));
+      }
+    };
+    if constexpr (UNROLL == 16) {
+      // one CTA per SM: two batches of 8, the next one's loads in flight
+      // while the current one is summed
+      float4 va[H], vb[H];
+      int ra[H], rb[H];
+      fetch(va, ra);
+      while (ra[0] >= 0) {
+        fetch(vb, rb);
+        consume(va, ra);
+        if (rb[0] < 0) break;
+        fetch(va, ra);
+        consume(vb, rb);
+      }
+    } else {
+      float4 v[H];
+      int vr[H];
+      for (;;) {
+        fetch(v, vr);
+        if (vr[0] < 0) break;
+        consume(v, vr);
       }
     }
     if (f0 + 32 * warp < f1) flush();
@@ -294,7 +334,9 @@ __global__ void __launch_bounds__(kSampThreads, 2) accept_sampled_kernel(
   cluster.sync();
 
   // ---- phase 2: weights of row a.  CTA c takes a range of units of the
-  // row, warp w a contiguous part of that, and the lanes stride through it.
+  // row and warp w a contiguous part of that, in steps of 32 units (one per
+  // lane, coalesced); the warp keeps the weight of every macro-step of M
+  // steps, at most kSampMacros of them, so that the draw walks one macro.
   const int a = a_sh;
   bool resid = a < gamma;
   const float* trow = tgt + (static_cast<size_t>(b) * (gamma + 1) + a) * vocab;
@@ -304,15 +346,16 @@ __global__ void __launch_bounds__(kSampThreads, 2) accept_sampled_kernel(
   const int W = VEC ? (vocab >> 2) : vocab;
   const int per_c = (W + CL - 1) / CL;
   const int c0 = min(W, c * per_c), c1 = min(W, c0 + per_c);
-  const int per_w = (c1 - c0 + kSampWarps - 1) / kSampWarps;
+  const int per_w = (((c1 - c0 + kSampWarps - 1) / kSampWarps) + 31) & ~31;
   const int w0 = min(c1, c0 + warp * per_w), w1 = min(c1, w0 + per_w);
+  const int nsteps = (w1 - w0 + 31) >> 5;
+  const int M = max(1, (nsteps + kSampMacros - 1) / kSampMacros);
+  const int nmac = (nsteps + M - 1) / M;
   // the four weights of a unit (the scalar layout has one column per unit)
-  auto weights = [&](int unit) -> float4 {
-    const float4 xt = load_unit<VEC>(trow, unit);
+  auto weights = [&](const float4& xt, const float4& xd) -> float4 {
     float4 w = make_float4(ex2(fmaf(xt.x, zscale, nmt)) * it, ex2(fmaf(xt.y, zscale, nmt)) * it,
                            ex2(fmaf(xt.z, zscale, nmt)) * it, ex2(fmaf(xt.w, zscale, nmt)) * it);
     if (resid) {
-      const float4 xd = load_unit<VEC>(drow, unit);
       w.x = fmaxf(0.f, w.x - ex2(fmaf(xd.x, zscale, nmd)) * id);
       w.y = fmaxf(0.f, w.y - ex2(fmaf(xd.y, zscale, nmd)) * id);
       w.z = fmaxf(0.f, w.z - ex2(fmaf(xd.z, zscale, nmd)) * id);
@@ -320,18 +363,40 @@ __global__ void __launch_bounds__(kSampThreads, 2) accept_sampled_kernel(
     }
     return w;
   };
+  const float4 kNone = make_float4(-INFINITY, -INFINITY, -INFINITY, -INFINITY);
+  // loads of 4 steps from step i0 (units past the part give weight 0)
+  auto load4 = [&](int i0, float4(&xt)[4], float4(&xd)[4]) {
+#pragma unroll
+    for (int j = 0; j < 4; ++j) {
+      const int u = w0 + 32 * (i0 + j) + lane;
+      const bool ok = u < w1;
+      xt[j] = ok ? load_unit_cached<VEC>(trow, u) : kNone;
+      xd[j] = ok && resid ? load_unit_cached<VEC>(drow, u) : kNone;
+    }
+  };
   // an empty residual (p_theta = p_phi to fp32 precision) cannot reject:
   // the draw then falls back to p_theta (second pass)
   for (int pass = 0; pass < 2; ++pass) {
-    float ws = 0.f;
-#pragma unroll 4
-    for (int u = w0 + lane; u < w1; u += 32) {
-      const float4 w = weights(u);
-      ws += (w.x + w.y) + (w.z + w.w);
-    }
+    float acc = 0.f, wt = 0.f;
+    for (int i0 = 0; i0 < nsteps; i0 += 4) {
+      float4 xt[4], xd[4];
+      load4(i0, xt, xd);
 #pragma unroll
-    for (int o = 16; o > 0; o >>= 1) ws += __shfl_xor_sync(full, ws, o);
-    if (lane == 0) warp_tot[warp] = ws;
+      for (int j = 0; j < 4; ++j) {
+        const int i = i0 + j;
+        if (i >= nsteps) break;
+        const float4 w = weights(xt[j], xd[j]);
+        acc += (w.x + w.y) + (w.z + w.w);
+        if ((i + 1) % M == 0 || i + 1 == nsteps) {
+#pragma unroll
+          for (int o = 16; o > 0; o >>= 1) acc += __shfl_xor_sync(full, acc, o);
+          if (lane == 0) mac[warp][i / M] = acc;
+          wt += acc;
+          acc = 0.f;
+        }
+      }
+    }
+    if (lane == 0) warp_tot[warp] = wt;
     __syncthreads();
     if (tid == 0) {
       float t = 0.f;
@@ -379,7 +444,7 @@ __global__ void __launch_bounds__(kSampThreads, 2) accept_sampled_kernel(
     for (int w = 0; w < kSampWarps; ++w) {
       const float t = warp_tot[w];
       if (t > 0.f) {
-        if (owner_w < 0 && thr < lo + t) {
+        if (thr < lo + t) {
           owner_w = w;
           break;
         }
@@ -393,22 +458,38 @@ __global__ void __launch_bounds__(kSampThreads, 2) accept_sampled_kernel(
       lo = last_lo;
     }
     if (warp == owner_w) {
-      // walk the part in order, 32 units a step: lane sums, a warp scan, and
-      // the first lane whose cumulative weight passes the threshold
-      float base = lo;
-      int tok = -1, last_pos = -1;
-      for (int k0 = w0; k0 < w1 && tok < 0; k0 += 32 * 4) {
-        float4 wv[4];
+      // the macro-step that holds the threshold, by a scan of the macro
+      // weights (lane k holds macros k and 32 + k), with the same fallback
+      const float ma = lane < nmac ? mac[warp][lane] : 0.f;
+      const float mb = lane + 32 < nmac ? mac[warp][lane + 32] : 0.f;
+      float ia = ma, ib = mb;
 #pragma unroll
-        for (int j = 0; j < 4; ++j) {
-          const int u = k0 + 32 * j + lane;
-          wv[j] = u < w1 ? weights(u) : make_float4(0.f, 0.f, 0.f, 0.f);
+      for (int o = 1; o < 32; o <<= 1) {
+        const float ya = __shfl_up_sync(full, ia, o), yb = __shfl_up_sync(full, ib, o);
+        if (lane >= o) {
+          ia += ya;
+          ib += yb;
         }
+      }
+      ib += __shfl_sync(full, ia, 31);
+      const unsigned ha = __ballot_sync(full, ma > 0.f && thr < lo + ia);
+      const unsigned hb = __ballot_sync(full, mb > 0.f && thr < lo + ib);
+      const unsigned pa = __ballot_sync(full, ma > 0.f), pb = __ballot_sync(full, mb > 0.f);
+      int k = ha ? __ffs(ha) - 1 : hb ? 32 + __ffs(hb) - 1 : pb ? 63 - __clz(pb) : pa ? 31 - __clz(pa) : 0;
+      float base = lo + __shfl_sync(full, k < 32 ? ia - ma : ib - mb, k & 31);
+      // walk the macro's steps in order: lane sums, a warp scan, and the
+      // first lane whose cumulative weight passes the threshold
+      int tok = -1, last_pos = -1;
+      const int s_end = min(nsteps, (k + 1) * M);
+      for (int i0 = k * M; i0 < s_end && tok < 0; i0 += 4) {
+        float4 xt[4], xd[4];
+        load4(i0, xt, xd);
 #pragma unroll
         for (int j = 0; j < 4; ++j) {
-          if (tok >= 0) break;
-          const int u = k0 + 32 * j + lane;
-          const float w4[4] = {wv[j].x, wv[j].y, wv[j].z, wv[j].w};
+          if (tok >= 0 || i0 + j >= s_end) break;
+          const int u = w0 + 32 * (i0 + j) + lane;
+          const float4 w = weights(xt[j], xd[j]);
+          const float w4[4] = {w.x, w.y, w.z, w.w};
           const float ls = (w4[0] + w4[1]) + (w4[2] + w4[3]);
           float incl = ls;
 #pragma unroll
@@ -443,8 +524,37 @@ __global__ void __launch_bounds__(kSampThreads, 2) accept_sampled_kernel(
 
 struct SampCapacity {
   bool ready = false;
-  int resident[kSampMaxCluster + 1] = {};
+  int resident8[kSampMaxCluster + 1] = {};   // clusters resident at once, UNROLL 8
+  int resident16[kSampMaxCluster + 1] = {};  // UNROLL 16
 };
+
+template <bool VEC, int UNROLL>
+cudaError_t max_clusters(int cl, int* n) {
+  auto kern = accept_sampled_kernel<VEC, UNROLL>;
+  cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
+  if (e != cudaSuccess) return e;
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(static_cast<unsigned>(cl));
+  cfg.blockDim = dim3(kSampThreads);
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeClusterDimension;
+  attr[0].val.clusterDim.x = static_cast<unsigned>(cl);
+  attr[0].val.clusterDim.y = 1;
+  attr[0].val.clusterDim.z = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  return cudaOccupancyMaxActiveClusters(n, kern, &cfg);
+}
+
+template <int UNROLL>
+cudaError_t min_clusters(int cl, int* n) {
+  int n1 = 0, n2 = 0;
+  cudaError_t e = max_clusters<true, UNROLL>(cl, &n1);
+  if (e != cudaSuccess) return e;
+  e = max_clusters<false, UNROLL>(cl, &n2);
+  *n = n1 < n2 ? n1 : n2;
+  return e;
+}
 
 cudaError_t samp_capacity(const SampCapacity** out) {
   static std::mutex mu;
@@ -456,32 +566,24 @@ cudaError_t samp_capacity(const SampCapacity** out) {
   std::lock_guard<std::mutex> lk(mu);
   SampCapacity& cp = cap[dev];
   if (!cp.ready) {
-    e = cudaFuncSetAttribute(accept_sampled_kernel<true>, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
-    if (e != cudaSuccess) return e;
-    e = cudaFuncSetAttribute(accept_sampled_kernel<false>, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
-    if (e != cudaSuccess) return e;
-    for (int cl = 1; cl <= kSampMaxCluster; ++cl) {
-      cudaLaunchConfig_t cfg = {};
-      cfg.gridDim = dim3(static_cast<unsigned>(cl));
-      cfg.blockDim = dim3(kSampThreads);
-      cudaLaunchAttribute attr[1];
-      attr[0].id = cudaLaunchAttributeClusterDimension;
-      attr[0].val.clusterDim.x = static_cast<unsigned>(cl);
-      attr[0].val.clusterDim.y = 1;
-      attr[0].val.clusterDim.z = 1;
-      cfg.attrs = attr;
-      cfg.numAttrs = 1;
-      int n = 0, n2 = 0;
-      e = cudaOccupancyMaxActiveClusters(&n, accept_sampled_kernel<true>, &cfg);
+    for (int cl = 1; cl <= kSampMaxCluster; cl <<= 1) {
+      e = min_clusters<8>(cl, &cp.resident8[cl]);
       if (e != cudaSuccess) return e;
-      e = cudaOccupancyMaxActiveClusters(&n2, accept_sampled_kernel<false>, &cfg);
+      e = min_clusters<16>(cl, &cp.resident16[cl]);
       if (e != cudaSuccess) return e;
-      cp.resident[cl] = n < n2 ? n : n2;
     }
     cp.ready = true;
   }
   *out = &cp;
   return cudaSuccess;
+}
+
+template <bool VEC, int UNROLL>
+cudaError_t launch_samp(dim3 grid, unsigned CL, cudaStream_t stream, const float* tl, const float* dl,
+                        const int32_t* draft, const float* ua, const float* us, float zscale, int gamma, int vocab,
+                        int32_t* accepted_len, int32_t* out_tokens, int32_t* err_word) {
+  return launch_overlapped(accept_sampled_kernel<VEC, UNROLL>, grid, dim3(kSampThreads), 0, stream, CL, tl, dl,
+                           draft, ua, us, zscale, gamma, vocab, accepted_len, out_tokens, err_word);
 }
 
 }  // namespace
@@ -493,24 +595,29 @@ cudaError_t launch_accept_sampled(const float* target_logits, const float* draft
   const SampCapacity* cap = nullptr;
   cudaError_t e = samp_capacity(&cap);
   if (e != cudaSuccess) return e;
-  // the largest cluster with which the whole batch is resident at once
+  // the largest cluster with which the whole batch is resident at once; the
+  // deeper unroll when that still holds with one CTA per SM
   int CL = 1;
   for (int cl = kSampMaxCluster; cl >= 1; cl >>= 1)
-    if (cap->resident[cl] >= Bt) {
+    if (cap->resident8[cl] >= Bt) {
       CL = cl;
       break;
     }
+  const bool deep = cap->resident16[CL] >= Bt;
   const bool vec4 = (vocab % 4 == 0) && ((reinterpret_cast<uintptr_t>(target_logits) & 15u) == 0) &&
                     ((reinterpret_cast<uintptr_t>(draft_logits) & 15u) == 0);
   const dim3 grid(static_cast<unsigned>(Bt) * CL);
   const float zscale = kLog2e / temperature;
+  const unsigned ucl = static_cast<unsigned>(CL);
   if (vec4)
-    return launch_overlapped(accept_sampled_kernel<true>, grid, dim3(kSampThreads), 0, stream,
-                             static_cast<unsigned>(CL), target_logits, draft_logits, draft, u_accept, u_sample,
-                             zscale, gamma, vocab, accepted_len, out_tokens, err_word);
-  return launch_overlapped(accept_sampled_kernel<false>, grid, dim3(kSampThreads), 0, stream,
-                           static_cast<unsigned>(CL), target_logits, draft_logits, draft, u_accept, u_sample, zscale,
-                           gamma, vocab, accepted_len, out_tokens, err_word);
+    return deep ? launch_samp<true, 16>(grid, ucl, stream, target_logits, draft_logits, draft, u_accept, u_sample,
+                                        zscale, gamma, vocab, accepted_len, out_tokens, err_word)
+                : launch_samp<true, 8>(grid, ucl, stream, target_logits, draft_logits, draft, u_accept, u_sample,
+                                       zscale, gamma, vocab, accepted_len, out_tokens, err_word);
+  return deep ? launch_samp<false, 16>(grid, ucl, stream, target_logits, draft_logits, draft, u_accept, u_sample,
+                                       zscale, gamma, vocab, accepted_len, out_tokens, err_word)
+              : launch_samp<false, 8>(grid, ucl, stream, target_logits, draft_logits, draft, u_accept, u_sample,
+                                      zscale, gamma, vocab, accepted_len, out_tokens, err_word);
 }
 
 }  // namespace simsd

@@ -99,10 +99,11 @@ def test_accept_sampled_matches_oracle(Bt, gamma, V, T, eta):
     _compare(si)
 
 
-@pytest.mark.parametrize("V", [1001, 30001])
-def test_accept_sampled_scalar_paths(V):
-    # a vocabulary that is not a multiple of 4, and base pointers off 16 bytes
-    si = inputs.make_sampled_inputs(6, 4, V, seed=V, device="cuda")
+@pytest.mark.parametrize("Bt,V", [(6, 1001), (6, 30001), (400, 1001)])
+def test_accept_sampled_scalar_paths(Bt, V):
+    # a vocabulary that is not a multiple of 4, and base pointers off 16 bytes;
+    # small and large batches take the one- and two-CTA-per-SM variants
+    si = inputs.make_sampled_inputs(Bt, 4, V, seed=V, device="cuda")
     _compare(si)
     for name in ("target_logits", "draft_logits"):
         t = getattr(si, name)
