@@ -64,10 +64,26 @@
 
 /* Checks that step_map row b is a partial permutation of 1..gamma (0 marks
  * padding).  Returns 1 when valid. */
+/* Step-map codes besides the drafted labels 1..gamma.  Sec. 3.2 verifies
+ * only the gamma drafted positions of a block; with fewer drafts than
+ * undecoded positions, and when the target completes the block itself
+ * (R < gamma), the block also holds positions that stay [MASK] through the
+ * step and positions decoded earlier in the block.
+ *    0  padding: both slots of the position are padding (Eq. (1), zeroed
+ *       rows and columns);
+ *   -1  undrafted: the position stays a mask placeholder; its data slot is
+ *       padding and its mask slot carries tau = gamma + 1, later than every
+ *       drafted step;
+ *   -2  decoded: the position already holds a clean token; its data slot
+ *       carries tau = 0 (known before every step, like a prompt token) and
+ *       its mask slot is padding. */
+#define OR_STEP_UNDRAFTED (-1)
+#define OR_STEP_DECODED (-2)
+
 static int step_map_row_valid(const int32_t *mu, int gamma) {
     for (int k = 0; k < gamma; ++k) {
-        if (mu[k] < 0 || mu[k] > gamma) return 0;
-        if (mu[k] == 0) continue;
+        if (mu[k] < OR_STEP_DECODED || mu[k] > gamma) return 0;
+        if (mu[k] <= 0) continue;
         for (int k2 = 0; k2 < k; ++k2)
             if (mu[k2] == mu[k]) return 0;
     }
@@ -75,19 +91,33 @@ static int step_map_row_valid(const int32_t *mu, int gamma) {
 }
 
 /* Per-slot labels for one sequence.  Slot k (k < gamma) is D_k, slot gamma+k
- * is D~_k; both carry tau = mu_k (Sec. 3.1 "Temporal Attention Mask").  A
- * zero entry or an invalid map marks the slot(s) as padding.  The RoPE index
- * of both D_k and D~_k is the absolute position of D_k, i.e. n + k, where n is
- * the cached prefix length (Sec. 3.1 "Position Encoding Alignment"). */
+ * is D~_k; a drafted position gives both tau = mu_k (Sec. 3.1 "Temporal
+ * Attention Mask"); the codes above set the other kinds.  An invalid map
+ * marks every slot as padding.  The RoPE index of both D_k and D~_k is the
+ * absolute position of D_k, i.e. n + k, where n is the cached prefix length
+ * (Sec. 3.1 "Position Encoding Alignment"). */
 static int labels_for_sequence(const int32_t *mu, int n, int gamma, int32_t *tau,
                                uint8_t *sect, int32_t *rope) {
     int ok = step_map_row_valid(mu, gamma);
     for (int k = 0; k < gamma; ++k) {
-        int pad = (!ok) || mu[k] == 0;
-        tau[k] = pad ? 0 : mu[k];
-        tau[gamma + k] = tau[k];
-        sect[k] = pad ? OR_SECT_PAD : OR_SECT_D;
-        sect[gamma + k] = pad ? OR_SECT_PAD : OR_SECT_DT;
+        int v = ok ? mu[k] : 0;
+        int td = 0, tm = 0;
+        uint8_t sd = OR_SECT_PAD, sm = OR_SECT_PAD;
+        if (v > 0) {
+            td = tm = v;
+            sd = OR_SECT_D;
+            sm = OR_SECT_DT;
+        } else if (v == OR_STEP_UNDRAFTED) {
+            tm = gamma + 1;
+            sm = OR_SECT_DT;
+        } else if (v == OR_STEP_DECODED) {
+            td = 0;
+            sd = OR_SECT_D;
+        }
+        tau[k] = td;
+        tau[gamma + k] = tm;
+        sect[k] = sd;
+        sect[gamma + k] = sm;
         rope[k] = n + k;
         rope[gamma + k] = n + k;
     }

@@ -43,6 +43,8 @@ ERR_DRAFT = 8
 ERR_ACCEPT_LEN = 32
 
 SECT_D, SECT_DT, SECT_PAD = 0, 1, 255
+# step-map codes besides the drafted labels 1..gamma (0 is padding)
+STEP_UNDRAFTED, STEP_DECODED = -1, -2
 
 
 def build(force: bool = False) -> str:
@@ -102,8 +104,11 @@ def max_threads() -> int:
 def build_mask(step_map, prefix_len, gamma: int) -> dict:
     """Eq. (1) mask plus per-slot labels.
 
-    step_map: int32 [Bt][gamma] (entries 1..gamma, 0 = padding) or None for
-    the identity map.  Returns tau, section, rope_pos ([Bt][2gamma]),
+    step_map: int32 [Bt][gamma] or None for the identity map.  Entries:
+    1..gamma drafted labels (distinct), 0 padding, STEP_UNDRAFTED (-1) a
+    position that stays [MASK] (mask slot only, tau = gamma + 1),
+    STEP_DECODED (-2) a clean token decoded earlier in the block (data slot
+    only, tau = 0).  Returns tau, section, rope_pos ([Bt][2gamma]),
     mask_bits (uint64 [Bt][2gamma]), dense (uint8 [Bt][2gamma][2gamma]) and
     the error bits.
     """

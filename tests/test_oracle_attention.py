@@ -285,6 +285,55 @@ def test_single_layer_equals_step_by_step_decode(seed):
     np.testing.assert_array_equal(ot[0, :gamma], drafts)
 
 
+@pytest.mark.parametrize("seed,n_draft", [(0, 3), (1, 1), (2, 5), (3, 0), (4, 0), (5, 2)])
+def test_single_layer_with_undrafted_and_decoded_positions(seed, n_draft):
+    """A block of B positions: some decoded earlier in the block (code -2),
+    n_draft drafted along a random order, the rest left [MASK] (code -1).
+    Each prediction row must equal plain bidirectional attention over the
+    block as it stands when that row predicts: positions known before its
+    step hold their clean token, every other position its [MASK] input.
+    Each data row equals the same after its own step.  n_draft = 0 is the
+    target completing the block itself (Sec. 3.2)."""
+    rng = np.random.default_rng(500 + seed)
+    toy = _Toy.make(40 + seed)
+    B = 6
+    n = int(rng.integers(0, 30))
+    order = rng.permutation(B)
+    codes = np.full(B, orc.STEP_UNDRAFTED, np.int32)
+    codes[order[:n_draft]] = rng.permutation(n_draft) + 1
+    n_dec = int(rng.integers(1, B - n_draft + 1)) if n_draft < B else 0
+    codes[order[n_draft:n_draft + n_dec]] = orc.STEP_DECODED
+    tok = rng.integers(0, toy.E.shape[0], B)
+    big = 10 ** 9
+    known = [0 if c == orc.STEP_DECODED else (big if c == orc.STEP_UNDRAFTED else int(c)) for c in codes]
+    hp = toy.E[rng.integers(0, toy.E.shape[0], n)] + toy.pos[:n]
+    _, Kp, Vp = toy.qkv(hp)
+
+    def block_hidden(t):
+        # the block when every position known before step t is decoded
+        return np.stack([(toy.E[tok[k]] if known[k] < t else toy.emask) + toy.pos[n + k] for k in range(B)])
+
+    hD = np.stack([toy.E[tok[k]] + toy.pos[n + k] for k in range(B)])
+    hM = np.stack([toy.emask + toy.pos[n + k] for k in range(B)])
+    q, k, v = toy.qkv(np.concatenate([hD, hM]))
+    kc, vc, bt = _paged(Kp, Vp, 8, rng)
+    out, err = orc.verify_attention(q[None], k[None], v[None], kc, vc, bt, [n], codes[None], B)
+    assert err == 0
+    for j in range(B):
+        if codes[j] != orc.STEP_DECODED:        # a prediction row, at its step
+            qb, Kb, Vb = toy.qkv(block_hidden(known[j]))
+            want = _bidir(qb[j], np.concatenate([Kp, Kb]), np.concatenate([Vp, Vb]))
+            np.testing.assert_allclose(out[0, B + j], want, rtol=1e-12, atol=1e-13)
+        else:
+            assert (out[0, B + j] == 0).all()
+        if codes[j] != orc.STEP_UNDRAFTED:      # a data row, just after its step
+            qb, Kb, Vb = toy.qkv(block_hidden(known[j] + 1))
+            want = _bidir(qb[j], np.concatenate([Kp, Kb]), np.concatenate([Vp, Vb]))
+            np.testing.assert_allclose(out[0, j], want, rtol=1e-12, atol=1e-13)
+        else:
+            assert (out[0, j] == 0).all()
+
+
 def test_two_layers_are_only_approximate():
     # With two layers the data slots' hidden states were formed under their
     # own decoding step, not the current one, so the match is no longer exact

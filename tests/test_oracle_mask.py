@@ -203,9 +203,102 @@ def test_mask_bits_match_dense():
             np.testing.assert_array_equal(got, r["dense"][b, i])
 
 
-@pytest.mark.parametrize("bad", [[1, 1, 2, 3], [1, 2, 5, 3], [1, -1, 2, 3], [4, 2, 2, 0]])
+@pytest.mark.parametrize("bad", [[1, 1, 2, 3], [1, 2, 5, 3], [1, -3, 2, 3], [4, 2, 2, 0], [-1, 1, 1, -2]])
 def test_invalid_step_map_is_flagged_and_padded(bad):
     r = orc.build_mask(np.array([bad], np.int32), [3], 4)
     assert r["err"] & orc.ERR_STEP_MAP
     assert (r["section"][0] == orc.SECT_PAD).all()
     assert (r["dense"][0] == 0).all()
+
+
+# ---- blocks with fewer drafts than positions, and the target completing
+# the block itself (Sec. 3.2, last sentences of "Target Model Verification")
+
+INF = 10 ** 9
+
+
+def _prose_mask_block(codes):
+    """Visible sets by the step at which each position becomes known.
+
+    A position decoded earlier in the block is known before every step
+    (step 0), a drafted position at its draft step, an undrafted one never
+    within this step.  Its data slot exists iff it holds a token (decoded or
+    drafted), its mask slot iff a prediction is made there (drafted or
+    undrafted).  A data token sees the data tokens known no later than it and
+    the placeholders of positions still unknown at that time; a prediction
+    slot sees the data tokens known strictly earlier and the placeholders of
+    positions unresolved at its step (Sec. 3.1).
+    """
+    B = len(codes)
+    known = [0 if c == orc.STEP_DECODED else (INF if c == orc.STEP_UNDRAFTED else c) for c in codes]
+    has_d = [c > 0 or c == orc.STEP_DECODED for c in codes]
+    has_m = [c > 0 or c == orc.STEP_UNDRAFTED for c in codes]
+    A = np.zeros((2 * B, 2 * B), np.uint8)
+    for i in range(B):
+        for k in range(B):
+            if has_d[i] and has_d[k] and known[k] <= known[i]:
+                A[i, k] = 1
+            if has_d[i] and has_m[k] and known[k] > known[i]:
+                A[i, B + k] = 1
+            if has_m[i] and has_d[k] and known[k] < known[i]:
+                A[B + i, k] = 1
+            if has_m[i] and has_m[k] and known[k] >= known[i]:
+                A[B + i, B + k] = 1
+    return A
+
+
+def _random_block(rng, B, n_draft, n_decoded):
+    codes = np.full(B, orc.STEP_UNDRAFTED, np.int32)
+    pos = rng.permutation(B)
+    codes[pos[:n_draft]] = rng.permutation(n_draft) + 1
+    codes[pos[n_draft:n_draft + n_decoded]] = orc.STEP_DECODED
+    return codes
+
+
+@pytest.mark.parametrize("B", [1, 2, 4, 5, 8, 16, 32])
+def test_undrafted_and_decoded_positions_match_prose(B):
+    rng = np.random.default_rng(300 + B)
+    maps = []
+    for _ in range(30):
+        n_draft = int(rng.integers(0, B + 1))
+        n_dec = int(rng.integers(0, B - n_draft + 1))
+        codes = _random_block(rng, B, n_draft, n_dec)
+        codes[rng.random(B) < 0.1] = 0       # some padding as well
+        maps.append(codes)
+    maps = np.stack(maps)
+    r = orc.build_mask(maps, np.zeros(len(maps), np.int32), B)
+    assert r["err"] == 0
+    for b, codes in enumerate(maps):
+        np.testing.assert_array_equal(r["dense"][b], _prose_mask_block(list(codes)), err_msg=str(codes))
+
+
+@pytest.mark.parametrize("B", [1, 3, 4, 8, 32])
+def test_target_completing_the_block_is_bidirectional(B):
+    # With no drafts (decoded tokens and [MASK] placeholders only) the step
+    # is the dLLM's own block decoding: every real slot sees every other.
+    rng = np.random.default_rng(400 + B)
+    for _ in range(10):
+        codes = _random_block(rng, B, 0, int(rng.integers(0, B + 1)))
+        r = orc.build_mask(codes[None], [5], B)
+        assert r["err"] == 0
+        real = np.concatenate([codes == orc.STEP_DECODED, codes == orc.STEP_UNDRAFTED])
+        A = r["dense"][0].astype(bool)
+        assert real.sum() == B
+        assert A[np.ix_(real, real)].all()
+        assert not A[~real].any() and not A[:, ~real].any()
+
+
+def test_drafted_part_is_the_mask_of_the_drafts_alone():
+    # Removing the undrafted and decoded positions leaves the plain mask of
+    # the drafted permutation: the extra kinds change nothing among drafts.
+    rng = np.random.default_rng(9)
+    for _ in range(20):
+        B = int(rng.integers(2, 17))
+        codes = _random_block(rng, B, int(rng.integers(1, B + 1)), 0)
+        codes[codes == orc.STEP_UNDRAFTED] = np.where(rng.random((codes == orc.STEP_UNDRAFTED).sum()) < 0.5,
+                                                      orc.STEP_UNDRAFTED, orc.STEP_DECODED)
+        d = np.nonzero(codes > 0)[0]
+        full = orc.build_mask(codes[None], [0], B)["dense"][0]
+        alone = orc.build_mask(codes[d][None], [0], len(d))["dense"][0]
+        idx = np.concatenate([d, B + d])
+        np.testing.assert_array_equal(full[np.ix_(idx, idx)], alone)
