@@ -66,8 +66,15 @@ extern "C" {
 #define SIMSD_SECT_MASK 1 /* D~: prediction slot */
 #define SIMSD_SECT_PAD 255 /* padding: row outputs zero, column never visible */
 
+/* step-map codes besides the drafted labels 1..gamma and 0 (padding).
+ * Sec. 3.2 verifies only the drafted positions of a block and has the target
+ * complete the block itself when fewer than gamma positions remain; these
+ * codes put the block's other positions into the same layout. */
+#define SIMSD_STEP_UNDRAFTED (-1) /* stays [MASK]: mask slot only, tau = gamma+1 */
+#define SIMSD_STEP_DECODED (-2)   /* decoded earlier in the block: data slot only, tau = 0 */
+
 /* device error-word bits */
-#define SIMSD_EW_STEP_MAP 1u    /* step map is not a partial permutation of 1..gamma */
+#define SIMSD_EW_STEP_MAP 1u    /* step map entry outside the codes above, or a repeated label */
 #define SIMSD_EW_PREFIX_LEN 2u  /* prefix length < 0 or beyond the block table */
 #define SIMSD_EW_PAGE 4u        /* a needed page id is outside [0, num_pages) */
 #define SIMSD_EW_DRAFT 8u       /* a draft id is outside [0, vocab) */
@@ -79,16 +86,22 @@ extern "C" {
  * Sec. 3.1 "Temporal Attention Mask" and Eq. (1); "Position Encoding
  * Alignment" (RoPE copy); Sec. 3.2 (the slot of the r-th draft gets tau=r).
  *
- *   step_map   [Bt][gamma] int32, mu_k in 1..gamma (a permutation), 0 marks a
- *              padding position; NULL means the identity mu_k = k+1.
+ *   step_map   [Bt][gamma] int32: mu_k in 1..gamma for a drafted position
+ *              (distinct labels), 0 for padding, SIMSD_STEP_UNDRAFTED or
+ *              SIMSD_STEP_DECODED; NULL means the identity mu_k = k+1.  A
+ *              map of undrafted and decoded entries only is the target's own
+ *              block decoding: every real slot sees every other.
  *   prefix_len [Bt] int32, cached prefix length n_b.
- *   tau        [Bt][2gamma] int32 out: tau of D_k and D~_k is mu_k (0 if pad).
+ *   tau        [Bt][2gamma] int32 out: tau of D_k and D~_k is mu_k for a
+ *              drafted position; gamma+1 for an undrafted mask slot, 0 for
+ *              a decoded data slot and for padding.
  *   section    [Bt][2gamma] uint8 out: SIMSD_SECT_DATA / _MASK / _PAD.
  *   rope_pos   [Bt][2gamma] int32 out: n_b + k for both D_k and D~_k.
  *   mask_bits  [Bt][2gamma] uint64 out or NULL: bit j of row i is A_ij of
  *              Eq. (1) over the new slots (prefix columns are always visible).
- *   1 <= gamma <= 32.  A step map row that is not a partial permutation sets
- *   SIMSD_EW_STEP_MAP and turns every slot of that sequence into padding.
+ *   1 <= gamma <= 32.  A step map row with an entry outside these codes or a
+ *   repeated label sets SIMSD_EW_STEP_MAP and turns every slot of that
+ *   sequence into padding.
  */
 SIMSD_API int simsd_build_mask(const int32_t* step_map, const int32_t* prefix_len, int Bt, int gamma,
                      int32_t* tau, uint8_t* section, int32_t* rope_pos, uint64_t* mask_bits,

@@ -24,21 +24,35 @@ __global__ void __launch_bounds__(64) build_mask_kernel(const int32_t* __restric
   if (i == 0) map_ok = 1;
   if (i < gamma) mu[i] = step_map ? step_map[static_cast<size_t>(b) * gamma + i] : i + 1;
   __syncthreads();
-  // the step map must be a partial permutation of 1..gamma (0 = padding)
+  // the drafted labels must be distinct values in 1..gamma; the other
+  // entries are 0 (padding), SIMSD_STEP_UNDRAFTED or SIMSD_STEP_DECODED
   if (i < gamma) {
     const int v = mu[i];
-    bool bad = v < 0 || v > gamma;
-    if (!bad && v != 0)
+    bool bad = v < SIMSD_STEP_DECODED || v > gamma;
+    if (!bad && v > 0)
       for (int k = 0; k < i; ++k) bad |= (mu[k] == v);
     if (bad) map_ok = 0;
   }
   __syncthreads();
   if (i == 0 && !map_ok) raise_error(err_word, SIMSD_EW_STEP_MAP);
   if (i < S) {
-    const int k = i < gamma ? i : i - gamma;
-    const bool pad = !map_ok || mu[k] == 0;
-    const int t = pad ? 0 : mu[k];
-    const uint8_t sec = pad ? kSectPad : (i < gamma ? kSectData : kSectMask);
+    const bool is_data = i < gamma;
+    const int k = is_data ? i : i - gamma;
+    const int v = map_ok ? mu[k] : 0;
+    // drafted: both slots at tau = v; undrafted: a mask placeholder after
+    // every draft step; decoded: a data token known before every step
+    int t = 0;
+    uint8_t sec = kSectPad;
+    if (v > 0) {
+      t = v;
+      sec = is_data ? kSectData : kSectMask;
+    } else if (v == SIMSD_STEP_UNDRAFTED && !is_data) {
+      t = gamma + 1;
+      sec = kSectMask;
+    } else if (v == SIMSD_STEP_DECODED && is_data) {
+      t = 0;
+      sec = kSectData;
+    }
     s_tau[i] = t;
     s_sect[i] = sec;
     const size_t o = static_cast<size_t>(b) * S + i;

@@ -23,7 +23,8 @@ Recipe (one per workload, all values seeded):
   * drafts: with probability p the row's argmax (torch.argmax), otherwise a
     uniform token in [0, V);
   * step map: the identity (left-to-right) unless a random permutation is
-    requested;
+    requested; blocks with fewer drafts than positions draw the number of
+    drafted, earlier-decoded and still-[MASK] positions uniformly;
   * stochastic acceptance: target logits ~ N(0, sigma^2); the draft model's
     logits are the target's plus N(0, (eta sigma)^2) noise (eta sets how
     often drafts are accepted); each draft is drawn from the draft model's
@@ -209,6 +210,30 @@ def make_step_inputs(w: Workload, device="cpu", seed: Optional[int] = None, pref
     dev = torch.device(device)
     return StepInputs(w, n.to(dev), bt.to(dev), num_pages, sm.to(dev), q, k_new, v_new, k_cache, v_cache,
                       logits, draft.to(dev), row_valid)
+
+
+STEP_UNDRAFTED, STEP_DECODED = -1, -2
+
+
+def block_step_maps(Bt: int, gamma: int, seed: int, n_draft=None, pad_frac: float = 0.0) -> torch.Tensor:
+    """Step maps of blocks with fewer drafts than positions: per sequence a
+    random number of drafted positions (labels 1..n in a random order, or
+    exactly n_draft), a random number of positions decoded earlier in the
+    block (-2), the rest left [MASK] (-1), then padding (0) with probability
+    pad_frac.  n_draft = 0 gives the target's own block decoding."""
+    g = _cpu_gen(seed)
+    out = torch.empty(Bt, gamma, dtype=torch.int32)
+    for b in range(Bt):
+        nd = int(torch.randint(0, gamma + 1, (1,), generator=g)) if n_draft is None else min(n_draft, gamma)
+        ndec = int(torch.randint(0, gamma - nd + 1, (1,), generator=g))
+        pos = torch.randperm(gamma, generator=g)
+        row = torch.full((gamma,), STEP_UNDRAFTED, dtype=torch.int32)
+        row[pos[:nd]] = (torch.randperm(nd, generator=g) + 1).to(torch.int32)
+        row[pos[nd:nd + ndec]] = STEP_DECODED
+        if pad_frac > 0:
+            row[torch.rand(gamma, generator=g) < pad_frac] = 0
+        out[b] = row
+    return out
 
 
 @dataclasses.dataclass

@@ -22,6 +22,7 @@ SIMSD_OK, SIMSD_ERR_INVALID_ARG, SIMSD_ERR_UNSUPPORTED, SIMSD_ERR_CUDA, SIMSD_ER
 SIMSD_F32, SIMSD_BF16 = 0, 1
 SECT_DATA, SECT_MASK, SECT_PAD = 0, 1, 255
 EW_STEP_MAP, EW_PREFIX_LEN, EW_PAGE, EW_DRAFT, EW_TIMEOUT, EW_ACCEPT_LEN = 1, 2, 4, 8, 16, 32
+STEP_UNDRAFTED, STEP_DECODED = -1, -2
 
 EXPORTED = ("simsd_build_mask", "simsd_verify_workspace_bytes", "simsd_verify_attention",
             "simsd_verify_attention_noalloc", "simsd_accept", "simsd_accept_sampled", "simsd_kv_commit",

@@ -6,6 +6,8 @@ tails, page-boundary prefixes, every page size the kernel takes, split and
 unsplit prefixes, row blocks, non-identity step maps, padding, poisoned
 unused cache rows, harder score distributions, and the error paths.
 """
+import dataclasses
+
 import numpy as np
 import pytest
 import torch
@@ -123,6 +125,27 @@ def test_padding_slots_and_error_paths():
     assert word == werr and word & simsd.EW_PREFIX_LEN and word & simsd.EW_PAGE and word & simsd.EW_STEP_MAP
     assert_attention_close(out, want, "bf16")
     assert (out[1:4].float() == 0).all() and (out[0, [2, 6]].float() == 0).all()
+
+
+@pytest.mark.parametrize("dtype,gamma,n_draft", [("f32", 4, None), ("bf16", 4, None), ("bf16", 8, None),
+                                                 ("bf16", 16, 0), ("bf16", 32, None), ("bf16", 8, 0)])
+def test_undrafted_and_decoded_positions(dtype, gamma, n_draft):
+    # blocks with fewer drafts than positions; n_draft 0 is the target's own
+    # (bidirectional) block decoding
+    w = _w(dtype, Bt=6, gamma=gamma, prefix=(0, 700), seed=gamma)
+    si = inputs.make_step_inputs(w, device="cuda", random_step_map=True)
+    si.step_map = inputs.block_step_maps(w.Bt, gamma, seed=gamma + 1, n_draft=n_draft, pad_frac=0.1).cuda()
+    _check(si)
+
+
+@pytest.mark.parametrize("name", ["c2", "c3"])
+def test_full_size_target_block_decoding(name):
+    # the target's own block decoding at full size: every sequence's block
+    # is decoded-or-[MASK]; the oracle checks a few sequences
+    w = dataclasses.replace(inputs.WORKLOADS[name], layers=1)
+    si = inputs.make_step_inputs(w, device="cuda", with_logits=False)
+    si.step_map = inputs.block_step_maps(w.Bt, w.gamma, seed=5, n_draft=0).cuda()
+    _check(si, seqs=[0, w.Bt // 2, w.Bt - 1])
 
 
 def test_deterministic():

@@ -40,6 +40,31 @@ def test_commit_bit_exact(dtype, L, gamma, P):
     np.testing.assert_array_equal(inputs.host_bits(si.v_cache), rv)
 
 
+@pytest.mark.parametrize("gamma", [4, 16])
+def test_commit_with_undrafted_and_decoded_positions(gamma):
+    # only drafted data slots are ever committed: a decoded slot (tau 0) and
+    # an undrafted one (no data slot) never match an accepted step
+    n = [0, 63, 64, 5, 200, 127, 31, 9]
+    si = _commit_case("bf16", 2, gamma, 16, n, seed=gamma)
+    si.step_map = inputs.block_step_maps(len(n), gamma, seed=gamma + 3).cuda()
+    drafted = (si.step_map > 0).sum(1).cpu().numpy()
+    rng = np.random.default_rng(gamma)
+    a = torch.as_tensor(np.array([rng.integers(0, k + 1) for k in drafted], np.int32), device="cuda")
+    tau, sect, _, _, err = gpu_mask(si, mask_bits=False)
+    kc0, vc0 = si.k_cache.clone(), si.v_cache.clone()
+    nn = si.prefix_len.clone()
+    simsd.simsd_kv_commit(si.k_new, si.v_new, tau, sect, a, si.k_cache, si.v_cache, si.block_table, nn, err)
+    word = simsd.simsd_check_error(err)
+    rk, rv, rn, rerr = orc.kv_commit(inputs.host_bits(si.k_new), inputs.host_bits(si.v_new),
+                                     si.step_map.cpu().numpy(), a.cpu().numpy(), inputs.host_bits(kc0),
+                                     inputs.host_bits(vc0), si.block_table.cpu().numpy(),
+                                     si.prefix_len.cpu().numpy(), gamma)
+    assert word == rerr == 0
+    np.testing.assert_array_equal(nn.cpu().numpy(), rn)
+    np.testing.assert_array_equal(inputs.host_bits(si.k_cache), rk)
+    np.testing.assert_array_equal(inputs.host_bits(si.v_cache), rv)
+
+
 def test_commit_error_paths():
     si = _commit_case("bf16", 2, 4, 16, [0, 14, 30, 7], seed=1)
     sm = si.step_map.clone()

@@ -41,6 +41,29 @@ def test_build_mask_bit_exact(gamma, identity):
     assert word == r["err"]
 
 
+@pytest.mark.parametrize("gamma", [1, 2, 3, 4, 8, 16, 32])
+@pytest.mark.parametrize("n_draft", [None, 0])
+def test_build_mask_undrafted_and_decoded_bit_exact(gamma, n_draft):
+    # blocks with fewer drafts than positions (n_draft None: random counts)
+    # and the target's own block decoding (n_draft 0)
+    Bt = 41
+    mu = inputs.block_step_maps(Bt, gamma, seed=7 * gamma, n_draft=n_draft, pad_frac=0.1).numpy()
+    mu[0] = [simsd.STEP_DECODED - 1] + [1] * (gamma - 1) if gamma > 1 else [-3]   # invalid: flagged, all padding
+    n = np.random.default_rng(gamma).integers(0, 5000, Bt).astype(np.int32)
+    w = inputs.Workload("m", "bf16", Bt, 2, 1, 128, gamma, (0, 0), 1, 8, 0.5, 1.0, 1.0, 0)
+    dev = torch.device("cuda")
+    si = inputs.StepInputs(w, torch.as_tensor(n, device=dev), None, 0, torch.as_tensor(mu, device=dev),
+                           *([None] * 7), None)
+    tau, sect, rope, bits, err = gpu_mask(si)
+    word = simsd.simsd_check_error(err)
+    r = orc.build_mask(mu, n, gamma)
+    np.testing.assert_array_equal(tau.cpu().numpy(), r["tau"])
+    np.testing.assert_array_equal(sect.cpu().numpy(), r["section"])
+    np.testing.assert_array_equal(rope.cpu().numpy(), r["rope_pos"])
+    np.testing.assert_array_equal(bits.cpu().numpy().view(np.uint64), r["mask_bits"])
+    assert word == r["err"] == simsd.EW_STEP_MAP
+
+
 def _accept_case(Bt, gamma, V, seed, p=0.6, std=2.0):
     g = torch.Generator(device="cuda").manual_seed(seed)
     logits = torch.randn(Bt, gamma + 1, V, generator=g, device="cuda") * std
