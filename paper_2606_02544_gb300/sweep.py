@@ -4,7 +4,9 @@ agreement (32 query / 8 KV heads, d 128, bf16, one layer, V 151936).
 
     python -m paper_2606_02544_gb300.sweep [--out table.md] [--steps 10]
         [--batch 1,8,32,128] [--prefix 512,2048,8192,32768]
-        [--gamma 4,8,16,32] [--agree 0.3,0.6,0.9]
+        [--gamma 4,8,16,32] [--agree 0.3,0.6,0.9] [--sampled]
+
+--sampled times the stochastic acceptance alone over batch x gamma instead.
 
 One JSON line per point on stdout.  Each point captures its step (mask,
 attention, acceptance, commit; the prefix lengths reset before every step)
@@ -83,6 +85,55 @@ def run_point(w: inputs.Workload, steps: int, peak: float) -> dict:
     return row
 
 
+def run_sampled_point(Bt: int, gamma: int, vocab: int, steps: int, peak: float) -> dict:
+    """Times simsd_accept_sampled alone (Sec. 3.2, Eq. (2)): one CUDA graph
+    of `steps` launches, L2 flushed before each when the logits fit in 4x L2,
+    every launch timed by events inside the graph."""
+    si = inputs.make_sampled_inputs(Bt, gamma, vocab, seed=Bt * 100 + gamma, device="cuda")
+    a = torch.empty(Bt, dtype=torch.int32, device="cuda")
+    ot = torch.empty(Bt, gamma + 1, dtype=torch.int32, device="cuda")
+    err = torch.zeros(1, dtype=torch.int32, device="cuda")
+    nbytes = Bt * (2 * gamma + 1) * vocab * 4          # every row read once
+    need_flush = nbytes < 4 * L2_BYTES
+    flush = torch.empty(2 * L2_BYTES, dtype=torch.uint8, device="cuda") if need_flush else None
+    ev = [[torch.cuda.Event(enable_timing=True, external=True) for _ in range(2)] for _ in range(steps)]
+
+    def call():
+        simsd.simsd_accept_sampled(si.target_logits, si.draft_logits, si.draft, si.u_accept, si.u_sample, a, ot,
+                                   temperature=si.temperature, err_word=err)
+
+    stream = torch.cuda.Stream()
+    stream.wait_stream(torch.cuda.current_stream())
+    with torch.cuda.stream(stream):
+        call()
+    torch.cuda.synchronize()
+    g = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(g, stream=stream):
+        for e in ev:
+            if flush is not None:
+                flush_l2(flush)
+            e[0].record()
+            call()
+            e[1].record()
+    for _ in range(2):
+        g.replay()
+    torch.cuda.synchronize()
+    ts = []
+    for _ in range(2):
+        g.replay()
+        torch.cuda.synchronize()
+        ts += [e[0].elapsed_time(e[1]) for e in ev]
+    assert simsd.simsd_check_error(err) == 0
+    t = statistics.median(ts)
+    gbs = nbytes / (t * 1e-3) / 1e9
+    row = {"kernel": "accept_sampled", "Bt": Bt, "gamma": gamma, "vocab": vocab, "us": round(t * 1e3, 2),
+           "algorithmic_bytes": nbytes, "gbs": round(gbs, 1), "frac": round(gbs / peak, 4),
+           "l2": "flushed" if need_flush else "larger than L2"}
+    del g, si, flush
+    torch.cuda.empty_cache()
+    return row
+
+
 def main(argv=None):
     ap = argparse.ArgumentParser(description=__doc__.split("\n\n")[0])
     ap.add_argument("--out", default=None, help="also write a markdown table here")
@@ -91,6 +142,8 @@ def main(argv=None):
     ap.add_argument("--prefix", default="512,2048,8192,32768")
     ap.add_argument("--gamma", default="4,8,16,32")
     ap.add_argument("--agree", default="0.3,0.6,0.9")
+    ap.add_argument("--sampled", action="store_true",
+                    help="time the stochastic acceptance alone over --batch x --gamma (V 151936)")
     args = ap.parse_args(argv)
     sel = lambda s, cast: {cast(x) for x in s.split(",")}
     bts, ns, gs, ps = sel(args.batch, int), sel(args.prefix, int), sel(args.gamma, int), sel(args.agree, float)
@@ -98,6 +151,20 @@ def main(argv=None):
     simsd.load_library()
     peak, kind = _hbm_peak()
     rows = []
+    if args.sampled:
+        for Bt in sorted(bts):
+            for gm in sorted(gs):
+                row = run_sampled_point(Bt, gm, 151936, args.steps, peak)
+                row["peak_gbs"], row["peak_source"] = peak, kind
+                print(json.dumps(row), flush=True)
+                rows.append(row)
+        if args.out:
+            with open(args.out, "w") as f:
+                f.write(f"| Bt | gamma | us | GB/s (rows read once) | of {peak:.0f} GB/s |\n|---|---|---|---|---|\n")
+                for r in rows:
+                    f.write(f"| {r['Bt']} | {r['gamma']} | {r['us']:.1f} | {r['gbs']:.0f} | "
+                            f"{100 * r['frac']:.1f}% |\n")
+        return
     for w in inputs.sweep_points():
         if w.Bt in bts and w.prefix[0] in ns and w.gamma in gs and w.p_agree in ps:
             row = run_point(w, args.steps, peak)

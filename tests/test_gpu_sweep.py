@@ -35,3 +35,10 @@ def test_sweep_point(Bt, n, gamma, p, seqs):
     assert_attention_close(st.out[0][torch.as_tensor(seqs, device="cuda")], want, "bf16")
     np.testing.assert_array_equal(st.accepted_len.cpu().numpy(), ra)
     np.testing.assert_array_equal(st.out_tokens.cpu().numpy(), rot)
+
+
+def test_sampled_sweep_point_runs_and_reports():
+    from paper_2606_02544_gb300 import sweep
+    row = sweep.run_sampled_point(4, 4, 151936, steps=3, peak=6800.0)
+    assert row["us"] > 0 and row["algorithmic_bytes"] == 4 * 9 * 151936 * 4
+    assert 0 < row["frac"] < 2
