@@ -8,7 +8,7 @@
 // row with plain float compares, and folds it into a 64-bit key per row in
 // shared memory when its row changes.
 // CTA 0 then gathers the CL partial keys per row through distributed shared
-// memory and walks the draft order.  No global scratch memory is used.
+// memory (one warp per row, one lane per CTA) and walks the draft order.  No global scratch memory is used.
 #include <cooperative_groups.h>
 #include <cuda_runtime.h>
 
@@ -159,17 +159,21 @@ __global__ void __launch_bounds__(kAcceptThreads) accept_kernel(const float* __r
   cluster.sync();
 
   if (c == 0) {
-    for (int r = tid; r < rows; r += kAcceptThreads) {
-      unsigned long long k = best[r];
-#pragma unroll 1
-      for (int peer = 1; peer < CL; ++peer) {
-        const unsigned long long* pb = cluster.map_shared_rank(best, peer);
-        const unsigned long long kp = pb[r];
+    // warp w gathers rows w, w+16, ...: lane p reads CTA p's key (all remote
+    // reads of a row in flight at once), then a shuffle maximum
+    const int warp = tid >> 5, lane = tid & 31;
+    for (int r = warp; r < rows; r += kAcceptThreads / 32) {
+      unsigned long long k = lane < CL ? *cluster.map_shared_rank(&best[r], lane) : 0ull;
+#pragma unroll
+      for (int o = 16; o > 0; o >>= 1) {
+        const unsigned long long kp = __shfl_xor_sync(0xffffffffu, k, o);
         k = k > kp ? k : kp;
       }
-      const int idx = static_cast<int>(~static_cast<uint32_t>(k & 0xFFFFFFFFull));
-      am[r] = idx;
-      if (row_argmax) row_argmax[static_cast<size_t>(b) * rows + r] = idx;
+      if (lane == 0) {
+        const int idx = static_cast<int>(~static_cast<uint32_t>(k & 0xFFFFFFFFull));
+        am[r] = idx;
+        if (row_argmax) row_argmax[static_cast<size_t>(b) * rows + r] = idx;
+      }
     }
     __syncthreads();
     if (tid < 32) {
