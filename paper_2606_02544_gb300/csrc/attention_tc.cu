@@ -80,6 +80,7 @@ struct TcParams {
   int32_t* err_word;
   int max_pages, page_size, num_pages;
   int Bt, gamma, S, Hq, Hkv, g, rb, rows_blk, s_blk, nsplit;
+  int sort;  // order sequences longest prefix first (grids of more than one wave)
   float scale_log2;
   RopeTable rope;
 };
@@ -91,7 +92,7 @@ struct alignas(1024) Smem {
   uint32_t tmem_base;
   int abort_flag;
   int seq_bad;
-  int b_sel;
+  int b_sel, n_sel;
   int32_t tau[64];
   uint8_t sect[64];
   int32_t pages[kPageCache];
@@ -154,13 +155,15 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm)
   // kernel's results are needed
   pdl_wait();
   pdl_launch_next();
-  // prefix lengths, staged in the (still unused) ring for the ranking
-  int32_t* nval = reinterpret_cast<int32_t*>(sm.ring[0]);
-  const bool sort = p.Bt <= 256;
-  if (sort)
+  // When the grid takes more than one wave, the sequences go longest prefix
+  // first: the prefix lengths are staged in the (still unused) ring and
+  // ranked.  In a single wave every CTA is resident at once and the order
+  // does not matter, so the CTA reads its own sequence's length only.
+  int b, n;
+  if (p.sort) {
+    int32_t* nval = reinterpret_cast<int32_t*>(sm.ring[0]);
     for (int i = tid; i < p.Bt; i += kThreads) nval[i] = p.prefix_len[i];
-  __syncthreads();
-  if (sort) {
+    __syncthreads();
     for (int i = tid; i < p.Bt; i += kThreads) {
       const int ni = nval[i];
       int r = 0;
@@ -168,14 +171,20 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm)
         const int nj = nval[j];
         r += (nj > ni) || (nj == ni && j < i);
       }
-      if (r == rank) sm.b_sel = i;
+      if (r == rank) {
+        sm.b_sel = i;
+        sm.n_sel = ni;
+      }
     }
     // the staging area is overwritten by TMA later
     fence_proxy_async_smem();
+    __syncthreads();
+    b = sm.b_sel;
+    n = sm.n_sel;
+  } else {
+    b = rank;
+    n = p.prefix_len[b];
   }
-  __syncthreads();
-  const int b = sm.b_sel;
-  const int n = p.prefix_len[b];
   const bool n_bad = n < 0 || static_cast<long long>(n) > static_cast<long long>(p.max_pages) * p.page_size;
   const int32_t* bt = p.block_table + static_cast<size_t>(b) * p.max_pages;
 
@@ -756,6 +765,7 @@ bool plan_attention_tc(int Bt, int gamma, int Hq, int Hkv, int max_pages, int pa
     ns = std::min(ns, 64);
   }
   pl.nsplit = ns;
+  pl.sort = (units * ns > slots && Bt <= 256) ? 1 : 0;
   pl.ws_bytes = ns > 1 ? static_cast<size_t>(units) * ns * pl.rows_blk * (kD + 2) * sizeof(float) : 0;
   *plan = pl;
   return true;
@@ -812,6 +822,7 @@ cudaError_t launch_attention_tc(const AttnTcArgs& a, const AttnTcPlan& pl, Encod
   p.rows_blk = pl.rows_blk;
   p.s_blk = pl.s_blk;
   p.nsplit = pl.nsplit;
+  p.sort = pl.sort;
   p.scale_log2 = a.scale * 1.4426950408889634f;
 
   {
