@@ -493,11 +493,16 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm)
 #pragma unroll
       for (int c = 0; c < kTile; ++c) x[c] = __uint_as_float(c < 32 ? sa[c] : sb[c - 32]);
       if (is_new || valid < kTile) {
-        // partial prefix tile or the tile of new slots: hide what the row may not see
+        // partial prefix tile or the tile of new slots: hide what the row may
+        // not see.  One bit word per row and a select per column: the rows of
+        // a warp see different new slots, so a per-column branch would
+        // diverge (it cost microseconds on the first tile).
+        const unsigned long long keep = is_new ? vis : (valid >= kTile ? ~0ull : ((1ull << valid) - 1ull));
+        const uint32_t klo = static_cast<uint32_t>(keep), khi = static_cast<uint32_t>(keep >> 32);
 #pragma unroll
         for (int c = 0; c < kTile; ++c) {
-          const bool see = c < valid && (!is_new || ((vis >> c) & 1ull));
-          x[c] = see ? x[c] : -INFINITY;
+          const uint32_t bit = ((c < 32 ? klo : khi) >> (c & 31)) & 1u;
+          x[c] = bit ? x[c] : -INFINITY;
         }
       }
       // raw-score maximum (pairwise tree); scale_log2 > 0 commutes with max
