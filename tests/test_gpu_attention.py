@@ -78,6 +78,38 @@ def test_bf16_split_and_unsplit(Bt):
     _check(si, seqs)
 
 
+@pytest.mark.parametrize("gamma,Hq,Hkv,P,prefix,Bt", [
+    (32, 32, 8, 64, [0, 1, 64, 700, 3000], 5),    # 256 rows: two row blocks, prefix split
+    (32, 32, 8, 16, [129, 2000], 2),               # small pages
+    (16, 64, 8, 64, [500, 4100, 63], 3),           # g = 8: two row blocks as well
+    (32, 32, 8, 256, None, 40),                    # many units, no split
+])
+def test_two_row_blocks(gamma, Hq, Hkv, P, prefix, Bt):
+    # more than 128 query rows per KV head: each unit runs as two row blocks
+    w = _w(Bt=Bt, Hq=Hq, Hkv=Hkv, gamma=gamma, P=P, prefix=(0, 1500), seed=gamma + P)
+    si = inputs.make_step_inputs(w, device="cuda", prefix_override=prefix, random_step_map=True,
+                                 poison_unused_rows=True)
+    seqs = None if Bt <= 5 else [0, 13, 27, 39]
+    _check(si, seqs)
+
+
+def test_two_row_blocks_error_paths():
+    w = _w(Bt=4, Hq=32, Hkv=8, gamma=32, seed=11)
+    si = inputs.make_step_inputs(w, device="cuda", prefix_override=[10, 100, 70, 5])
+    sm = si.step_map.clone()
+    sm[0, 2] = 0                                  # padding slot in sequence 0
+    sm[3, :2] = 1                                 # invalid map: all padding
+    si.step_map = sm
+    bt = si.block_table.clone()
+    bt[2, 1] = si.num_pages + 5                   # page id outside the pool
+    si.block_table = bt
+    out, word, _ = gpu_attention(si)
+    want, werr = oracle_attention(si)
+    assert word == werr and word & simsd.EW_PAGE and word & simsd.EW_STEP_MAP
+    assert_attention_close(out, want, "bf16")
+    assert (out[2:4].float() == 0).all() and (out[0, [2, 34]].float() == 0).all()
+
+
 @pytest.mark.parametrize("kind", ["unit_scores", "peaked", "growing"])
 def test_bf16_hard_score_distributions(kind):
     # Q,K ~ N(0,1): scores ~ N(0,1) after the 1/sqrt(d) scale; "peaked": one
