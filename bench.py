@@ -362,7 +362,7 @@ def _oracle_sample_step(orc, inputs, si, seqs, layers):
     return int(np.sum(a)) + len(seqs)
 
 
-def run_cpu_baseline(args, si, max_seconds=15.0):
+def run_cpu_baseline(args, si, max_seconds=12.0):
     """The oracle as it stands, on this host's cores, on a bounded sample of
     the workload: whole sequences (all layers), repeated until about
     max_seconds of CPU work.  Host-side marshalling is excluded: only the
@@ -383,8 +383,6 @@ def run_cpu_baseline(args, si, max_seconds=15.0):
         done_tokens += _oracle_sample_step(orc, inputs, si, [b], layers)
         t_used += time.perf_counter() - t0
         seqs_done += 1
-        if i >= w.Bt and t_used >= 1.0 and seqs_done >= w.Bt:
-            break
     return {"value": round(done_tokens / t_used, 2), "unit": UNIT, "cores": orc.max_threads(), "kind": "oracle",
             "sample": f"{seqs_done} whole sequences x {len(layers)} layers of {w.name} (mask, attention, accept, "
                       f"commit), one sequence per oracle call, {t_used:.1f} s"}
@@ -443,7 +441,8 @@ def main():
     ap.add_argument("--warmup", type=int, default=5)
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
     ap.add_argument("--workload", default=DEFAULT_WORKLOAD, choices=["c1", "c2", "c3", "c4"])
-    ap.add_argument("--cpu-seconds", type=float, default=15.0)
+    ap.add_argument("--cpu-seconds", type=float, default=12.0,
+                    help="oracle time of the cpu_baseline sample (whole sequences until this much is spent)")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--layers", type=int, default=None,
                     help="run only this many layers of the workload (a smaller case of the same per-layer "
