@@ -155,6 +155,9 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm)
   // kernel's results are needed
   pdl_wait();
   pdl_launch_next();
+  // the barriers and flags set by thread 0 above must be in place before the
+  // producer (another warp) issues its first load on them
+  __syncthreads();
   // When the grid takes more than one wave, the sequences go longest prefix
   // first: the prefix lengths are staged in the (still unused) ring and
   // ranked.  In a single wave every CTA is resident at once and the order
