@@ -73,6 +73,22 @@ def _traffic(workload, kernel):
         return None
 
 
+def combine_over_ranks(total_ms, local_tokens, world):
+    """Whole-job figures of N independent replicas (one per GPU, no data
+    exchange): the slowest rank's timed milliseconds and every rank's
+    verified tokens.  Needs an initialised process group when world > 1."""
+    if world <= 1:
+        return float(total_ms), float(local_tokens)
+    import torch
+    import torch.distributed as dist
+
+    t = torch.tensor([float(total_ms), float(local_tokens)], dtype=torch.float64)
+    tmax = t.clone()
+    dist.all_reduce(tmax, op=dist.ReduceOp.MAX)
+    dist.all_reduce(t, op=dist.ReduceOp.SUM)
+    return float(tmax[0]), float(t[1])
+
+
 class ClockSampler:
     """nvidia-smi clocks / throttle reasons sampled while the timed loop runs."""
 
@@ -225,16 +241,7 @@ def run_gpu(args):
 
     total_ms = sum(step_ms)
     local_tokens = tokens_per_step * K
-    if world > 1:
-        import torch.distributed as dist
-        t = torch.tensor([total_ms, float(local_tokens)], dtype=torch.float64)
-        tmax = t.clone()
-        dist.all_reduce(tmax, op=dist.ReduceOp.MAX)
-        dist.all_reduce(t, op=dist.ReduceOp.SUM)
-        total_ms_max = float(tmax[0])
-        all_tokens = float(t[1])
-    else:
-        total_ms_max, all_tokens = total_ms, float(local_tokens)
+    total_ms_max, all_tokens = combine_over_ranks(total_ms, local_tokens, world)
     value = all_tokens / (total_ms_max / 1e3)
 
     # ---- end to end through the public API with host buffers
@@ -251,10 +258,14 @@ def run_gpu(args):
                  "peak_source": peak_kind, "algorithmic_bytes_per_launch": int(attn_bytes),
                  "launch_us": round(attn_launch_ms * 1e3, 3),
                  "tensor_tflops": round(attn_flops / (attn_launch_ms * 1e-3) / 1e12, 2),
+                 "tensor_frac": round(attn_flops / (attn_launch_ms * 1e-3) / 1e12 / tf_peak, 4),
                  "traffic": _traffic(args.workload, "attention")}
     acc_roof = {"kernel": "simsd_accept (accept_kernel)", "bound": "hbm", "achieved": round(acc_gbs, 1),
                 "peak": hbm_peak, "unit": "GB/s", "frac": round(acc_gbs / hbm_peak, 4), "peak_source": peak_kind,
                 "algorithmic_bytes_per_launch": int(acc_bytes), "launch_us": round(acc_launch_ms * 1e3, 3),
+                # rows up to the first rejection only: what a kernel that stopped
+                # at the first mismatch would have to read
+                "early_stop_bytes": int(tokens_per_step) * int(wl.vocab) * 4,
                 "traffic": _traffic(args.workload, "accept")}
     dominant, other = (attn_roof, acc_roof) if attn_launch_ms * st.L >= acc_launch_ms else (acc_roof, attn_roof)
 

@@ -39,6 +39,14 @@ def _hbm_peak():
         return 6800.0, "fallback"
 
 
+def _tensor_peak():
+    try:
+        with open(os.path.join(_HERE, "..", "MEASURED_PEAKS.json")) as f:
+            return float(json.load(f)["bf16_tflops"])
+    except Exception:
+        return 1900.0
+
+
 def run_point(w: inputs.Workload, steps: int, peak: float) -> dict:
     si = inputs.make_step_inputs(w, device="cuda")
     st = VerifyStep(si, restore_prefix=True)
@@ -79,6 +87,7 @@ def run_point(w: inputs.Workload, steps: int, peak: float) -> dict:
            "step_us": round(t_step * 1e3, 2), "attention_us": round(t_attn * 1e3, 2),
            "attention_gbs": round(gbs, 1), "attention_frac": round(gbs / peak, 4),
            "attention_tflops": round(attn_flops / (t_attn * 1e-3) / 1e12, 1),
+           "attention_tensor_frac": round(attn_flops / (t_attn * 1e-3) / 1e12 / _tensor_peak(), 4),
            "l2": "flushed" if need_flush else "larger than L2"}
     del g, st, si, flush
     torch.cuda.empty_cache()
@@ -174,11 +183,13 @@ def main(argv=None):
     if args.out:
         with open(args.out, "w") as f:
             f.write("| Bt | prefix | gamma | p | tokens/s | step us | attention us | attention GB/s | "
-                    f"of {peak:.0f} GB/s |\n|---|---|---|---|---|---|---|---|---|\n")
+                    f"of {peak:.0f} GB/s | TFLOP/s | of {_tensor_peak():.0f} |\n"
+                    "|---|---|---|---|---|---|---|---|---|---|---|\n")
             for r in rows:
                 f.write(f"| {r['Bt']} | {r['prefix']} | {r['gamma']} | {r['p_agree']} | {r['tokens_per_s']:.0f} | "
                         f"{r['step_us']:.1f} | {r['attention_us']:.1f} | {r['attention_gbs']:.0f} | "
-                        f"{100 * r['attention_frac']:.1f}% |\n")
+                        f"{100 * r['attention_frac']:.1f}% | {r['attention_tflops']:.0f} | "
+                        f"{100 * r['attention_tensor_frac']:.1f}% |\n")
 
 
 if __name__ == "__main__":
