@@ -80,7 +80,6 @@ __global__ void __launch_bounds__(kAcceptThreads) accept_kernel(const float* __r
   __shared__ unsigned long long best[kMaxRows];
   __shared__ int am[kMaxRows];
   pdl_wait();
-  pdl_launch_next();
   cg::cluster_group cluster = cg::this_cluster();
   const int c = static_cast<int>(cluster.block_rank());
   const int CL = static_cast<int>(cluster.num_blocks());
@@ -155,6 +154,9 @@ __global__ void __launch_bounds__(kAcceptThreads) accept_kernel(const float* __r
     }
   }
   if (f0 + tid < f1) atomicMax(&best[cur], rb.key());
+  // the next kernel may be scheduled once the stream of logits is done
+  // (earlier, its waiting CTAs would sit beside this one's)
+  pdl_launch_next();
   __syncthreads();
   cluster.sync();
 

@@ -129,7 +129,6 @@ __global__ void __launch_bounds__(kSampThreads, UNROLL == 8 ? 2 : 1) accept_samp
   __shared__ int w_state;          // 1: the total weight was positive (set by CTA 0)
   __shared__ float mac[kSampWarps][kSampMacros];     // phase 2: weight of each macro-step
   pdl_wait();
-  pdl_launch_next();
   cg::cluster_group cluster = cg::this_cluster();
   const int CL = static_cast<int>(cluster.num_blocks());
   const int c = static_cast<int>(cluster.block_rank());
@@ -263,6 +262,8 @@ __global__ void __launch_bounds__(kSampThreads, UNROLL == 8 ? 2 : 1) accept_samp
     }
     if (f0 + 32 * warp < f1) flush();
   }
+  // the next kernel may be scheduled once the logits have streamed through
+  pdl_launch_next();
   __syncthreads();
   for (int r = tid; r < rows; r += kSampThreads) {
     float m = kEmpty, s = 0.f;

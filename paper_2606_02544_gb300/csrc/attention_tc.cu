@@ -81,6 +81,7 @@ struct TcParams {
   int max_pages, page_size, num_pages;
   int Bt, gamma, S, Hq, Hkv, g, rb, rows_blk, s_blk, nsplit;
   int sort;  // order sequences longest prefix first (grids of more than one wave)
+  int slots;  // CTAs resident at once: blocks past this start in a later wave
   float scale_log2;
   RopeTable rope;
 };
@@ -154,7 +155,12 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm)
   // the set-up above touches no global memory; from here on the previous
   // kernel's results are needed
   pdl_wait();
-  pdl_launch_next();
+  // A CTA of a later wave lets the next kernel in at once: the next grid can
+  // then fill the slots this grid's last wave leaves idle (consecutive
+  // layers).  First-wave CTAs let it in after their tile loop (below), so
+  // that in a single-wave grid no waiting CTA of the next kernel sits beside
+  // this one for its whole run (that cost up to 30 us at c3).
+  if (static_cast<int>(blockIdx.x) >= p.slots) pdl_launch_next();
   // the barriers and flags set by thread 0 above must be in place before the
   // producer (another warp) issues its first load on them
   __syncthreads();
@@ -591,6 +597,9 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm)
       if (lane == 0) mbar_arrive(smem_u32(&sm.bar_p));
     }
     if (!ok && lane == 0) signal_abort(sm, p.err_word);
+    // the next kernel on the stream may be scheduled now (its CTAs wait for
+    // this grid to finish anyway)
+    pdl_launch_next();
     // ---- epilogue: O of the last PV, scaled by 1/l
     const bool have_o = ok && ntiles > 0 && mbar_wait_warp(smem_u32(&sm.bar_pv), (ntiles - 1) & 1, abort_flag);
     if (have_o) tc_fence_after();
@@ -774,6 +783,7 @@ bool plan_attention_tc(int Bt, int gamma, int Hq, int Hkv, int max_pages, int pa
   }
   pl.nsplit = ns;
   pl.sort = (units * ns > slots && Bt <= 256) ? 1 : 0;
+  pl.slots = static_cast<int>(slots);
   pl.ws_bytes = ns > 1 ? static_cast<size_t>(units) * ns * pl.rows_blk * (kD + 2) * sizeof(float) : 0;
   *plan = pl;
   return true;
@@ -831,6 +841,7 @@ cudaError_t launch_attention_tc(const AttnTcArgs& a, const AttnTcPlan& pl, Encod
   p.s_blk = pl.s_blk;
   p.nsplit = pl.nsplit;
   p.sort = pl.sort;
+  p.slots = pl.slots;
   p.scale_log2 = a.scale * 1.4426950408889634f;
 
   {

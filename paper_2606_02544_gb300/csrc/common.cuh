@@ -32,8 +32,11 @@ __host__ __device__ __forceinline__ bool temporal_visible(uint8_t si, int ti, ui
 // launched so that it may start (set-up only) while the previous kernel on
 // the stream finishes: it calls pdl_wait() before it reads or writes any
 // memory that earlier work may touch, and pdl_launch_next() to let the next
-// kernel start its own set-up early.  The wait returns once the previous
-// grid has completed and its memory operations are visible.
+// kernel be scheduled (one thread per CTA is enough).  The wait returns once
+// the previous grid has completed and its memory operations are visible.
+// Short kernels trigger at once; the attention and acceptance kernels only
+// after their main loop, since CTAs of the next kernel that wait beside a
+// long-running one slowed it down.
 __device__ __forceinline__ void pdl_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
 __device__ __forceinline__ void pdl_launch_next() { asm volatile("griddepcontrol.launch_dependents;" ::: "memory"); }
 

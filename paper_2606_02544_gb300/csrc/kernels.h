@@ -54,6 +54,7 @@ struct AttnTcPlan {
   int rows_blk;     // query rows per row block (<= 128)
   int s_blk;        // slots per row block
   int sort;         // more CTAs than resident slots: longest prefix first
+  int slots;        // CTAs resident at once (SMs x CTAs per SM)
   size_t ws_bytes;  // workspace bytes for the split partials (0 if nsplit == 1)
 };
 // Returns false if the shape is not supported by the tensor-core kernel.

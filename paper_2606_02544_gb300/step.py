@@ -71,11 +71,7 @@ class VerifyStep:
         rope = self.rope_pos if self.rope_theta > 0 else None
         if attn_events is not None:
             attn_events[0].record()
-        for l in range(self.L):
-            simsd.simsd_verify_attention(si.q[l], si.k_new[l], si.v_new[l], si.k_cache[l], si.v_cache[l],
-                                         si.block_table, self.n, self.tau, self.section, self.out[l],
-                                         workspace=self.workspace, err_word=self.err, rope_pos=rope,
-                                         rope_theta=self.rope_theta)
+        self.run_attention()
         if attn_events is not None:
             attn_events[1].record()
         simsd.simsd_accept(si.logits, si.draft, self.accepted_len, self.out_tokens, self.row_argmax,
@@ -83,6 +79,17 @@ class VerifyStep:
         simsd.simsd_kv_commit(si.k_new, si.v_new, self.tau, self.section, self.accepted_len, si.k_cache,
                               si.v_cache, si.block_table, self.n, err_word=self.err, rope_pos=rope,
                               rope_theta=self.rope_theta)
+
+    def run_attention(self):
+        """The layers' verification attention alone, on the step's current
+        mask metadata (the last step's simsd_build_mask)."""
+        si = self.si
+        rope = self.rope_pos if self.rope_theta > 0 else None
+        for l in range(self.L):
+            simsd.simsd_verify_attention(si.q[l], si.k_new[l], si.v_new[l], si.k_cache[l], si.v_cache[l],
+                                         si.block_table, self.n, self.tau, self.section, self.out[l],
+                                         workspace=self.workspace, err_word=self.err, rope_pos=rope,
+                                         rope_theta=self.rope_theta)
 
     def launches_per_step(self) -> int:
         """Kernels of this library launched by one step."""

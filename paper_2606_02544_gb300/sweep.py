@@ -6,13 +6,13 @@ agreement (32 query / 8 KV heads, d 128, bf16, one layer, V 151936).
         [--batch 1,8,32,128] [--prefix 512,2048,8192,32768]
         [--gamma 4,8,16,32] [--agree 0.3,0.6,0.9] [--sampled]
 
---sampled times the stochastic acceptance alone over batch x gamma instead.
-
 One JSON line per point on stdout.  Each point captures its step (mask,
 attention, acceptance, commit; the prefix lengths reset before every step)
-in a CUDA graph and times every step with CUDA events; attention is timed
-by events inside the same graph.  When a step's bytes are below 4x the L2
-size, L2 is flushed before every step.
+in a CUDA graph and times every step with CUDA events; the attention
+launches are timed in a graph of their own.  When a step's bytes are below
+4x the L2 size, L2 is flushed before every step.
+
+--sampled times the stochastic acceptance alone over batch x gamma instead.
 """
 from __future__ import annotations
 
@@ -53,12 +53,13 @@ def run_point(w: inputs.Workload, steps: int, peak: float) -> dict:
     attn_bytes, attn_flops, acc_bytes = algorithmic_bytes(si)
     need_flush = attn_bytes + acc_bytes < 4 * L2_BYTES
     flush = torch.empty(2 * L2_BYTES, dtype=torch.uint8, device="cuda") if need_flush else None
-    ev = [[torch.cuda.Event(enable_timing=True, external=True) for _ in range(4)] for _ in range(steps)]
+    ev = [[torch.cuda.Event(enable_timing=True, external=True) for _ in range(2)] for _ in range(steps)]
     stream = torch.cuda.Stream()
     stream.wait_stream(torch.cuda.current_stream())
     with torch.cuda.stream(stream):
         st.run()
     torch.cuda.synchronize()
+    # the steps (no event inside a step) and, apart, the attention launches
     g = torch.cuda.CUDAGraph()
     with torch.cuda.graph(g, stream=stream):
         for e in ev:
@@ -66,17 +67,29 @@ def run_point(w: inputs.Workload, steps: int, peak: float) -> dict:
                 flush_l2(flush)
             st.restore()
             e[0].record()
-            st.run(attn_events=(e[1], e[2]), restore=False)
-            e[3].record()
+            st.run(restore=False)
+            e[1].record()
+    ea = [[torch.cuda.Event(enable_timing=True, external=True) for _ in range(2)] for _ in range(steps)]
+    ga = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(ga, stream=stream):
+        for e in ea:
+            if flush is not None:
+                flush_l2(flush)
+            e[0].record()
+            st.run_attention()
+            e[1].record()
     for _ in range(2):
         g.replay()
+        ga.replay()
     torch.cuda.synchronize()
     step_ms, attn_ms = [], []
     for _ in range(2):
         g.replay()
         torch.cuda.synchronize()
-        step_ms += [e[0].elapsed_time(e[3]) for e in ev]
-        attn_ms += [e[1].elapsed_time(e[2]) for e in ev]
+        step_ms += [e[0].elapsed_time(e[1]) for e in ev]
+        ga.replay()
+        torch.cuda.synchronize()
+        attn_ms += [e[0].elapsed_time(e[1]) for e in ea]
     assert simsd.simsd_check_error(st.err) == 0
     tokens = st.verified_tokens()
     t_step = statistics.median(step_ms)
