@@ -317,39 +317,80 @@ def run_gpu(args):
 def run_e2e(args, si, st, stream):
     """Verified tokens/s through the public API with pinned host inputs:
     every step copies Q, K_new, V_new, logits, drafts and the step map host ->
-    device, runs the step graph and reads accepted lengths + tokens back."""
+    device, runs the step and reads accepted lengths + tokens back.  Two input
+    sets alternate so that the copy of step k+1 (on a copy stream) overlaps
+    step k (on the compute stream); the host reads step k's results while
+    step k+1 runs."""
+    import dataclasses
+
     import torch
 
-    g1 = torch.cuda.CUDAGraph()
-    with torch.cuda.graph(g1, stream=stream):
-        st.run()
-    host_in = {k: getattr(si, k).cpu().pin_memory() for k in ("q", "k_new", "v_new", "logits", "draft", "step_map")}
-    h_a = torch.empty_like(st.accepted_len, device="cpu").pin_memory()
-    h_t = torch.empty_like(st.out_tokens, device="cpu").pin_memory()
+    from paper_2606_02544_gb300.step import VerifyStep
+
+    keys = ("q", "k_new", "v_new", "logits", "draft", "step_map")
+    host_in = {k: getattr(si, k).cpu().pin_memory() for k in keys}
+    # the second set has its own inputs and outputs and shares the caches;
+    # steps still run one after the other on the compute stream
+    si_b = dataclasses.replace(si, **{k: getattr(si, k).clone() for k in keys})
+    sets = [st, VerifyStep(si_b, restore_prefix=True, rope_theta=st.rope_theta)]
+    graphs = []
+    for s_ in sets:
+        with torch.cuda.stream(stream):
+            s_.run()
+        torch.cuda.synchronize()
+        g = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(g, stream=stream):
+            s_.run()
+        graphs.append(g)
+    h_a = [torch.empty_like(st.accepted_len, device="cpu").pin_memory() for _ in sets]
+    h_t = [torch.empty_like(st.out_tokens, device="cpu").pin_memory() for _ in sets]
     bi = sum(t.numel() * t.element_size() for t in host_in.values())
-    bo = h_a.numel() * 4 + h_t.numel() * 4
+    bo = h_a[0].numel() * 4 + h_t[0].numel() * 4
     steps = max(3, min(args.steps, 200 if si.w.layers == 1 else 10))
+    copy_stream = torch.cuda.Stream()
+    copied = [torch.cuda.Event() for _ in sets]
+    done = [torch.cuda.Event() for _ in sets]
     e0 = torch.cuda.Event(enable_timing=True)
     e1 = torch.cuda.Event(enable_timing=True)
+
+    def issue(k):
+        x = k % 2
+        s_ = sets[x]
+        with torch.cuda.stream(copy_stream):
+            if k >= 2:
+                copy_stream.wait_event(done[x])          # step k-2 is done with this set
+            for name, t in host_in.items():
+                getattr(s_.si, name).copy_(t, non_blocking=True)
+            copied[x].record(copy_stream)
+        with torch.cuda.stream(stream):
+            stream.wait_event(copied[x])
+            graphs[x].replay()
+            h_a[x].copy_(s_.accepted_len, non_blocking=True)
+            h_t[x].copy_(s_.out_tokens, non_blocking=True)
+            done[x].record(stream)
+
     tokens = 0
-    with torch.cuda.stream(stream):
-        for i in range(steps + 2):
-            if i == 2:
-                torch.cuda.synchronize()
-                e0.record(stream)
-                tokens = 0
-            for k, t in host_in.items():
-                getattr(si, k).copy_(t, non_blocking=True)
-            g1.replay()
-            h_a.copy_(st.accepted_len, non_blocking=True)
-            h_t.copy_(st.out_tokens, non_blocking=True)
-            stream.synchronize()
-            tokens += int(h_a.sum()) + si.w.Bt
-        e1.record(stream)
+    warm = 2
+    torch.cuda.synchronize()
+    for k in range(warm + steps):
+        if k == warm:
+            done[(k - 1) % 2].synchronize()
+            e0.record(stream)
+            tokens = 0
+        issue(k)
+        if k >= warm + 1:
+            x = (k - 1) % 2
+            done[x].synchronize()                         # step k-1's results on the host
+            tokens += int(h_a[x].sum()) + si.w.Bt
+    x = (warm + steps - 1) % 2
+    done[x].synchronize()
+    tokens += int(h_a[x].sum()) + si.w.Bt
+    e1.record(stream)
     torch.cuda.synchronize()
     ms = e0.elapsed_time(e1)
     return {"value": round(tokens / (ms / 1e3), 1), "unit": UNIT, "h2d_bytes_per_step": int(bi),
-            "d2h_bytes_per_step": int(bo), "steps": steps, "ms_per_step": round(ms / steps, 4)}
+            "d2h_bytes_per_step": int(bo), "steps": steps, "ms_per_step": round(ms / steps, 4),
+            "overlap": "inputs of step k+1 copied (copy stream) while step k runs"}
 
 
 # ----------------------------------------------------------------------------
