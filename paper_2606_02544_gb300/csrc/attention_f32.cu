@@ -1,11 +1,13 @@
 // attention_f32.cu -- fp32 verification attention on CUDA cores (the paper's
-// own runs are fp32, Sec. 4.1).  One warp per query row.  Keys go in chunks
-// of 32: the paged prefix rows, then the new slots admitted by Eq. (1);
-// each lane scores one key of the chunk, the warp folds the chunk into a
-// running max / sum (online softmax) and accumulates V with lanes over the
-// head dimension.  When the inputs are not rotated yet (Sec. 3.1 RoPE copy),
-// the query row is rotated once in shared memory and each new key on the
-// fly while it is scored; cached keys are stored rotated.
+// own runs are fp32, Sec. 4.1).  One CTA per query row; its warps split the
+// keys in chunks of 32 (chunk c goes to warp c mod kF32Warps): the paged
+// prefix rows, then the new slots admitted by Eq. (1).  Each lane scores
+// one key of the chunk, the warp folds the chunk into its running max / sum
+// (online softmax) and accumulates V with lanes over the head dimension; the
+// warps' partial (max, sum, accumulator) are merged through shared memory at
+// the end.  When the inputs are not rotated yet (Sec. 3.1 RoPE copy), the
+// query row is rotated once in shared memory and each new key on the fly
+// while it is scored; cached keys are stored rotated.
 #include <cuda_runtime.h>
 
 #include "common.cuh"
@@ -17,15 +19,16 @@ constexpr int kF32Warps = 4;
 
 template <int DPL>  // head-dim elements per lane (d = 32 * DPL)
 __global__ void __launch_bounds__(kF32Warps * 32) attention_f32_kernel(const __grid_constant__ AttnF32Args a) {
-  __shared__ __align__(16) float q_s[kF32Warps][32 * DPL];
+  constexpr int d = 32 * DPL;
+  __shared__ __align__(16) float q_s[d];
+  __shared__ float acc_s[kF32Warps][d];
+  __shared__ float m_s[kF32Warps], l_s[kF32Warps];
+  __shared__ int ok_s;
   pdl_wait();
   pdl_launch_next();
   const int lane = threadIdx.x & 31, wib = threadIdx.x >> 5;
-  const long long row = (static_cast<long long>(blockIdx.x) * blockDim.x + threadIdx.x) >> 5;
+  const long long row = blockIdx.x;
   const int S = 2 * a.gamma, g = a.Hq / a.Hkv;
-  constexpr int d = 32 * DPL;
-  const long long rows = static_cast<long long>(a.Bt) * S * a.Hq;
-  if (row >= rows) return;
   const int h = static_cast<int>(row % a.Hq);
   const int s = static_cast<int>((row / a.Hq) % S);
   const int b = static_cast<int>(row / (static_cast<long long>(a.Hq) * S));
@@ -33,48 +36,48 @@ __global__ void __launch_bounds__(kF32Warps * 32) attention_f32_kernel(const __g
   float* o = a.out + row * d;
 
   const int n = a.prefix_len[b];
-  bool ok = n >= 0 && static_cast<long long>(n) <= static_cast<long long>(a.max_pages) * a.page_size;
-  if (!ok && lane == 0 && s == 0 && h == 0) raise_error(a.err_word, SIMSD_EW_PREFIX_LEN);
-  if (ok) {
-    const int npages = (n + a.page_size - 1) / a.page_size;
-    bool bad = false;
-    for (int p = lane; p < npages; p += 32) {
-      const int pg = a.block_table[static_cast<size_t>(b) * a.max_pages + p];
-      bad |= (pg < 0 || pg >= a.num_pages);
-    }
-    if (__any_sync(0xffffffffu, bad)) {
-      ok = false;
-      if (lane == 0 && s == 0 && h == 0) raise_error(a.err_word, SIMSD_EW_PAGE);
-    }
-  }
   const uint8_t si = a.section[static_cast<size_t>(b) * S + s];
-  if (!ok || si == kSectPad) {
-#pragma unroll
-    for (int c = 0; c < DPL; ++c) o[lane + 32 * c] = 0.f;
+  if (wib == 0) {
+    bool ok = n >= 0 && static_cast<long long>(n) <= static_cast<long long>(a.max_pages) * a.page_size;
+    if (!ok && lane == 0 && s == 0 && h == 0) raise_error(a.err_word, SIMSD_EW_PREFIX_LEN);
+    if (ok) {
+      const int npages = (n + a.page_size - 1) / a.page_size;
+      bool bad = false;
+      for (int p = lane; p < npages; p += 32) {
+        const int pg = a.block_table[static_cast<size_t>(b) * a.max_pages + p];
+        bad |= (pg < 0 || pg >= a.num_pages);
+      }
+      if (__any_sync(0xffffffffu, bad)) {
+        ok = false;
+        if (lane == 0 && s == 0 && h == 0) raise_error(a.err_word, SIMSD_EW_PAGE);
+      }
+    }
+    if (lane == 0) ok_s = ok && si != kSectPad;
+  }
+  for (int c = threadIdx.x; c < d; c += blockDim.x) q_s[c] = a.q[row * d + c];
+  __syncthreads();
+  if (!ok_s) {
+    for (int c = threadIdx.x; c < d; c += blockDim.x) o[c] = 0.f;
     return;
   }
   const int ti = a.tau[static_cast<size_t>(b) * S + s];
-#pragma unroll
-  for (int c = 0; c < DPL; ++c) q_s[wib][lane + 32 * c] = a.q[row * d + lane + 32 * c];
-  __syncwarp();
   if (a.rope_pos) {
     const int pos = a.rope_pos[static_cast<size_t>(b) * S + s];
-#pragma unroll
-    for (int i = lane; i < d / 2; i += 32) {
+    for (int i = threadIdx.x; i < d / 2; i += blockDim.x) {
       float sn, cs;
       rope_sincos(pos, a.rope.f[i], &sn, &cs);
-      rope_pair(q_s[wib][i], q_s[wib][i + d / 2], sn, cs);
+      rope_pair(q_s[i], q_s[i + d / 2], sn, cs);
     }
-    __syncwarp();
+    __syncthreads();
   }
   float acc[DPL];
 #pragma unroll
   for (int c = 0; c < DPL; ++c) acc[c] = 0.f;
   float m = -INFINITY, l = 0.f;
   // keys 0..n-1 are the prefix rows, keys n..n+S-1 the new slots; lane j of
-  // each chunk of 32 scores key base+j, then the warp folds the chunk in
+  // a chunk of 32 scores key base+j, then the warp folds the chunk in
   const int nkeys = n + S;
-  for (int base = 0; base < nkeys; base += 32) {
+  for (int base = 32 * wib; base < nkeys; base += 32 * kF32Warps) {
     const int j = base + lane;
     const float* kr = nullptr;
     long long voff = -1;
@@ -96,7 +99,7 @@ __global__ void __launch_bounds__(kF32Warps * 32) attention_f32_kernel(const __g
     if (kr) {
       float dot = 0.f;
       const float4* k4 = reinterpret_cast<const float4*>(kr);
-      const float4* q4 = reinterpret_cast<const float4*>(q_s[wib]);
+      const float4* q4 = reinterpret_cast<const float4*>(q_s);
       if (!from_cache && a.rope_pos) {
         // new key: rotate each (i, i + d/2) pair at its slot's position
         const int pos = a.rope_pos[static_cast<size_t>(b) * S + (j - n)];
@@ -164,14 +167,35 @@ __global__ void __launch_bounds__(kF32Warps * 32) attention_f32_kernel(const __g
     }
     m = m_new;
   }
-  const float inv = l > 0.f ? 1.f / l : 0.f;
+  // merge the warps: O = sum_w e^(m_w - M) acc_w / sum_w e^(m_w - M) l_w
+  if (lane == 0) {
+    m_s[wib] = m;
+    l_s[wib] = l;
+  }
 #pragma unroll
-  for (int c = 0; c < DPL; ++c) o[lane + 32 * c] = acc[c] * inv;
+  for (int c = 0; c < DPL; ++c) acc_s[wib][lane + 32 * c] = acc[c];
+  __syncthreads();
+  float M = -INFINITY;
+#pragma unroll
+  for (int w = 0; w < kF32Warps; ++w) M = fmaxf(M, m_s[w]);
+  float L = 0.f, f[kF32Warps];
+#pragma unroll
+  for (int w = 0; w < kF32Warps; ++w) {
+    f[w] = m_s[w] == -INFINITY ? 0.f : expf(m_s[w] - M);
+    L = fmaf(f[w], l_s[w], L);
+  }
+  const float inv = L > 0.f ? 1.f / L : 0.f;
+  for (int c = threadIdx.x; c < d; c += blockDim.x) {
+    float v = 0.f;
+#pragma unroll
+    for (int w = 0; w < kF32Warps; ++w) v = fmaf(f[w], acc_s[w][c], v);
+    o[c] = v * inv;
+  }
 }
 
 cudaError_t launch_attention_f32(const AttnF32Args& a, cudaStream_t stream) {
   const long long rows = static_cast<long long>(a.Bt) * 2 * a.gamma * a.Hq;
-  const unsigned blocks = static_cast<unsigned>((rows + kF32Warps - 1) / kF32Warps);
+  const unsigned blocks = static_cast<unsigned>(rows);  // one CTA per query row
   if (a.d == 64) return launch_overlapped(attention_f32_kernel<2>, dim3(blocks), dim3(kF32Warps * 32), 0, stream, 1, a);
   return launch_overlapped(attention_f32_kernel<4>, dim3(blocks), dim3(kF32Warps * 32), 0, stream, 1, a);
 }
