@@ -35,6 +35,7 @@
 // and makes the whole CTA stop, drain its async work and free its TMEM.
 #include <cuda.h>
 #include <cuda_bf16.h>
+#include <cooperative_groups.h>
 #include <cuda_runtime.h>
 
 #include <algorithm>
@@ -51,6 +52,8 @@
 // the runtime for the device address once per device (below).
 static __device__ __align__(256) unsigned char g_noalloc_scratch[12u << 20];
 
+namespace cg = cooperative_groups;
+
 namespace simsd {
 namespace {
 
@@ -65,6 +68,11 @@ constexpr int kWarpMma = 5;
 constexpr uint32_t kTmemCols = 256;
 constexpr uint32_t kColQ = 0, kColS = 64, kColO = 128;
 constexpr int kHalfBytes = kTile * 128;     // 64 rows x 64 bf16 (one d-half of K or V)
+// Split merge in place (fused): per-row partials in the ring, padded rows
+constexpr int kMaxSplitFuse = 8;            // cluster of at most 8 splits
+constexpr int kPartStride = kD + 4;         // floats per partial row (no bank conflicts)
+constexpr int kPartMl = kRows * kPartStride;              // (m, l) per row
+constexpr int kPartWts = kPartMl + 2 * kRows;             // merge weights [row][split]
 constexpr int kSlotBytes = 4 * kHalfBytes;  // K0 K1 V0 V1, or Q0 Q1 (16 KB each)
 constexpr int kPageCache = 512;             // page ids of one sequence kept in shared memory
 constexpr float kRescaleThreshold = 8.0f;   // log2 units: rescale when the max grows by > 2^8
@@ -82,6 +90,7 @@ struct TcParams {
   int Bt, gamma, S, Hq, Hkv, g, rb, rows_blk, s_blk, nsplit;
   int sort;  // order sequences longest prefix first (grids of more than one wave)
   int slots;  // CTAs resident at once: blocks past this start in a later wave
+  int fuse;   // the prefix splits of a unit form a cluster and merge in shared memory
   float scale_log2;
   RopeTable rope;
 };
@@ -101,6 +110,8 @@ struct alignas(1024) Smem {
 
 constexpr size_t smem_bytes() { return sizeof(Smem) + 1024; }
 static_assert(kCtasPerSm * (smem_bytes() + 1024) <= 233472, "two CTAs per SM");
+static_assert((kPartWts + (kRows / 2) * kMaxSplitFuse) * sizeof(float) <= sizeof(Smem::ring),
+              "the fused split merge fits in the ring");
 
 __device__ __forceinline__ void signal_abort(Smem& sm, int32_t* err_word) {
   raise_error(err_word, SIMSD_EW_TIMEOUT);
@@ -112,6 +123,10 @@ __device__ __forceinline__ uint4 ld_sw128_chunk(const uint8_t* half, int r, int 
   return *reinterpret_cast<const uint4*>(half + r * 128 + ((c ^ (r & 7)) << 4));
 }
 
+// kFuse: the prefix splits of a unit form a cluster and merge their partials
+// in shared memory (a separate instantiation, so that the unclustered kernel
+// carries no cluster barriers).
+template <bool kFuse>
 __global__ void __launch_bounds__(kThreads, kCtasPerSm)
     attention_tc_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ CUtensorMap tm_kn,
                         const __grid_constant__ CUtensorMap tm_vn, const __grid_constant__ CUtensorMap tm_kc,
@@ -121,12 +136,20 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm)
   volatile int* abort_flag = &sm.abort_flag;
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
 
-  // ---- which unit this CTA computes; sequences go longest prefix first
+  // ---- which unit this CTA computes; sequences go longest prefix first.
+  // Merged in place, the splits of a unit are adjacent (one cluster);
+  // otherwise the splits of a sequence follow one another.
   const int per_seq = p.nsplit * p.Hkv * p.rb;
   const int rank = blockIdx.x / per_seq;
   int rem = blockIdx.x - rank * per_seq;
-  const int split = rem / (p.Hkv * p.rb);
-  rem -= split * p.Hkv * p.rb;
+  int split;
+  if (kFuse) {
+    split = rem % p.nsplit;
+    rem /= p.nsplit;
+  } else {
+    split = rem / (p.Hkv * p.rb);
+    rem -= split * p.Hkv * p.rb;
+  }
   const int kvh = rem / p.rb;
   const int rblk = rem - kvh * p.rb;
 
@@ -159,7 +182,8 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm)
   // then fill the slots this grid's last wave leaves idle (consecutive
   // layers).  First-wave CTAs let it in after their tile loop (below), so
   // that in a single-wave grid no waiting CTA of the next kernel sits beside
-  // this one for its whole run (that cost up to 30 us at c3).
+  // this one for its whole run (that cost up to 30 us with 32 sequences of
+  // 4096-token prefixes).
   if (static_cast<int>(blockIdx.x) >= p.slots) pdl_launch_next();
   // the barriers and flags set by thread 0 above must be in place before the
   // producer (another warp) issues its first load on them
@@ -308,6 +332,10 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm)
   const int t0 = static_cast<int>(static_cast<long long>(split) * T_all / p.nsplit);
   const int t1 = static_cast<int>(static_cast<long long>(split + 1) * T_all / p.nsplit);
   const int ntiles = t1 - t0;
+
+  // fused split merge: what the softmax thread of this row hands over
+  bool fz_any = false, fz_have = false;
+  float fz_m = -INFINITY, fz_l = 0.f;
 
   if (warp == kWarpProducer) {
     // ------------------------------------------------------------ producer
@@ -598,14 +626,22 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm)
     }
     if (!ok && lane == 0) signal_abort(sm, p.err_word);
     // the next kernel on the stream may be scheduled now (its CTAs wait for
-    // this grid to finish anyway)
-    pdl_launch_next();
+    // this grid to finish anyway).  A clustered grid lets it in only when
+    // its CTAs exit: next-kernel CTAs placed beside clusters still merging
+    // cost more than they gain (measured at 8 sequences, 4 splits each).
+    if (!kFuse) pdl_launch_next();
     // ---- epilogue: O of the last PV, scaled by 1/l
     const bool have_o = ok && ntiles > 0 && mbar_wait_warp(smem_u32(&sm.bar_pv), (ntiles - 1) & 1, abort_flag);
     if (have_o) tc_fence_after();
     const bool any = have_o && active && l_sum > 0.f;
     const int h = kvh * p.g + hl;
-    if (p.nsplit == 1) {
+    if (kFuse) {
+      // written to the ring after the whole CTA is done with it (below)
+      fz_any = any;
+      fz_have = have_o;
+      fz_m = m_ref;
+      fz_l = l_sum;
+    } else if (p.nsplit == 1) {
       const float inv = any ? 1.0f / l_sum : 0.f;
       __nv_bfloat16* orow = p.out + ((static_cast<size_t>(b) * p.S + s) * p.Hq + h) * kD;
 #pragma unroll 1
@@ -655,6 +691,102 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm)
         wml[1] = any ? l_sum : 0.f;
       }
     }
+  }
+
+  if (kFuse) {
+    // Merge of the splits of this unit, O = sum_i 2^(m_i - M) O_i / sum_i
+    // 2^(m_i - M) l_i: CTA c of the cluster takes rows c, c + nsplit, ...,
+    // reading every split's partials through distributed shared memory.
+    // First this CTA's partial O (unnormalised) and (m, l) of each row go
+    // into the ring, once every load and MMA of the CTA has completed.
+    cg::cluster_group cluster = cg::this_cluster();
+    float* part = reinterpret_cast<float*>(sm.ring[0]);
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    if (warp < 4) {
+      const int row = tid;
+      const uint32_t lane_tmem = tmem + (static_cast<uint32_t>(warp * 32) << 16);
+#pragma unroll 1
+      for (int ch = 0; ch < kD / 32; ++ch) {
+        uint32_t o[32];
+        if (fz_have) {
+          tmem_ld32(lane_tmem + kColO + 32 * ch, o);
+          tmem_wait_ld();
+        }
+        if (row < p.rows_blk) {
+          float4* dst = reinterpret_cast<float4*>(part + row * kPartStride + 32 * ch);
+#pragma unroll
+          for (int c = 0; c < 8; ++c)
+            dst[c] = fz_any ? make_float4(__uint_as_float(o[4 * c]), __uint_as_float(o[4 * c + 1]),
+                                          __uint_as_float(o[4 * c + 2]), __uint_as_float(o[4 * c + 3]))
+                            : make_float4(0.f, 0.f, 0.f, 0.f);
+        }
+      }
+      if (row < p.rows_blk) {
+        part[kPartMl + 2 * row] = fz_any ? fz_m : -INFINITY;
+        part[kPartMl + 2 * row + 1] = fz_any ? fz_l : 0.f;
+      }
+    }
+    cluster.sync();  // every split's partials are in place
+    if (warp < 4) {
+      // Every remote load of a step is issued before its first use, so one
+      // round trip through distributed shared memory serves all splits.
+      const int nsp = p.nsplit;
+      float* wts = part + kPartWts;  // [row of this CTA][split]
+      const int nrows = (p.rows_blk - split + nsp - 1) / nsp;
+      for (int k = tid; k < nrows; k += 128) {
+        const int r = split + k * nsp;
+        float2 ml[kMaxSplitFuse];
+#pragma unroll
+        for (int i = 0; i < kMaxSplitFuse; ++i)
+          ml[i] = i < nsp ? *reinterpret_cast<const float2*>(cluster.map_shared_rank(part, i) + kPartMl + 2 * r)
+                          : make_float2(-INFINITY, 0.f);
+        float M = -INFINITY;
+#pragma unroll
+        for (int i = 0; i < kMaxSplitFuse; ++i)
+          if (ml[i].y > 0.f) M = fmaxf(M, ml[i].x);
+        float w[kMaxSplitFuse], L = 0.f;
+#pragma unroll
+        for (int i = 0; i < kMaxSplitFuse; ++i) {
+          w[i] = (M != -INFINITY && ml[i].y > 0.f) ? exp2f(ml[i].x - M) : 0.f;
+          L = fmaf(w[i], ml[i].y, L);
+        }
+        const float inv = L > 0.f ? 1.f / L : 0.f;
+#pragma unroll
+        for (int i = 0; i < kMaxSplitFuse; ++i) wts[k * kMaxSplitFuse + i] = w[i] * inv;
+      }
+      asm volatile("bar.sync 1, 128;" ::: "memory");
+      constexpr int kVec = kD / 4;
+      for (int e = tid; e < nrows * kVec; e += 128) {
+        const int k = e / kVec, c4 = e - k * kVec;
+        const int r = split + k * nsp;
+        float4 x[kMaxSplitFuse];
+#pragma unroll
+        for (int i = 0; i < kMaxSplitFuse; ++i)
+          if (i < nsp) x[i] = *reinterpret_cast<const float4*>(cluster.map_shared_rank(part, i) + r * kPartStride + 4 * c4);
+        float4 v = make_float4(0.f, 0.f, 0.f, 0.f);
+#pragma unroll
+        for (int i = 0; i < kMaxSplitFuse; ++i) {
+          if (i < nsp) {
+            const float wi = wts[k * kMaxSplitFuse + i];
+            v.x = fmaf(wi, x[i].x, v.x);
+            v.y = fmaf(wi, x[i].y, v.y);
+            v.z = fmaf(wi, x[i].z, v.z);
+            v.w = fmaf(wi, x[i].w, v.w);
+          }
+        }
+        const int sr = rblk * p.s_blk + r / p.g;
+        if (sr < p.S) {
+          const int hr = kvh * p.g + r % p.g;
+          uint2 pk;
+          pk.x = pack_bf16x2(v.x, v.y);
+          pk.y = pack_bf16x2(v.z, v.w);
+          *reinterpret_cast<uint2*>(p.out + ((static_cast<size_t>(b) * p.S + sr) * p.Hq + hr) * kD + 4 * c4) = pk;
+        }
+      }
+    }
+    cluster.sync();  // no CTA leaves while a peer may still read its partials
   }
 
   tc_fence_before();
@@ -734,13 +866,15 @@ __global__ void __launch_bounds__(128) combine_kernel(const __grid_constant__ Tc
 cudaError_t ensure_smem_attr() {
   static bool done = false;
   if (done) return cudaSuccess;
-  cudaError_t e = cudaFuncSetAttribute(attention_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                       static_cast<int>(smem_bytes()));
-  if (e != cudaSuccess) return e;
-  e = cudaFuncSetAttribute(attention_tc_kernel, cudaFuncAttributePreferredSharedMemoryCarveout,
-                           cudaSharedmemCarveoutMaxShared);
-  if (e == cudaSuccess) done = true;
-  return e;
+  for (auto kern : {attention_tc_kernel<false>, attention_tc_kernel<true>}) {
+    cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                         static_cast<int>(smem_bytes()));
+    if (e != cudaSuccess) return e;
+    e = cudaFuncSetAttribute(kern, cudaFuncAttributePreferredSharedMemoryCarveout, cudaSharedmemCarveoutMaxShared);
+    if (e != cudaSuccess) return e;
+  }
+  done = true;
+  return cudaSuccess;
 }
 
 bool make_map(EncodeTiledFn encode, CUtensorMap* m, const void* base, int rank, const cuuint64_t* dims,
@@ -783,8 +917,11 @@ bool plan_attention_tc(int Bt, int gamma, int Hq, int Hkv, int max_pages, int pa
   }
   pl.nsplit = ns;
   pl.sort = (units * ns > slots && Bt <= 256) ? 1 : 0;
+  // up to 8 splits merge in place (a cluster per unit), more through the
+  // workspace and combine_kernel
+  pl.fuse = (ns >= 2 && ns <= kMaxSplitFuse) ? 1 : 0;
   pl.slots = static_cast<int>(slots);
-  pl.ws_bytes = ns > 1 ? static_cast<size_t>(units) * ns * pl.rows_blk * (kD + 2) * sizeof(float) : 0;
+  pl.ws_bytes = (ns > 1 && !pl.fuse) ? static_cast<size_t>(units) * ns * pl.rows_blk * (kD + 2) * sizeof(float) : 0;
   *plan = pl;
   return true;
 }
@@ -841,6 +978,7 @@ cudaError_t launch_attention_tc(const AttnTcArgs& a, const AttnTcPlan& pl, Encod
   p.s_blk = pl.s_blk;
   p.nsplit = pl.nsplit;
   p.sort = pl.sort;
+  p.fuse = pl.fuse;
   p.slots = pl.slots;
   p.scale_log2 = a.scale * 1.4426950408889634f;
 
@@ -849,9 +987,12 @@ cudaError_t launch_attention_tc(const AttnTcArgs& a, const AttnTcPlan& pl, Encod
     if (e != cudaSuccess) return e;
   }
   const long long grid = static_cast<long long>(a.Bt) * pl.nsplit * a.Hkv * pl.rb;
-  cudaError_t e = launch_overlapped(attention_tc_kernel, dim3(static_cast<unsigned>(grid)), dim3(kThreads),
-                                    smem_bytes(), stream, 1, tq, tkn, tvn, tkc, tvc, p);
-  if (e != cudaSuccess || pl.nsplit == 1) return e;
+  cudaError_t e = pl.fuse ? launch_overlapped(attention_tc_kernel<true>, dim3(static_cast<unsigned>(grid)),
+                                               dim3(kThreads), smem_bytes(), stream,
+                                               static_cast<unsigned>(pl.nsplit), tq, tkn, tvn, tkc, tvc, p)
+                          : launch_overlapped(attention_tc_kernel<false>, dim3(static_cast<unsigned>(grid)),
+                                              dim3(kThreads), smem_bytes(), stream, 1u, tq, tkn, tvn, tkc, tvc, p);
+  if (e != cudaSuccess || pl.nsplit == 1 || pl.fuse) return e;
   const long long warps = static_cast<long long>(a.Bt) * a.Hkv * pl.rb * pl.rows_blk;
   return launch_overlapped(combine_kernel, dim3(static_cast<unsigned>((warps + 3) / 4)), dim3(128), 0, stream, 1, p);
 }

@@ -55,6 +55,7 @@ struct AttnTcPlan {
   int s_blk;        // slots per row block
   int sort;         // more CTAs than resident slots: longest prefix first
   int slots;        // CTAs resident at once (SMs x CTAs per SM)
+  int fuse;         // 2..8 splits merge in place (cluster per unit), no workspace
   size_t ws_bytes;  // workspace bytes for the split partials (0 if nsplit == 1)
 };
 // Returns false if the shape is not supported by the tensor-core kernel.

@@ -78,6 +78,25 @@ def test_bf16_split_and_unsplit(Bt):
     _check(si, seqs)
 
 
+@pytest.mark.parametrize("Bt,prefix,fused", [
+    (1, 150, True), (1, 450, True), (1, 1000, True), (3, 900, True), (5, 2000, True), (6, 2000, True),
+    (10, 1500, True), (13, 1500, True), (1, 1200, False), (2, 3000, False), (4, 2500, False), (1, 5000, False),
+])
+def test_split_counts_merged_in_place_and_through_workspace(Bt, prefix, fused):
+    # Bt * Hkv units split their prefixes to fill the GPU: 2 to 8 splits of
+    # a unit form a cluster and merge in shared memory (no workspace), more
+    # write partials to the workspace for the combine kernel.  The prefix
+    # lengths fall from the given one, so short sequences leave some splits
+    # without a tile.
+    w = _w(Bt=Bt, Hq=32, Hkv=8, gamma=8, prefix=(0, prefix), seed=prefix + Bt)
+    lens = [max(0, prefix - 137 * i) for i in range(Bt)]
+    si = inputs.make_step_inputs(w, device="cuda", prefix_override=lens, random_step_map=True,
+                                 poison_unused_rows=True)
+    ws = simsd.simsd_verify_workspace_bytes(simsd.SIMSD_BF16, Bt, 8, 32, 8, 128, si.block_table.shape[1], 64)
+    assert (ws == 0) == fused
+    _check(si)
+
+
 @pytest.mark.parametrize("gamma,Hq,Hkv,P,prefix,Bt", [
     (32, 32, 8, 64, [0, 1, 64, 700, 3000], 5),    # 256 rows: two row blocks, prefix split
     (32, 32, 8, 16, [129, 2000], 2),               # small pages
