@@ -175,6 +175,14 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm)
     tmem_alloc(smem_u32(&sm.tmem_base), kTmemCols);
     tmem_relinquish();
   }
+  if (warp == kWarpProducer && lane == 0) {
+    // the tensor maps are kernel parameters, not results of earlier work
+    tma_prefetch_desc(&tm_q);
+    tma_prefetch_desc(&tm_kn);
+    tma_prefetch_desc(&tm_vn);
+    tma_prefetch_desc(&tm_kc);
+    tma_prefetch_desc(&tm_vc);
+  }
   // the set-up above touches no global memory; from here on the previous
   // kernel's results are needed
   pdl_wait();
@@ -192,7 +200,7 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm)
   // first: the prefix lengths are staged in the (still unused) ring and
   // ranked.  In a single wave every CTA is resident at once and the order
   // does not matter, so the CTA reads its own sequence's length only.
-  int b, n;
+  int b, n = 0;
   if (p.sort) {
     int32_t* nval = reinterpret_cast<int32_t*>(sm.ring[0]);
     for (int i = tid; i < p.Bt; i += kThreads) nval[i] = p.prefix_len[i];
@@ -216,9 +224,7 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm)
     n = sm.n_sel;
   } else {
     b = rank;
-    n = p.prefix_len[b];
   }
-  const bool n_bad = n < 0 || static_cast<long long>(n) > static_cast<long long>(p.max_pages) * p.page_size;
   const int32_t* bt = p.block_table + static_cast<size_t>(b) * p.max_pages;
 
   // ---- TMA issue of ring items (producer thread only): item 0 is Q, item
@@ -281,26 +287,35 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm)
       tma_load_3d(v1, &tm_vn, bv, 64, kvh, b * p.S);
     }
   };
-  // Q and the tile of new slots need no page id: they are issued before the
-  // page table is checked.  If the check fails they are drained unused.
+  // Q, and in split 0 the tile of new slots, need neither the prefix length
+  // nor a page id: they go out first.  If the sequence turns out to be
+  // invalid they are drained unused.
   int early = 0;
   if (warp == kWarpProducer && lane == 0) {
-    tma_prefetch_desc(&tm_q);
-    tma_prefetch_desc(&tm_kc);
-    tma_prefetch_desc(&tm_vc);
-    if (!n_bad) {
-      issue_q();
-      early = 1;
-      const int tg = (n + kTile - 1) / kTile + 1;  // tiles of a valid sequence
-      const int t0g = static_cast<int>(static_cast<long long>(split) * tg / p.nsplit);
-      const int t1g = static_cast<int>(static_cast<long long>(split + 1) * tg / p.nsplit);
-      if (t0g == 0 && t1g > 0) {
-        issue_tile(1, 0);
-        early = 2;
-      }
+    issue_q();
+    early = 1;
+    if (split == 0) {
+      issue_tile(1, 0);
+      early = 2;
     }
   }
-
+  // The prefix length, the sequence's page ids (up to the page cache) and
+  // its slot labels are read together: one memory latency instead of a
+  // chain.  Page ids past the prefix are loaded but not used.
+  if (!p.sort) n = p.prefix_len[b];
+  constexpr int kPgRegs = (kPageCache + kThreads - 1) / kThreads;
+  int pg_reg[kPgRegs];
+  const int pg_lim = min(p.max_pages, kPageCache);
+#pragma unroll
+  for (int j = 0; j < kPgRegs; ++j) {
+    const int i = tid + j * kThreads;
+    pg_reg[j] = i < pg_lim ? bt[i] : -1;
+  }
+  for (int i = tid; i < p.S; i += kThreads) {
+    sm.tau[i] = p.tau[static_cast<size_t>(b) * p.S + i];
+    sm.sect[i] = p.section[static_cast<size_t>(b) * p.S + i];
+  }
+  const bool n_bad = n < 0 || static_cast<long long>(n) > static_cast<long long>(p.max_pages) * p.page_size;
   if (n_bad) {
     if (tid == 0) {
       sm.seq_bad = 1;
@@ -308,18 +323,25 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm)
     }
   } else {
     const int npages = (n + p.page_size - 1) / p.page_size;
-    for (int i = tid; i < npages; i += kThreads) {
+#pragma unroll
+    for (int j = 0; j < kPgRegs; ++j) {
+      const int i = tid + j * kThreads;
+      if (i < npages && i < kPageCache) {
+        const int pg = pg_reg[j];
+        sm.pages[i] = pg;
+        if (pg < 0 || pg >= p.num_pages) {
+          sm.seq_bad = 1;
+          raise_error(p.err_word, SIMSD_EW_PAGE);
+        }
+      }
+    }
+    for (int i = kPageCache + tid; i < npages; i += kThreads) {
       const int pg = bt[i];
-      if (i < kPageCache) sm.pages[i] = pg;
       if (pg < 0 || pg >= p.num_pages) {
         sm.seq_bad = 1;
         raise_error(p.err_word, SIMSD_EW_PAGE);
       }
     }
-  }
-  for (int i = tid; i < p.S; i += kThreads) {
-    sm.tau[i] = p.tau[static_cast<size_t>(b) * p.S + i];
-    sm.sect[i] = p.section[static_cast<size_t>(b) * p.S + i];
   }
   tc_fence_before();
   __syncthreads();
@@ -329,8 +351,10 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm)
   const bool seq_bad = sm.seq_bad != 0;
   const int T = seq_bad ? 0 : (n + kTile - 1) / kTile;  // prefix tiles
   const int T_all = seq_bad ? 0 : T + 1;                 // tile 0: new slots, tiles 1..T: prefix
-  const int t0 = static_cast<int>(static_cast<long long>(split) * T_all / p.nsplit);
-  const int t1 = static_cast<int>(static_cast<long long>(split + 1) * T_all / p.nsplit);
+  // split i takes tiles [ceil(i T_all / nsplit), ceil((i + 1) T_all / nsplit)):
+  // split 0 always holds tile 0 (issued above)
+  const int t0 = static_cast<int>((static_cast<long long>(split) * T_all + p.nsplit - 1) / p.nsplit);
+  const int t1 = static_cast<int>((static_cast<long long>(split + 1) * T_all + p.nsplit - 1) / p.nsplit);
   const int ntiles = t1 - t0;
 
   // fused split merge: what the softmax thread of this row hands over
@@ -342,7 +366,7 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm)
     if (lane == 0) {
       int issued = early;
       if (ntiles > 0) {
-        // a valid sequence: Q (and the tile of new slots) went out already
+        // Q (and in split 0 the tile of new slots) went out already
         for (int i = issued - 1; i < ntiles; ++i) {
           const int it = i + 1, st = it % kStages;
           if (it >= kStages && !mbar_wait(smem_u32(&sm.bar_empty[st]), ((it / kStages) - 1) & 1, abort_flag)) {
@@ -426,10 +450,10 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm)
 
     // ---- Q: shared memory (ring slot 0) -> TMEM columns [0, 64)
     if (ntiles > 0) {
+      const int pos = p.rope_pos ? p.rope_pos[static_cast<size_t>(b) * p.S + (s < p.S ? s : 0)] : 0;
       ok = mbar_wait_warp(smem_u32(&sm.bar_k[0]), 0, abort_flag);
       if (ok && p.rope_pos) {
         // rotate this row's query at its slot's position on the way
-        const int pos = p.rope_pos[static_cast<size_t>(b) * p.S + (s < p.S ? s : 0)];
         const uint8_t* h0 = sm.ring[0];
         const uint8_t* h1 = sm.ring[0] + 2 * kHalfBytes;
         uint32_t q0r[32], q1r[32];
