@@ -7,8 +7,10 @@
 // streams 16-byte loads (8 in flight), keeps a running (value, index) per
 // row with plain float compares, and folds it into a 64-bit key per row in
 // shared memory when its row changes.
-// CTA 0 then gathers the CL partial keys per row through distributed shared
-// memory (one warp per row, one lane per CTA) and walks the draft order.  No global scratch memory is used.
+// Each CTA then writes its keys into CTA 0's shared memory (distributed
+// shared memory) and arrives on an mbarrier there, and exits; CTA 0 waits for
+// the CL arrivals, takes the maximum per row and walks the draft order.  No
+// global scratch memory is used.
 #include <cooperative_groups.h>
 #include <cuda_runtime.h>
 
@@ -16,6 +18,7 @@
 
 #include "common.cuh"
 #include "kernels.h"
+#include "ptx.cuh"
 
 namespace cg = cooperative_groups;
 
@@ -23,6 +26,7 @@ namespace simsd {
 
 constexpr int kAcceptThreads = 512;
 constexpr int kMaxRows = 33;  // gamma + 1 <= 33
+constexpr int kMaxCluster = 16;  // CTAs per sequence (non-portable cluster size)
 
 // Total order used by the argmax: larger key = better.  NaN ranks above every
 // number, -0.0 equals +0.0, and among equal values the lower index wins
@@ -78,8 +82,9 @@ __global__ void __launch_bounds__(kAcceptThreads) accept_kernel(const float* __r
                                                                 int32_t* __restrict__ out_tokens,
                                                                 int32_t* __restrict__ row_argmax, int32_t* err_word) {
   __shared__ unsigned long long best[kMaxRows];
+  __shared__ unsigned long long gath[kMaxCluster][kMaxRows];  // CTA 0: every CTA's keys
+  __shared__ __align__(8) unsigned long long gbar;              // CTA 0: one arrival per CTA
   __shared__ int am[kMaxRows];
-  pdl_wait();
   cg::cluster_group cluster = cg::this_cluster();
   const int c = static_cast<int>(cluster.block_rank());
   const int CL = static_cast<int>(cluster.num_blocks());
@@ -87,6 +92,16 @@ __global__ void __launch_bounds__(kAcceptThreads) accept_kernel(const float* __r
   const int rows = gamma + 1;
   const int tid = threadIdx.x;
   for (int r = tid; r < rows; r += kAcceptThreads) best[r] = 0ull;
+  if (c == 0 && tid == 0) {
+    mbar_init(smem_u32(&gbar), static_cast<uint32_t>(CL));
+    fence_mbar_init();
+  }
+  // CTA 0's barrier must be initialised before any CTA arrives on it: every
+  // thread arrives here and waits just before its first remote write
+  cluster_arrive_relaxed();
+  pdl_wait();
+  // the drafts are needed only at the end; their load is issued now
+  const int dr_lane = (c == 0 && tid < gamma) ? draft[static_cast<size_t>(b) * gamma + tid] : 0;
   __syncthreads();
 
   // This CTA owns one contiguous span of the sequence's [rows][vocab] block
@@ -158,53 +173,50 @@ __global__ void __launch_bounds__(kAcceptThreads) accept_kernel(const float* __r
   // (earlier, its waiting CTAs would sit beside this one's)
   pdl_launch_next();
   __syncthreads();
-  cluster.sync();
-
-  if (c == 0) {
-    // warp w gathers rows w, w+16, ...: lane p reads CTA p's key (all remote
-    // reads of a row in flight at once), then a shuffle maximum
-    const int warp = tid >> 5, lane = tid & 31;
-    for (int r = warp; r < rows; r += kAcceptThreads / 32) {
-      unsigned long long k = lane < CL ? *cluster.map_shared_rank(&best[r], lane) : 0ull;
-#pragma unroll
-      for (int o = 16; o > 0; o >>= 1) {
-        const unsigned long long kp = __shfl_xor_sync(0xffffffffu, k, o);
-        k = k > kp ? k : kp;
-      }
-      if (lane == 0) {
-        const int idx = static_cast<int>(~static_cast<uint32_t>(k & 0xFFFFFFFFull));
-        am[r] = idx;
-        if (row_argmax) row_argmax[static_cast<size_t>(b) * rows + r] = idx;
-      }
-    }
-    __syncthreads();
-    if (tid < 32) {
-      // drafts in tau order; lane r checks draft r (gamma <= 32)
-      const int lane = tid;
-      int dr = 0;
-      bool in_range = true, match = false;
-      if (lane < gamma) {
-        dr = draft[static_cast<size_t>(b) * gamma + lane];
-        in_range = dr >= 0 && dr < vocab;
-        match = in_range && dr == am[lane];
-      }
-      const unsigned bad = __ballot_sync(0xffffffffu, !in_range);
-      const unsigned miss = __ballot_sync(0xffffffffu, lane < gamma && !match);
-      const int a = miss ? (__ffs(miss) - 1) : gamma;
-      if (lane == 0) {
-        if (bad) raise_error(err_word, SIMSD_EW_DRAFT);
-        accepted_len[b] = a;
-      }
-      int32_t* ot = out_tokens + static_cast<size_t>(b) * rows;
-      for (int r = lane; r < rows; r += 32) ot[r] = r < a ? draft[static_cast<size_t>(b) * gamma + r] : (r == a ? am[a] : -1);
-    }
+  cluster_wait();
+  if (tid < 32) {
+    // warp 0 pushes this CTA's keys into CTA 0 and arrives there (release:
+    // the pushes of all lanes, ordered by the __syncwarp, go with it)
+    unsigned long long* dst = cluster.map_shared_rank(&gath[c][0], 0);
+    for (int r = tid; r < rows; r += 32) dst[r] = best[r];
+    __syncwarp();
+    if (tid == 0) mbar_arrive_cluster(smem_u32(&gbar), 0);
   }
-  cluster.sync();  // peers stay resident until CTA 0 has read their keys
+  // Nothing reads this CTA's shared memory: every CTA but CTA 0 is done.
+  if (c != 0 || tid >= 32) return;
+
+  // CTA 0, warp 0: lane r takes row r (and row 32 on lane 0)
+  const int lane = tid;
+  if (!mbar_wait_cluster_warp(smem_u32(&gbar), 0)) {
+    if (lane == 0) raise_error(err_word, SIMSD_EW_TIMEOUT);
+    return;
+  }
+  for (int r = lane; r < rows; r += 32) {
+    unsigned long long k = 0ull;
+    for (int p = 0; p < CL; ++p) k = gath[p][r] > k ? gath[p][r] : k;
+    const int idx = static_cast<int>(~static_cast<uint32_t>(k & 0xFFFFFFFFull));
+    am[r] = idx;
+    if (row_argmax) row_argmax[static_cast<size_t>(b) * rows + r] = idx;
+  }
+  __syncwarp();
+  // drafts in tau order; lane r checks draft r (gamma <= 32)
+  bool in_range = true, match = false;
+  if (lane < gamma) {
+    in_range = dr_lane >= 0 && dr_lane < vocab;
+    match = in_range && dr_lane == am[lane];
+  }
+  const unsigned bad = __ballot_sync(0xffffffffu, !in_range);
+  const unsigned miss = __ballot_sync(0xffffffffu, lane < gamma && !match);
+  const int a = miss ? (__ffs(miss) - 1) : gamma;
+  if (lane == 0) {
+    if (bad) raise_error(err_word, SIMSD_EW_DRAFT);
+    accepted_len[b] = a;
+  }
+  int32_t* ot = out_tokens + static_cast<size_t>(b) * rows;
+  for (int r = lane; r < rows; r += 32) ot[r] = r < a ? dr_lane : (r == a ? am[a] : -1);
 }
 
 namespace {
-
-constexpr int kMaxCluster = 16;
 
 // How many clusters of each size (1..16) the device keeps resident at once,
 // asked once per device from the occupancy calculator (clusters must fit in

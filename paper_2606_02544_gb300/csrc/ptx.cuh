@@ -51,6 +51,49 @@ __device__ __forceinline__ bool mbar_try_wait(uint32_t bar, uint32_t parity) {
   return done != 0;
 }
 
+// Arrive on the mbarrier at the same shared-memory offset in CTA `rank` of
+// the cluster, releasing this thread's earlier writes at cluster scope.
+__device__ __forceinline__ void mbar_arrive_cluster(uint32_t bar, uint32_t rank) {
+  uint32_t remote;
+  asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(remote) : "r"(bar), "r"(rank));
+  asm volatile("mbarrier.arrive.release.cluster.shared::cluster.b64 _, [%0];" ::"r"(remote) : "memory");
+}
+
+// try_wait that acquires at cluster scope (arrivals from other CTAs).
+__device__ __forceinline__ bool mbar_try_wait_cluster(uint32_t bar, uint32_t parity) {
+  uint32_t done;
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "mbarrier.try_wait.parity.acquire.cluster.shared::cta.b64 p, [%1], %2;\n\t"
+      "selp.u32 %0, 1, 0, p;\n\t}"
+      : "=r"(done)
+      : "r"(bar), "r"(parity)
+      : "memory");
+  return done != 0;
+}
+
+// Warp-uniform bounded wait (1 s) for arrivals from other CTAs of the
+// cluster; false on timeout.
+__device__ __forceinline__ bool mbar_wait_cluster_warp(uint32_t bar, uint32_t parity) {
+  const unsigned full = 0xffffffffu;
+  if (__all_sync(full, mbar_try_wait_cluster(bar, parity))) return true;
+  const unsigned long long t0 = globaltimer_ns();
+  for (uint32_t it = 1;; ++it) {
+    if (__all_sync(full, mbar_try_wait_cluster(bar, parity))) return true;
+    if ((it & 63u) == 0) {
+      int give_up = 0;
+      if ((threadIdx.x & 31) == 0) give_up = globaltimer_ns() - t0 > kWaitLimitNs;
+      if (__shfl_sync(full, give_up, 0)) return false;
+    }
+  }
+}
+
+// Split cluster barrier: arrive (no ordering) now, wait later.
+__device__ __forceinline__ void cluster_arrive_relaxed() {
+  asm volatile("barrier.cluster.arrive.relaxed.aligned;" ::: "memory");
+}
+__device__ __forceinline__ void cluster_wait() { asm volatile("barrier.cluster.wait.aligned;" ::: "memory"); }
+
 // Single-thread bounded wait for the phase with the given parity to
 // complete.  Returns false on timeout or when *abort becomes non-zero
 // (abort == nullptr: only the time limit ends the wait, as when draining).
