@@ -73,6 +73,13 @@ def _traffic(workload, kernel):
         return None
 
 
+def workload_config(wl, layers):
+    """The workload description both arms print in ``config``."""
+    return {"workload": wl.name, "Bt": wl.Bt, "Hq": wl.Hq, "Hkv": wl.Hkv, "head_dim": wl.d, "gamma": wl.gamma,
+            "prefix": list(wl.prefix), "layers": layers, "vocab": wl.vocab, "page_size": wl.page_size,
+            "p_agree": wl.p_agree, "seed": wl.seed, "draft_tokens_per_step": wl.Bt * wl.gamma}
+
+
 def combine_over_ranks(total_ms, local_tokens, world):
     """Whole-job figures of N independent replicas (one per GPU, no data
     exchange): the slowest rank's timed milliseconds and every rank's
@@ -294,10 +301,8 @@ def run_gpu(args):
             "warmup": warm_reps * M, "ms_per_step": round(total_ms_max / K, 5), "higher_is_better": True,
             "scaling": "weak", "vs_baseline": None, "dtype": "bf16" if wl.dtype == "bf16" else "f32",
             "data": "synthetic (seeded; SDAR-shaped Q/K/V, logits and drafts; no weights)",
-            "config": {"workload": wl.name, "Bt": wl.Bt, "Hq": wl.Hq, "Hkv": wl.Hkv, "head_dim": wl.d,
-                       "gamma": wl.gamma, "prefix": list(wl.prefix), "layers": st.L, "vocab": wl.vocab,
-                       "page_size": wl.page_size, "p_agree": wl.p_agree, "seed": wl.seed,
-                       "verified_tokens_per_step": tokens_per_step, "draft_tokens_per_step": wl.Bt * wl.gamma,
+            "config": {**workload_config(wl, st.L),
+                       "verified_tokens_per_step": tokens_per_step,
                        "l2": "flushed before every step (258 MB write + read)" if need_flush else
                        "inputs larger than L2 (no flush)",
                        "timing": f"CUDA graph of {M} steps; per-step CUDA events (the reset of the prefix "
@@ -497,7 +502,9 @@ def run_reference(args):
     line = {"impl": "reference", "metric": METRIC, "value": round(value, 2), "unit": UNIT, "n_gpus": world,
             "steps": args.steps, "warmup": args.warmup, "ms_per_step": round(1e3 * sum(times) / len(times), 3),
             "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
-            "dtype": "f64", "data": "synthetic (seeded)", "config": {"workload": wl.name},
+            "dtype": "f64", "data": "synthetic (seeded)",
+            "config": {**workload_config(wl, wl.layers),
+                       "timing": "the oracle on the host cores, wall clock per step of whole sequences"},
             "cpu_baseline": cpu,
             "e2e": {"value": round(value, 2), "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
     print(json.dumps(line), flush=True)
