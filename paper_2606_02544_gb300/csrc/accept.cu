@@ -4,7 +4,7 @@
 //
 // One thread-block cluster per sequence.  The CTAs of a cluster split the
 // sequence's [gamma+1][vocab] block into contiguous spans; each thread
-// streams 16-byte loads (8 in flight), keeps a running (value, index) per
+// streams 16-byte loads (8 or 16 in flight), keeps a running (value, index) per
 // row with plain float compares, and folds it into a 64-bit key per row in
 // shared memory when its row changes.
 // Each CTA then writes its keys into CTA 0's shared memory (distributed
