@@ -1,5 +1,7 @@
-// ptx.cuh -- thin inline-PTX wrappers for sm_103a: mbarrier, TMA tensor
-// loads, tcgen05 (TMEM allocation, MMA, commit, loads/stores, fences).
+// ptx.cuh -- thin inline-PTX wrappers for sm_103a: mbarrier (this CTA's
+// and, for arrivals from other CTAs of a cluster, cluster scope), the split
+// cluster barrier, TMA tensor loads, tcgen05 (TMEM allocation, MMA, commit,
+// loads/stores, fences).
 //
 // Every wait is bounded: after kWaitLimitNs of wall-clock time (read from
 // %globaltimer) the wait gives up and reports failure, so a protocol error
