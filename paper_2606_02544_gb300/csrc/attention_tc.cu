@@ -351,10 +351,26 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm)
   const bool seq_bad = sm.seq_bad != 0;
   const int T = seq_bad ? 0 : (n + kTile - 1) / kTile;  // prefix tiles
   const int T_all = seq_bad ? 0 : T + 1;                 // tile 0: new slots, tiles 1..T: prefix
-  // split i takes tiles [ceil(i T_all / nsplit), ceil((i + 1) T_all / nsplit)):
-  // split 0 always holds tile 0 (issued above)
-  const int t0 = static_cast<int>((static_cast<long long>(split) * T_all + p.nsplit - 1) / p.nsplit);
-  const int t1 = static_cast<int>((static_cast<long long>(split + 1) * T_all + p.nsplit - 1) / p.nsplit);
+  // Split 0 always holds tile 0 (issued above).  Split i takes tiles
+  // [ceil(i T_all / nsplit), ceil((i + 1) T_all / nsplit)); merged in a
+  // cluster, where the slowest split sets the pace, split 0 instead holds
+  // tile 0, the costliest (the Eq. (1) mask, zeroed V rows), plus tiles up
+  // to floor(T_all / nsplit) in all, and splits 1.. share the rest evenly,
+  // so the extra tiles of an uneven split go to splits without tile 0.
+  int t0, t1;
+  if (kFuse) {
+    const int first = T_all == 0 ? 0 : max(1, T_all / p.nsplit);
+    t0 = 0;
+    t1 = first;
+    if (split > 0) {
+      const long long rest = T_all - first, ns1 = p.nsplit - 1;
+      t0 = first + static_cast<int>(((split - 1) * rest + ns1 - 1) / ns1);
+      t1 = first + static_cast<int>((split * rest + ns1 - 1) / ns1);
+    }
+  } else {
+    t0 = static_cast<int>((static_cast<long long>(split) * T_all + p.nsplit - 1) / p.nsplit);
+    t1 = static_cast<int>((static_cast<long long>(split + 1) * T_all + p.nsplit - 1) / p.nsplit);
+  }
   const int ntiles = t1 - t0;
 
   // fused split merge: what the softmax thread of this row hands over
