@@ -94,12 +94,12 @@ def _run_accept(logits, draft):
 
 @pytest.mark.parametrize("Bt,gamma,V", [(1, 4, 1024), (8, 4, 151936), (32, 8, 151936), (64, 16, 151936),
                                         (3, 1, 151936), (5, 32, 50000), (200, 4, 4096), (7, 3, 1001),
-                                        (2, 5, 3), (1, 32, 151936), (2, 4, 64), (19, 8, 151936), (4, 16, 65540)])
+                                        (2, 5, 3), (1, 32, 151936), (2, 4, 64), (19, 8, 151936), (4, 16, 65540),
+                                        (700, 2, 512)])
 def test_accept_bit_exact(Bt, gamma, V):
-    # up to one sequence per 8 SMs the span of each CTA comes in through a
-    # ring of bulk copies (one sequence of 33 rows: 26 refills per CTA; a
-    # 64-token vocabulary: CTAs with a few units or none); more sequences, an
-    # odd vocabulary or an unaligned base stream through registers
+    # one cluster per sequence, from 16 CTAs (one sequence of 33 rows) down
+    # to single CTAs in several waves (700 sequences); a 64-token vocabulary
+    # leaves CTAs with a few units or none; odd vocabularies stream scalars
     logits, draft = _accept_case(Bt, gamma, V, seed=Bt * 100 + gamma)
     _run_accept(logits, draft)
 
