@@ -55,8 +55,11 @@ class VerifyStep:
 
     # ------------------------------------------------------------------
     def restore(self):
-        """Puts the original prefix lengths back (a 4*Bt-byte device copy)."""
-        self.n.copy_(self.n_orig, non_blocking=True)
+        """Puts the original prefix lengths back (4*Bt bytes).  An
+        elementwise kernel, not a memcpy: a memcpy would be queued on a copy
+        engine behind the next step's host-to-device input copies and hold
+        this step back until they finish."""
+        torch.mul(self.n_orig, 1, out=self.n)
 
     def run(self, attn_events=None, restore=None):
         """Issues the whole step on the current stream (eager or captured).
