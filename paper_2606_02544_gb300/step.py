@@ -22,7 +22,7 @@ class VerifyStep:
     """Device buffers and the call sequence of one verification step.
 
     ``restore_prefix`` copies the original prefix lengths back before each
-    step (a 4*Bt-byte device copy) so that repeated steps verify the same
+    step (4*Bt bytes, an elementwise kernel) so that repeated steps verify the same
     block against the same prefix: the commit writes rows past the original
     prefix, which the restored lengths never read.
     """
