@@ -43,12 +43,16 @@ __global__ void __launch_bounds__(kCommitWarps * 32) kv_commit_kernel(
   const int rank = static_cast<int>(cluster.block_rank());
   const int b = blockIdx.x / CL;
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  const int S = 2 * gamma;
   const int a = accepted_len[b];
   const int n = prefix_len[b];
+  // the labels of the data slots (lane k: slot k) do not depend on a or n:
+  // their loads go out together with those two
+  const bool lane_data = lane < gamma && section[static_cast<size_t>(b) * S + lane] == kSectData;
+  const int lane_tau = lane < gamma ? tau[static_cast<size_t>(b) * S + lane] : 0;
   // "n_b has been read"
   asm volatile("barrier.cluster.arrive.release;" ::: "memory");
   const bool ok = a >= 0 && a <= gamma && n >= 0;
-  const int S = 2 * gamma;
   if (ok) {
     const long long rows = static_cast<long long>(a) * L * Hkv;
     for (long long row = static_cast<long long>(rank) * kCommitWarps + warp; row < rows;
@@ -57,8 +61,7 @@ __global__ void __launch_bounds__(kCommitWarps * 32) kv_commit_kernel(
       const int r = static_cast<int>((row / Hkv) % a);
       const int l = static_cast<int>(row / (static_cast<long long>(Hkv) * a));
       // source: the data slot whose label is r+1
-      const bool hit = lane < gamma && section[static_cast<size_t>(b) * S + lane] == kSectData &&
-                       tau[static_cast<size_t>(b) * S + lane] == r + 1;
+      const bool hit = lane_data && lane_tau == r + 1;
       const unsigned m = __ballot_sync(0xffffffffu, hit);
       if (!m) {
         if (lane == 0) raise_error(err_word, SIMSD_EW_STEP_MAP);
