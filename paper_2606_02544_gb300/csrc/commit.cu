@@ -50,6 +50,9 @@ __global__ void __launch_bounds__(kCommitWarps * 32) kv_commit_kernel(
   // their loads go out together with those two
   const bool lane_data = lane < gamma && section[static_cast<size_t>(b) * S + lane] == kSectData;
   const int lane_tau = lane < gamma ? tau[static_cast<size_t>(b) * S + lane] : 0;
+  // the sequence's first 32 page ids (lane p: page p), likewise: a row that
+  // lands there takes its page id by a shuffle instead of a dependent load
+  const int lane_pg = lane < max_pages ? block_table[static_cast<size_t>(b) * max_pages + lane] : -1;
   // "n_b has been read"
   asm volatile("barrier.cluster.arrive.release;" ::: "memory");
   const bool ok = a >= 0 && a <= gamma && n >= 0;
@@ -74,7 +77,8 @@ __global__ void __launch_bounds__(kCommitWarps * 32) kv_commit_kernel(
         if (lane == 0) raise_error(err_word, SIMSD_EW_PAGE);
         continue;
       }
-      const int pg = block_table[static_cast<size_t>(b) * max_pages + pidx];
+      const int pg = pidx < 32 ? __shfl_sync(0xffffffffu, lane_pg, static_cast<int>(pidx))
+                               : block_table[static_cast<size_t>(b) * max_pages + pidx];
       if (pg < 0 || pg >= num_pages) {
         if (lane == 0) raise_error(err_word, SIMSD_EW_PAGE);
         continue;
