@@ -51,8 +51,10 @@ __global__ void __launch_bounds__(kCommitWarps * 32) kv_commit_kernel(
   const bool lane_data = lane < gamma && section[static_cast<size_t>(b) * S + lane] == kSectData;
   const int lane_tau = lane < gamma ? tau[static_cast<size_t>(b) * S + lane] : 0;
   // the sequence's first 32 page ids (lane p: page p), likewise: a row that
-  // lands there takes its page id by a shuffle instead of a dependent load
-  const int lane_pg = lane < max_pages ? block_table[static_cast<size_t>(b) * max_pages + lane] : -1;
+  // lands there takes its page id by a shuffle instead of a dependent load.
+  // With no layer there is no row to place, and the caller may pass no
+  // block table at all.
+  const int lane_pg = (L > 0 && lane < max_pages) ? block_table[static_cast<size_t>(b) * max_pages + lane] : -1;
   // "n_b has been read"
   asm volatile("barrier.cluster.arrive.release;" ::: "memory");
   const bool ok = a >= 0 && a <= gamma && n >= 0;
