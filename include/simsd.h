@@ -173,7 +173,9 @@ SIMSD_API int simsd_verify_attention(int dtype, const void* q, const void* k_new
  * library owns (every GPU that loads libsimsd.so holds it until the process
  * exits).  It allocates nothing and calls no allocating routine.
  *   - The first call on each device looks up the array's device address
- *     (cudaGetSymbolAddress); make that first call before any stream capture.
+ *     (cudaGetSymbolAddress) and keeps it for the life of the process; make
+ *     that first call before any stream capture.  Because the address is
+ *     kept, a cudaDeviceReset between calls is not supported.
  *   - Sizes whose scratch would exceed 12 MiB are rejected with
  *     SIMSD_ERR_UNSUPPORTED (see simsd_last_error); use
  *     simsd_verify_attention with a caller workspace for those.
@@ -274,6 +276,26 @@ SIMSD_API int simsd_kv_commit(int dtype, const void* k_new, const void* v_new, i
  * non-zero, SIMSD_OK otherwise.  The only call that synchronises.
  */
 SIMSD_API int simsd_check_error(const int32_t* err_word, int32_t* host_word, void* stream);
+
+/*
+ * simsd_debug_expire_next_wait -- test hook for failure detection; the paper
+ * has no counterpart.  Arms the next bf16 simsd_verify_attention
+ * (which = SIMSD_DEBUG_WAIT_ATTENTION) or simsd_accept
+ * (which = SIMSD_DEBUG_WAIT_ACCEPT) call made by this host thread so that
+ * one of its on-device barriers expects one arrival more than ever comes
+ * and its waits give up after limit_us microseconds (10..10^6) instead of
+ * 1 s.  The wait then runs out: the kernel sets SIMSD_EW_TIMEOUT, stops
+ * every warp, waits (with the full limit) for its own copies and MMAs in
+ * flight, frees its tensor memory and returns; the outputs of that call are
+ * undefined and the context stays usable.  Attention: the softmax warps'
+ * hand-off of P to the MMA issuer.  Acceptance: CTA 0's wait for the
+ * per-CTA row maxima; armed only where every sequence runs as a single CTA
+ * (a batch too large for one cluster per sequence to be resident), else the
+ * call returns SIMSD_ERR_UNSUPPORTED.  The arm is consumed by that call.
+ */
+#define SIMSD_DEBUG_WAIT_ATTENTION 1
+#define SIMSD_DEBUG_WAIT_ACCEPT 2
+SIMSD_API int simsd_debug_expire_next_wait(int which, unsigned int limit_us);
 
 /* Text of the last CUDA error seen by this thread (empty if none). */
 SIMSD_API const char* simsd_last_error(void);

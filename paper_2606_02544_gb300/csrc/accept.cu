@@ -80,7 +80,8 @@ __global__ void __launch_bounds__(kAcceptThreads) accept_kernel(const float* __r
                                                                 const int32_t* __restrict__ draft, int gamma,
                                                                 int vocab, int vec4, int32_t* __restrict__ accepted_len,
                                                                 int32_t* __restrict__ out_tokens,
-                                                                int32_t* __restrict__ row_argmax, int32_t* err_word) {
+                                                                int32_t* __restrict__ row_argmax, int32_t* err_word,
+                                                                uint32_t extra_arrivals, unsigned long long wait_ns) {
   __shared__ unsigned long long best[kMaxRows];
   __shared__ unsigned long long gath[kMaxCluster][kMaxRows];  // CTA 0: every CTA's keys
   __shared__ __align__(8) unsigned long long gbar;              // CTA 0: one arrival per CTA
@@ -93,7 +94,7 @@ __global__ void __launch_bounds__(kAcceptThreads) accept_kernel(const float* __r
   const int tid = threadIdx.x;
   for (int r = tid; r < rows; r += kAcceptThreads) best[r] = 0ull;
   if (c == 0 && tid == 0) {
-    mbar_init(smem_u32(&gbar), static_cast<uint32_t>(CL));
+    mbar_init(smem_u32(&gbar), static_cast<uint32_t>(CL) + extra_arrivals);
     fence_mbar_init();
   }
   // CTA 0's barrier must be initialised before any CTA arrives on it: every
@@ -187,7 +188,7 @@ __global__ void __launch_bounds__(kAcceptThreads) accept_kernel(const float* __r
 
   // CTA 0, warp 0: lane r takes row r (and row 32 on lane 0)
   const int lane = tid;
-  if (!mbar_wait_cluster_warp(smem_u32(&gbar), 0)) {
+  if (!mbar_wait_cluster_warp(smem_u32(&gbar), 0, wait_ns)) {
     if (lane == 0) raise_error(err_word, SIMSD_EW_TIMEOUT);
     return;
   }
@@ -265,7 +266,8 @@ cudaError_t cluster_capacity(const ClusterCapacity** out) {
 
 cudaError_t launch_accept(const float* logits, const int32_t* draft, int Bt, int gamma, int vocab,
                           int32_t* accepted_len, int32_t* out_tokens, int32_t* row_argmax, int32_t* err_word,
-                          int num_sms, cudaStream_t stream) {
+                          int num_sms, cudaStream_t stream, const WaitFault& fault) {
+  const unsigned long long wait_ns = fault.wait_ns ? fault.wait_ns : kWaitLimitNs;
   const int vec4 = (vocab % 4 == 0) && ((reinterpret_cast<uintptr_t>(logits) & 15u) == 0);
   const ClusterCapacity* cap = nullptr;
   // few sequences: the largest clusters still leave SMs idle, so each CTA
@@ -273,10 +275,12 @@ cudaError_t launch_accept(const float* logits, const int32_t* draft, int Bt, int
   if (Bt * kMaxCluster <= num_sms) {
     cudaError_t e = cluster_capacity<16>(&cap);
     if (e != cudaSuccess) return e;
-    if (cap->resident[kMaxCluster] >= Bt)
+    if (cap->resident[kMaxCluster] >= Bt) {
+      if (fault.extra) return cudaErrorNotSupported;
       return launch_overlapped(accept_kernel<16>, dim3(static_cast<unsigned>(Bt) * kMaxCluster),
                                dim3(kAcceptThreads), 0, stream, static_cast<unsigned>(kMaxCluster), logits, draft,
-                               gamma, vocab, vec4, accepted_len, out_tokens, row_argmax, err_word);
+                               gamma, vocab, vec4, accepted_len, out_tokens, row_argmax, err_word, 0u, wait_ns);
+    }
   }
   cudaError_t e = cluster_capacity<8>(&cap);
   if (e != cudaSuccess) return e;
@@ -289,9 +293,10 @@ cudaError_t launch_accept(const float* logits, const int32_t* draft, int Bt, int
       break;
     }
   }
+  if (fault.extra && CL > 1) return cudaErrorNotSupported;
   return launch_overlapped(accept_kernel<8>, dim3(static_cast<unsigned>(Bt) * CL), dim3(kAcceptThreads), 0, stream,
                            static_cast<unsigned>(CL), logits, draft, gamma, vocab, vec4, accepted_len, out_tokens,
-                           row_argmax, err_word);
+                           row_argmax, err_word, fault.extra, wait_ns);
 }
 
 }  // namespace simsd

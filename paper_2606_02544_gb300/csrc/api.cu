@@ -17,6 +17,16 @@ namespace {
 
 thread_local char g_last_error[256] = "";
 
+// Planted wait expiry armed by simsd_debug_expire_next_wait for the next
+// launch of one kernel on this thread (index: SIMSD_DEBUG_WAIT_*).
+thread_local simsd::WaitFault g_armed[3];
+
+simsd::WaitFault take_armed(int which) {
+  const simsd::WaitFault f = g_armed[which];
+  g_armed[which] = simsd::WaitFault{};
+  return f;
+}
+
 int cuda_fail(cudaError_t e, const char* where) {
   std::snprintf(g_last_error, sizeof(g_last_error), "%s: %s", where, cudaGetErrorString(e));
   return SIMSD_ERR_CUDA;
@@ -93,7 +103,7 @@ int verify_attention_impl(int dtype, const void* q, const void* k_new, const voi
                           int page_size, const int32_t* prefix_len, const int32_t* tau, const uint8_t* section,
                           const int32_t* rope_pos, float rope_theta, int Bt, int gamma, int Hq, int Hkv, int d,
                           float softmax_scale, void* out, void* workspace, size_t workspace_bytes,
-                          bool static_scratch, int32_t* err_word, void* stream) {
+                          bool static_scratch, const simsd::WaitFault& fault, int32_t* err_word, void* stream) {
   if (Bt < 0) return arg_fail("Bt < 0");
   if (gamma < 1 || gamma > 32) return arg_fail("gamma must be in [1, 32]");
   if (Hq <= 0 || Hkv <= 0 || Hq % Hkv != 0) return arg_fail("Hq must be a positive multiple of Hkv");
@@ -194,6 +204,7 @@ int verify_attention_impl(int dtype, const void* q, const void* k_new, const voi
   a.Hq = Hq;
   a.Hkv = Hkv;
   a.scale = scale;
+  a.fault = fault;
   if (num_pages == 0) {
     a.max_pages = 0;
     a.num_pages = 0;
@@ -256,9 +267,11 @@ int simsd_verify_attention(int dtype, const void* q, const void* k_new, const vo
                            const int32_t* rope_pos, float rope_theta, int Bt, int gamma, int Hq, int Hkv, int d,
                            float softmax_scale, void* out, void* workspace, size_t workspace_bytes,
                            int32_t* err_word, void* stream) {
+  // an armed wait expiry is consumed by this call whatever its outcome
+  const simsd::WaitFault fault = take_armed(SIMSD_DEBUG_WAIT_ATTENTION);
   return verify_attention_impl(dtype, q, k_new, v_new, k_cache, v_cache, num_pages, block_table, max_pages,
                                page_size, prefix_len, tau, section, rope_pos, rope_theta, Bt, gamma, Hq, Hkv, d,
-                               softmax_scale, out, workspace, workspace_bytes, false, err_word, stream);
+                               softmax_scale, out, workspace, workspace_bytes, false, fault, err_word, stream);
 }
 
 int simsd_verify_attention_noalloc(int dtype, const void* q, const void* k_new, const void* v_new,
@@ -269,11 +282,13 @@ int simsd_verify_attention_noalloc(int dtype, const void* q, const void* k_new, 
                                    int d, float softmax_scale, void* out, int32_t* err_word, void* stream) {
   return verify_attention_impl(dtype, q, k_new, v_new, k_cache, v_cache, num_pages, block_table, max_pages,
                                page_size, prefix_len, tau, section, rope_pos, rope_theta, Bt, gamma, Hq, Hkv, d,
-                               softmax_scale, out, nullptr, 0, true, err_word, stream);
+                               softmax_scale, out, nullptr, 0, true, simsd::WaitFault{}, err_word, stream);
 }
 
 int simsd_accept(const float* logits, const int32_t* draft, int Bt, int gamma, int vocab, int32_t* accepted_len,
                  int32_t* out_tokens, int32_t* row_argmax, int32_t* err_word, void* stream) {
+  // an armed wait expiry is consumed by this call whatever its outcome
+  const simsd::WaitFault fault = take_armed(SIMSD_DEBUG_WAIT_ACCEPT);
   if (Bt < 0) return arg_fail("Bt < 0");
   if (gamma < 1 || gamma > 32) return arg_fail("gamma must be in [1, 32]");
   if (vocab < 1 || vocab > (1 << 28)) return arg_fail("vocab must be in [1, 2^28]");
@@ -283,7 +298,9 @@ int simsd_accept(const float* logits, const int32_t* draft, int Bt, int gamma, i
   int rc = require_sm103(&info);
   if (rc != SIMSD_OK) return rc;
   cudaError_t e = simsd::launch_accept(logits, draft, Bt, gamma, vocab, accepted_len, out_tokens, row_argmax,
-                                       err_word, info.num_sms, as_stream(stream));
+                                       err_word, info.num_sms, as_stream(stream), fault);
+  if (e == cudaErrorNotSupported && fault.extra)
+    return unsupported("a planted wait expiry needs one CTA per sequence (a batch too large for clusters)");
   return e == cudaSuccess ? SIMSD_OK : cuda_fail(e, "accept launch");
 }
 
@@ -333,6 +350,14 @@ int simsd_kv_commit(int dtype, const void* k_new, const void* v_new, int L, cons
                                           num_pages, block_table, max_pages, page_size, prefix_len, Bt, gamma, Hkv,
                                           d, rope_pos, table, err_word, as_stream(stream));
   return e == cudaSuccess ? SIMSD_OK : cuda_fail(e, "kv_commit launch");
+}
+
+int simsd_debug_expire_next_wait(int which, unsigned int limit_us) {
+  if (which != SIMSD_DEBUG_WAIT_ATTENTION && which != SIMSD_DEBUG_WAIT_ACCEPT) return arg_fail("which");
+  if (limit_us < 10 || limit_us > 1000000) return arg_fail("limit_us must be in [10, 10^6]");
+  g_armed[which].extra = 1;
+  g_armed[which].wait_ns = 1000ull * limit_us;
+  return SIMSD_OK;
 }
 
 int simsd_check_error(const int32_t* err_word, int32_t* host_word, void* stream) {

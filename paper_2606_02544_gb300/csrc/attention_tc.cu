@@ -92,6 +92,10 @@ struct TcParams {
   int slots;  // CTAs resident at once: blocks past this start in a later wave
   int fuse;   // the prefix splits of a unit form a cluster and merge in shared memory
   float scale_log2;
+  // bounded waits: time limit and extra arrivals expected on bar_p (0 in
+  // normal use; a test arms one launch so that a wait runs out)
+  unsigned long long wait_ns;
+  uint32_t extra_p;
   RopeTable rope;
 };
 
@@ -166,7 +170,7 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm)
     }
     mbar_init(smem_u32(&sm.bar_qt), 1);
     mbar_init(smem_u32(&sm.bar_s_full), 1);
-    mbar_init(smem_u32(&sm.bar_p), 4);
+    mbar_init(smem_u32(&sm.bar_p), 4 + p.extra_p);
     mbar_init(smem_u32(&sm.bar_pv), 1);
     mbar_init(smem_u32(&sm.bar_drain), 1);
     fence_mbar_init();
@@ -385,7 +389,8 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm)
         // Q (and in split 0 the tile of new slots) went out already
         for (int i = issued - 1; i < ntiles; ++i) {
           const int it = i + 1, st = it % kStages;
-          if (it >= kStages && !mbar_wait(smem_u32(&sm.bar_empty[st]), ((it / kStages) - 1) & 1, abort_flag)) {
+          if (it >= kStages &&
+              !mbar_wait(smem_u32(&sm.bar_empty[st]), ((it / kStages) - 1) & 1, abort_flag, p.wait_ns)) {
             signal_abort(sm, p.err_word);
             break;
           }
@@ -394,7 +399,8 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm)
         }
       }
       // Drain: every issued load must have landed before the CTA may exit.
-      // In a normal run these phases completed long ago.
+      // In a normal run these phases completed long ago.  These waits keep
+      // the full limit even when a test shortens the others.
       for (int it = max(0, issued - kStages); it < issued; ++it) {
         const int st = it % kStages;
         mbar_wait(smem_u32(&sm.bar_k[st]), (it / kStages) & 1, nullptr);
@@ -407,13 +413,13 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm)
     if (lane == 0 && ntiles > 0) {
       constexpr uint32_t kIdescQK = idesc_bf16_f32(kRows, kTile, 0, 0);
       constexpr uint32_t kIdescPV = idesc_bf16_f32(kRows, kD, 0, 1);
-      bool ok = mbar_wait(smem_u32(&sm.bar_qt), 0, abort_flag);
+      bool ok = mbar_wait(smem_u32(&sm.bar_qt), 0, abort_flag, p.wait_ns);
       for (int i = 0; ok && i < ntiles; ++i) {
         const int it = i + 1, st = it % kStages;
         const uint32_t par = (it / kStages) & 1;
         // S overwrites P of the previous tile; tcgen05.mma ops issued by one
         // thread run in issue order, so that PV has read P before this S lands
-        if (!mbar_wait(smem_u32(&sm.bar_k[st]), par, abort_flag)) {
+        if (!mbar_wait(smem_u32(&sm.bar_k[st]), par, abort_flag, p.wait_ns)) {
           ok = false;
           break;
         }
@@ -425,8 +431,8 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm)
           tc_mma_ts(tmem + kColS, tmem + kColQ + 8 * kk, sdesc_sw128(ka, 16, 1024), kIdescQK, kk > 0);
         }
         tc_commit(smem_u32(&sm.bar_s_full));
-        if (!mbar_wait(smem_u32(&sm.bar_p), i & 1, abort_flag) ||
-            !mbar_wait(smem_u32(&sm.bar_v[st]), par, abort_flag)) {
+        if (!mbar_wait(smem_u32(&sm.bar_p), i & 1, abort_flag, p.wait_ns) ||
+            !mbar_wait(smem_u32(&sm.bar_v[st]), par, abort_flag, p.wait_ns)) {
           ok = false;
           break;
         }
@@ -467,7 +473,7 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm)
     // ---- Q: shared memory (ring slot 0) -> TMEM columns [0, 64)
     if (ntiles > 0) {
       const int pos = p.rope_pos ? p.rope_pos[static_cast<size_t>(b) * p.S + (s < p.S ? s : 0)] : 0;
-      ok = mbar_wait_warp(smem_u32(&sm.bar_k[0]), 0, abort_flag);
+      ok = mbar_wait_warp(smem_u32(&sm.bar_k[0]), 0, abort_flag, p.wait_ns);
       if (ok && p.rope_pos) {
         // rotate this row's query at its slot's position on the way
         const uint8_t* h0 = sm.ring[0];
@@ -514,7 +520,7 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm)
         // the new keys (ring item 1, the unit's first tile) are rotated in
         // place before the first S = Q K^T reads them
         constexpr int st1 = 1 % kStages;
-        ok = mbar_wait_warp(smem_u32(&sm.bar_k[st1]), 0, abort_flag);
+        ok = mbar_wait_warp(smem_u32(&sm.bar_k[st1]), 0, abort_flag, p.wait_ns);
         if (ok) {
           uint8_t* h0 = sm.ring[st1];
           uint8_t* h1 = sm.ring[st1] + kHalfBytes;
@@ -554,7 +560,7 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm)
     for (int i = 0; ok && i < ntiles; ++i) {
       const int it = i + 1, st = it % kStages;
       const int t = t0 + i;
-      if (!mbar_wait_warp(smem_u32(&sm.bar_s_full), i & 1, abort_flag)) {
+      if (!mbar_wait_warp(smem_u32(&sm.bar_s_full), i & 1, abort_flag, p.wait_ns)) {
         ok = false;
         break;
       }
@@ -642,7 +648,7 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm)
       if (warp < 2 && (valid < kTile || is_new)) {
         // rows of V that no query may use are zeroed so that 0 * (stale or
         // non-finite data) cannot reach O
-        if (!mbar_wait_warp(smem_u32(&sm.bar_v[st]), (it / kStages) & 1, abort_flag)) {
+        if (!mbar_wait_warp(smem_u32(&sm.bar_v[st]), (it / kStages) & 1, abort_flag, p.wait_ns)) {
           ok = false;
           break;
         }
@@ -671,7 +677,8 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm)
     // cost more than they gain (measured at 8 sequences, 4 splits each).
     if (!kFuse) pdl_launch_next();
     // ---- epilogue: O of the last PV, scaled by 1/l
-    const bool have_o = ok && ntiles > 0 && mbar_wait_warp(smem_u32(&sm.bar_pv), (ntiles - 1) & 1, abort_flag);
+    const bool have_o =
+        ok && ntiles > 0 && mbar_wait_warp(smem_u32(&sm.bar_pv), (ntiles - 1) & 1, abort_flag, p.wait_ns);
     if (have_o) tc_fence_after();
     const bool any = have_o && active && l_sum > 0.f;
     const int h = kvh * p.g + hl;
@@ -1021,6 +1028,8 @@ cudaError_t launch_attention_tc(const AttnTcArgs& a, const AttnTcPlan& pl, Encod
   p.fuse = pl.fuse;
   p.slots = pl.slots;
   p.scale_log2 = a.scale * 1.4426950408889634f;
+  p.wait_ns = a.fault.wait_ns ? a.fault.wait_ns : kWaitLimitNs;
+  p.extra_p = a.fault.extra;
 
   {
     cudaError_t e = ensure_smem_attr();
@@ -1041,7 +1050,8 @@ size_t noalloc_scratch_capacity() { return sizeof(g_noalloc_scratch); }
 
 cudaError_t noalloc_scratch_pointer(void** out) {
   // Set-up, once per device and with that device current: the device
-  // address of the static scratch array.
+  // address of the static scratch array.  It is kept for the life of the
+  // process (a device reset, which would move the array, is not supported).
   static std::mutex mu;
   static void* ptr[64] = {};
   int dev = 0;

@@ -15,13 +15,24 @@ struct RopeTable {
 };
 RopeTable make_rope_table(double theta, int d);
 
+// A planted wait expiry for one launch (tests of failure detection): the
+// kernel expects `extra` more arrivals than ever come on one of its
+// barriers and its waits give up after wait_ns.  {0, 0}: normal launch.
+struct WaitFault {
+  uint32_t extra = 0;
+  unsigned long long wait_ns = 0;
+};
+
 cudaError_t launch_build_mask(const int32_t* step_map, const int32_t* prefix_len, int Bt, int gamma, int32_t* tau,
                               uint8_t* section, int32_t* rope_pos, uint64_t* mask_bits, int32_t* err_word,
                               cudaStream_t stream);
 
+// fault.extra > 0 is applied only when every sequence runs as a single
+// CTA (no other CTA then writes into the waiting CTA's shared memory);
+// otherwise cudaErrorNotSupported.
 cudaError_t launch_accept(const float* logits, const int32_t* draft, int Bt, int gamma, int vocab,
                           int32_t* accepted_len, int32_t* out_tokens, int32_t* row_argmax, int32_t* err_word,
-                          int num_sms, cudaStream_t stream);
+                          int num_sms, cudaStream_t stream, const WaitFault& fault = WaitFault{});
 
 cudaError_t launch_accept_sampled(const float* target_logits, const float* draft_logits, const int32_t* draft,
                                   const float* u_accept, const float* u_sample, float temperature, int Bt,
@@ -73,6 +84,7 @@ struct AttnTcArgs {
   int32_t* err_word;
   int num_pages, max_pages, page_size, Bt, gamma, Hq, Hkv;
   float scale;
+  WaitFault fault;
 };
 // The tensor-map encoder is the driver's cuTensorMapEncodeTiled.
 typedef CUresult (*EncodeTiledFn)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*, const cuuint64_t*,

@@ -74,9 +74,10 @@ __device__ __forceinline__ bool mbar_try_wait_cluster(uint32_t bar, uint32_t par
   return done != 0;
 }
 
-// Warp-uniform bounded wait (1 s) for arrivals from other CTAs of the
-// cluster; false on timeout.
-__device__ __forceinline__ bool mbar_wait_cluster_warp(uint32_t bar, uint32_t parity) {
+// Warp-uniform bounded wait (limit_ns, 1 s by default) for arrivals from
+// other CTAs of the cluster; false on timeout.
+__device__ __forceinline__ bool mbar_wait_cluster_warp(uint32_t bar, uint32_t parity,
+                                                       unsigned long long limit_ns = kWaitLimitNs) {
   const unsigned full = 0xffffffffu;
   if (__all_sync(full, mbar_try_wait_cluster(bar, parity))) return true;
   const unsigned long long t0 = globaltimer_ns();
@@ -84,7 +85,7 @@ __device__ __forceinline__ bool mbar_wait_cluster_warp(uint32_t bar, uint32_t pa
     if (__all_sync(full, mbar_try_wait_cluster(bar, parity))) return true;
     if ((it & 63u) == 0) {
       int give_up = 0;
-      if ((threadIdx.x & 31) == 0) give_up = globaltimer_ns() - t0 > kWaitLimitNs;
+      if ((threadIdx.x & 31) == 0) give_up = globaltimer_ns() - t0 > limit_ns;
       if (__shfl_sync(full, give_up, 0)) return false;
     }
   }
@@ -97,22 +98,25 @@ __device__ __forceinline__ void cluster_arrive_relaxed() {
 __device__ __forceinline__ void cluster_wait() { asm volatile("barrier.cluster.wait.aligned;" ::: "memory"); }
 
 // Single-thread bounded wait for the phase with the given parity to
-// complete.  Returns false on timeout or when *abort becomes non-zero
-// (abort == nullptr: only the time limit ends the wait, as when draining).
-__device__ __forceinline__ bool mbar_wait(uint32_t bar, uint32_t parity, volatile int* abort) {
+// complete.  Returns false on timeout (limit_ns, 1 s by default) or when
+// *abort becomes non-zero (abort == nullptr: only the time limit ends the
+// wait, as when draining).
+__device__ __forceinline__ bool mbar_wait(uint32_t bar, uint32_t parity, volatile int* abort,
+                                          unsigned long long limit_ns = kWaitLimitNs) {
   if (mbar_try_wait(bar, parity)) return true;
   const unsigned long long t0 = globaltimer_ns();
   for (uint32_t it = 1;; ++it) {
     if (mbar_try_wait(bar, parity)) return true;
     if ((it & 63u) == 0) {
       if (abort && *abort) return false;
-      if (globaltimer_ns() - t0 > kWaitLimitNs) return false;
+      if (globaltimer_ns() - t0 > limit_ns) return false;
     }
   }
 }
 
 // Warp-uniform bounded wait: every lane polls, all lanes leave together.
-__device__ __forceinline__ bool mbar_wait_warp(uint32_t bar, uint32_t parity, volatile int* abort) {
+__device__ __forceinline__ bool mbar_wait_warp(uint32_t bar, uint32_t parity, volatile int* abort,
+                                               unsigned long long limit_ns = kWaitLimitNs) {
   const unsigned full = 0xffffffffu;
   if (__all_sync(full, mbar_try_wait(bar, parity))) return true;
   const unsigned long long t0 = globaltimer_ns();
@@ -120,7 +124,7 @@ __device__ __forceinline__ bool mbar_wait_warp(uint32_t bar, uint32_t parity, vo
     if (__all_sync(full, mbar_try_wait(bar, parity))) return true;
     if ((it & 63u) == 0) {
       int give_up = 0;
-      if ((threadIdx.x & 31) == 0) give_up = (*abort) || (globaltimer_ns() - t0 > kWaitLimitNs);
+      if ((threadIdx.x & 31) == 0) give_up = (*abort) || (globaltimer_ns() - t0 > limit_ns);
       if (__shfl_sync(full, give_up, 0)) return false;
     }
   }

@@ -26,8 +26,9 @@ STEP_UNDRAFTED, STEP_DECODED = -1, -2
 
 EXPORTED = ("simsd_build_mask", "simsd_verify_workspace_bytes", "simsd_verify_attention",
             "simsd_verify_attention_noalloc", "simsd_accept", "simsd_accept_sampled", "simsd_kv_commit",
-            "simsd_check_error",
+            "simsd_check_error", "simsd_debug_expire_next_wait",
             "simsd_last_error", "simsd_version")
+DEBUG_WAIT_ATTENTION, DEBUG_WAIT_ACCEPT = 1, 2
 
 
 class SimsdError(RuntimeError):
@@ -61,10 +62,11 @@ def load_library(path: str = LIB_PATH):
             lib.simsd_accept_sampled.argtypes = [P, P, P, P, P, F, I, I, I, P, P, P, P]
             lib.simsd_kv_commit.argtypes = [I, P, P, I, P, P, P, F, P, P, P, I, P, I, I, P, I, I, I, I, P, P]
             lib.simsd_check_error.argtypes = [P, P, P]
+            lib.simsd_debug_expire_next_wait.argtypes = [I, ctypes.c_uint]
             lib.simsd_last_error.restype = ctypes.c_char_p
             for name in ("simsd_build_mask", "simsd_verify_attention", "simsd_verify_attention_noalloc",
                          "simsd_accept", "simsd_accept_sampled", "simsd_kv_commit", "simsd_check_error",
-                         "simsd_version"):
+                         "simsd_debug_expire_next_wait", "simsd_version"):
                 getattr(lib, name).restype = ctypes.c_int
             _lib = lib
     return _lib
@@ -172,6 +174,13 @@ def simsd_kv_commit(k_new, v_new, tau, section, accepted_len, k_cache, v_cache, 
         _p(v_cache), num_pages, _p(block_table), block_table.shape[1], P, _p(prefix_len), Bt, S // 2, Hkv, d,
         _p(err_word), _stream(stream))
     _check(rc, "simsd_kv_commit")
+
+
+def simsd_debug_expire_next_wait(which, limit_us):
+    """Test hook: the next attention (DEBUG_WAIT_ATTENTION) or acceptance
+    (DEBUG_WAIT_ACCEPT) call of this thread waits for an arrival that never
+    comes and gives up after limit_us."""
+    _check(load_library().simsd_debug_expire_next_wait(int(which), int(limit_us)), "simsd_debug_expire_next_wait")
 
 
 def simsd_check_error(err_word, stream=None):

@@ -66,6 +66,11 @@ def test_host_validation_without_gpu(lib):
     assert lib.simsd_accept_sampled(None, None, None, None, None, F(1.0), 0, 4, 10, None, None, None, None) == 0
     # empty batches are no-ops that touch nothing
     assert lib.simsd_accept(None, None, 0, 4, 10, None, None, None, None, None) == 0
+    # the wait-expiry test hook validates its arguments on the host
+    assert lib.simsd_debug_expire_next_wait(0, 200) == 1
+    assert lib.simsd_debug_expire_next_wait(3, 200) == 1
+    assert lib.simsd_debug_expire_next_wait(1, 5) == 1
+    assert lib.simsd_debug_expire_next_wait(2, 2000000) == 1
     assert lib.simsd_check_error(None, None, None) == 1
     assert b"null error word" in lib.simsd_last_error()
 
