@@ -3,7 +3,32 @@ same call through the oracle, on the same seeded inputs.
 
 The oracle only ever sees host copies of the generator's tensors; it builds
 its own mask from the step map and never reads anything the CUDA path made.
+
+Attention tolerance.  Every output element must pass two bars:
+
+* the stated one: |g - r| <= 2e-2 + 2e-2 |r| for bf16, |g - r| <= 1e-5 for
+  fp32 (r is the fp64 oracle);
+* for bf16, a bound derived from the arithmetic of the tensor-core kernel,
+  which scales with the output.  The kernel rounds each probability p_j to
+  bf16 (8 significant bits, round to nearest: relative error <= u = 2^-8)
+  before P V, sums l = sum p_j unrounded
+  in fp32, and rounds O / l to bf16 (again <= u).  So
+
+      |g - r| <= u (A + |r|) + (e^(2 Delta) - 1)(A + |r|) + c (A + |r|)
+
+  with A = sum_j p_j |v_j| / sum_j p_j (the oracle's attention over |V|,
+  computed by a second oracle call), Delta a bound on the error of the
+  scores in natural-log units (fp32 accumulation of d products, the FFMA
+  and ex2.approx of the softmax, and when the kernel rotates q / k_new
+  itself, their bf16 rounding: Delta_rope = 2^-7 scale |q| |k|), and c the
+  fp32 accumulation over T key tiles, (T + 70) 2^-23.  At the SDAR input
+  scale (Q/K/V ~ N(0, 1/128)) this is ~3e-4 against outputs of 1e-3 to
+  1e-2, so an all-zero output or a dropped key tile fails it.
 """
+import dataclasses
+import math
+import os
+
 import numpy as np
 import torch
 
@@ -13,6 +38,11 @@ from paper_2606_02544_gb300 import inputs, simsd
 BF16_ATOL = 2e-2
 BF16_RTOL = 2e-2
 F32_ATOL = 1e-5
+U_BF16 = 2.0 ** -8          # unit roundoff of bf16 (8 significant bits, round to nearest)
+LOG2E = 1.4426950408889634
+
+# (test id, statistics) of every attention comparison of this process
+PARITY_LOG = []
 
 
 def gpu_mask(si, mask_bits=True):
@@ -49,51 +79,135 @@ def gpu_attention(si, layer=0, mask=None, err=None, rope_pos=None, rope_theta=0.
     return out, word, ws
 
 
-def oracle_attention(si, layer=0, seqs=None, rope_theta=0.0, rope_mode=1):
-    """Oracle attention for all sequences, or for the listed ones only (a
-    sub-batch with its own compact page pool).  rope_theta > 0: q and k_new
-    are rotated by the oracle first (rope_mode 1: RoPE copy, 2: physical
-    positions)."""
-    rope = dict(rope_theta=rope_theta, rope_mode=rope_mode)
+@dataclasses.dataclass
+class OracleRef:
+    """The oracle's attention and what the derived bound needs."""
+    out: np.ndarray          # fp64 [Bt'][2g][Hq][d]
+    err: int                 # oracle error bits
+    absv: np.ndarray         # oracle attention over |V| (same shape)
+    delta: float             # bound on the kernel's score error, natural-log units
+    tiles: int               # key tiles of the longest row (prefix tiles + the new-slot tile)
+    dtype: str
+
+
+def _abs_bits(x):
+    """|x| of host storage: clears the sign bit of bf16 bit patterns."""
+    if x.dtype == np.uint16:
+        return x & np.uint16(0x7FFF)
+    return np.abs(x)
+
+
+def _sub_batch(si, layer, seqs):
+    """Host arrays of the listed sequences with their own compact page pool."""
+    w = si.w
+    P = w.page_size
     if seqs is None:
-        return orc.verify_attention(
-            inputs.host_bits(si.q[layer]), inputs.host_bits(si.k_new[layer]), inputs.host_bits(si.v_new[layer]),
-            inputs.host_bits(si.k_cache[layer]), inputs.host_bits(si.v_cache[layer]),
-            si.block_table.cpu().numpy(), si.prefix_len.cpu().numpy(), si.step_map.cpu().numpy(), si.w.gamma,
-            **rope)
+        return (inputs.host_bits(si.q[layer]), inputs.host_bits(si.k_new[layer]), inputs.host_bits(si.v_new[layer]),
+                inputs.host_bits(si.k_cache[layer]), inputs.host_bits(si.v_cache[layer]),
+                si.block_table.cpu().numpy(), si.prefix_len.cpu().numpy(), si.step_map.cpu().numpy())
     idx = torch.as_tensor(seqs, device=si.q.device)
     bt = si.block_table[idx].cpu()
     n = si.prefix_len[idx].cpu()
-    P = si.w.page_size
     used = []
     for r in range(len(seqs)):
-        cnt = (int(n[r]) + P - 1) // P
+        cnt = max(0, (int(n[r]) + P - 1) // P)
         used.append(bt[r, :cnt])
     used = torch.cat(used) if used else torch.zeros(0, dtype=torch.int32)
     uniq, inv = torch.unique(used, return_inverse=True)
     new_bt = torch.full_like(bt, -1)
     pos = 0
     for r in range(len(seqs)):
-        cnt = (int(n[r]) + P - 1) // P
+        cnt = max(0, (int(n[r]) + P - 1) // P)
         new_bt[r, :cnt] = inv[pos:pos + cnt].to(torch.int32)
         pos += cnt
     pages = uniq.to(si.q.device).long()
     kc = si.k_cache[layer][pages] if len(pages) else si.k_cache[layer][:1]
     vc = si.v_cache[layer][pages] if len(pages) else si.v_cache[layer][:1]
-    return orc.verify_attention(
-        inputs.host_bits(si.q[layer][idx]), inputs.host_bits(si.k_new[layer][idx]),
-        inputs.host_bits(si.v_new[layer][idx]), inputs.host_bits(kc), inputs.host_bits(vc), new_bt.numpy(),
-        n.numpy(), si.step_map[idx].cpu().numpy(), si.w.gamma, **rope)
+    return (inputs.host_bits(si.q[layer][idx]), inputs.host_bits(si.k_new[layer][idx]),
+            inputs.host_bits(si.v_new[layer][idx]), inputs.host_bits(kc), inputs.host_bits(vc), new_bt.numpy(),
+            n.numpy(), si.step_map[idx].cpu().numpy())
 
 
-def assert_attention_close(got, want, dtype):
+def _max_row_norm(t):
+    return float(t.float().reshape(-1, t.shape[-1]).norm(dim=1).nan_to_num(0.0).max()) if t.numel() else 0.0
+
+
+def _max_prefix_key_norm(si, layer):
+    """Largest norm of a cached key that holds a prefix row (in chunks of
+    pages, so that large pools need no full fp32 copy)."""
+    valid = torch.as_tensor(si.row_valid, device=si.q.device)
+    kc = si.k_cache[layer]
+    best = 0.0
+    for p0 in range(0, kc.shape[0], 2048):
+        x = kc[p0:p0 + 2048].float().pow(2).sum(-1).sqrt()          # [pages][Hkv][P]
+        x = torch.where(valid[p0:p0 + 2048, None, :], x.nan_to_num(0.0), torch.zeros_like(x))
+        if x.numel():
+            best = max(best, float(x.max()))
+    return best
+
+
+def oracle_attention(si, layer=0, seqs=None, rope_theta=0.0, rope_mode=1, prefix_override=None):
+    """Oracle attention for all sequences, or for the listed ones only (a
+    sub-batch with its own compact page pool), plus the oracle's attention
+    over |V| for the derived bound.  rope_theta > 0: q and k_new are rotated
+    by the oracle first (rope_mode 1: RoPE copy, 2: physical positions).
+    ``prefix_override`` (one length per listed sequence) plants a different
+    prefix length in the oracle's input only (negative controls)."""
+    q, kn, vn, kc, vc, bt, n, sm = _sub_batch(si, layer, seqs)
+    if prefix_override is not None:
+        n = np.asarray(prefix_override, dtype=np.int32)
+    rope = dict(rope_theta=rope_theta, rope_mode=rope_mode)
+    out, err = orc.verify_attention(q, kn, vn, kc, vc, bt, n, sm, si.w.gamma, **rope)
+    absv, _ = orc.verify_attention(q, kn, _abs_bits(vn), kc, _abs_bits(vc), bt, n, sm, si.w.gamma, **rope)
+    # score error bound: |q| |k| over the rows involved (prefix rows through
+    # the valid-row map, NaN-poisoned unused rows excluded)
+    d = si.w.d
+    scale = 1.0 / math.sqrt(d)
+    idx = None if seqs is None else torch.as_tensor(seqs, device=si.q.device)
+    qsel = si.q[layer] if idx is None else si.q[layer][idx]
+    knsel = si.k_new[layer] if idx is None else si.k_new[layer][idx]
+    qn = _max_row_norm(qsel)
+    kn_max = max(_max_row_norm(knsel), _max_prefix_key_norm(si, layer))
+    qk = scale * qn * kn_max
+    delta = 2.0 ** -16 * qk + 2.0 ** -22 + 2.0 ** -24 * math.log(2) * (2 * LOG2E * qk + 8)
+    if rope_theta > 0:
+        delta += 2.0 ** -7 * qk
+    tiles = int(np.max(n)) // 64 + 2 if len(n) else 2
+    return OracleRef(out, int(err), absv, delta, tiles, si.w.dtype)
+
+
+def attention_check(got, ref):
+    """Compares a kernel output with the oracle under both bars; returns the
+    statistics (no assertion)."""
     g = got.float().cpu().numpy().astype(np.float64)
-    assert np.isfinite(g).all(), "non-finite output"
-    if dtype == "f32":
-        err = np.abs(g - want).max()
-        assert err <= F32_ATOL, f"max abs error {err}"
+    r = ref.out
+    diff = np.abs(g - r)
+    finite = bool(np.isfinite(g).all())
+    rms_r = float(np.sqrt(np.mean(r * r))) if r.size else 0.0
+    st = {"elements": int(r.size), "finite": finite, "max_abs": float(np.nanmax(diff)) if r.size else 0.0,
+          "rms_rel": float(np.sqrt(np.nanmean(diff * diff)) / rms_r) if rms_r > 0 else 0.0,
+          "max_abs_r": float(np.max(np.abs(r))) if r.size else 0.0}
+    if ref.dtype == "f32":
+        st["north_star_ok"] = finite and st["max_abs"] <= F32_ATOL
+        st["bound_ok"] = st["north_star_ok"]
+        st["max_ratio"] = st["max_abs"] / F32_ATOL
     else:
-        bad = np.abs(g - want) > BF16_ATOL + BF16_RTOL * np.abs(want)
-        assert not bad.any(), (f"{bad.sum()} elements out of tolerance; max abs "
-                               f"{np.abs(g - want).max():.3g}")
-    return float(np.abs(g - want).max())
+        st["north_star_ok"] = finite and bool((diff <= BF16_ATOL + BF16_RTOL * np.abs(r)).all())
+        mag = ref.absv + np.abs(r)
+        tol = mag * (U_BF16 * (1 + 2.0 ** -7) + math.expm1(2 * ref.delta) + (ref.tiles + 70) * 2.0 ** -23) + 1e-12
+        ratio = diff / tol
+        st["bound_ok"] = finite and bool((ratio <= 1.0).all())
+        st["max_ratio"] = float(np.nanmax(ratio)) if r.size else 0.0
+        st["bound_median"] = float(np.median(tol)) if r.size else 0.0
+        st["out_of_bound"] = int((~(ratio <= 1.0)).sum())
+    st["ok"] = st["north_star_ok"] and st["bound_ok"]
+    return st
+
+
+def assert_attention_close(got, ref):
+    st = attention_check(got, ref)
+    PARITY_LOG.append((os.environ.get("PYTEST_CURRENT_TEST", "?").split(" ")[0], st))
+    assert st["finite"], "non-finite output"
+    assert st["north_star_ok"], f"outside the stated tolerance: {st}"
+    assert st["bound_ok"], f"outside the derived bf16 bound: {st}"
+    return st["max_abs"]

@@ -6,7 +6,6 @@ tails, page-boundary prefixes, every page size the kernel takes, split and
 unsplit prefixes, row blocks, non-identity step maps, padding, poisoned
 unused cache rows, harder score distributions, and the error paths.
 """
-import dataclasses
 
 import numpy as np
 import pytest
@@ -25,10 +24,10 @@ def _w(dtype="bf16", Bt=3, Hq=16, Hkv=8, d=128, gamma=4, prefix=(0, 300), P=64, 
 
 def _check(si, seqs=None):
     out, word, _ = gpu_attention(si)
-    want, werr = oracle_attention(si, seqs=seqs)
-    assert word == werr
+    ref = oracle_attention(si, seqs=seqs)
+    assert word == ref.err
     got = out if seqs is None else out[torch.as_tensor(seqs, device=out.device)]
-    return assert_attention_close(got, want, si.w.dtype)
+    return assert_attention_close(got, ref)
 
 
 def test_c1_tiny_fp32():
@@ -123,9 +122,9 @@ def test_two_row_blocks_error_paths():
     bt[2, 1] = si.num_pages + 5                   # page id outside the pool
     si.block_table = bt
     out, word, _ = gpu_attention(si)
-    want, werr = oracle_attention(si)
-    assert word == werr and word & simsd.EW_PAGE and word & simsd.EW_STEP_MAP
-    assert_attention_close(out, want, "bf16")
+    ref = oracle_attention(si)
+    assert word == ref.err and word & simsd.EW_PAGE and word & simsd.EW_STEP_MAP
+    assert_attention_close(out, ref)
     assert (out[2:4].float() == 0).all() and (out[0, [2, 34]].float() == 0).all()
 
 
@@ -172,9 +171,9 @@ def test_padding_slots_and_error_paths():
     bt[2, 1] = si.num_pages + 5                              # page id outside the pool
     si.block_table = bt
     out, word, _ = gpu_attention(si)
-    want, werr = oracle_attention(si)
-    assert word == werr and word & simsd.EW_PREFIX_LEN and word & simsd.EW_PAGE and word & simsd.EW_STEP_MAP
-    assert_attention_close(out, want, "bf16")
+    ref = oracle_attention(si)
+    assert word == ref.err and word & simsd.EW_PREFIX_LEN and word & simsd.EW_PAGE and word & simsd.EW_STEP_MAP
+    assert_attention_close(out, ref)
     assert (out[1:4].float() == 0).all() and (out[0, [2, 6]].float() == 0).all()
 
 
@@ -189,41 +188,9 @@ def test_undrafted_and_decoded_positions(dtype, gamma, n_draft):
     _check(si)
 
 
-@pytest.mark.parametrize("name", ["c2", "c3"])
-def test_full_size_target_block_decoding(name):
-    # the target's own block decoding at full size: every sequence's block
-    # is decoded-or-[MASK]; the oracle checks a few sequences
-    w = dataclasses.replace(inputs.WORKLOADS[name], layers=1)
-    si = inputs.make_step_inputs(w, device="cuda", with_logits=False)
-    si.step_map = inputs.block_step_maps(w.Bt, w.gamma, seed=5, n_draft=0).cuda()
-    _check(si, seqs=[0, w.Bt // 2, w.Bt - 1])
-
-
 def test_deterministic():
     w = _w(Bt=5, Hq=32, Hkv=8, gamma=8, prefix=(100, 900), seed=3)
     si = inputs.make_step_inputs(w, device="cuda", random_step_map=True)
     a, _, _ = gpu_attention(si)
     b, _, _ = gpu_attention(si)
     assert torch.equal(a, b)
-
-
-@pytest.mark.parametrize("name", ["c2", "c3"])
-def test_full_size_configs(name):
-    wl = inputs.WORKLOADS[name]
-    si = inputs.make_step_inputs(wl, device="cuda", poison_unused_rows=True)
-    seqs = None if name == "c2" else [0, 11, 31]
-    _check(si, seqs)
-
-
-def test_c4_sampled_layers():
-    # SDAR-8B shapes at full batch and prefix range; two of the 36 layers
-    # (each layer is one independent launch with the same configuration)
-    wl = inputs.WORKLOADS["c4"]
-    si = inputs.make_step_inputs(wl, device="cuda", layers=2)
-    n = si.prefix_len.cpu()
-    seqs = [int(torch.argmax(n)), int(torch.argmin(n)), 17]
-    for layer in (0, 1):
-        out, word, _ = gpu_attention(si, layer=layer)
-        want, werr = oracle_attention(si, layer=layer, seqs=seqs)
-        assert word == werr == 0
-        assert_attention_close(out[torch.as_tensor(seqs, device="cuda")], want, "bf16")

@@ -30,9 +30,9 @@ def _rope_check(si, theta, mode=1):
         n = si.prefix_len.long()[:, None]
         rope = (n + torch.arange(si.w.S, device=n.device)[None]).to(torch.int32).contiguous()
     out, word, _ = gpu_attention(si, mask=(tau, sect), rope_pos=rope, rope_theta=theta)
-    want, werr = oracle_attention(si, rope_theta=theta, rope_mode=mode)
-    assert word == werr == 0
-    return assert_attention_close(out, want, si.w.dtype)
+    ref = oracle_attention(si, rope_theta=theta, rope_mode=mode)
+    assert word == ref.err == 0
+    return assert_attention_close(out, ref)
 
 
 @pytest.mark.parametrize("gamma,Hq,Hkv", [(4, 16, 8), (8, 32, 8), (16, 32, 8), (32, 32, 8)])
@@ -83,8 +83,7 @@ def test_noalloc_with_rope():
                                          si.block_table, si.prefix_len, tau, sect, out, err_word=err,
                                          rope_pos=rope, rope_theta=1e6)
     assert simsd.simsd_check_error(err) == 0
-    want, _ = oracle_attention(si, rope_theta=1e6)
-    assert_attention_close(out, want, "bf16")
+    assert_attention_close(out, oracle_attention(si, rope_theta=1e6))
 
 
 def _values(bits, dtype):
@@ -133,7 +132,7 @@ def test_commit_rotates_keys(dtype, P):
 def test_whole_step_with_rope(name, theta):
     wl = inputs.WORKLOADS[name]
     si = inputs.make_step_inputs(wl, device="cuda")
-    want_out, werr = oracle_attention(si, rope_theta=theta)
+    ref = oracle_attention(si, rope_theta=theta)
     ra, rot, _, aerr = orc.accept(si.logits.cpu().numpy(), si.draft.cpu().numpy(), wl.gamma)
     kc0, vc0 = inputs.host_bits(si.k_cache), inputs.host_bits(si.v_cache)
     st = VerifyStep(si, restore_prefix=True, rope_theta=theta)
@@ -141,8 +140,8 @@ def test_whole_step_with_rope(name, theta):
     for _ in range(2):
         st.replay()
     word = simsd.simsd_check_error(st.err)
-    assert word == werr == aerr == 0
-    assert_attention_close(st.out[0], want_out, wl.dtype)
+    assert word == ref.err == aerr == 0
+    assert_attention_close(st.out[0], ref)
     np.testing.assert_array_equal(st.accepted_len.cpu().numpy(), ra)
     np.testing.assert_array_equal(st.out_tokens.cpu().numpy(), rot)
     rk, rv, rn, _ = orc.kv_commit(inputs.host_bits(si.k_new), inputs.host_bits(si.v_new),
