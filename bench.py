@@ -4,7 +4,7 @@ One step = the whole verification hot path over one batch: temporal-mask
 metadata, the masked attention of every layer, greedy acceptance and the KV
 commit, all through the C ABI (libsimsd.so), captured in a CUDA graph.
 
-    python bench.py [--gpus N] [--steps K] [--warmup W] [--workload c2|c3|c4|c1]
+    python bench.py [--gpus N] [--steps K] [--warmup W] [--workload c4|c3|c2|c1]
     python bench.py --impl reference ...     # the fp64 CPU oracle on the host cores
 
 Prints one JSON line.  ``value`` = verified tokens/s = sum_b (a_b + 1) per
@@ -31,7 +31,9 @@ if ROOT not in sys.path:
 
 METRIC = "verified draft tokens/sec per GB300; attention HBM GB/s vs 8 TB/s"
 UNIT = "tokens/s"
-DEFAULT_WORKLOAD = "c2"
+# the largest configuration that fits one GPU: SDAR-8B head shapes, 64
+# sequences, 36 layers (48.3 GB of KV cache), the KV-bound shape
+DEFAULT_WORKLOAD = "c4"
 DEFAULT_STEPS = {"c1": 2000, "c2": 2000, "c3": 400, "c4": 60}
 UNROLL = {"c1": 50, "c2": 50, "c3": 20, "c4": 1}
 
@@ -58,6 +60,10 @@ def _kernel_sha():
         with open(os.path.join(ROOT, "paper_2606_02544_gb300", "csrc", fn), "rb") as f:
             h.update(f.read())
     return h.hexdigest()[:16]
+
+
+TRAFFIC_SOURCE = ("stored: profiles/traffic.json (ncu dram__bytes_read.sum + dram__bytes_write.sum per launch), "
+                  "used only while the kernel sources hash to the value recorded there")
 
 
 def _traffic(workload, kernel):
@@ -282,14 +288,14 @@ def run_gpu(args):
                  "launch_us": round(attn_launch_ms * 1e3, 3),
                  "tensor_tflops": round(attn_flops / (attn_launch_ms * 1e-3) / 1e12, 2),
                  "tensor_frac": round(attn_flops / (attn_launch_ms * 1e-3) / 1e12 / tf_peak, 4),
-                 "traffic": _traffic(args.workload, "attention")}
+                 "traffic": _traffic(args.workload, "attention"), "traffic_source": TRAFFIC_SOURCE}
     acc_roof = {"kernel": "simsd_accept (accept_kernel)", "bound": "hbm", "achieved": round(acc_gbs, 1),
                 "peak": hbm_peak, "unit": "GB/s", "frac": round(acc_gbs / hbm_peak, 4), "peak_source": peak_kind,
                 "algorithmic_bytes_per_launch": int(acc_bytes), "launch_us": round(acc_launch_ms * 1e3, 3),
                 # rows up to the first rejection only: what a kernel that stopped
                 # at the first mismatch would have to read
                 "early_stop_bytes": int(tokens_per_step) * int(wl.vocab) * 4,
-                "traffic": _traffic(args.workload, "accept")}
+                "traffic": _traffic(args.workload, "accept"), "traffic_source": TRAFFIC_SOURCE}
     dominant, other = (attn_roof, acc_roof) if attn_launch_ms * st.L >= acc_launch_ms else (acc_roof, attn_roof)
 
     if rank == 0:
@@ -459,7 +465,9 @@ def run_cpu_baseline(args, si, max_seconds=12.0):
         seqs_done += 1
     return {"value": round(done_tokens / t_used, 2), "unit": UNIT, "cores": orc.max_threads(), "kind": "oracle",
             "sample": f"{seqs_done} whole sequences x {len(layers)} layers of {w.name} (mask, attention, accept, "
-                      f"commit), one sequence per oracle call, {t_used:.1f} s"}
+                      f"commit), one sequence per oracle call, {t_used:.1f} s; the value is extrapolated to the "
+                      f"workload as verified tokens of the sample / oracle seconds of the sample",
+            "extrapolated": True}
 
 
 def run_reference(args):
