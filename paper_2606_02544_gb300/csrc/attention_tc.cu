@@ -926,13 +926,18 @@ cudaError_t ensure_smem_attr() {
 
 bool make_map(EncodeTiledFn encode, CUtensorMap* m, const void* base, int rank, const cuuint64_t* dims,
               const cuuint64_t* strides, const cuuint32_t* box) {
+  return make_bf16_map(encode, m, base, rank, dims, strides, box);
+}
+
+}  // namespace
+
+bool make_bf16_map(EncodeTiledFn encode, CUtensorMap* m, const void* base, int rank, const cuuint64_t* dims,
+                   const cuuint64_t* strides, const cuuint32_t* box) {
   cuuint32_t es[3] = {1, 1, 1};
   return encode(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, rank, const_cast<void*>(base), dims, strides, box, es,
                 CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
                 CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
-
-}  // namespace
 
 bool plan_attention_tc(int Bt, int gamma, int Hq, int Hkv, int max_pages, int page_size, int num_sms,
                        AttnTcPlan* plan) {
@@ -949,6 +954,19 @@ bool plan_attention_tc(int Bt, int gamma, int Hq, int Hkv, int max_pages, int pa
   }
   pl.rows_blk = g * pl.s_blk;
   if (pl.rows_blk > kRows || g > 256 || pl.s_blk > 256) return false;
+  pl.num_sms = num_sms;
+  if (tc256_applies(Bt, Hkv, pl.rb, num_sms)) {
+    // two row blocks share one CTA and its K/V stream; enough units to
+    // give every SM one, so no split
+    pl.kind = 1;
+    pl.nsplit = 1;
+    pl.sort = 0;
+    pl.fuse = 0;
+    pl.slots = num_sms;
+    pl.ws_bytes = 0;
+    *plan = pl;
+    return true;
+  }
   // split the prefix only when the units alone cannot fill the GPU (the
   // occupancy calculator reports one CTA per SM for this kernel although two
   // are resident, so the budget the kernel is built for is used instead)
@@ -975,6 +993,7 @@ bool plan_attention_tc(int Bt, int gamma, int Hq, int Hkv, int max_pages, int pa
 
 cudaError_t launch_attention_tc(const AttnTcArgs& a, const AttnTcPlan& pl, EncodeTiledFn encode,
                                 cudaStream_t stream) {
+  if (pl.kind == 1) return launch_attention_tc256(a, pl.s_blk, encode, pl.num_sms, stream);
   const int S = 2 * a.gamma, g = a.Hq / a.Hkv;
   CUtensorMap tq, tkn, tvn, tkc, tvc;
   {

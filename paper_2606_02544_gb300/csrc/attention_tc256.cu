@@ -1,0 +1,752 @@
+// attention_tc256.cu -- bf16 verification attention for units of 256 query
+// rows on the sm_103a tensor cores (Sec. 3.2 "Target Model Verification",
+// Sec. 3.3 KV cache; cost Eqs. (4)-(5)).
+//
+// A unit is (sequence b, KV head) when its g = Hq/Hkv heads x 2*gamma slots
+// make two row blocks of 128 (32 drafts with g = 4, 16 with g = 8).  One CTA
+// owns both row blocks, so every K/V tile crosses HBM and L2 once and feeds
+// four MMAs: S_A = Q_A K^T, S_B = Q_B K^T, O_A += P_A V, O_B += P_B V.  At
+// this intensity (about 256 flop per K/V byte, the ridge of the GPU) the
+// tensor pipe must stay busy while the softmax runs, so S is double-buffered
+// per row block: the MMAs of tile i+1 run while the softmax works on tile i.
+//
+// The kernel is persistent: one CTA per SM (512 TMEM columns, ~197 KB of
+// shared memory) walks units blockIdx.x, blockIdx.x + gridDim.x, ... in
+// longest-prefix-first order.  Tensor memory, barriers and the K/V ring
+// carry over from unit to unit; the producer loads the next unit's Q and
+// tiles while the softmax warps finish the previous one.
+//
+// Warp roles (384 threads):
+//   warps 0-3  softmax of row block A, warps 4-7 of row block B; thread i of
+//              a block owns query row i (TMEM lane i).  Per tile: read S,
+//              update the running max / sum, write P (bf16) over the first
+//              half of its S buffer, hand it to the MMA issuer.  Per unit:
+//              O / l to the output.
+//   warp 8     TMA producer of Q (both blocks, into a region of its own, per
+//              unit) and of the K half of every tile; warp 11 of the V
+//              half.  The ring has 5 slots of 32 KB whose halves are
+//              refilled apart: K is free once the tile's S MMAs are done, a
+//              softmax before V.  Each producer's lanes hold a window of 32
+//              page ids.
+//   warps 9-10 MMA issuers, one thread per row block (issuing a tcgen05.mma
+//              takes longer than an N = 64 MMA runs, so one thread for both
+//              blocks left the tensor pipe idle); warp 9 owns TMEM.
+// TMEM (512 columns): S_A[2] [0,128), S_B[2] [128,256), O_A [256,384),
+// O_B [384,512); S buffers hold fp32 scores, P overwrites their first 32
+// columns.
+//
+// Every mbarrier wait is bounded; after a wait expires the CTA raises
+// SIMSD_EW_TIMEOUT, every role leaves its loops (the softmax warps still
+// meet at their named barriers), drains its copies and MMAs and frees TMEM.
+#include <cuda.h>
+#include <cuda_bf16.h>
+#include <cuda_runtime.h>
+
+#include <algorithm>
+
+#include "common.cuh"
+#include "kernels.h"
+#include "ptx.cuh"
+
+namespace simsd {
+namespace {
+
+constexpr int kTile = 64;        // keys per tile
+constexpr int kD = 128;          // head dimension
+constexpr int kRows = 128;       // query rows per row block (MMA M)
+constexpr int kStages = 5;       // K/V ring slots
+constexpr int kThreads = 384;
+constexpr int kSoftmaxThreads = 256;
+constexpr int kWarpProducer = 8;
+constexpr int kWarpMma = 9;  // issuer of block A's MMAs and TMEM owner; warp 10 issues block B's
+constexpr int kWarpProducerV = 11;
+constexpr uint32_t kTmemCols = 512;
+constexpr uint32_t kColS = 0;    // S of block X, buffer u: kColS + 64 * (2X + u)
+constexpr uint32_t kColO = 256;  // O of block X: kColO + 128 X
+constexpr int kHalfBytes = kTile * 128;      // 64 rows x 64 bf16 (one d-half of K or V)
+constexpr int kSlotBytes = 4 * kHalfBytes;   // K0 K1 V0 V1
+constexpr int kQHalfBytes = kRows * 128;     // 128 rows x 64 bf16
+constexpr int kQBlockBytes = 2 * kQHalfBytes;
+constexpr int kMaxSort = 256;                // sequences ranked by prefix length (longest first)
+constexpr float kRescaleThreshold = 8.0f;    // log2 units: rescale when the max grows by > 2^8
+
+struct Tc256Params {
+  const int32_t* block_table;
+  const int32_t* prefix_len;
+  const int32_t* tau;
+  const uint8_t* section;
+  const int32_t* rope_pos;  // [Bt][2*gamma] or null (inputs rotated already)
+  __nv_bfloat16* out;
+  int32_t* err_word;
+  int max_pages, page_size, num_pages;
+  int Bt, S, Hq, Hkv, g, s_blk;
+  int units;  // Bt * Hkv
+  int sort;   // rank sequences by prefix length (Bt <= kMaxSort)
+  float scale_log2;
+  unsigned long long wait_ns;
+  uint32_t extra_p;  // planted extra arrivals on bar_p (a test of the bounded waits)
+  RopeTable rope;
+};
+
+struct alignas(1024) Smem256 {
+  uint8_t ring[kStages][kSlotBytes];
+  uint8_t q[2][kQBlockBytes];
+  // K and V of a slot are released apart: K once the tile's S MMAs have
+  // completed, V once its PV MMAs have
+  uint64_t bar_k[kStages], bar_v[kStages], bar_kfree[kStages], bar_vfree[kStages];
+  uint64_t bar_q, bar_qr, bar_qfree;
+  uint64_t bar_s[2][2], bar_p[2][2], bar_pv[2], bar_ofree[2];
+  uint64_t bar_drain[2];
+  uint32_t tmem_base;
+  int abort_flag;
+  int bad[2];           // per unit parity: a needed page id is out of range
+  int32_t tau[2][64];   // per unit parity: slot labels of the unit's sequence
+  uint8_t sect[2][64];
+  int32_t order[kMaxSort];
+};
+
+constexpr size_t smem_bytes() { return sizeof(Smem256) + 1024; }
+static_assert(smem_bytes() <= 232448, "one CTA per SM");
+
+__device__ __forceinline__ void signal_abort(Smem256& sm, int32_t* err_word) {
+  raise_error(err_word, SIMSD_EW_TIMEOUT);
+  *reinterpret_cast<volatile int*>(&sm.abort_flag) = 1;
+}
+
+// Row r of a 128-byte-swizzled tile: 16-byte chunk c sits at chunk c ^ (r & 7).
+__device__ __forceinline__ uint4* sw128_chunk(uint8_t* half, int r, int c) {
+  return reinterpret_cast<uint4*>(half + r * 128 + ((c ^ (r & 7)) << 4));
+}
+
+// Rotates the pairs (x_i, x_{i+64}) held in chunk c of two d-halves in place.
+__device__ __forceinline__ void rope_chunk_pair(uint4* pa, uint4* pb, int pos, int c, const RopeTable& rope) {
+  const uint4 va = *pa, vb = *pb;
+  uint32_t wa[4] = {va.x, va.y, va.z, va.w}, wb[4] = {vb.x, vb.y, vb.z, vb.w};
+#pragma unroll
+  for (int w = 0; w < 4; ++w) {
+    float x0 = __uint_as_float(wa[w] << 16), x1 = __uint_as_float(wa[w] & 0xffff0000u);
+    float y0 = __uint_as_float(wb[w] << 16), y1 = __uint_as_float(wb[w] & 0xffff0000u);
+    float sn, cs;
+    rope_sincos(pos, rope.f[8 * c + 2 * w], &sn, &cs);
+    rope_pair(x0, y0, sn, cs);
+    rope_sincos(pos, rope.f[8 * c + 2 * w + 1], &sn, &cs);
+    rope_pair(x1, y1, sn, cs);
+    wa[w] = pack_bf16x2(x0, x1);
+    wb[w] = pack_bf16x2(y0, y1);
+  }
+  *pa = make_uint4(wa[0], wa[1], wa[2], wa[3]);
+  *pb = make_uint4(wb[0], wb[1], wb[2], wb[3]);
+}
+
+// The unit at position U of the walk: sequence (longest prefix first when
+// ranked), KV head, prefix length and number of key tiles (0 when the
+// prefix length is out of range: the unit then only writes zeros).
+struct Unit {
+  int b, kvh, n, tiles;
+  bool n_bad;
+};
+
+__device__ __forceinline__ Unit unit_at(const Tc256Params& p, const Smem256& sm, int U) {
+  Unit u;
+  const int rank = U / p.Hkv;
+  u.kvh = U - rank * p.Hkv;
+  u.b = p.sort ? sm.order[rank] : rank;
+  u.n = p.prefix_len[u.b];
+  u.n_bad = u.n < 0 || static_cast<long long>(u.n) > static_cast<long long>(p.max_pages) * p.page_size;
+  u.tiles = u.n_bad ? 0 : (u.n + kTile - 1) / kTile + 1;  // tile 0: the new slots, 1..: the prefix
+  return u;
+}
+
+__global__ void __launch_bounds__(kThreads, 1)
+    attention_tc256_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ CUtensorMap tm_kn,
+                           const __grid_constant__ CUtensorMap tm_vn, const __grid_constant__ CUtensorMap tm_kc,
+                           const __grid_constant__ CUtensorMap tm_vc, const __grid_constant__ Tc256Params p) {
+  extern __shared__ uint8_t smem_raw[];
+  Smem256& sm =
+      *reinterpret_cast<Smem256*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~static_cast<uintptr_t>(1023));
+  volatile int* abort_flag = &sm.abort_flag;
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+
+  if (tid == 0) {
+    sm.abort_flag = 0;
+    sm.bad[0] = sm.bad[1] = 0;
+    for (int s = 0; s < kStages; ++s) {
+      mbar_init(smem_u32(&sm.bar_k[s]), 1);
+      mbar_init(smem_u32(&sm.bar_v[s]), 1);
+      mbar_init(smem_u32(&sm.bar_kfree[s]), 2);  // one commit per MMA issuer
+      mbar_init(smem_u32(&sm.bar_vfree[s]), 2);
+    }
+    mbar_init(smem_u32(&sm.bar_q), 1);
+    mbar_init(smem_u32(&sm.bar_qr), 1);
+    mbar_init(smem_u32(&sm.bar_qfree), 2);
+    for (int x = 0; x < 2; ++x) {
+      for (int u = 0; u < 2; ++u) {
+        mbar_init(smem_u32(&sm.bar_s[x][u]), 1);
+        mbar_init(smem_u32(&sm.bar_p[x][u]), 4 + p.extra_p);
+      }
+      mbar_init(smem_u32(&sm.bar_pv[x]), 1);
+      mbar_init(smem_u32(&sm.bar_ofree[x]), 4);
+    }
+    mbar_init(smem_u32(&sm.bar_drain[0]), 1);
+    mbar_init(smem_u32(&sm.bar_drain[1]), 1);
+    fence_mbar_init();
+  }
+  if (warp == kWarpMma) {
+    tmem_alloc(smem_u32(&sm.tmem_base), kTmemCols);
+    tmem_relinquish();
+  }
+  if (warp == kWarpProducer && lane == 0) {
+    tma_prefetch_desc(&tm_q);
+    tma_prefetch_desc(&tm_kn);
+    tma_prefetch_desc(&tm_vn);
+    tma_prefetch_desc(&tm_kc);
+    tma_prefetch_desc(&tm_vc);
+  }
+  // from here on the previous kernel's results (prefix lengths, labels) are read
+  pdl_wait();
+  if (p.sort) {
+    // rank sequences by prefix length, longest first (ties: lower index first)
+    int32_t* nval = reinterpret_cast<int32_t*>(sm.ring[0]);
+    for (int i = tid; i < p.Bt; i += kThreads) nval[i] = p.prefix_len[i];
+    __syncthreads();
+    for (int i = tid; i < p.Bt; i += kThreads) {
+      const int ni = nval[i];
+      int r = 0;
+      for (int j = 0; j < p.Bt; ++j) {
+        const int nj = nval[j];
+        r += (nj > ni) || (nj == ni && j < i);
+      }
+      sm.order[r] = i;
+    }
+    // the staging area is overwritten by TMA later
+    fence_proxy_async_smem();
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = sm.tmem_base;
+  const int first_unit = blockIdx.x, step = gridDim.x;
+  // the last unit this CTA takes (for the dependent-launch trigger)
+  const int last_unit = first_unit + ((p.units - 1 - first_unit) / step) * step;
+
+  if (warp == kWarpProducer || warp == kWarpProducerV) {
+    // ----------------------------------------------------------- producers
+    // warp 8 loads Q and the K half of every tile, warp 11 the V half; each
+    // refills a slot's half as soon as that half is released, so K runs
+    // ahead of V (K is consumed a softmax earlier than V)
+    const int kv = warp == kWarpProducer ? 0 : 1;
+    uint32_t g = 0, jq = 0;  // tiles and units (with tiles) issued so far
+    bool ok = true;
+    for (int U = first_unit; ok && U < p.units; U += step) {
+      const Unit u = unit_at(p, sm, U);
+      if (u.tiles == 0) continue;
+      if (kv == 0) {
+        if (lane == 0 && jq > 0 && !mbar_wait(smem_u32(&sm.bar_qfree), (jq - 1) & 1, abort_flag, p.wait_ns))
+          ok = false;
+        ok = __shfl_sync(0xffffffffu, ok, 0);
+        if (!ok) break;
+        if (lane == 0) {
+          const uint32_t bq = smem_u32(&sm.bar_q);
+          const int z = u.b * p.S;
+          mbar_arrive_expect_tx(bq, 2u * kQBlockBytes);
+          tma_load_3d(smem_u32(sm.q[0]), &tm_q, bq, 0, u.kvh * p.g, z);
+          tma_load_3d(smem_u32(sm.q[0]) + kQHalfBytes, &tm_q, bq, 64, u.kvh * p.g, z);
+          tma_load_3d(smem_u32(sm.q[1]), &tm_q, bq, 0, u.kvh * p.g, z + p.s_blk);
+          tma_load_3d(smem_u32(sm.q[1]) + kQHalfBytes, &tm_q, bq, 64, u.kvh * p.g, z + p.s_blk);
+        }
+        ++jq;
+      }
+      const int32_t* bt = p.block_table + static_cast<size_t>(u.b) * p.max_pages;
+      const int P = p.page_size;
+      int win_base = -(1 << 30), win = -1;  // lane i holds the page id of page win_base + i
+      for (int t = 0; t < u.tiles; ++t) {
+        const int st = g % kStages;
+        // page ids this tile needs (prefix tiles), loaded by the whole warp
+        int pi0 = 0, nsub = 0, key0 = 0, valid = 0;
+        if (t > 0) {
+          key0 = (t - 1) * kTile;
+          valid = min(kTile, u.n - key0);
+          pi0 = key0 / P;
+          nsub = P >= kTile ? 1 : (valid + P - 1) / P;
+          if (pi0 < win_base || pi0 + nsub > win_base + 32) {
+            win_base = pi0;
+            const int pi = win_base + lane;
+            win = pi < p.max_pages ? bt[pi] : -1;
+          }
+        }
+        int pgs[kTile / 8];
+#pragma unroll
+        for (int sb = 0; sb < kTile / 8; ++sb) {
+          const int pg = __shfl_sync(0xffffffffu, win, (pi0 + sb - win_base) & 31);
+          // a page id out of range is replaced by page 0 (the softmax warps
+          // zero that sequence's output and the error bit is set there)
+          pgs[sb] = (pg < 0 || pg >= p.num_pages) ? 0 : pg;
+        }
+        if (lane == 0) {
+          const uint64_t* freed = kv == 0 ? &sm.bar_kfree[st] : &sm.bar_vfree[st];
+          if (g >= static_cast<uint32_t>(kStages) &&
+              !mbar_wait(smem_u32(freed), ((g / kStages) - 1) & 1, abort_flag, p.wait_ns)) {
+            ok = false;
+          } else {
+            const uint32_t bar = smem_u32(kv == 0 ? &sm.bar_k[st] : &sm.bar_v[st]);
+            const uint32_t d0 = smem_u32(sm.ring[st]) + 2 * kv * kHalfBytes, d1 = d0 + kHalfBytes;
+            if (t == 0) {
+              const CUtensorMap* m = kv == 0 ? &tm_kn : &tm_vn;
+              mbar_arrive_expect_tx(bar, 2u * static_cast<uint32_t>(p.S) * 128u);
+              tma_load_3d(d0, m, bar, 0, u.kvh, u.b * p.S);
+              tma_load_3d(d1, m, bar, 64, u.kvh, u.b * p.S);
+            } else {
+              const CUtensorMap* m = kv == 0 ? &tm_kc : &tm_vc;
+              if (P >= kTile) {
+                const int row = (pgs[0] * p.Hkv + u.kvh) * P + (key0 % P);
+                mbar_arrive_expect_tx(bar, 2u * kHalfBytes);
+                tma_load_2d(d0, m, bar, 0, row);
+                tma_load_2d(d1, m, bar, 64, row);
+              } else {
+                const uint32_t sub_bytes = static_cast<uint32_t>(P) * 128u;
+                mbar_arrive_expect_tx(bar, 2u * nsub * sub_bytes);
+#pragma unroll
+                for (int sb = 0; sb < kTile / 8; ++sb) {
+                  if (sb < nsub) {  // (a constant index keeps pgs in registers)
+                    const int row = (pgs[sb] * p.Hkv + u.kvh) * P;
+                    tma_load_2d(d0 + sb * sub_bytes, m, bar, 0, row);
+                    tma_load_2d(d1 + sb * sub_bytes, m, bar, 64, row);
+                  }
+                }
+              }
+            }
+          }
+        }
+        ok = __shfl_sync(0xffffffffu, ok, 0);
+        if (!ok) break;  // nothing was issued for tile g
+        ++g;
+      }
+    }
+    if (!ok && lane == 0) signal_abort(sm, p.err_word);
+    // Drain: every issued load of this warp must have landed before the CTA
+    // may exit (full limit, whatever the other waits use).
+    if (lane == 0) {
+      for (uint32_t it = g > static_cast<uint32_t>(kStages) ? g - kStages : 0; it < g; ++it) {
+        const int st = it % kStages;
+        mbar_wait(smem_u32(kv == 0 ? &sm.bar_k[st] : &sm.bar_v[st]), (it / kStages) & 1, nullptr);
+      }
+      if (kv == 0 && jq > 0) mbar_wait(smem_u32(&sm.bar_q), (jq - 1) & 1, nullptr);
+    }
+    __syncwarp();
+  } else if (warp == kWarpMma || warp == kWarpMma + 1) {
+    // ---------------------------------------------------------- MMA issuers
+    // one thread per row block; each issues its block's S and PV MMAs
+    const int x = warp - kWarpMma;
+    if (lane == 0) {
+      constexpr uint32_t kIdescQK = idesc_bf16_f32(kRows, kTile, 0, 0);
+      constexpr uint32_t kIdescPV = idesc_bf16_f32(kRows, kD, 0, 1);
+      uint32_t g = 0, jq = 0;
+      bool ok = true;
+      const uint32_t qb0 = smem_u32(sm.q[x]), qb1 = qb0 + kQHalfBytes;
+      const uint32_t ocol = tmem + kColO + 128u * x;
+      for (int U = first_unit; ok && U < p.units; U += step) {
+        const Unit u = unit_at(p, sm, U);
+        if (u.tiles == 0) continue;
+        ++jq;
+        // Q landed (rotated by the softmax warps when RoPE is applied here)
+        if (!mbar_wait(smem_u32(p.rope_pos ? &sm.bar_qr : &sm.bar_q), (jq - 1) & 1, abort_flag, p.wait_ns)) {
+          ok = false;
+          break;
+        }
+        // Issue loop of this unit: S of the next tile once its K has landed
+        // (and its S buffer's previous P has gone into a PV), PV of the
+        // oldest tile once its P is written and its V has landed, whichever
+        // is ready first.  A PV that waits for the next K would hold its V
+        // slot and stall the loads behind it.
+        const uint32_t g0 = g, g_end = g + u.tiles;
+        uint32_t s_next = g, pv_next = g;
+        unsigned long long t_last = globaltimer_ns();
+        uint32_t spins = 0;
+        while (pv_next < g_end) {
+          bool progressed = false;
+          if (s_next < g_end && s_next < pv_next + 2) {
+            const int st = s_next % kStages;
+            if (mbar_test_wait(smem_u32(&sm.bar_k[st]), (s_next / kStages) & 1)) {
+              tc_fence_after();
+              const uint32_t kb0 = smem_u32(sm.ring[st]), kb1 = kb0 + kHalfBytes;
+              const uint32_t scol = tmem + kColS + 64u * (2 * x + (s_next & 1));
+#pragma unroll
+              for (int kk = 0; kk < kD / 16; ++kk) {
+                const uint32_t off = (kk & 3) * 32;
+                tc_mma_ss(scol, sdesc_sw128((kk < 4 ? qb0 : qb1) + off, 16, 1024),
+                          sdesc_sw128((kk < 4 ? kb0 : kb1) + off, 16, 1024), kIdescQK, kk > 0);
+              }
+              tc_commit(smem_u32(&sm.bar_s[x][s_next & 1]));
+              // K of this slot may be replaced once both blocks' S have completed
+              tc_commit(smem_u32(&sm.bar_kfree[st]));
+              // the unit's last S: Q may be replaced once it has completed
+              if (s_next == g_end - 1) tc_commit(smem_u32(&sm.bar_qfree));
+              ++s_next;
+              progressed = true;
+            }
+          }
+          if (pv_next < s_next) {
+            const uint32_t gg = pv_next;
+            const int st = gg % kStages;
+            const bool first = gg == g0;
+            // P written; the previous unit's epilogue has read O_X; V landed
+            if (mbar_test_wait(smem_u32(&sm.bar_p[x][gg & 1]), (gg >> 1) & 1) &&
+                (!first || jq <= 1 || mbar_test_wait(smem_u32(&sm.bar_ofree[x]), (jq - 2) & 1)) &&
+                mbar_test_wait(smem_u32(&sm.bar_v[st]), (gg / kStages) & 1)) {
+              tc_fence_after();
+              const uint32_t vb = smem_u32(sm.ring[st]) + 2 * kHalfBytes;
+              const uint32_t pcol = tmem + kColS + 64u * (2 * x + (gg & 1));
+#pragma unroll
+              for (int kk = 0; kk < kTile / 16; ++kk)
+                tc_mma_ts(ocol, pcol + 8 * kk, sdesc_sw128(vb + kk * 2048, kHalfBytes, 1024), kIdescPV,
+                          (first && kk == 0) ? 0u : 1u);
+              tc_commit(smem_u32(&sm.bar_pv[x]));
+              tc_commit(smem_u32(&sm.bar_vfree[st]));
+              ++pv_next;
+              progressed = true;
+            }
+          }
+          if (progressed) {
+            spins = 0;
+          } else if ((++spins & 63u) == 0) {
+            const unsigned long long now = globaltimer_ns();
+            if (spins == 64) t_last = now;  // the first check of a stall starts its clock
+            if (*abort_flag || now - t_last > p.wait_ns) {
+              ok = false;
+              break;
+            }
+          }
+        }
+        g = g_end;
+      }
+      if (!ok) signal_abort(sm, p.err_word);
+      // every MMA issued by this thread has completed once this fires
+      tc_commit(smem_u32(&sm.bar_drain[x]));
+      mbar_wait(smem_u32(&sm.bar_drain[x]), 0, nullptr);
+    }
+    __syncwarp();
+  } else {
+    // -------------------------------------------------------------- softmax
+    const int x = warp >> 2;          // row block
+    const int row = tid & (kRows - 1);  // TMEM lane / query row of the block
+    const int hl = row % p.g;
+    const uint32_t lane_tmem = tmem + (static_cast<uint32_t>((warp & 3) * 32) << 16);
+    const uint32_t o_tmem = lane_tmem + kColO + 128u * x;
+    uint32_t g = 0, jq = 0, mu = 0;
+    bool ok = true;
+    for (int U = first_unit; U < p.units; U += step, ++mu) {
+      const Unit u = unit_at(p, sm, U);
+      const int par = mu & 1;  // metadata buffer of this unit
+      // every softmax thread is done with the previous unit: its flag
+      // (the other buffer) is cleared for the next one
+      asm volatile("bar.sync 1, 256;" ::: "memory");
+      if (tid == 0) sm.bad[par ^ 1] = 0;
+      if (tid < p.S) {
+        sm.tau[par][tid] = p.tau[static_cast<size_t>(u.b) * p.S + tid];
+        sm.sect[par][tid] = p.section[static_cast<size_t>(u.b) * p.S + tid];
+      }
+      if (u.n_bad) {
+        if (tid == 0 && u.kvh == 0) raise_error(p.err_word, SIMSD_EW_PREFIX_LEN);
+      } else {
+        const int npages = (u.n + p.page_size - 1) / p.page_size;
+        const int32_t* bt = p.block_table + static_cast<size_t>(u.b) * p.max_pages;
+        bool bad = false;
+        for (int i = tid; i < npages; i += kSoftmaxThreads) {
+          const int pg = bt[i];
+          bad |= pg < 0 || pg >= p.num_pages;
+        }
+        if (bad) {
+          atomicOr(&sm.bad[par], 1);
+          if (u.kvh == 0) raise_error(p.err_word, SIMSD_EW_PAGE);
+        }
+      }
+      asm volatile("bar.sync 1, 256;" ::: "memory");
+      const bool seq_bad = u.n_bad || sm.bad[par] != 0;
+      const int s = x * p.s_blk + row / p.g;
+      const bool row_exists = s < p.S;
+      const bool active = row_exists && !seq_bad && sm.sect[par][s] != kSectPad;
+      unsigned long long vis = 0ull;
+      if (active) {
+        const uint8_t si = sm.sect[par][s];
+        const int ti = sm.tau[par][s];
+        for (int t = 0; t < p.S; ++t)
+          if (temporal_visible(si, ti, sm.sect[par][t], sm.tau[par][t])) vis |= 1ull << t;
+      }
+      float m_ref = -INFINITY, l_sum = 0.f;
+      if (u.tiles > 0) {
+        ++jq;
+        if (p.rope_pos) {
+          // Q of both blocks and the new keys (the unit's first tile) are
+          // rotated in shared memory before the first S reads them
+          const int pos = p.rope_pos[static_cast<size_t>(u.b) * p.S + (row_exists ? s : 0)];
+          if (ok) ok = mbar_wait_warp(smem_u32(&sm.bar_q), (jq - 1) & 1, abort_flag, p.wait_ns);
+          if (ok) {
+            uint8_t* h0 = sm.q[x];
+            uint8_t* h1 = sm.q[x] + kQHalfBytes;
+#pragma unroll 1
+            for (int c = 0; c < 8; ++c) rope_chunk_pair(sw128_chunk(h0, row, c), sw128_chunk(h1, row, c), pos, c, p.rope);
+          }
+          const int st0 = g % kStages;
+          if (ok) ok = mbar_wait_warp(smem_u32(&sm.bar_k[st0]), (g / kStages) & 1, abort_flag, p.wait_ns);
+          if (ok) {
+            uint8_t* h0 = sm.ring[st0];
+            uint8_t* h1 = sm.ring[st0] + kHalfBytes;
+            for (int task = tid; task < p.S * 8; task += kSoftmaxThreads) {
+              const int r = task >> 3, c = task & 7;
+              const int kpos = p.rope_pos[static_cast<size_t>(u.b) * p.S + r];
+              rope_chunk_pair(sw128_chunk(h0, r, c), sw128_chunk(h1, r, c), kpos, c, p.rope);
+            }
+          }
+          fence_proxy_async_smem();
+          asm volatile("bar.sync 1, 256;" ::: "memory");
+          if (tid == 0 && !*abort_flag) mbar_arrive(smem_u32(&sm.bar_qr));
+        }
+        for (int i = 0; ok && i < u.tiles; ++i) {
+          const uint32_t gg = g + i;
+          const int st = gg % kStages;
+          const uint32_t buf = gg & 1;
+          const uint32_t s_tmem = lane_tmem + kColS + 64u * (2 * x + buf);
+          if (!mbar_wait_warp(smem_u32(&sm.bar_s[x][buf]), (gg >> 1) & 1, abort_flag, p.wait_ns)) {
+            ok = false;
+            break;
+          }
+          tc_fence_after();
+          uint32_t sa[32], sb[32];
+          tmem_ld32(s_tmem, sa);
+          tmem_ld32(s_tmem + 32, sb);
+          tmem_wait_ld();
+          const bool is_new = (i == 0);
+          const int valid = is_new ? p.S : min(kTile, u.n - (i - 1) * kTile);
+          float xs[kTile];
+#pragma unroll
+          for (int c = 0; c < kTile; ++c) xs[c] = __uint_as_float(c < 32 ? sa[c] : sb[c - 32]);
+          if (is_new || valid < kTile) {
+            // one bit word per row and a select per column (no divergence)
+            const unsigned long long keep = is_new ? vis : ((1ull << valid) - 1ull);
+            const uint32_t klo = static_cast<uint32_t>(keep), khi = static_cast<uint32_t>(keep >> 32);
+#pragma unroll
+            for (int c = 0; c < kTile; ++c) {
+              const uint32_t bit = ((c < 32 ? klo : khi) >> (c & 31)) & 1u;
+              xs[c] = bit ? xs[c] : -INFINITY;
+            }
+          }
+          float mx;
+          {
+            float r[kTile / 2];
+#pragma unroll
+            for (int c = 0; c < kTile / 2; ++c) r[c] = fmaxf(xs[2 * c], xs[2 * c + 1]);
+#pragma unroll
+            for (int w2 = kTile / 4; w2 >= 1; w2 >>= 1)
+#pragma unroll
+              for (int c = 0; c < w2; ++c) r[c] = fmaxf(r[c], r[c + w2]);
+            mx = active ? r[0] * p.scale_log2 : -INFINITY;
+          }
+          bool need = false;
+          if (active && mx != -INFINITY) {
+            if (m_ref == -INFINITY)
+              m_ref = mx;
+            else if (mx > m_ref + kRescaleThreshold)
+              need = true;
+          }
+          if (__any_sync(0xffffffffu, need)) {
+            // O holds the unit's earlier tiles: wait until the last PV of
+            // this block has completed, then scale it
+            if (i > 0 && !mbar_wait_warp(smem_u32(&sm.bar_pv[x]), (gg - 1) & 1, abort_flag, p.wait_ns)) {
+              ok = false;
+              break;
+            }
+            tc_fence_after();
+            const float f = need ? fast_exp2(m_ref - mx) : 1.0f;
+            if (need) {
+              l_sum *= f;
+              m_ref = mx;
+            }
+            if (i > 0) {
+#pragma unroll 1
+              for (int ch = 0; ch < kD / 32; ++ch) {
+                uint32_t o[32];
+                tmem_ld32(o_tmem + 32 * ch, o);
+                tmem_wait_ld();
+#pragma unroll
+                for (int c = 0; c < 32; ++c) o[c] = __float_as_uint(__uint_as_float(o[c]) * f);
+                tmem_st32(o_tmem + 32 * ch, o);
+              }
+            }
+          }
+          const float neg_m = (active && m_ref != -INFINITY) ? -m_ref : 0.f;
+          uint32_t pk[32];
+          float ps[kTile / 2];
+#pragma unroll
+          for (int c = 0; c < kTile / 2; ++c) {
+            const float p0 = fast_exp2(fmaf(xs[2 * c], p.scale_log2, neg_m));
+            const float p1 = fast_exp2(fmaf(xs[2 * c + 1], p.scale_log2, neg_m));
+            ps[c] = p0 + p1;
+            pk[c] = pack_bf16x2(p0, p1);
+          }
+#pragma unroll
+          for (int w2 = kTile / 4; w2 >= 1; w2 >>= 1)
+#pragma unroll
+            for (int c = 0; c < w2; ++c) ps[c] += ps[c + w2];
+          l_sum += ps[0];
+          tmem_st32(s_tmem, pk);
+          tmem_wait_st();
+          if ((warp & 3) < 2 && (valid < kTile || is_new)) {
+            // rows of V that no query may use are zeroed so that 0 * (stale
+            // or non-finite data) cannot reach O.  The first two warps of
+            // each block zero them (writing the same zeros), so that each
+            // block's PV, which waits only for its own P, sees them zeroed.
+            if (!mbar_wait_warp(smem_u32(&sm.bar_v[st]), (gg / kStages) & 1, abort_flag, p.wait_ns)) {
+              ok = false;
+              break;
+            }
+            const bool zero = row >= valid || (is_new && sm.sect[par][row] == kSectPad);
+            if (zero) {
+              const uint4 z = make_uint4(0u, 0u, 0u, 0u);
+              uint4* r0 = reinterpret_cast<uint4*>(sm.ring[st] + 2 * kHalfBytes + row * 128);
+              uint4* r1 = reinterpret_cast<uint4*>(sm.ring[st] + 3 * kHalfBytes + row * 128);
+#pragma unroll
+              for (int c = 0; c < 8; ++c) {
+                r0[c] = z;
+                r1[c] = z;
+              }
+            }
+            fence_proxy_async_smem();
+          }
+          tc_fence_before();
+          __syncwarp();
+          if (lane == 0) mbar_arrive(smem_u32(&sm.bar_p[x][buf]));
+        }
+        if (U == last_unit) pdl_launch_next();
+        // ---- epilogue: O of the unit's last PV, scaled by 1/l.  The S of
+        // the last tile implies that the PV two tiles back has completed,
+        // not the one just before: a parity wait for the last PV alone could
+        // see that earlier phase still open and pass at once, so the PVs of
+        // the last two tiles are awaited in order.
+        const uint32_t last = g + u.tiles - 1;
+        bool have_o = ok;
+        if (have_o && u.tiles >= 2)
+          have_o = mbar_wait_warp(smem_u32(&sm.bar_pv[x]), (last - 1) & 1, abort_flag, p.wait_ns);
+        if (have_o) have_o = mbar_wait_warp(smem_u32(&sm.bar_pv[x]), last & 1, abort_flag, p.wait_ns);
+        if (!have_o) ok = false;
+        if (have_o) tc_fence_after();
+        const bool any = have_o && active && l_sum > 0.f;
+        const float inv = any ? 1.0f / l_sum : 0.f;
+        const int h = u.kvh * p.g + hl;
+        __nv_bfloat16* orow = p.out + ((static_cast<size_t>(u.b) * p.S + (row_exists ? s : 0)) * p.Hq + h) * kD;
+#pragma unroll 1
+        for (int ch = 0; ch < kD / 32; ++ch) {
+          uint32_t o[32];
+          if (have_o) {
+            tmem_ld32(o_tmem + 32 * ch, o);
+            tmem_wait_ld();
+          }
+          if (row_exists) {
+            uint4 pkd[4];
+            uint32_t* wv = reinterpret_cast<uint32_t*>(pkd);
+#pragma unroll
+            for (int c = 0; c < 16; ++c) {
+              const float r0 = any ? __uint_as_float(o[2 * c]) * inv : 0.f;
+              const float r1 = any ? __uint_as_float(o[2 * c + 1]) * inv : 0.f;
+              wv[c] = pack_bf16x2(r0, r1);
+            }
+            uint4* dst = reinterpret_cast<uint4*>(orow + 32 * ch);
+#pragma unroll
+            for (int c = 0; c < 4; ++c) dst[c] = pkd[c];
+          }
+        }
+        // O_X may be overwritten by the next unit's first PV
+        tc_fence_before();
+        __syncwarp();
+        if (lane == 0) mbar_arrive(smem_u32(&sm.bar_ofree[x]));
+        g += u.tiles;
+      } else {
+        // a prefix length out of range: this unit's rows are zero
+        if (U == last_unit) pdl_launch_next();
+        if (row_exists) {
+          const int h = u.kvh * p.g + hl;
+          uint4* dst = reinterpret_cast<uint4*>(p.out + ((static_cast<size_t>(u.b) * p.S + s) * p.Hq + h) * kD);
+#pragma unroll
+          for (int c = 0; c < kD / 8; ++c) dst[c] = make_uint4(0u, 0u, 0u, 0u);
+        }
+      }
+    }
+    if (!ok && lane == 0) signal_abort(sm, p.err_word);
+  }
+
+  tc_fence_before();
+  __syncthreads();
+  if (warp == kWarpMma) {
+    tc_fence_after();
+    tmem_dealloc(tmem, kTmemCols);
+  }
+}
+
+}  // namespace
+
+bool tc256_applies(int Bt, int Hkv, int rb, int num_sms) {
+  return rb == 2 && static_cast<long long>(Bt) * Hkv >= num_sms;
+}
+
+cudaError_t launch_attention_tc256(const AttnTcArgs& a, int s_blk, EncodeTiledFn encode, int num_sms,
+                                   cudaStream_t stream) {
+  const int S = 2 * a.gamma, g = a.Hq / a.Hkv;
+  CUtensorMap tq, tkn, tvn, tkc, tvc;
+  {
+    const cuuint64_t dims[3] = {static_cast<cuuint64_t>(kD), static_cast<cuuint64_t>(a.Hq),
+                                static_cast<cuuint64_t>(a.Bt) * S};
+    const cuuint64_t strides[2] = {kD * 2ull, static_cast<cuuint64_t>(a.Hq) * kD * 2ull};
+    const cuuint32_t box[3] = {64u, static_cast<cuuint32_t>(g), static_cast<cuuint32_t>(s_blk)};
+    if (!make_bf16_map(encode, &tq, a.q, 3, dims, strides, box)) return cudaErrorInvalidValue;
+  }
+  {
+    const cuuint64_t dims[3] = {static_cast<cuuint64_t>(kD), static_cast<cuuint64_t>(a.Hkv),
+                                static_cast<cuuint64_t>(a.Bt) * S};
+    const cuuint64_t strides[2] = {kD * 2ull, static_cast<cuuint64_t>(a.Hkv) * kD * 2ull};
+    const cuuint32_t box[3] = {64u, 1u, static_cast<cuuint32_t>(S)};
+    if (!make_bf16_map(encode, &tkn, a.k_new, 3, dims, strides, box)) return cudaErrorInvalidValue;
+    if (!make_bf16_map(encode, &tvn, a.v_new, 3, dims, strides, box)) return cudaErrorInvalidValue;
+  }
+  {
+    const cuuint64_t dims[2] = {static_cast<cuuint64_t>(kD),
+                                std::max<cuuint64_t>(1, static_cast<cuuint64_t>(a.num_pages) * a.Hkv * a.page_size)};
+    const cuuint64_t strides[1] = {kD * 2ull};
+    const cuuint32_t box[2] = {64u, static_cast<cuuint32_t>(std::min(a.page_size, kTile))};
+    if (!make_bf16_map(encode, &tkc, a.k_cache, 2, dims, strides, box)) return cudaErrorInvalidValue;
+    if (!make_bf16_map(encode, &tvc, a.v_cache, 2, dims, strides, box)) return cudaErrorInvalidValue;
+  }
+  Tc256Params p{};
+  p.block_table = a.block_table;
+  p.prefix_len = a.prefix_len;
+  p.tau = a.tau;
+  p.section = a.section;
+  p.rope_pos = a.rope_pos;
+  p.rope = a.rope;
+  p.out = static_cast<__nv_bfloat16*>(a.out);
+  p.err_word = a.err_word;
+  p.max_pages = a.max_pages;
+  p.page_size = a.page_size;
+  p.num_pages = a.num_pages;
+  p.Bt = a.Bt;
+  p.S = S;
+  p.Hq = a.Hq;
+  p.Hkv = a.Hkv;
+  p.g = g;
+  p.s_blk = s_blk;
+  p.units = a.Bt * a.Hkv;
+  p.sort = a.Bt <= kMaxSort ? 1 : 0;
+  p.scale_log2 = a.scale * 1.4426950408889634f;
+  p.wait_ns = a.fault.wait_ns ? a.fault.wait_ns : kWaitLimitNs;
+  p.extra_p = a.fault.extra;
+  static bool attr_done = false;
+  if (!attr_done) {
+    cudaError_t e = cudaFuncSetAttribute(attention_tc256_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                         static_cast<int>(smem_bytes()));
+    if (e != cudaSuccess) return e;
+    attr_done = true;
+  }
+  const int grid = std::min(p.units, num_sms);
+  return launch_overlapped(attention_tc256_kernel, dim3(static_cast<unsigned>(grid)), dim3(kThreads), smem_bytes(),
+                           stream, 1u, tq, tkn, tvn, tkc, tvc, p);
+}
+
+}  // namespace simsd

@@ -67,6 +67,8 @@ struct AttnTcPlan {
   int sort;         // more CTAs than resident slots: longest prefix first
   int slots;        // CTAs resident at once (SMs x CTAs per SM)
   int fuse;         // 2..8 splits merge in place (cluster per unit), no workspace
+  int kind;         // 0: one row block per CTA; 1: 256-row units, one persistent CTA per SM
+  int num_sms;
   size_t ws_bytes;  // workspace bytes for the split partials (0 if nsplit == 1)
 };
 // Returns false if the shape is not supported by the tensor-core kernel.
@@ -92,6 +94,16 @@ typedef CUresult (*EncodeTiledFn)(CUtensorMap*, CUtensorMapDataType, cuuint32_t,
                                   CUtensorMapSwizzle, CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
 cudaError_t launch_attention_tc(const AttnTcArgs& a, const AttnTcPlan& plan, EncodeTiledFn encode,
                                 cudaStream_t stream);
+
+// bf16 tensor map with the 128-byte swizzle (shared by the attention kernels)
+bool make_bf16_map(EncodeTiledFn encode, CUtensorMap* m, const void* base, int rank, const cuuint64_t* dims,
+                   const cuuint64_t* strides, const cuuint32_t* box);
+
+// 256-row units (two row blocks per KV head) on one persistent CTA per SM,
+// used when there are at least as many units as SMs.
+bool tc256_applies(int Bt, int Hkv, int rb, int num_sms);
+cudaError_t launch_attention_tc256(const AttnTcArgs& a, int s_blk, EncodeTiledFn encode, int num_sms,
+                                   cudaStream_t stream);
 
 // Static device scratch of simsd_verify_attention_noalloc.
 size_t noalloc_scratch_capacity();

@@ -108,17 +108,23 @@ def _sub_batch(si, layer, seqs):
     idx = torch.as_tensor(seqs, device=si.q.device)
     bt = si.block_table[idx].cpu()
     n = si.prefix_len[idx].cpu()
-    used = []
-    for r in range(len(seqs)):
-        cnt = max(0, (int(n[r]) + P - 1) // P)
-        used.append(bt[r, :cnt])
+    max_pages = bt.shape[1]
+
+    def needed(r):
+        return min(max_pages, max(0, (int(n[r]) + P - 1) // P))
+
+    used = [bt[r, :needed(r)] for r in range(len(seqs))]
     used = torch.cat(used) if used else torch.zeros(0, dtype=torch.int32)
-    uniq, inv = torch.unique(used, return_inverse=True)
+    in_pool = (used >= 0) & (used < si.num_pages)
+    uniq, inv = torch.unique(used[in_pool], return_inverse=True)
+    # page ids outside the pool stay outside the compact pool
+    compact = torch.full_like(used, len(uniq) + 5)
+    compact[in_pool] = inv.to(used.dtype)
     new_bt = torch.full_like(bt, -1)
     pos = 0
     for r in range(len(seqs)):
-        cnt = max(0, (int(n[r]) + P - 1) // P)
-        new_bt[r, :cnt] = inv[pos:pos + cnt].to(torch.int32)
+        cnt = needed(r)
+        new_bt[r, :cnt] = compact[pos:pos + cnt].to(torch.int32)
         pos += cnt
     pages = uniq.to(si.q.device).long()
     kc = si.k_cache[layer][pages] if len(pages) else si.k_cache[layer][:1]

@@ -1,0 +1,129 @@
+"""GPU parity of the 256-row attention kernel (two row blocks of one KV head
+in one persistent CTA per SM) against the fp64 oracle, both bars of
+tests/_gpu.py.
+
+The kernel serves units of 129..256 query rows per KV head (32 drafts with
+32/8 heads, 16 drafts with 64/8 heads, 20 drafts with 32/8 heads, where the
+second block is partly empty) when the batch has at least one unit per SM;
+smaller batches keep the one-block-per-CTA kernel.  Cases: ragged prefixes
+across tile and page edges, every page size, random step maps, padding,
+undrafted and decoded positions, RoPE applied in the kernel (both position
+rules), NaN-poisoned unused cache rows, more sequences than the ranking
+handles, and the error paths.
+"""
+import numpy as np
+import pytest
+import torch
+
+from paper_2606_02544_gb300 import inputs, simsd
+from tests._gpu import assert_attention_close, gpu_attention, gpu_mask, oracle_attention
+
+pytestmark = pytest.mark.gpu
+
+
+def _w(Bt, gamma=32, Hq=32, Hkv=8, P=64, prefix=(0, 700), seed=0, std=None):
+    std = 1 / np.sqrt(128) if std is None else std
+    return inputs.Workload("t256", "bf16", Bt, Hq, Hkv, 128, gamma, prefix, 1, 64, 0.5, std, 1.0, seed, P)
+
+
+def _uses_tc256(si):
+    # at least one unit (sequence, KV head) per SM and two row blocks
+    w = si.w
+    sms = torch.cuda.get_device_properties(0).multi_processor_count
+    rows = w.g * w.S
+    return 128 < rows <= 256 and 128 % w.g == 0 and w.Bt * w.Hkv >= sms
+
+
+def _check(si, seqs=None, rope=None):
+    assert _uses_tc256(si)
+    if rope is None:
+        out, word, ws = gpu_attention(si)
+        ref = oracle_attention(si, seqs=seqs)
+    else:
+        theta, mode = rope
+        tau, sect, pos, _, merr = gpu_mask(si, mask_bits=False)
+        assert simsd.simsd_check_error(merr) == 0
+        if mode == 2:
+            n = si.prefix_len.long()[:, None]
+            pos = (n + torch.arange(si.w.S, device=n.device)[None]).to(torch.int32).contiguous()
+        out, word, ws = gpu_attention(si, mask=(tau, sect), rope_pos=pos, rope_theta=theta)
+        ref = oracle_attention(si, seqs=seqs, rope_theta=theta, rope_mode=mode)
+    assert ws == 0 and word == ref.err
+    got = out if seqs is None else out[torch.as_tensor(seqs, device=out.device)]
+    assert_attention_close(got, ref)
+    return out, word
+
+
+@pytest.mark.parametrize("P", [8, 16, 32, 64, 128, 256])
+def test_page_sizes_and_ragged_prefixes(P):
+    rng = np.random.default_rng(P)
+    n = rng.integers(0, 700, 20)
+    n[:6] = [0, 1, 63, 64, 65, 129]
+    si = inputs.make_step_inputs(_w(20, P=P, seed=P), device="cuda", prefix_override=n, random_step_map=True,
+                                 poison_unused_rows=True)
+    _check(si, seqs=[0, 1, 2, 3, 4, 5, 11, 19])
+
+
+@pytest.mark.parametrize("gamma,Hq", [(32, 32), (16, 64), (20, 32), (17, 32)])
+def test_row_layouts(gamma, Hq):
+    # 64/8 heads with 16 drafts: 256 rows of 8 heads x 32 slots; 20 or 17
+    # drafts with 32/8 heads: the second block is partly empty
+    si = inputs.make_step_inputs(_w(24, gamma=gamma, Hq=Hq, seed=gamma + Hq), device="cuda", random_step_map=True,
+                                 poison_unused_rows=True)
+    _check(si, seqs=[0, 7, 13, 23])
+
+
+def test_many_units_per_cta_and_long_prefixes():
+    # 64 sequences x 8 KV heads = 512 units: several units per CTA, prefixes
+    # from 0 to 4000 ranked longest first
+    si = inputs.make_step_inputs(_w(64, prefix=(0, 4000), seed=3), device="cuda", random_step_map=True)
+    n = si.prefix_len.cpu().numpy()
+    _check(si, seqs=sorted({int(np.argmax(n)), int(np.argmin(n)), 5, 40, 63}))
+
+
+def test_more_sequences_than_ranked():
+    # beyond 256 sequences the walk keeps the batch order
+    si = inputs.make_step_inputs(_w(300, prefix=(0, 300), seed=4), device="cuda")
+    _check(si, seqs=[0, 150, 299])
+
+
+@pytest.mark.parametrize("n_draft", [None, 0])
+def test_undrafted_decoded_and_padding(n_draft):
+    si = inputs.make_step_inputs(_w(20, prefix=(0, 500), seed=5), device="cuda")
+    si.step_map = inputs.block_step_maps(20, 32, seed=6, n_draft=n_draft, pad_frac=0.1).cuda()
+    _check(si, seqs=[0, 3, 9, 19])
+
+
+@pytest.mark.parametrize("mode", [1, 2])
+def test_rope_in_kernel(mode):
+    si = inputs.make_step_inputs(_w(20, prefix=(0, 600), seed=7 + mode), device="cuda", random_step_map=True)
+    _check(si, seqs=[0, 10, 19], rope=(1e6, mode))
+
+
+def test_unit_scale_scores():
+    si = inputs.make_step_inputs(_w(20, prefix=(100, 900), seed=9, std=1.0), device="cuda", random_step_map=True)
+    _check(si, seqs=[2, 17])
+
+
+def test_error_paths():
+    si = inputs.make_step_inputs(_w(20, prefix=(10, 300), seed=10), device="cuda")
+    sm = si.step_map.clone()
+    sm[0, 2] = 0                                    # padding slot in sequence 0
+    sm[3, :2] = 1                                   # invalid map: all padding
+    si.step_map = sm
+    n = si.prefix_len.clone()
+    n[1] = si.block_table.shape[1] * si.w.page_size + 3    # beyond the block table
+    si.prefix_len = n
+    bt = si.block_table.clone()
+    bt[2, 1] = si.num_pages + 5                     # page id outside the pool
+    si.block_table = bt
+    out, word = _check(si, seqs=[0, 1, 2, 3, 4])
+    assert word & simsd.EW_PREFIX_LEN and word & simsd.EW_PAGE and word & simsd.EW_STEP_MAP
+    assert (out[1:4].float() == 0).all() and (out[0, [2, 34]].float() == 0).all()
+
+
+def test_deterministic_and_equal_to_rerun():
+    si = inputs.make_step_inputs(_w(24, prefix=(100, 900), seed=11), device="cuda", random_step_map=True)
+    a, _, _ = gpu_attention(si)
+    b, _, _ = gpu_attention(si)
+    assert torch.equal(a, b)
