@@ -56,7 +56,7 @@ def _peaks():
 
 def _kernel_sha():
     h = hashlib.sha256()
-    for fn in ("attention_tc.cu", "ptx.cuh", "common.cuh", "accept.cu"):
+    for fn in ("attention_tc.cu", "attention_tc256.cu", "ptx.cuh", "common.cuh", "accept.cu"):
         with open(os.path.join(ROOT, "paper_2606_02544_gb300", "csrc", fn), "rb") as f:
             h.update(f.read())
     return h.hexdigest()[:16]
