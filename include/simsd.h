@@ -164,14 +164,14 @@ SIMSD_API int simsd_verify_attention(int dtype, const void* q, const void* k_new
  * cannot allocate device memory.  The paper has no counterpart; this is a
  * deployment convenience.
  *
- * Some callers cannot call cudaMalloc: a serving loop that is being captured
- * into a CUDA graph (allocation is not allowed inside stream capture), or an
- * engine that hands all device memory to its own pool at start-up and must
- * not stall on the allocator (cudaMalloc may synchronise the device).  This
- * entry point takes the same arguments minus the workspace: the scratch for
- * the split partials comes from a 12 MiB array in device memory that the
- * library owns (every GPU that loads libsimsd.so holds it until the process
- * exits).  It allocates nothing and calls no allocating routine.
+ * Some callers cannot call cudaMalloc: an engine that hands all device
+ * memory to its own pool at start-up and must not stall on the allocator
+ * (cudaMalloc may synchronise the device), or a process under a memory
+ * budget that forbids further device allocation.  This entry point takes
+ * the same arguments minus the workspace: the scratch for the split
+ * partials comes from a 12 MiB array in device memory that the library owns
+ * (every GPU that loads libsimsd.so holds it until the process exits).  It
+ * allocates nothing and calls no allocating routine.
  *   - The first call on each device looks up the array's device address
  *     (cudaGetSymbolAddress) and keeps it for the life of the process; make
  *     that first call before any stream capture.  Because the address is
