@@ -58,7 +58,12 @@ def _draw_is_valid(tl, dl, a, gamma, u, tok, t):
     return lo <= thr + DRAW_BAND * tot and c[tok] >= thr - DRAW_BAND * tot
 
 
-def _compare(si, expect_err=0, min_exact=0.5):
+def _compare(si, expect_err=0):
+    """Every sequence whose decisions all lie outside the fp32 band (by the
+    oracle's own fp64 numbers) must match the oracle exactly; a sequence
+    with a decision inside the band must make a valid choice.  Band hits
+    are rare (each decision lands in the band with probability ~2 * 2e-5)
+    and are counted."""
     tl = si.target_logits.cpu().numpy()
     dl = si.draft_logits.cpu().numpy()
     dr = si.draft.cpu().numpy()
@@ -69,23 +74,29 @@ def _compare(si, expect_err=0, min_exact=0.5):
     ga, got, gerr = _gpu(si)
     ra, rot, ral, rmg, rerr = orc.accept_sampled(tl, dl, dr, ua, us, gamma, temperature=si.temperature)
     assert gerr == rerr == expect_err
-    exact = 0
+    band_hits = 0
     for b in range(Bt):
         a = int(ga[b])
         assert 0 <= a <= gamma
+        # the acceptance decisions that matter: rows up to the first rejection
+        last = min(max(a, int(ra[b])), gamma - 1)
+        near_alpha = any(abs(float(ua[b, r]) - ral[b, r]) < ALPHA_BAND for r in range(last + 1))
+        near_draw = rmg[b] < DRAW_BAND
+        if not (near_alpha or near_draw):
+            assert a == ra[b], (b, a, ra[b])
+            np.testing.assert_array_equal(got[b], rot[b])
+            continue
+        band_hits += 1
         if a != ra[b]:
-            # only a decision inside the band may differ
             r = min(a, int(ra[b]))
             assert abs(float(ua[b, r]) - ral[b, r]) < ALPHA_BAND, (b, a, ra[b], ua[b, r], ral[b, r])
         np.testing.assert_array_equal(got[b, :a], dr[b, :a])
         assert (got[b, a + 1:] == -1).all()
-        if a == ra[b] and got[b, a] == rot[b, a]:
-            exact += 1
-            continue
-        if a == ra[b]:
-            assert rmg[b] < DRAW_BAND, (b, a, got[b, a], rot[b, a], rmg[b])
+        if a == ra[b] and got[b, a] != rot[b, a]:
+            assert near_draw, (b, a, got[b, a], rot[b, a], rmg[b])
         assert _draw_is_valid(tl[b], dl[b], a, gamma, us[b], int(got[b, a]), si.temperature), (b, a, got[b, a])
-    assert exact >= min_exact * Bt, (exact, Bt)
+    print(f"accept_sampled Bt={Bt} gamma={gamma}: {band_hits} sequence(s) with a decision in the fp32 band")
+    assert band_hits <= max(2, Bt // 100), band_hits
     return ga, got
 
 
