@@ -61,9 +61,9 @@ def _draw_is_valid(tl, dl, a, gamma, u, tok, t):
 def _compare(si, expect_err=0):
     """Every sequence whose decisions all lie outside the fp32 band (by the
     oracle's own fp64 numbers) must match the oracle exactly; a sequence
-    with a decision inside the band must make a valid choice.  Band hits
-    are rare (each decision lands in the band with probability ~2 * 2e-5)
-    and are counted."""
+    with a decision inside the band must make a valid choice.  Band hits are
+    counted: at V = 151936 most draws are band hits, since one token's
+    probability (~7e-6 of the total) is below the band."""
     tl = si.target_logits.cpu().numpy()
     dl = si.draft_logits.cpu().numpy()
     dr = si.draft.cpu().numpy()
@@ -95,8 +95,13 @@ def _compare(si, expect_err=0):
         if a == ra[b] and got[b, a] != rot[b, a]:
             assert near_draw, (b, a, got[b, a], rot[b, a], rmg[b])
         assert _draw_is_valid(tl[b], dl[b], a, gamma, us[b], int(got[b, a]), si.temperature), (b, a, got[b, a])
-    print(f"accept_sampled Bt={Bt} gamma={gamma}: {band_hits} sequence(s) with a decision in the fp32 band")
-    assert band_hits <= max(2, Bt // 100), band_hits
+    exact = int(sum(int(ga[b]) == int(ra[b]) and np.array_equal(got[b], rot[b]) for b in range(Bt)))
+    print(f"accept_sampled Bt={Bt} gamma={gamma} V={V}: {band_hits} sequence(s) with a decision in the fp32 band, "
+          f"{exact} of {Bt} equal to the oracle")
+    # measured on the GB300: every sequence of every case equal to the oracle
+    # (band hits included, 0-79% of the sequences at V 151936); a valid
+    # in-band choice may still differ on at most 2% of them
+    assert exact >= Bt - max(1, Bt // 50), (exact, Bt, band_hits)
     return ga, got
 
 
