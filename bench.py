@@ -357,7 +357,7 @@ def run_e2e(args, si, st, stream):
     h_t = [torch.empty_like(st.out_tokens, device="cpu").pin_memory() for _ in sets]
     bi = sum(t.numel() * t.element_size() for t in host_in.values())
     bo = h_a[0].numel() * 4 + h_t[0].numel() * 4
-    steps = max(3, min(args.steps, 200 if si.w.layers == 1 else 20))
+    steps = max(3, min(args.steps, 200 if si.w.layers == 1 else 10))
     copy_stream = torch.cuda.Stream()
     copied = [torch.cuda.Event() for _ in sets]
     done = [torch.cuda.Event() for _ in sets]
