@@ -20,9 +20,13 @@ from tests._gpu import assert_attention_close, gpu_attention, gpu_mask, oracle_a
 pytestmark = pytest.mark.gpu
 
 
-def test_attention_wait_runs_out_and_the_context_stays_usable():
-    # 40 sequences x 8 KV heads: 320 unsplit units in two waves
-    w = inputs.Workload("we", "bf16", 40, 16, 8, 128, 4, (100, 300), 1, 64, 0.5, 1 / np.sqrt(128), 1.0, 31)
+@pytest.mark.parametrize("Bt,Hq,gamma", [(40, 16, 4), (20, 32, 32)])
+def test_attention_wait_runs_out_and_the_context_stays_usable(Bt, Hq, gamma):
+    # 40 sequences x 8 KV heads of 16 rows: 320 unsplit units in two waves
+    # of the one-row-block kernel; 20 x 8 units of 256 rows: the persistent
+    # two-row-block kernel (each block's MMA issuer waits for P that the
+    # planted count never completes)
+    w = inputs.Workload("we", "bf16", Bt, Hq, 8, 128, gamma, (100, 300), 1, 64, 0.5, 1 / np.sqrt(128), 1.0, 31)
     si = inputs.make_step_inputs(w, device="cuda", random_step_map=True, with_logits=False)
     tau, sect, _, _, merr = gpu_mask(si, mask_bits=False)
     assert simsd.simsd_check_error(merr) == 0
