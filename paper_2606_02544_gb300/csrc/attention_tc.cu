@@ -62,7 +62,14 @@ constexpr int kD = 128;              // head dimension
 constexpr int kRows = 128;           // MMA M (query rows per CTA)
 constexpr int kStages = 3;           // ring slots of one CTA
 constexpr int kThreads = 192;
-constexpr int kCtasPerSm = 2;        // register (launch bounds) and shared-memory budget of one CTA
+constexpr int kCtasPerSm = 2;        // shared-memory budget of one CTA
+// Registers per thread: at most 128, so that two CTAs fit one SM by the
+// per-scheduler register file (each CTA's warps 0, 1, 4, 5 share two of the
+// four schedulers).  With more, the block scheduler counts one CTA per SM: a
+// launch still starts two per SM, but a freed slot is refilled only once its
+// SM is empty, which left SMs idle for tens of microseconds on ragged
+// prefixes.
+constexpr int kMaxRegs = 128;
 constexpr int kWarpProducer = 4;
 constexpr int kWarpMma = 5;
 constexpr uint32_t kTmemCols = 256;
@@ -131,7 +138,7 @@ __device__ __forceinline__ uint4 ld_sw128_chunk(const uint8_t* half, int r, int 
 // in shared memory (a separate instantiation, so that the unclustered kernel
 // carries no cluster barriers).
 template <bool kFuse>
-__global__ void __launch_bounds__(kThreads, kCtasPerSm)
+__global__ void __maxnreg__(kMaxRegs)
     attention_tc_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ CUtensorMap tm_kn,
                         const __grid_constant__ CUtensorMap tm_vn, const __grid_constant__ CUtensorMap tm_kc,
                         const __grid_constant__ CUtensorMap tm_vc, const __grid_constant__ TcParams p) {
