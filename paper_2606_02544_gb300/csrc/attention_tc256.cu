@@ -16,7 +16,7 @@
 // carry over from unit to unit; the producer loads the next unit's Q and
 // tiles while the softmax warps finish the previous one.
 //
-// Warp roles (384 threads):
+// Warp roles (512 threads):
 //   warps 0-3  softmax of row block A, warps 4-7 of row block B; thread i of
 //              a block owns query row i (TMEM lane i).  Per tile: read S,
 //              update the running max / sum, write P (bf16) over the first
@@ -28,9 +28,11 @@
 //              refilled apart: K is free once the tile's S MMAs are done, a
 //              softmax before V.  Each producer's lanes hold a window of 32
 //              page ids.
-//   warps 9-10 MMA issuers, one thread per row block (issuing a tcgen05.mma
-//              takes longer than an N = 64 MMA runs, so one thread for both
-//              blocks left the tensor pipe idle); warp 9 owns TMEM.
+//   warps 9, 10, 12, 13  MMA issuers, one thread each: S of row block A, S
+//              of B, PV of A, PV of B (a thread that issues a tcgen05.mma
+//              is held about as long as the MMA runs, so a thread serving
+//              two of these streams delays one behind the other); warp 9
+//              owns TMEM.
 // TMEM (512 columns): S_A[2] [0,128), S_B[2] [128,256), O_A [256,384),
 // O_B [384,512); S buffers hold fp32 scores, P overwrites their first 32
 // columns.
@@ -55,10 +57,11 @@ constexpr int kTile = 64;        // keys per tile
 constexpr int kD = 128;          // head dimension
 constexpr int kRows = 128;       // query rows per row block (MMA M)
 constexpr int kStages = 5;       // K/V ring slots
-constexpr int kThreads = 384;
+constexpr int kThreads = 512;  // warps 14-15 only meet the final barrier
 constexpr int kSoftmaxThreads = 256;
 constexpr int kWarpProducer = 8;
-constexpr int kWarpMma = 9;  // issuer of block A's MMAs and TMEM owner; warp 10 issues block B's
+constexpr int kWarpMma = 9;  // S issuer of row block A and TMEM owner; warp 10: S of block B
+constexpr int kWarpPv = 12;  // PV issuer of row block A; warp 13: PV of block B
 constexpr int kWarpProducerV = 11;
 constexpr uint32_t kTmemCols = 512;
 constexpr uint32_t kColS = 0;    // S of block X, buffer u: kColS + 64 * (2X + u)
@@ -69,6 +72,7 @@ constexpr int kQHalfBytes = kRows * 128;     // 128 rows x 64 bf16
 constexpr int kQBlockBytes = 2 * kQHalfBytes;
 constexpr int kMaxSort = 256;                // sequences ranked by prefix length (longest first)
 constexpr float kRescaleThreshold = 8.0f;    // log2 units: rescale when the max grows by > 2^8
+static_assert(kTile == 64, "the softmax reductions are written out for 64 keys");
 
 struct Tc256Params {
   const int32_t* block_table;
@@ -95,8 +99,10 @@ struct alignas(1024) Smem256 {
   // completed, V once its PV MMAs have
   uint64_t bar_k[kStages], bar_v[kStages], bar_kfree[kStages], bar_vfree[kStages];
   uint64_t bar_q, bar_qr, bar_qfree;
-  uint64_t bar_s[2][2], bar_p[2][2], bar_pv[2], bar_ofree[2];
-  uint64_t bar_drain[2];
+  uint64_t bar_s[2][2], bar_p[2][2], bar_ofree[2];
+  // PV_X of the tiles that use S buffer u have completed (one phase per PV)
+  uint64_t bar_pvs[2][2];
+  uint64_t bar_drain[4];
   uint32_t tmem_base;
   int abort_flag;
   int bad[2];           // per unit parity: a needed page id is out of range
@@ -178,17 +184,16 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
     mbar_init(smem_u32(&sm.bar_q), 1);
     mbar_init(smem_u32(&sm.bar_qr), 1);
-    mbar_init(smem_u32(&sm.bar_qfree), 2);
+    mbar_init(smem_u32(&sm.bar_qfree), 2);  // one commit per S issuer
     for (int x = 0; x < 2; ++x) {
       for (int u = 0; u < 2; ++u) {
         mbar_init(smem_u32(&sm.bar_s[x][u]), 1);
         mbar_init(smem_u32(&sm.bar_p[x][u]), 4 + p.extra_p);
+        mbar_init(smem_u32(&sm.bar_pvs[x][u]), 1);
       }
-      mbar_init(smem_u32(&sm.bar_pv[x]), 1);
       mbar_init(smem_u32(&sm.bar_ofree[x]), 4);
     }
-    mbar_init(smem_u32(&sm.bar_drain[0]), 1);
-    mbar_init(smem_u32(&sm.bar_drain[1]), 1);
+    for (int d = 0; d < 4; ++d) mbar_init(smem_u32(&sm.bar_drain[d]), 1);
     fence_mbar_init();
   }
   if (warp == kWarpMma) {
@@ -226,206 +231,201 @@ __global__ void __launch_bounds__(kThreads, 1)
   tc_fence_after();
   const uint32_t tmem = sm.tmem_base;
   const int first_unit = blockIdx.x, step = gridDim.x;
+
   // the last unit this CTA takes (for the dependent-launch trigger)
   const int last_unit = first_unit + ((p.units - 1 - first_unit) / step) * step;
 
-  if (warp == kWarpProducer || warp == kWarpProducerV) {
-    // ----------------------------------------------------------- producers
-    // warp 8 loads Q and the K half of every tile, warp 11 the V half; each
-    // refills a slot's half as soon as that half is released, so K runs
-    // ahead of V (K is consumed a softmax earlier than V)
-    const int kv = warp == kWarpProducer ? 0 : 1;
-    uint32_t g = 0, jq = 0;  // tiles and units (with tiles) issued so far
-    bool ok = true;
-    for (int U = first_unit; ok && U < p.units; U += step) {
-      const Unit u = unit_at(p, sm, U);
-      if (u.tiles == 0) continue;
-      if (kv == 0) {
-        if (lane == 0 && jq > 0 && !mbar_wait(smem_u32(&sm.bar_qfree), (jq - 1) & 1, abort_flag, p.wait_ns))
-          ok = false;
-        ok = __shfl_sync(0xffffffffu, ok, 0);
-        if (!ok) break;
-        if (lane == 0) {
-          const uint32_t bq = smem_u32(&sm.bar_q);
-          const int z = u.b * p.S;
-          mbar_arrive_expect_tx(bq, 2u * kQBlockBytes);
-          tma_load_3d(smem_u32(sm.q[0]), &tm_q, bq, 0, u.kvh * p.g, z);
-          tma_load_3d(smem_u32(sm.q[0]) + kQHalfBytes, &tm_q, bq, 64, u.kvh * p.g, z);
-          tma_load_3d(smem_u32(sm.q[1]), &tm_q, bq, 0, u.kvh * p.g, z + p.s_blk);
-          tma_load_3d(smem_u32(sm.q[1]) + kQHalfBytes, &tm_q, bq, 64, u.kvh * p.g, z + p.s_blk);
-        }
-        ++jq;
-      }
-      const int32_t* bt = p.block_table + static_cast<size_t>(u.b) * p.max_pages;
-      const int P = p.page_size;
-      int win_base = -(1 << 30), win = -1;  // lane i holds the page id of page win_base + i
-      for (int t = 0; t < u.tiles; ++t) {
-        const int st = g % kStages;
-        // page ids this tile needs (prefix tiles), loaded by the whole warp
-        int pi0 = 0, nsub = 0, key0 = 0, valid = 0;
-        if (t > 0) {
-          key0 = (t - 1) * kTile;
-          valid = min(kTile, u.n - key0);
-          pi0 = key0 / P;
-          nsub = P >= kTile ? 1 : (valid + P - 1) / P;
-          if (pi0 < win_base || pi0 + nsub > win_base + 32) {
-            win_base = pi0;
-            const int pi = win_base + lane;
-            win = pi < p.max_pages ? bt[pi] : -1;
-          }
-        }
-        int pgs[kTile / 8];
-#pragma unroll
-        for (int sb = 0; sb < kTile / 8; ++sb) {
-          const int pg = __shfl_sync(0xffffffffu, win, (pi0 + sb - win_base) & 31);
-          // a page id out of range is replaced by page 0 (the softmax warps
-          // zero that sequence's output and the error bit is set there)
-          pgs[sb] = (pg < 0 || pg >= p.num_pages) ? 0 : pg;
-        }
-        if (lane == 0) {
-          const uint64_t* freed = kv == 0 ? &sm.bar_kfree[st] : &sm.bar_vfree[st];
-          if (g >= static_cast<uint32_t>(kStages) &&
-              !mbar_wait(smem_u32(freed), ((g / kStages) - 1) & 1, abort_flag, p.wait_ns)) {
+  // Register split (setmaxnreg, per warpgroup): the two softmax warpgroups
+  // take 200 registers a thread, the two control warpgroups give theirs
+  // down to 56 (2 x 128 x 200 + 2 x 128 x 56 = 65,536, the 512 x 128 the
+  // block is launched with).
+  if (warp >= 8) {
+    asm volatile("setmaxnreg.dec.sync.aligned.u32 56;");
+    if (warp == kWarpProducer || warp == kWarpProducerV) {
+      // ----------------------------------------------------------- producers
+      // warp 8 loads Q and the K half of every tile, warp 11 the V half; each
+      // refills a slot's half as soon as that half is released, so K runs
+      // ahead of V (K is consumed a softmax earlier than V)
+      const int kv = warp == kWarpProducer ? 0 : 1;
+      uint32_t g = 0, jq = 0;  // tiles and units (with tiles) issued so far
+      bool ok = true;
+      for (int U = first_unit; ok && U < p.units; U += step) {
+        const Unit u = unit_at(p, sm, U);
+        if (u.tiles == 0) continue;
+        if (kv == 0) {
+          if (lane == 0 && jq > 0 && !mbar_wait(smem_u32(&sm.bar_qfree), (jq - 1) & 1, abort_flag, p.wait_ns))
             ok = false;
-          } else {
-            const uint32_t bar = smem_u32(kv == 0 ? &sm.bar_k[st] : &sm.bar_v[st]);
-            const uint32_t d0 = smem_u32(sm.ring[st]) + 2 * kv * kHalfBytes, d1 = d0 + kHalfBytes;
-            if (t == 0) {
-              const CUtensorMap* m = kv == 0 ? &tm_kn : &tm_vn;
-              mbar_arrive_expect_tx(bar, 2u * static_cast<uint32_t>(p.S) * 128u);
-              tma_load_3d(d0, m, bar, 0, u.kvh, u.b * p.S);
-              tma_load_3d(d1, m, bar, 64, u.kvh, u.b * p.S);
+          ok = __shfl_sync(0xffffffffu, ok, 0);
+          if (!ok) break;
+          if (lane == 0) {
+            const uint32_t bq = smem_u32(&sm.bar_q);
+            const int z = u.b * p.S;
+            mbar_arrive_expect_tx(bq, 2u * kQBlockBytes);
+            tma_load_3d(smem_u32(sm.q[0]), &tm_q, bq, 0, u.kvh * p.g, z);
+            tma_load_3d(smem_u32(sm.q[0]) + kQHalfBytes, &tm_q, bq, 64, u.kvh * p.g, z);
+            tma_load_3d(smem_u32(sm.q[1]), &tm_q, bq, 0, u.kvh * p.g, z + p.s_blk);
+            tma_load_3d(smem_u32(sm.q[1]) + kQHalfBytes, &tm_q, bq, 64, u.kvh * p.g, z + p.s_blk);
+          }
+          ++jq;
+        }
+        const int32_t* bt = p.block_table + static_cast<size_t>(u.b) * p.max_pages;
+        const int P = p.page_size;
+        int win_base = -(1 << 30), win = -1;  // lane i holds the page id of page win_base + i
+        for (int t = 0; t < u.tiles; ++t) {
+          const int st = g % kStages;
+          // page ids this tile needs (prefix tiles), loaded by the whole warp
+          int pi0 = 0, nsub = 0, key0 = 0, valid = 0;
+          if (t > 0) {
+            key0 = (t - 1) * kTile;
+            valid = min(kTile, u.n - key0);
+            pi0 = key0 / P;
+            nsub = P >= kTile ? 1 : (valid + P - 1) / P;
+            if (pi0 < win_base || pi0 + nsub > win_base + 32) {
+              win_base = pi0;
+              const int pi = win_base + lane;
+              win = pi < p.max_pages ? bt[pi] : -1;
+            }
+          }
+          int pgs[kTile / 8];
+  #pragma unroll
+          for (int sb = 0; sb < kTile / 8; ++sb) {
+            const int pg = __shfl_sync(0xffffffffu, win, (pi0 + sb - win_base) & 31);
+            // a page id out of range is replaced by page 0 (the softmax warps
+            // zero that sequence's output and the error bit is set there)
+            pgs[sb] = (pg < 0 || pg >= p.num_pages) ? 0 : pg;
+          }
+          if (lane == 0) {
+            const uint64_t* freed = kv == 0 ? &sm.bar_kfree[st] : &sm.bar_vfree[st];
+            if (g >= static_cast<uint32_t>(kStages) &&
+                !mbar_wait(smem_u32(freed), ((g / kStages) - 1) & 1, abort_flag, p.wait_ns)) {
+              ok = false;
             } else {
-              const CUtensorMap* m = kv == 0 ? &tm_kc : &tm_vc;
-              if (P >= kTile) {
-                const int row = (pgs[0] * p.Hkv + u.kvh) * P + (key0 % P);
-                mbar_arrive_expect_tx(bar, 2u * kHalfBytes);
-                tma_load_2d(d0, m, bar, 0, row);
-                tma_load_2d(d1, m, bar, 64, row);
+              const uint32_t bar = smem_u32(kv == 0 ? &sm.bar_k[st] : &sm.bar_v[st]);
+              const uint32_t d0 = smem_u32(sm.ring[st]) + 2 * kv * kHalfBytes, d1 = d0 + kHalfBytes;
+              if (t == 0) {
+                const CUtensorMap* m = kv == 0 ? &tm_kn : &tm_vn;
+                mbar_arrive_expect_tx(bar, 2u * static_cast<uint32_t>(p.S) * 128u);
+                tma_load_3d(d0, m, bar, 0, u.kvh, u.b * p.S);
+                tma_load_3d(d1, m, bar, 64, u.kvh, u.b * p.S);
               } else {
-                const uint32_t sub_bytes = static_cast<uint32_t>(P) * 128u;
-                mbar_arrive_expect_tx(bar, 2u * nsub * sub_bytes);
-#pragma unroll
-                for (int sb = 0; sb < kTile / 8; ++sb) {
-                  if (sb < nsub) {  // (a constant index keeps pgs in registers)
-                    const int row = (pgs[sb] * p.Hkv + u.kvh) * P;
-                    tma_load_2d(d0 + sb * sub_bytes, m, bar, 0, row);
-                    tma_load_2d(d1 + sb * sub_bytes, m, bar, 64, row);
+                const CUtensorMap* m = kv == 0 ? &tm_kc : &tm_vc;
+                if (P >= kTile) {
+                  const int row = (pgs[0] * p.Hkv + u.kvh) * P + (key0 % P);
+                  mbar_arrive_expect_tx(bar, 2u * kHalfBytes);
+                  tma_load_2d(d0, m, bar, 0, row);
+                  tma_load_2d(d1, m, bar, 64, row);
+                } else {
+                  const uint32_t sub_bytes = static_cast<uint32_t>(P) * 128u;
+                  mbar_arrive_expect_tx(bar, 2u * nsub * sub_bytes);
+  #pragma unroll
+                  for (int sb = 0; sb < kTile / 8; ++sb) {
+                    if (sb < nsub) {  // (a constant index keeps pgs in registers)
+                      const int row = (pgs[sb] * p.Hkv + u.kvh) * P;
+                      tma_load_2d(d0 + sb * sub_bytes, m, bar, 0, row);
+                      tma_load_2d(d1 + sb * sub_bytes, m, bar, 64, row);
+                    }
                   }
                 }
               }
             }
           }
+          ok = __shfl_sync(0xffffffffu, ok, 0);
+          if (!ok) break;  // nothing was issued for tile g
+          ++g;
         }
-        ok = __shfl_sync(0xffffffffu, ok, 0);
-        if (!ok) break;  // nothing was issued for tile g
-        ++g;
       }
-    }
-    if (!ok && lane == 0) signal_abort(sm, p.err_word);
-    // Drain: every issued load of this warp must have landed before the CTA
-    // may exit (full limit, whatever the other waits use).
-    if (lane == 0) {
-      for (uint32_t it = g > static_cast<uint32_t>(kStages) ? g - kStages : 0; it < g; ++it) {
-        const int st = it % kStages;
-        mbar_wait(smem_u32(kv == 0 ? &sm.bar_k[st] : &sm.bar_v[st]), (it / kStages) & 1, nullptr);
-      }
-      if (kv == 0 && jq > 0) mbar_wait(smem_u32(&sm.bar_q), (jq - 1) & 1, nullptr);
-    }
-    __syncwarp();
-  } else if (warp == kWarpMma || warp == kWarpMma + 1) {
-    // ---------------------------------------------------------- MMA issuers
-    // one thread per row block; each issues its block's S and PV MMAs
-    const int x = warp - kWarpMma;
-    if (lane == 0) {
-      constexpr uint32_t kIdescQK = idesc_bf16_f32(kRows, kTile, 0, 0);
-      constexpr uint32_t kIdescPV = idesc_bf16_f32(kRows, kD, 0, 1);
-      uint32_t g = 0, jq = 0;
-      bool ok = true;
-      const uint32_t qb0 = smem_u32(sm.q[x]), qb1 = qb0 + kQHalfBytes;
-      const uint32_t ocol = tmem + kColO + 128u * x;
-      for (int U = first_unit; ok && U < p.units; U += step) {
-        const Unit u = unit_at(p, sm, U);
-        if (u.tiles == 0) continue;
-        ++jq;
-        // Q landed (rotated by the softmax warps when RoPE is applied here)
-        if (!mbar_wait(smem_u32(p.rope_pos ? &sm.bar_qr : &sm.bar_q), (jq - 1) & 1, abort_flag, p.wait_ns)) {
-          ok = false;
-          break;
+      if (!ok && lane == 0) signal_abort(sm, p.err_word);
+      // Drain: every issued load of this warp must have landed before the CTA
+      // may exit (full limit, whatever the other waits use).
+      if (lane == 0) {
+        for (uint32_t it = g > static_cast<uint32_t>(kStages) ? g - kStages : 0; it < g; ++it) {
+          const int st = it % kStages;
+          mbar_wait(smem_u32(kv == 0 ? &sm.bar_k[st] : &sm.bar_v[st]), (it / kStages) & 1, nullptr);
         }
-        // Issue loop of this unit: S of the next tile once its K has landed
-        // (and its S buffer's previous P has gone into a PV), PV of the
-        // oldest tile once its P is written and its V has landed, whichever
-        // is ready first.  A PV that waits for the next K would hold its V
-        // slot and stall the loads behind it.
-        const uint32_t g0 = g, g_end = g + u.tiles;
-        uint32_t s_next = g, pv_next = g;
-        unsigned long long t_last = globaltimer_ns();
-        uint32_t spins = 0;
-        while (pv_next < g_end) {
-          bool progressed = false;
-          if (s_next < g_end && s_next < pv_next + 2) {
-            const int st = s_next % kStages;
-            if (mbar_test_wait(smem_u32(&sm.bar_k[st]), (s_next / kStages) & 1)) {
+        if (kv == 0 && jq > 0) mbar_wait(smem_u32(&sm.bar_q), (jq - 1) & 1, nullptr);
+      }
+      __syncwarp();
+    } else if (warp >= kWarpMma && warp <= kWarpPv + 1) {
+      // ---------------------------------------------------------- MMA issuers
+      // four threads: the S MMAs of row block A (warp 9) and B (warp 10), the
+      // PV MMAs of A (warp 12) and B (warp 13).  A thread that issues a
+      // tcgen05.mma is held about as long as the MMA runs, so a thread that
+      // served two of these streams kept a request of one waiting behind the
+      // MMAs of the other (a written P behind the next tile's S, or one
+      // block's P behind the other's PV).  Each thread waits on one barrier
+      // at a time.
+      const bool is_s = warp < kWarpProducerV;
+      const int x = is_s ? warp - kWarpMma : warp - kWarpPv;
+      if (lane == 0) {
+        constexpr uint32_t kIdescQK = idesc_bf16_f32(kRows, kTile, 0, 0);
+        constexpr uint32_t kIdescPV = idesc_bf16_f32(kRows, kD, 0, 1);
+        const uint32_t qb0 = smem_u32(sm.q[x]), qb1 = qb0 + kQHalfBytes;
+        const uint32_t ocol = tmem + kColO + 128u * x;
+        uint32_t g = 0, jq = 0;
+        bool ok = true;
+        for (int U = first_unit; ok && U < p.units; U += step) {
+          const Unit u = unit_at(p, sm, U);
+          if (u.tiles == 0) continue;
+          ++jq;
+          const uint32_t g0 = g, g_end = g + u.tiles;
+          if (is_s) {
+            // Q landed (rotated by the softmax warps when RoPE is applied here)
+            ok = mbar_wait(smem_u32(p.rope_pos ? &sm.bar_qr : &sm.bar_q), (jq - 1) & 1, abort_flag, p.wait_ns);
+            for (uint32_t gg = g0; ok && gg < g_end; ++gg) {
+              // S_X(t) needs K(t) and the completion of PV_X(t - 2), which read
+              // the P held in the same S buffer
+              const int st = gg % kStages;
+              ok = mbar_wait(smem_u32(&sm.bar_k[st]), (gg / kStages) & 1, abort_flag, p.wait_ns) &&
+                   (gg < 2 || mbar_wait(smem_u32(&sm.bar_pvs[x][gg & 1]), ((gg - 2) >> 1) & 1, abort_flag, p.wait_ns));
+              if (!ok) break;
               tc_fence_after();
               const uint32_t kb0 = smem_u32(sm.ring[st]), kb1 = kb0 + kHalfBytes;
-              const uint32_t scol = tmem + kColS + 64u * (2 * x + (s_next & 1));
-#pragma unroll
+              const uint32_t scol = tmem + kColS + 64u * (2 * x + (gg & 1));
+  #pragma unroll
               for (int kk = 0; kk < kD / 16; ++kk) {
                 const uint32_t off = (kk & 3) * 32;
                 tc_mma_ss(scol, sdesc_sw128((kk < 4 ? qb0 : qb1) + off, 16, 1024),
                           sdesc_sw128((kk < 4 ? kb0 : kb1) + off, 16, 1024), kIdescQK, kk > 0);
               }
-              tc_commit(smem_u32(&sm.bar_s[x][s_next & 1]));
+              tc_commit(smem_u32(&sm.bar_s[x][gg & 1]));
               // K of this slot may be replaced once both blocks' S have completed
               tc_commit(smem_u32(&sm.bar_kfree[st]));
-              // the unit's last S: Q may be replaced once it has completed
-              if (s_next == g_end - 1) tc_commit(smem_u32(&sm.bar_qfree));
-              ++s_next;
-              progressed = true;
             }
-          }
-          if (pv_next < s_next) {
-            const uint32_t gg = pv_next;
-            const int st = gg % kStages;
-            const bool first = gg == g0;
-            // P written; the previous unit's epilogue has read O_X; V landed
-            if (mbar_test_wait(smem_u32(&sm.bar_p[x][gg & 1]), (gg >> 1) & 1) &&
-                (!first || jq <= 1 || mbar_test_wait(smem_u32(&sm.bar_ofree[x]), (jq - 2) & 1)) &&
-                mbar_test_wait(smem_u32(&sm.bar_v[st]), (gg / kStages) & 1)) {
+            // the unit's last S MMAs: Q may be replaced once both blocks' have completed
+            if (ok) tc_commit(smem_u32(&sm.bar_qfree));
+          } else {
+            for (uint32_t gg = g0; ok && gg < g_end; ++gg) {
+              // PV_X(t) needs P_X(t), V(t) and, for the unit's first tile, the
+              // previous unit's O_X read out by the epilogue
+              const int st = gg % kStages;
+              const bool first = gg == g0;
+              ok = mbar_wait(smem_u32(&sm.bar_p[x][gg & 1]), (gg >> 1) & 1, abort_flag, p.wait_ns) &&
+                   (!first || jq <= 1 || mbar_wait(smem_u32(&sm.bar_ofree[x]), (jq - 2) & 1, abort_flag, p.wait_ns)) &&
+                   mbar_wait(smem_u32(&sm.bar_v[st]), (gg / kStages) & 1, abort_flag, p.wait_ns);
+              if (!ok) break;
               tc_fence_after();
               const uint32_t vb = smem_u32(sm.ring[st]) + 2 * kHalfBytes;
               const uint32_t pcol = tmem + kColS + 64u * (2 * x + (gg & 1));
-#pragma unroll
+  #pragma unroll
               for (int kk = 0; kk < kTile / 16; ++kk)
                 tc_mma_ts(ocol, pcol + 8 * kk, sdesc_sw128(vb + kk * 2048, kHalfBytes, 1024), kIdescPV,
                           (first && kk == 0) ? 0u : 1u);
-              tc_commit(smem_u32(&sm.bar_pv[x]));
+              tc_commit(smem_u32(&sm.bar_pvs[x][gg & 1]));
               tc_commit(smem_u32(&sm.bar_vfree[st]));
-              ++pv_next;
-              progressed = true;
             }
           }
-          if (progressed) {
-            spins = 0;
-          } else if ((++spins & 63u) == 0) {
-            const unsigned long long now = globaltimer_ns();
-            if (spins == 64) t_last = now;  // the first check of a stall starts its clock
-            if (*abort_flag || now - t_last > p.wait_ns) {
-              ok = false;
-              break;
-            }
-          }
+          g = g_end;
         }
-        g = g_end;
+        if (!ok) signal_abort(sm, p.err_word);
+        // every MMA issued by this thread has completed once this fires
+        const int d = (is_s ? 0 : 2) + x;
+        tc_commit(smem_u32(&sm.bar_drain[d]));
+        mbar_wait(smem_u32(&sm.bar_drain[d]), 0, nullptr);
       }
-      if (!ok) signal_abort(sm, p.err_word);
-      // every MMA issued by this thread has completed once this fires
-      tc_commit(smem_u32(&sm.bar_drain[x]));
-      mbar_wait(smem_u32(&sm.bar_drain[x]), 0, nullptr);
+      __syncwarp();
     }
-    __syncwarp();
   } else {
+    asm volatile("setmaxnreg.inc.sync.aligned.u32 200;");
     // -------------------------------------------------------------- softmax
     const int x = warp >> 2;          // row block
     const int row = tid & (kRows - 1);  // TMEM lane / query row of the block
@@ -532,14 +532,16 @@ __global__ void __launch_bounds__(kThreads, 1)
           }
           float mx;
           {
-            float r[kTile / 2];
+            // 64 -> 22 -> 8 -> 3 -> 1 with three-input maxima
+            float r[22], r2[8];
 #pragma unroll
-            for (int c = 0; c < kTile / 2; ++c) r[c] = fmaxf(xs[2 * c], xs[2 * c + 1]);
+            for (int c = 0; c < 21; ++c) r[c] = fmax3(xs[3 * c], xs[3 * c + 1], xs[3 * c + 2]);
+            r[21] = xs[63];
 #pragma unroll
-            for (int w2 = kTile / 4; w2 >= 1; w2 >>= 1)
-#pragma unroll
-              for (int c = 0; c < w2; ++c) r[c] = fmaxf(r[c], r[c + w2]);
-            mx = active ? r[0] * p.scale_log2 : -INFINITY;
+            for (int c = 0; c < 7; ++c) r2[c] = fmax3(r[3 * c], r[3 * c + 1], r[3 * c + 2]);
+            r2[7] = r[21];
+            const float m3 = fmax3(fmax3(r2[0], r2[1], r2[2]), fmax3(r2[3], r2[4], r2[5]), fmaxf(r2[6], r2[7]));
+            mx = active ? m3 * p.scale_log2 : -INFINITY;
           }
           bool need = false;
           if (active && mx != -INFINITY) {
@@ -551,7 +553,8 @@ __global__ void __launch_bounds__(kThreads, 1)
           if (__any_sync(0xffffffffu, need)) {
             // O holds the unit's earlier tiles: wait until the last PV of
             // this block has completed, then scale it
-            if (i > 0 && !mbar_wait_warp(smem_u32(&sm.bar_pv[x]), (gg - 1) & 1, abort_flag, p.wait_ns)) {
+            if (i > 0 && !mbar_wait_warp(smem_u32(&sm.bar_pvs[x][(gg - 1) & 1]), ((gg - 1) >> 1) & 1, abort_flag,
+                                         p.wait_ns)) {
               ok = false;
               break;
             }
@@ -575,19 +578,27 @@ __global__ void __launch_bounds__(kThreads, 1)
           }
           const float neg_m = (active && m_ref != -INFINITY) ? -m_ref : 0.f;
           uint32_t pk[32];
-          float ps[kTile / 2];
+          unsigned long long ps[kTile / 2];
+          {
+            const unsigned long long sc2 = f32x2(p.scale_log2, p.scale_log2), nm2 = f32x2(neg_m, neg_m);
 #pragma unroll
-          for (int c = 0; c < kTile / 2; ++c) {
-            const float p0 = fast_exp2(fmaf(xs[2 * c], p.scale_log2, neg_m));
-            const float p1 = fast_exp2(fmaf(xs[2 * c + 1], p.scale_log2, neg_m));
-            ps[c] = p0 + p1;
-            pk[c] = pack_bf16x2(p0, p1);
+            for (int c = 0; c < kTile / 2; ++c) {
+              float e0, e1;
+              f32x2_split(fma_f32x2(f32x2(xs[2 * c], xs[2 * c + 1]), sc2, nm2), e0, e1);
+              const float p0 = fast_exp2(e0), p1 = fast_exp2(e1);
+              ps[c] = f32x2(p0, p1);
+              pk[c] = pack_bf16x2(p0, p1);
+            }
           }
 #pragma unroll
           for (int w2 = kTile / 4; w2 >= 1; w2 >>= 1)
 #pragma unroll
-            for (int c = 0; c < w2; ++c) ps[c] += ps[c + w2];
-          l_sum += ps[0];
+            for (int c = 0; c < w2; ++c) ps[c] = add_f32x2(ps[c], ps[c + w2]);
+          {
+            float s0, s1;
+            f32x2_split(ps[0], s0, s1);
+            l_sum += s0 + s1;
+          }
           tmem_st32(s_tmem, pk);
           tmem_wait_st();
           if ((warp & 3) < 2 && (valid < kTile || is_new)) {
@@ -619,14 +630,17 @@ __global__ void __launch_bounds__(kThreads, 1)
         if (U == last_unit) pdl_launch_next();
         // ---- epilogue: O of the unit's last PV, scaled by 1/l.  The S of
         // the last tile implies that the PV two tiles back has completed,
-        // not the one just before: a parity wait for the last PV alone could
-        // see that earlier phase still open and pass at once, so the PVs of
-        // the last two tiles are awaited in order.
+        // not the one just before, so the PVs of the last two tiles are
+        // awaited, each on the barrier of its S buffer: neither barrier can
+        // complete a later phase before this epilogue has ended (their next
+        // PVs need P of the next unit), so no parity wait can be misread.
         const uint32_t last = g + u.tiles - 1;
         bool have_o = ok;
         if (have_o && u.tiles >= 2)
-          have_o = mbar_wait_warp(smem_u32(&sm.bar_pv[x]), (last - 1) & 1, abort_flag, p.wait_ns);
-        if (have_o) have_o = mbar_wait_warp(smem_u32(&sm.bar_pv[x]), last & 1, abort_flag, p.wait_ns);
+          have_o = mbar_wait_warp(smem_u32(&sm.bar_pvs[x][(last - 1) & 1]), ((last - 1) >> 1) & 1, abort_flag,
+                                  p.wait_ns);
+        if (have_o)
+          have_o = mbar_wait_warp(smem_u32(&sm.bar_pvs[x][last & 1]), (last >> 1) & 1, abort_flag, p.wait_ns);
         if (!have_o) ok = false;
         if (have_o) tc_fence_after();
         const bool any = have_o && active && l_sum > 0.f;
