@@ -26,10 +26,12 @@ struct CommitRope {
 
 // One thread-block cluster per sequence.  Every thread reads n_b and a_b and
 // arrives on the cluster barrier; the cluster's warps then share the
-// sequence's accepted rows (layer, accepted row, KV head), one row per warp
-// at a time (16-byte chunks, or pairs when rotating keys); after every
-// thread of the cluster has arrived, thread 0 of CTA 0 writes
-// n_b + a_b (no thread reads n_b after that).
+// sequence's accepted rows.  Without RoPE a warp copies one (layer, accepted
+// row) at a time: the KV heads of that row are adjacent in K_new/V_new, and
+// each lane keeps several 16-byte chunks in flight.  With RoPE a warp
+// rotates one (layer, accepted row, KV head) row at a time.  After every
+// thread of the cluster has arrived, thread 0 of CTA 0 writes n_b + a_b (no
+// thread reads n_b after that).
 __global__ void __launch_bounds__(kCommitWarps * 32) kv_commit_kernel(
     const uint8_t* __restrict__ k_new, const uint8_t* __restrict__ v_new, int L, const int32_t* __restrict__ tau,
     const uint8_t* __restrict__ section, const int32_t* __restrict__ accepted_len, uint8_t* __restrict__ k_cache,
@@ -50,21 +52,30 @@ __global__ void __launch_bounds__(kCommitWarps * 32) kv_commit_kernel(
   // their loads go out together with those two
   const bool lane_data = lane < gamma && section[static_cast<size_t>(b) * S + lane] == kSectData;
   const int lane_tau = lane < gamma ? tau[static_cast<size_t>(b) * S + lane] : 0;
-  // the sequence's first 32 page ids (lane p: page p), likewise: a row that
-  // lands there takes its page id by a shuffle instead of a dependent load.
-  // With no layer there is no row to place, and the caller may pass no
-  // block table at all.
-  const int lane_pg = (L > 0 && lane < max_pages) ? block_table[static_cast<size_t>(b) * max_pages + lane] : -1;
+  const int32_t* bt = block_table + static_cast<size_t>(b) * max_pages;
+  // page ids of a 32-page window (lane i: page win + i) that holds every
+  // destination row n_b .. n_b + a_b - 1 (a_b <= 32): the first 32 pages,
+  // loaded beside n_b and a_b, or, when the rows lie beyond them, the 32
+  // pages from the first destination page.  With no layer there is no row
+  // to place, and the caller may pass no block table at all.
+  int win = 0;
+  int lane_pg = (L > 0 && lane < max_pages) ? bt[lane] : -1;
   // "n_b has been read"
   asm volatile("barrier.cluster.arrive.release;" ::: "memory");
   const bool ok = a >= 0 && a <= gamma && n >= 0;
-  if (ok) {
-    const long long rows = static_cast<long long>(a) * L * Hkv;
-    for (long long row = static_cast<long long>(rank) * kCommitWarps + warp; row < rows;
-         row += static_cast<long long>(CL) * kCommitWarps) {
-      const int kvh = static_cast<int>(row % Hkv);
-      const int r = static_cast<int>((row / Hkv) % a);
-      const int l = static_cast<int>(row / (static_cast<long long>(Hkv) * a));
+  if (ok && a > 0 && L > 0) {
+    const int last_page = (n + a - 1) / page_size;
+    if (last_page >= 32) {
+      win = n / page_size;
+      lane_pg = win + lane < max_pages ? bt[win + lane] : -1;
+    }
+    const size_t Bt = gridDim.x / CL;
+    const int chunks = row_bytes >> 4;  // 16-byte chunks of one KV head's row
+    const int rows = rope.pos ? a * L * Hkv : a * L;
+    for (int row = rank * kCommitWarps + warp; row < rows; row += CL * kCommitWarps) {
+      const int kvh = rope.pos ? row % Hkv : 0;
+      const int q = rope.pos ? row / Hkv : row;  // (layer, accepted row)
+      const int r = q % a, l = q / a;
       // source: the data slot whose label is r+1
       const bool hit = lane_data && lane_tau == r + 1;
       const unsigned m = __ballot_sync(0xffffffffu, hit);
@@ -73,27 +84,26 @@ __global__ void __launch_bounds__(kCommitWarps * 32) kv_commit_kernel(
         continue;
       }
       const int src = __ffs(m) - 1;
-      const long long dst_row = static_cast<long long>(n) + r;
-      const long long pidx = dst_row / page_size;
+      const int dst_row = n + r;
+      const int pidx = dst_row / page_size;
       if (pidx >= max_pages) {
         if (lane == 0) raise_error(err_word, SIMSD_EW_PAGE);
         continue;
       }
-      const int pg = pidx < 32 ? __shfl_sync(0xffffffffu, lane_pg, static_cast<int>(pidx))
-                               : block_table[static_cast<size_t>(b) * max_pages + pidx];
+      const int pg = __shfl_sync(0xffffffffu, lane_pg, pidx - win);
       if (pg < 0 || pg >= num_pages) {
         if (lane == 0) raise_error(err_word, SIMSD_EW_PAGE);
         continue;
       }
-      const int off = static_cast<int>(dst_row % page_size);
-      const size_t Bt = gridDim.x / CL;
+      const int off = dst_row - pidx * page_size;
+      // row indices (in rows of row_bytes): K_new/V_new [L][Bt][S][Hkv],
+      // the pools [L][num_pages][Hkv][page_size]
       const size_t s_row = ((static_cast<size_t>(l) * Bt + b) * S + src) * Hkv + kvh;
       const size_t d_row = ((static_cast<size_t>(l) * num_pages + pg) * Hkv + kvh) * page_size + off;
       const uint4* ks = reinterpret_cast<const uint4*>(k_new + s_row * row_bytes);
       const uint4* vs = reinterpret_cast<const uint4*>(v_new + s_row * row_bytes);
       uint4* kd = reinterpret_cast<uint4*>(k_cache + d_row * row_bytes);
       uint4* vd = reinterpret_cast<uint4*>(v_cache + d_row * row_bytes);
-      const int chunks = row_bytes >> 4;
       if (rope.pos) {
         const int pos = rope.pos[static_cast<size_t>(b) * S + src];
         const int d = row_bytes / elem_bytes, half = d / 2;
@@ -118,9 +128,30 @@ __global__ void __launch_bounds__(kCommitWarps * 32) kv_commit_kernel(
         }
         for (int c = lane; c < chunks; c += 32) vd[c] = vs[c];
       } else {
-        for (int c = lane; c < chunks; c += 32) {
-          kd[c] = ks[c];
-          vd[c] = vs[c];
+        // every KV head of the row: chunk c of the Hkv * chunks source
+        // chunks (contiguous) lands in head c / chunks, page_size rows apart
+        const int total = Hkv * chunks;
+        const size_t head_step = static_cast<size_t>(page_size) * chunks;
+        for (int c0 = 0; c0 < total; c0 += 128) {
+          uint4 kx[4], vx[4];
+#pragma unroll
+          for (int j = 0; j < 4; ++j) {
+            const int c = c0 + 32 * j + lane;
+            if (c < total) {
+              kx[j] = ks[c];
+              vx[j] = vs[c];
+            }
+          }
+#pragma unroll
+          for (int j = 0; j < 4; ++j) {
+            const int c = c0 + 32 * j + lane;
+            if (c < total) {
+              const int h = c / chunks;
+              const size_t dc = h * head_step + (c - h * chunks);
+              kd[dc] = kx[j];
+              vd[dc] = vx[j];
+            }
+          }
         }
       }
     }

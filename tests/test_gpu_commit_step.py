@@ -40,6 +40,57 @@ def test_commit_bit_exact(dtype, L, gamma, P):
     np.testing.assert_array_equal(inputs.host_bits(si.v_cache), rv)
 
 
+@pytest.mark.parametrize("dtype,Hkv,d,gamma,P", [("bf16", 8, 128, 16, 8), ("f32", 8, 128, 8, 16),
+                                                 ("bf16", 2, 64, 32, 1)])
+def test_commit_rows_beyond_the_first_32_pages(dtype, Hkv, d, gamma, P):
+    # destination rows past a sequence's first 32 pages (their page ids come
+    # from a window that starts at the first destination page), rows that
+    # straddle a page boundary, one-row pages (32 accepted rows on 32
+    # pages), and rows of 8 heads x 128 fp32 (256 chunks of 16 bytes)
+    n = [32 * P - 1, 32 * P, 41 * P - 2, 500, 7, 33 * P + 1]
+    w = inputs.Workload("c", dtype, len(n), 2 * Hkv, Hkv, d, gamma, (0, 0), 2, 16, 0.5, 1.0, 1.0, gamma + P, P)
+    si = inputs.make_step_inputs(w, device="cuda", prefix_override=n, random_step_map=True, with_logits=False)
+    rng = np.random.default_rng(P)
+    a = rng.integers(1, gamma + 1, len(n)).astype(np.int32)
+    a[2] = gamma
+    a = torch.as_tensor(a, device="cuda")
+    tau, sect, _, _, err = gpu_mask(si, mask_bits=False)
+    kc0, vc0 = si.k_cache.clone(), si.v_cache.clone()
+    nn = si.prefix_len.clone()
+    simsd.simsd_kv_commit(si.k_new, si.v_new, tau, sect, a, si.k_cache, si.v_cache, si.block_table, nn, err)
+    word = simsd.simsd_check_error(err)
+    rk, rv, rn, rerr = orc.kv_commit(inputs.host_bits(si.k_new), inputs.host_bits(si.v_new),
+                                     si.step_map.cpu().numpy(), a.cpu().numpy(), inputs.host_bits(kc0),
+                                     inputs.host_bits(vc0), si.block_table.cpu().numpy(),
+                                     si.prefix_len.cpu().numpy(), gamma)
+    assert word == rerr == 0
+    np.testing.assert_array_equal(nn.cpu().numpy(), rn)
+    np.testing.assert_array_equal(inputs.host_bits(si.k_cache), rk)
+    np.testing.assert_array_equal(inputs.host_bits(si.v_cache), rv)
+
+
+def test_commit_bad_page_past_the_first_32():
+    P = 8
+    si = _commit_case("bf16", 2, 8, P, [300, 40 * P + 5, 9], seed=3)
+    bt = si.block_table.clone()
+    bt[1, (40 * P + 5) // P + 1] = -3               # a destination page id below zero
+    si.block_table = bt
+    a = torch.tensor([4, 8, 2], dtype=torch.int32, device="cuda")
+    tau, sect, _, _, err = gpu_mask(si, mask_bits=False)
+    kc0, vc0 = si.k_cache.clone(), si.v_cache.clone()
+    nn = si.prefix_len.clone()
+    simsd.simsd_kv_commit(si.k_new, si.v_new, tau, sect, a, si.k_cache, si.v_cache, si.block_table, nn, err)
+    word = simsd.simsd_check_error(err)
+    rk, rv, rn, rerr = orc.kv_commit(inputs.host_bits(si.k_new), inputs.host_bits(si.v_new),
+                                     si.step_map.cpu().numpy(), a.cpu().numpy(), inputs.host_bits(kc0),
+                                     inputs.host_bits(vc0), si.block_table.cpu().numpy(),
+                                     si.prefix_len.cpu().numpy(), 8)
+    assert word == rerr == simsd.EW_PAGE
+    np.testing.assert_array_equal(nn.cpu().numpy(), rn)
+    np.testing.assert_array_equal(inputs.host_bits(si.k_cache), rk)
+    np.testing.assert_array_equal(inputs.host_bits(si.v_cache), rv)
+
+
 @pytest.mark.parametrize("gamma", [4, 16])
 def test_commit_with_undrafted_and_decoded_positions(gamma):
     # only drafted data slots are ever committed: a decoded slot (tau 0) and
