@@ -857,7 +857,6 @@ __global__ void __maxnreg__(kMaxRegs)
 // lanes over the head dimension (independent loads, several in flight).
 __global__ void __launch_bounds__(128) combine_kernel(const __grid_constant__ TcParams p) {
   pdl_wait();
-  pdl_launch_next();
   const int lane = threadIdx.x & 31;
   const unsigned full = 0xffffffffu;
   const long long wid = (static_cast<long long>(blockIdx.x) * blockDim.x + threadIdx.x) >> 5;
@@ -915,6 +914,10 @@ __global__ void __launch_bounds__(128) combine_kernel(const __grid_constant__ Tc
   v.x = pack_bf16x2(acc.x * inv, acc.y * inv);
   v.y = pack_bf16x2(acc.z * inv, acc.w * inv);
   reinterpret_cast<uint2*>(orow)[lane] = v;
+  // the next kernel is let in only as this grid's blocks finish: launched
+  // at the start, its CTAs took SMs that thousands of these small blocks
+  // still needed
+  pdl_launch_next();
 }
 
 cudaError_t ensure_smem_attr() {
@@ -962,15 +965,18 @@ bool plan_attention_tc(int Bt, int gamma, int Hq, int Hkv, int max_pages, int pa
   pl.rows_blk = g * pl.s_blk;
   if (pl.rows_blk > kRows || g > 256 || pl.s_blk > 256) return false;
   pl.num_sms = num_sms;
-  if (tc256_applies(Bt, Hkv, pl.rb, num_sms)) {
-    // two row blocks share one CTA and its K/V stream; enough units to
-    // give every SM one, so no split
+  const long long max_tiles = (static_cast<long long>(max_pages) * page_size + kTile - 1) / kTile + 1;
+  if (const int ns256 = tc256_splits(Bt, Hkv, pl.rb, max_tiles, num_sms)) {
+    // two row blocks share one CTA and its K/V stream; with fewer units
+    // than SMs each unit's key tiles are split into ranges whose partials
+    // the combine kernel merges
     pl.kind = 1;
-    pl.nsplit = 1;
+    pl.nsplit = ns256;
     pl.sort = 0;
     pl.fuse = 0;
     pl.slots = num_sms;
-    pl.ws_bytes = 0;
+    pl.ws_bytes = ns256 > 1 ? static_cast<size_t>(Bt) * Hkv * pl.rb * ns256 * pl.rows_blk * (kD + 2) * sizeof(float)
+                            : 0;
     *plan = pl;
     return true;
   }
@@ -979,7 +985,6 @@ bool plan_attention_tc(int Bt, int gamma, int Hq, int Hkv, int max_pages, int pa
   // are resident, so the budget the kernel is built for is used instead)
   const long long units = static_cast<long long>(Bt) * Hkv * pl.rb;
   const long long slots = static_cast<long long>(num_sms) * kCtasPerSm;
-  const long long max_tiles = (static_cast<long long>(max_pages) * page_size + kTile - 1) / kTile + 1;
   int ns = 1;
   if (units < slots) {
     // as many splits as keep every CTA in one wave
@@ -998,9 +1003,27 @@ bool plan_attention_tc(int Bt, int gamma, int Hq, int Hkv, int max_pages, int pa
   return true;
 }
 
+cudaError_t launch_attention_combine(const AttnTcArgs& a, const AttnTcPlan& pl, cudaStream_t stream) {
+  TcParams p{};
+  p.out = static_cast<__nv_bfloat16*>(a.out);
+  p.ws = static_cast<float*>(a.workspace);
+  p.Bt = a.Bt;
+  p.gamma = a.gamma;
+  p.S = 2 * a.gamma;
+  p.Hq = a.Hq;
+  p.Hkv = a.Hkv;
+  p.g = a.Hq / a.Hkv;
+  p.rb = pl.rb;
+  p.rows_blk = pl.rows_blk;
+  p.s_blk = pl.s_blk;
+  p.nsplit = pl.nsplit;
+  const long long warps = static_cast<long long>(a.Bt) * a.Hkv * pl.rb * pl.rows_blk;
+  return launch_overlapped(combine_kernel, dim3(static_cast<unsigned>((warps + 3) / 4)), dim3(128), 0, stream, 1, p);
+}
+
 cudaError_t launch_attention_tc(const AttnTcArgs& a, const AttnTcPlan& pl, EncodeTiledFn encode,
                                 cudaStream_t stream) {
-  if (pl.kind == 1) return launch_attention_tc256(a, pl.s_blk, encode, pl.num_sms, stream);
+  if (pl.kind == 1) return launch_attention_tc256(a, pl, encode, stream);
   const int S = 2 * a.gamma, g = a.Hq / a.Hkv;
   CUtensorMap tq, tkn, tvn, tkc, tvc;
   {

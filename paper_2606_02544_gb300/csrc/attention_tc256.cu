@@ -84,8 +84,11 @@ struct Tc256Params {
   int32_t* err_word;
   int max_pages, page_size, num_pages;
   int Bt, S, Hq, Hkv, g, s_blk;
-  int units;  // Bt * Hkv
-  int sort;   // rank sequences by prefix length (Bt <= kMaxSort)
+  int units;   // Bt * Hkv
+  int nsplit;  // key-tile ranges per unit (work items = units * nsplit)
+  int items;
+  float* ws;   // nsplit > 1: partial O, (m, l) of each row block and range (the combine's layout)
+  int sort;    // rank sequences by prefix length (Bt <= kMaxSort)
   float scale_log2;
   unsigned long long wait_ns;
   uint32_t extra_p;  // planted extra arrivals on bar_p (a test of the bounded waits)
@@ -144,23 +147,45 @@ __device__ __forceinline__ void rope_chunk_pair(uint4* pa, uint4* pb, int pos, i
   *pb = make_uint4(wb[0], wb[1], wb[2], wb[3]);
 }
 
-// The unit at position U of the walk: sequence (longest prefix first when
-// ranked), KV head, prefix length and number of key tiles (0 when the
-// prefix length is out of range: the unit then only writes zeros).
+// The work item at position U of the walk: key-tile range `split` of the
+// unit (sequence b, KV head), sequences longest prefix first when ranked.
+// A unit has T = ceil(n / 64) + 1 tiles (tile 0: the new slots, 1..: the
+// prefix; none when the prefix length is out of range); range i holds tiles
+// [ceil(i T / nsplit), ceil((i + 1) T / nsplit)), so range 0 holds tile 0.
 struct Unit {
-  int b, kvh, n, tiles;
+  int b, kvh, n, split, t0, tiles;
   bool n_bad;
 };
 
 __device__ __forceinline__ Unit unit_at(const Tc256Params& p, const Smem256& sm, int U) {
   Unit u;
-  const int rank = U / p.Hkv;
-  u.kvh = U - rank * p.Hkv;
+  const int unit = U / p.nsplit;
+  u.split = U - unit * p.nsplit;
+  const int rank = unit / p.Hkv;
+  u.kvh = unit - rank * p.Hkv;
   u.b = p.sort ? sm.order[rank] : rank;
   u.n = p.prefix_len[u.b];
   u.n_bad = u.n < 0 || static_cast<long long>(u.n) > static_cast<long long>(p.max_pages) * p.page_size;
-  u.tiles = u.n_bad ? 0 : (u.n + kTile - 1) / kTile + 1;  // tile 0: the new slots, 1..: the prefix
+  // T < 2^25 and split < 64: the products fit 32 bits
+  const unsigned T = u.n_bad ? 0u : static_cast<unsigned>((u.n + kTile - 1) / kTile + 1);
+  const unsigned ns = static_cast<unsigned>(p.nsplit), sp = static_cast<unsigned>(u.split);
+  u.t0 = static_cast<int>((sp * T + ns - 1) / ns);
+  u.tiles = static_cast<int>(((sp + 1) * T + ns - 1) / ns) - u.t0;
   return u;
+}
+
+// Partial results of a split unit, in the layout the combine kernel reads:
+// O (unnormalised, fp32) [units * 2 * nsplit][128][d], then (m, l)
+// [units * 2 * nsplit][128][2]; entry ((b Hkv + kvh) 2 + x) nsplit + split,
+// row `row` of block x.  m is the row's reference maximum in log2 units.
+__device__ __forceinline__ float* partial_o(const Tc256Params& p, const Unit& u, int x, int row) {
+  const size_t e = ((static_cast<size_t>(u.b) * p.Hkv + u.kvh) * 2 + x) * p.nsplit + u.split;
+  return p.ws + (e * kRows + row) * kD;
+}
+__device__ __forceinline__ float* partial_ml(const Tc256Params& p, const Unit& u, int x, int row) {
+  const size_t e = ((static_cast<size_t>(u.b) * p.Hkv + u.kvh) * 2 + x) * p.nsplit + u.split;
+  const size_t entries = static_cast<size_t>(p.units) * 2 * p.nsplit;
+  return p.ws + entries * kRows * kD + (e * kRows + row) * 2;
 }
 
 __global__ void __launch_bounds__(kThreads, 1)
@@ -233,7 +258,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   const int first_unit = blockIdx.x, step = gridDim.x;
 
   // the last unit this CTA takes (for the dependent-launch trigger)
-  const int last_unit = first_unit + ((p.units - 1 - first_unit) / step) * step;
+  const int last_unit = first_unit + ((p.items - 1 - first_unit) / step) * step;
 
   // Register split (setmaxnreg, per warpgroup): the two softmax warpgroups
   // take 200 registers a thread, the two control warpgroups give theirs
@@ -249,7 +274,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       const int kv = warp == kWarpProducer ? 0 : 1;
       uint32_t g = 0, jq = 0;  // tiles and units (with tiles) issued so far
       bool ok = true;
-      for (int U = first_unit; ok && U < p.units; U += step) {
+      for (int U = first_unit; ok && U < p.items; U += step) {
         const Unit u = unit_at(p, sm, U);
         if (u.tiles == 0) continue;
         if (kv == 0) {
@@ -271,7 +296,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         const int32_t* bt = p.block_table + static_cast<size_t>(u.b) * p.max_pages;
         const int P = p.page_size;
         int win_base = -(1 << 30), win = -1;  // lane i holds the page id of page win_base + i
-        for (int t = 0; t < u.tiles; ++t) {
+        for (int t = u.t0; t < u.t0 + u.tiles; ++t) {
           const int st = g % kStages;
           // page ids this tile needs (prefix tiles), loaded by the whole warp
           int pi0 = 0, nsub = 0, key0 = 0, valid = 0;
@@ -363,7 +388,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         const uint32_t ocol = tmem + kColO + 128u * x;
         uint32_t g = 0, jq = 0;
         bool ok = true;
-        for (int U = first_unit; ok && U < p.units; U += step) {
+        for (int U = first_unit; ok && U < p.items; U += step) {
           const Unit u = unit_at(p, sm, U);
           if (u.tiles == 0) continue;
           ++jq;
@@ -434,7 +459,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     const uint32_t o_tmem = lane_tmem + kColO + 128u * x;
     uint32_t g = 0, jq = 0, mu = 0;
     bool ok = true;
-    for (int U = first_unit; U < p.units; U += step, ++mu) {
+    for (int U = first_unit; U < p.items; U += step, ++mu) {
       const Unit u = unit_at(p, sm, U);
       const int par = mu & 1;  // metadata buffer of this unit
       // every softmax thread is done with the previous unit: its flag
@@ -446,7 +471,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         sm.sect[par][tid] = p.section[static_cast<size_t>(u.b) * p.S + tid];
       }
       if (u.n_bad) {
-        if (tid == 0 && u.kvh == 0) raise_error(p.err_word, SIMSD_EW_PREFIX_LEN);
+        if (tid == 0 && u.kvh == 0 && u.split == 0) raise_error(p.err_word, SIMSD_EW_PREFIX_LEN);
       } else {
         const int npages = (u.n + p.page_size - 1) / p.page_size;
         const int32_t* bt = p.block_table + static_cast<size_t>(u.b) * p.max_pages;
@@ -457,7 +482,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
         if (bad) {
           atomicOr(&sm.bad[par], 1);
-          if (u.kvh == 0) raise_error(p.err_word, SIMSD_EW_PAGE);
+          if (u.kvh == 0 && u.split == 0) raise_error(p.err_word, SIMSD_EW_PAGE);
         }
       }
       asm volatile("bar.sync 1, 256;" ::: "memory");
@@ -476,8 +501,8 @@ __global__ void __launch_bounds__(kThreads, 1)
       if (u.tiles > 0) {
         ++jq;
         if (p.rope_pos) {
-          // Q of both blocks and the new keys (the unit's first tile) are
-          // rotated in shared memory before the first S reads them
+          // Q of both blocks and, in range 0, the new keys (its first tile)
+          // are rotated in shared memory before the first S reads them
           const int pos = p.rope_pos[static_cast<size_t>(u.b) * p.S + (row_exists ? s : 0)];
           if (ok) ok = mbar_wait_warp(smem_u32(&sm.bar_q), (jq - 1) & 1, abort_flag, p.wait_ns);
           if (ok) {
@@ -487,8 +512,8 @@ __global__ void __launch_bounds__(kThreads, 1)
             for (int c = 0; c < 8; ++c) rope_chunk_pair(sw128_chunk(h0, row, c), sw128_chunk(h1, row, c), pos, c, p.rope);
           }
           const int st0 = g % kStages;
-          if (ok) ok = mbar_wait_warp(smem_u32(&sm.bar_k[st0]), (g / kStages) & 1, abort_flag, p.wait_ns);
-          if (ok) {
+          if (ok && u.t0 == 0) ok = mbar_wait_warp(smem_u32(&sm.bar_k[st0]), (g / kStages) & 1, abort_flag, p.wait_ns);
+          if (ok && u.t0 == 0) {
             uint8_t* h0 = sm.ring[st0];
             uint8_t* h1 = sm.ring[st0] + kHalfBytes;
             for (int task = tid; task < p.S * 8; task += kSoftmaxThreads) {
@@ -515,8 +540,9 @@ __global__ void __launch_bounds__(kThreads, 1)
           tmem_ld32(s_tmem, sa);
           tmem_ld32(s_tmem + 32, sb);
           tmem_wait_ld();
-          const bool is_new = (i == 0);
-          const int valid = is_new ? p.S : min(kTile, u.n - (i - 1) * kTile);
+          const int t = u.t0 + i;  // tile of the unit
+          const bool is_new = (t == 0);
+          const int valid = is_new ? p.S : min(kTile, u.n - (t - 1) * kTile);
           float xs[kTile];
 #pragma unroll
           for (int c = 0; c < kTile; ++c) xs[c] = __uint_as_float(c < 32 ? sa[c] : sb[c - 32]);
@@ -647,6 +673,9 @@ __global__ void __launch_bounds__(kThreads, 1)
         const float inv = any ? 1.0f / l_sum : 0.f;
         const int h = u.kvh * p.g + hl;
         __nv_bfloat16* orow = p.out + ((static_cast<size_t>(u.b) * p.S + (row_exists ? s : 0)) * p.Hq + h) * kD;
+        // a split unit leaves its partial O (fp32) and (m, l) to the combine
+        const bool part = p.nsplit > 1;
+        float* wo = part ? partial_o(p, u, x, row) : nullptr;
 #pragma unroll 1
         for (int ch = 0; ch < kD / 32; ++ch) {
           uint32_t o[32];
@@ -654,7 +683,14 @@ __global__ void __launch_bounds__(kThreads, 1)
             tmem_ld32(o_tmem + 32 * ch, o);
             tmem_wait_ld();
           }
-          if (row_exists) {
+          if (row_exists && part) {
+            float4* dst = reinterpret_cast<float4*>(wo + 32 * ch);
+#pragma unroll
+            for (int c = 0; c < 8; ++c)
+              dst[c] = any ? make_float4(__uint_as_float(o[4 * c]), __uint_as_float(o[4 * c + 1]),
+                                         __uint_as_float(o[4 * c + 2]), __uint_as_float(o[4 * c + 3]))
+                           : make_float4(0.f, 0.f, 0.f, 0.f);
+          } else if (row_exists) {
             uint4 pkd[4];
             uint32_t* wv = reinterpret_cast<uint32_t*>(pkd);
 #pragma unroll
@@ -668,11 +704,28 @@ __global__ void __launch_bounds__(kThreads, 1)
             for (int c = 0; c < 4; ++c) dst[c] = pkd[c];
           }
         }
+        if (row_exists && part) {
+          float* wml = partial_ml(p, u, x, row);
+          wml[0] = any ? m_ref : -INFINITY;
+          wml[1] = any ? l_sum : 0.f;
+        }
         // O_X may be overwritten by the next unit's first PV
         tc_fence_before();
         __syncwarp();
         if (lane == 0) mbar_arrive(smem_u32(&sm.bar_ofree[x]));
         g += u.tiles;
+      } else if (p.nsplit > 1) {
+        // an empty tile range (or a prefix length out of range): an empty
+        // partial, which the combine skips
+        if (U == last_unit) pdl_launch_next();
+        if (row_exists) {
+          float4* dst = reinterpret_cast<float4*>(partial_o(p, u, x, row));
+#pragma unroll 4
+          for (int c = 0; c < kD / 4; ++c) dst[c] = make_float4(0.f, 0.f, 0.f, 0.f);
+          float* wml = partial_ml(p, u, x, row);
+          wml[0] = -INFINITY;
+          wml[1] = 0.f;
+        }
       } else {
         // a prefix length out of range: this unit's rows are zero
         if (U == last_unit) pdl_launch_next();
@@ -697,13 +750,36 @@ __global__ void __launch_bounds__(kThreads, 1)
 
 }  // namespace
 
-bool tc256_applies(int Bt, int Hkv, int rb, int num_sms) {
-  return rb == 2 && static_cast<long long>(Bt) * Hkv >= num_sms;
+int tc256_splits(int Bt, int Hkv, int rb, long long max_tiles, int num_sms) {
+  if (rb != 2) return 0;
+  const long long units = static_cast<long long>(Bt) * Hkv;
+  if (units >= num_sms) return 1;
+  // short units (under 16 key tiles) that would need splitting stay with
+  // the one-row-block kernel, whose splits merge in a cluster (at 512 keys
+  // it was ~3.5% faster per step)
+  if (max_tiles < 16) return 0;
+  // Fewer units than SMs: split each unit's key tiles into ns ranges (at
+  // least two tiles each).  A CTA walks ceil(units ns / SMs) items, each
+  // costing its tiles plus a fixed ~14 tiles (Q, the pipeline refill, the
+  // partial write); ns minimises that product (measured at 8 sequences x 8
+  // KV heads: ~0.9 us per tile, ~13 us per item).
+  const long long kItemCost = 14;
+  const long long ns_max = std::min<long long>(64, std::max<long long>(1, max_tiles / 2));
+  long long best = 1, best_cost = -1;
+  for (long long ns = 1; ns <= ns_max; ++ns) {
+    const long long per_cta = (units * ns + num_sms - 1) / num_sms;
+    const long long cost = per_cta * ((max_tiles + ns - 1) / ns + kItemCost);
+    if (best_cost < 0 || cost < best_cost) {
+      best = ns;
+      best_cost = cost;
+    }
+  }
+  return static_cast<int>(best);
 }
 
-cudaError_t launch_attention_tc256(const AttnTcArgs& a, int s_blk, EncodeTiledFn encode, int num_sms,
+cudaError_t launch_attention_tc256(const AttnTcArgs& a, const AttnTcPlan& pl, EncodeTiledFn encode,
                                    cudaStream_t stream) {
-  const int S = 2 * a.gamma, g = a.Hq / a.Hkv;
+  const int S = 2 * a.gamma, g = a.Hq / a.Hkv, s_blk = pl.s_blk;
   CUtensorMap tq, tkn, tvn, tkc, tvc;
   {
     const cuuint64_t dims[3] = {static_cast<cuuint64_t>(kD), static_cast<cuuint64_t>(a.Hq),
@@ -747,6 +823,9 @@ cudaError_t launch_attention_tc256(const AttnTcArgs& a, int s_blk, EncodeTiledFn
   p.g = g;
   p.s_blk = s_blk;
   p.units = a.Bt * a.Hkv;
+  p.nsplit = pl.nsplit;
+  p.items = p.units * pl.nsplit;
+  p.ws = static_cast<float*>(a.workspace);
   p.sort = a.Bt <= kMaxSort ? 1 : 0;
   p.scale_log2 = a.scale * 1.4426950408889634f;
   p.wait_ns = a.fault.wait_ns ? a.fault.wait_ns : kWaitLimitNs;
@@ -758,9 +837,11 @@ cudaError_t launch_attention_tc256(const AttnTcArgs& a, int s_blk, EncodeTiledFn
     if (e != cudaSuccess) return e;
     attr_done = true;
   }
-  const int grid = std::min(p.units, num_sms);
-  return launch_overlapped(attention_tc256_kernel, dim3(static_cast<unsigned>(grid)), dim3(kThreads), smem_bytes(),
-                           stream, 1u, tq, tkn, tvn, tkc, tvc, p);
+  const int grid = std::min(p.items, pl.num_sms);
+  cudaError_t e = launch_overlapped(attention_tc256_kernel, dim3(static_cast<unsigned>(grid)), dim3(kThreads),
+                                    smem_bytes(), stream, 1u, tq, tkn, tvn, tkc, tvc, p);
+  if (e != cudaSuccess || pl.nsplit == 1) return e;
+  return launch_attention_combine(a, pl, stream);
 }
 
 }  // namespace simsd

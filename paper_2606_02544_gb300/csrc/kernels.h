@@ -99,11 +99,15 @@ cudaError_t launch_attention_tc(const AttnTcArgs& a, const AttnTcPlan& plan, Enc
 bool make_bf16_map(EncodeTiledFn encode, CUtensorMap* m, const void* base, int rank, const cuuint64_t* dims,
                    const cuuint64_t* strides, const cuuint32_t* box);
 
-// 256-row units (two row blocks per KV head) on one persistent CTA per SM,
-// used when there are at least as many units as SMs.
-bool tc256_applies(int Bt, int Hkv, int rb, int num_sms);
-cudaError_t launch_attention_tc256(const AttnTcArgs& a, int s_blk, EncodeTiledFn encode, int num_sms,
+// 256-row units (two row blocks per KV head) on one persistent CTA per SM.
+// tc256_splits: 0 if the kernel does not take the shape (not two row
+// blocks, or fewer units than SMs with under 16 key tiles each), else the
+// key-tile ranges per unit (1 when there are at least as many units as SMs).
+int tc256_splits(int Bt, int Hkv, int rb, long long max_tiles, int num_sms);
+cudaError_t launch_attention_tc256(const AttnTcArgs& a, const AttnTcPlan& pl, EncodeTiledFn encode,
                                    cudaStream_t stream);
+// Merge of split partials (workspace layout of the plan) into the output.
+cudaError_t launch_attention_combine(const AttnTcArgs& a, const AttnTcPlan& pl, cudaStream_t stream);
 
 // Static device scratch of simsd_verify_attention_noalloc.
 size_t noalloc_scratch_capacity();

@@ -4,12 +4,13 @@ tests/_gpu.py.
 
 The kernel serves units of 129..256 query rows per KV head (32 drafts with
 32/8 heads, 16 drafts with 64/8 heads, 20 drafts with 32/8 heads, where the
-second block is partly empty) when the batch has at least one unit per SM;
-smaller batches keep the one-block-per-CTA kernel.  Cases: ragged prefixes
-across tile and page edges, every page size, random step maps, padding,
-undrafted and decoded positions, RoPE applied in the kernel (both position
-rules), NaN-poisoned unused cache rows, more sequences than the ranking
-handles, and the error paths.
+second block is partly empty).  With fewer units than SMs each unit's key
+tiles are split into ranges whose partials the combine kernel merges.
+Cases: ragged prefixes across tile and page edges, every page size, random
+step maps, padding, undrafted and decoded positions, RoPE applied in the
+kernel (both position rules), NaN-poisoned unused cache rows, more
+sequences than the ranking handles, split units (small batches, ranges with
+no tile, the new-slot tile in range 0 only), and the error paths.
 """
 import numpy as np
 import pytest
@@ -27,11 +28,26 @@ def _w(Bt, gamma=32, Hq=32, Hkv=8, P=64, prefix=(0, 700), seed=0, std=None):
 
 
 def _uses_tc256(si):
-    # at least one unit (sequence, KV head) per SM and two row blocks
+    # two row blocks of 128 rows per KV head
+    w = si.w
+    rows = w.g * w.S
+    return 128 < rows <= 256 and 128 % w.g == 0
+
+
+def _splits(si):
+    # key-tile ranges per unit: one with at least one unit per SM, else the
+    # count (at least two tiles a range) that minimises the items a CTA
+    # walks times their tiles plus a fixed 14
     w = si.w
     sms = torch.cuda.get_device_properties(0).multi_processor_count
-    rows = w.g * w.S
-    return 128 < rows <= 256 and 128 % w.g == 0 and w.Bt * w.Hkv >= sms
+    units = w.Bt * w.Hkv
+    if units >= sms:
+        return 1
+    max_tiles = (si.block_table.shape[1] * w.page_size + 63) // 64 + 1
+    if max_tiles < 16:
+        return 0  # the one-row-block kernel takes short units
+    cost = {ns: -(-units * ns // sms) * (-(-max_tiles // ns) + 14) for ns in range(1, min(64, max(1, max_tiles // 2)) + 1)}
+    return min(cost, key=lambda ns: (cost[ns], ns))
 
 
 def _check(si, seqs=None, rope=None):
@@ -48,7 +64,11 @@ def _check(si, seqs=None, rope=None):
             pos = (n + torch.arange(si.w.S, device=n.device)[None]).to(torch.int32).contiguous()
         out, word, ws = gpu_attention(si, mask=(tau, sect), rope_pos=pos, rope_theta=theta)
         ref = oracle_attention(si, seqs=seqs, rope_theta=theta, rope_mode=mode)
-    assert ws == 0 and word == ref.err
+    # a workspace when the units are split, none when the kernel takes
+    # them whole
+    ns = _splits(si)
+    assert (ns > 1 and ws > 0) or (ns == 1 and ws == 0) or ns == 0
+    assert word == ref.err
     got = out if seqs is None else out[torch.as_tensor(seqs, device=out.device)]
     assert_attention_close(got, ref)
     return out, word
@@ -120,6 +140,61 @@ def test_error_paths():
     out, word = _check(si, seqs=[0, 1, 2, 3, 4])
     assert word & simsd.EW_PREFIX_LEN and word & simsd.EW_PAGE and word & simsd.EW_STEP_MAP
     assert (out[1:4].float() == 0).all() and (out[0, [2, 34]].float() == 0).all()
+
+
+@pytest.mark.parametrize("Bt,prefix,P,split", [(1, (0, 0), 64, 0), (1, (3000, 3000), 64, 2),
+                                               (3, (1200, 1500), 16, 2), (8, (1500, 2000), 64, 2),
+                                               (8, (0, 40), 32, 0), (12, (2000, 6000), 64, 2),
+                                               (18, (500, 1500), 128, 1), (2, (1000, 1100), 8, 2)])
+def test_split_units(Bt, prefix, P, split):
+    # fewer units than SMs: ranges of key tiles per unit, merged by the
+    # combine kernel (ranges of short sequences can hold no tile); nearly
+    # one unit per SM stays whole (1), short units go to the one-row-block
+    # kernel (0)
+    si = inputs.make_step_inputs(_w(Bt, prefix=prefix, P=P, seed=Bt + P), device="cuda", random_step_map=True,
+                                 poison_unused_rows=True)
+    assert min(_splits(si), 2) == split
+    _check(si, seqs=sorted({0, Bt // 2, Bt - 1}))
+
+
+@pytest.mark.parametrize("gamma,Hq", [(16, 64), (20, 32)])
+def test_split_units_row_layouts(gamma, Hq):
+    si = inputs.make_step_inputs(_w(4, gamma=gamma, Hq=Hq, prefix=(1000, 1200), seed=gamma), device="cuda",
+                                 random_step_map=True, poison_unused_rows=True)
+    assert _splits(si) > 1
+    _check(si, seqs=[0, 3])
+
+
+@pytest.mark.parametrize("mode", [1, 2])
+def test_split_units_rope(mode):
+    si = inputs.make_step_inputs(_w(2, prefix=(1000, 1300), seed=20 + mode), device="cuda", random_step_map=True)
+    assert _splits(si) > 1
+    _check(si, seqs=[0, 1], rope=(1e6, mode))
+
+
+def test_split_units_error_paths():
+    si = inputs.make_step_inputs(_w(6, prefix=(1000, 1700), seed=30), device="cuda")
+    sm = si.step_map.clone()
+    sm[0, 5] = 0                                    # padding slot in sequence 0
+    sm[3, :2] = 1                                   # invalid map: all padding
+    si.step_map = sm
+    n = si.prefix_len.clone()
+    n[1] = si.block_table.shape[1] * si.w.page_size + 3    # beyond the block table
+    si.prefix_len = n
+    bt = si.block_table.clone()
+    bt[2, 1] = -1                                   # page id outside the pool
+    si.block_table = bt
+    assert _splits(si) > 1
+    out, word = _check(si, seqs=[0, 1, 2, 3, 4])
+    assert word & simsd.EW_PREFIX_LEN and word & simsd.EW_PAGE and word & simsd.EW_STEP_MAP
+    assert (out[1:4].float() == 0).all() and (out[0, [5, 37]].float() == 0).all()
+
+
+def test_split_units_deterministic():
+    si = inputs.make_step_inputs(_w(2, prefix=(900, 4000), seed=12), device="cuda", random_step_map=True)
+    a, _, _ = gpu_attention(si)
+    b, _, _ = gpu_attention(si)
+    assert torch.equal(a, b)
 
 
 def test_deterministic_and_equal_to_rerun():
