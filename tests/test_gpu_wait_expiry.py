@@ -20,23 +20,27 @@ from tests._gpu import assert_attention_close, gpu_attention, gpu_mask, oracle_a
 pytestmark = pytest.mark.gpu
 
 
-@pytest.mark.parametrize("Bt,Hq,gamma", [(40, 16, 4), (20, 32, 32)])
-def test_attention_wait_runs_out_and_the_context_stays_usable(Bt, Hq, gamma):
+@pytest.mark.parametrize("Bt,Hq,gamma,prefix", [(40, 16, 4, (100, 300)), (20, 32, 32, (100, 300)),
+                                               (2, 32, 32, (1500, 2000))])
+def test_attention_wait_runs_out_and_the_context_stays_usable(Bt, Hq, gamma, prefix):
     # 40 sequences x 8 KV heads of 16 rows: 320 unsplit units in two waves
     # of the one-row-block kernel; 20 x 8 units of 256 rows: the persistent
-    # two-row-block kernel (each block's MMA issuer waits for P that the
-    # planted count never completes)
-    w = inputs.Workload("we", "bf16", Bt, Hq, 8, 128, gamma, (100, 300), 1, 64, 0.5, 1 / np.sqrt(128), 1.0, 31)
+    # two-row-block kernel (each block's PV issuer waits for P that the
+    # planted count never completes); 2 x 8 units of 256 rows: the same
+    # kernel with key-tile ranges, then the combine kernel
+    w = inputs.Workload("we", "bf16", Bt, Hq, 8, 128, gamma, prefix, 1, 64, 0.5, 1 / np.sqrt(128), 1.0, 31)
     si = inputs.make_step_inputs(w, device="cuda", random_step_map=True, with_logits=False)
     tau, sect, _, _, merr = gpu_mask(si, mask_bits=False)
     assert simsd.simsd_check_error(merr) == 0
     before, word, ws = gpu_attention(si, mask=(tau, sect))
-    assert word == 0 and ws == 0
+    # a workspace only for the ranges of the small batch
+    assert word == 0 and (ws > 0) == (Bt == 2)
     simsd.simsd_debug_expire_next_wait(simsd.DEBUG_WAIT_ATTENTION, 200)
     out = torch.full_like(si.q[0], float("nan"))
     err = torch.zeros(1, dtype=torch.int32, device="cuda")
+    work = torch.zeros(ws, dtype=torch.uint8, device="cuda") if ws else None
     simsd.simsd_verify_attention(si.q[0], si.k_new[0], si.v_new[0], si.k_cache[0], si.v_cache[0], si.block_table,
-                                 si.prefix_len, tau, sect, out, err_word=err)
+                                 si.prefix_len, tau, sect, out, workspace=work, err_word=err)
     word = simsd.simsd_check_error(err)
     assert word == simsd.EW_TIMEOUT
     after, word, _ = gpu_attention(si, mask=(tau, sect))
