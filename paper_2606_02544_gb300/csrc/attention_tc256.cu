@@ -378,7 +378,8 @@ __global__ void __launch_bounds__(kThreads, 1)
       // served two of these streams kept a request of one waiting behind the
       // MMAs of the other (a written P behind the next tile's S, or one
       // block's P behind the other's PV).  Each thread waits on one barrier
-      // at a time.
+      // at a time, polling it with test_wait (a try_wait that suspends the
+      // thread woke it later; ~1% slower at 32 drafts).
       const bool is_s = warp < kWarpProducerV;
       const int x = is_s ? warp - kWarpMma : warp - kWarpPv;
       if (lane == 0) {
@@ -400,8 +401,8 @@ __global__ void __launch_bounds__(kThreads, 1)
               // S_X(t) needs K(t) and the completion of PV_X(t - 2), which read
               // the P held in the same S buffer
               const int st = gg % kStages;
-              ok = mbar_wait(smem_u32(&sm.bar_k[st]), (gg / kStages) & 1, abort_flag, p.wait_ns) &&
-                   (gg < 2 || mbar_wait(smem_u32(&sm.bar_pvs[x][gg & 1]), ((gg - 2) >> 1) & 1, abort_flag, p.wait_ns));
+              ok = mbar_wait_poll(smem_u32(&sm.bar_k[st]), (gg / kStages) & 1, abort_flag, p.wait_ns) &&
+                   (gg < 2 || mbar_wait_poll(smem_u32(&sm.bar_pvs[x][gg & 1]), ((gg - 2) >> 1) & 1, abort_flag, p.wait_ns));
               if (!ok) break;
               tc_fence_after();
               const uint32_t kb0 = smem_u32(sm.ring[st]), kb1 = kb0 + kHalfBytes;
@@ -424,9 +425,9 @@ __global__ void __launch_bounds__(kThreads, 1)
               // previous unit's O_X read out by the epilogue
               const int st = gg % kStages;
               const bool first = gg == g0;
-              ok = mbar_wait(smem_u32(&sm.bar_p[x][gg & 1]), (gg >> 1) & 1, abort_flag, p.wait_ns) &&
-                   (!first || jq <= 1 || mbar_wait(smem_u32(&sm.bar_ofree[x]), (jq - 2) & 1, abort_flag, p.wait_ns)) &&
-                   mbar_wait(smem_u32(&sm.bar_v[st]), (gg / kStages) & 1, abort_flag, p.wait_ns);
+              ok = mbar_wait_poll(smem_u32(&sm.bar_p[x][gg & 1]), (gg >> 1) & 1, abort_flag, p.wait_ns) &&
+                   (!first || jq <= 1 || mbar_wait_poll(smem_u32(&sm.bar_ofree[x]), (jq - 2) & 1, abort_flag, p.wait_ns)) &&
+                   mbar_wait_poll(smem_u32(&sm.bar_v[st]), (gg / kStages) & 1, abort_flag, p.wait_ns);
               if (!ok) break;
               tc_fence_after();
               const uint32_t vb = smem_u32(sm.ring[st]) + 2 * kHalfBytes;
