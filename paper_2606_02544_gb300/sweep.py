@@ -17,6 +17,7 @@ launches are timed in a graph of their own.  When a step's bytes are below
 from __future__ import annotations
 
 import argparse
+import dataclasses
 import json
 import os
 import statistics
@@ -156,6 +157,27 @@ def run_sampled_point(Bt: int, gamma: int, vocab: int, steps: int, peak: float) 
     return row
 
 
+def points(bts, ns, gs, ps, args):
+    """Workloads of batch x prefix x gamma x agreement: the preset sweep
+    point where one exists (its seed), else one of the same shape, with the
+    heads, page size, layer count and seed of the command line."""
+    hq, hkv = (int(v) for v in args.heads.split("/"))
+    preset = {(w.Bt, w.prefix[0], w.gamma, w.p_agree): w for w in inputs.sweep_points()}
+    out = []
+    for Bt in sorted(bts):
+        for n in sorted(ns):
+            for gm in sorted(gs):
+                for pa in sorted(ps):
+                    w = preset.get((Bt, n, gm, pa))
+                    if w is None:
+                        w = inputs.Workload(f"c5_b{Bt}_n{n}_g{gm}_p{pa}", "bf16", Bt, 32, 8, 128, gm, (n, n), 1,
+                                            151936, pa, inputs._SD, 2.0, 9000 + Bt + n + gm)
+                    w = dataclasses.replace(w, Hq=hq, Hkv=hkv, page_size=args.page_size, layers=args.layers,
+                                            seed=w.seed if args.seed is None else args.seed)
+                    out.append(w)
+    return out
+
+
 def main(argv=None):
     ap = argparse.ArgumentParser(description=__doc__.split("\n\n")[0])
     ap.add_argument("--out", default=None, help="also write a markdown table here")
@@ -164,6 +186,10 @@ def main(argv=None):
     ap.add_argument("--prefix", default="512,2048,8192,32768")
     ap.add_argument("--gamma", default="4,8,16,32")
     ap.add_argument("--agree", default="0.3,0.6,0.9")
+    ap.add_argument("--heads", default="32/8", help="query/KV heads, e.g. 64/8")
+    ap.add_argument("--page-size", type=int, default=64)
+    ap.add_argument("--layers", type=int, default=1, help="stacked layers per step (independent K/V per layer)")
+    ap.add_argument("--seed", type=int, default=None, help="seed of every point (default: the preset's)")
     ap.add_argument("--sampled", action="store_true",
                     help="time the stochastic acceptance alone over --batch x --gamma (V 151936)")
     args = ap.parse_args(argv)
@@ -187,14 +213,14 @@ def main(argv=None):
                     f.write(f"| {r['Bt']} | {r['gamma']} | {r['us']:.1f} | {r['gbs']:.0f} | "
                             f"{100 * r['frac']:.1f}% |\n")
         return
-    for w in inputs.sweep_points():
-        if w.Bt in bts and w.prefix[0] in ns and w.gamma in gs and w.p_agree in ps:
+    for w in points(bts, ns, gs, ps, args):
             row = run_point(w, args.steps, peak)
             row["peak_gbs"], row["peak_source"] = peak, kind
             print(json.dumps(row), flush=True)
             rows.append(row)
     if args.out:
         with open(args.out, "w") as f:
+            f.write(f"Heads {args.heads}, page size {args.page_size}, {args.layers} layer(s) per step.\n\n")
             f.write("| Bt | prefix | gamma | p | tokens/s | step us | attention us | attention GB/s | "
                     f"of {peak:.0f} GB/s | TFLOP/s | of {_tensor_peak():.0f} |\n"
                     "|---|---|---|---|---|---|---|---|---|---|---|\n")
