@@ -213,6 +213,31 @@ SIMSD_API int simsd_accept(const float* logits, const int32_t* draft, int Bt, in
                  int32_t* out_tokens, int32_t* row_argmax, int32_t* err_word, void* stream);
 
 /*
+ * simsd_accept_workspace_bytes -- bytes of scratch simsd_accept_ws uses for
+ * these sizes on the current device: 0 when the shape keeps the
+ * scratch-free kernel of simsd_accept (more than num_SMs / 16 sequences, or
+ * too few logits per sequence to split), else Bt x parts x (gamma+1) x 8.
+ * Returns 0 for invalid sizes or when no sm_103a device is current.
+ *
+ * simsd_accept_ws -- simsd_accept (same arguments, outputs and error rules)
+ * with a caller workspace.  For few sequences each sequence's logits are
+ * split over more CTAs than one thread-block cluster holds: a first launch
+ * writes one 64-bit argmax key per (sequence, part, row) to the workspace,
+ * a second takes the maximum per row and walks the drafts.  The results are
+ * identical to simsd_accept's (the argmax is a total order).
+ *   workspace   device memory of at least simsd_accept_workspace_bytes()
+ *               bytes, 8-byte aligned, owned by the caller; its contents
+ *               need no initial value and are overwritten.  NULL/0 is
+ *               accepted when that size is 0.
+ * A workspace smaller than needed returns SIMSD_ERR_INVALID_ARG before any
+ * launch.  Two calls that share a workspace must not overlap on the GPU.
+ */
+SIMSD_API size_t simsd_accept_workspace_bytes(int Bt, int gamma, int vocab);
+SIMSD_API int simsd_accept_ws(const float* logits, const int32_t* draft, int Bt, int gamma, int vocab,
+                              int32_t* accepted_len, int32_t* out_tokens, int32_t* row_argmax, void* workspace,
+                              size_t workspace_bytes, int32_t* err_word, void* stream);
+
+/*
  * simsd_accept_sampled -- stochastic acceptance (Sec. 3.2, Eq. (2)): with
  * p = softmax(logits / temperature), the r-th draft x_r is accepted iff
  * u_accept[b][r] < alpha_r = min(1, p_theta^(r)(x_r) / p_phi^(r)(x_r)),

@@ -14,6 +14,7 @@
 #include <cooperative_groups.h>
 #include <cuda_runtime.h>
 
+#include <algorithm>
 #include <mutex>
 
 #include "common.cuh"
@@ -73,41 +74,14 @@ struct RowBest {
   }
 };
 
-// UNROLL 16-byte loads are in flight per thread: 8 in general, 16 when the
-// grid leaves SMs idle (then each CTA has the SM to itself).
+// Span c of CL equal spans of one sequence's [rows][vocab] block (in 16-byte
+// units when rows are 16-byte aligned): each thread streams its elements
+// and folds a running (value, index) per row into best[row] (shared memory,
+// 64-bit keys, atomicMax) when its row changes.
 template <int UNROLL>
-__global__ void __launch_bounds__(kAcceptThreads) accept_kernel(const float* __restrict__ logits,
-                                                                const int32_t* __restrict__ draft, int gamma,
-                                                                int vocab, int vec4, int32_t* __restrict__ accepted_len,
-                                                                int32_t* __restrict__ out_tokens,
-                                                                int32_t* __restrict__ row_argmax, int32_t* err_word,
-                                                                uint32_t extra_arrivals, unsigned long long wait_ns) {
-  __shared__ unsigned long long best[kMaxRows];
-  __shared__ unsigned long long gath[kMaxCluster][kMaxRows];  // CTA 0: every CTA's keys
-  __shared__ __align__(8) unsigned long long gbar;              // CTA 0: one arrival per CTA
-  __shared__ int am[kMaxRows];
-  cg::cluster_group cluster = cg::this_cluster();
-  const int c = static_cast<int>(cluster.block_rank());
-  const int CL = static_cast<int>(cluster.num_blocks());
-  const int b = blockIdx.x / CL;
-  const int rows = gamma + 1;
+__device__ __forceinline__ void scan_span(const float* __restrict__ base, int rows, int vocab, int vec4, int c, int CL,
+                                          unsigned long long* best) {
   const int tid = threadIdx.x;
-  for (int r = tid; r < rows; r += kAcceptThreads) best[r] = 0ull;
-  if (c == 0 && tid == 0) {
-    mbar_init(smem_u32(&gbar), static_cast<uint32_t>(CL) + extra_arrivals);
-    fence_mbar_init();
-  }
-  // CTA 0's barrier must be initialised before any CTA arrives on it: every
-  // thread arrives here and waits just before its first remote write
-  cluster_arrive_relaxed();
-  pdl_wait();
-  // the drafts are needed only at the end; their load is issued now
-  const int dr_lane = (c == 0 && tid < gamma) ? draft[static_cast<size_t>(b) * gamma + tid] : 0;
-  __syncthreads();
-
-  // This CTA owns one contiguous span of the sequence's [rows][vocab] block
-  // (in 16-byte units when rows are 16-byte aligned).
-  const float* base = logits + static_cast<size_t>(b) * rows * vocab;
   const int W = vec4 ? (vocab >> 2) : vocab;   // units per row
   const long long F = static_cast<long long>(rows) * W;
   const long long per = (F + CL - 1) / CL;
@@ -170,6 +144,69 @@ __global__ void __launch_bounds__(kAcceptThreads) accept_kernel(const float* __r
     }
   }
   if (f0 + tid < f1) atomicMax(&best[cur], rb.key());
+}
+
+// One warp of sequence b, after am[r] (shared memory) holds the argmax of
+// every row: the accepted length (drafts in tau order, lane r checks draft
+// r; gamma <= 32) and the output tokens.
+__device__ __forceinline__ void walk_drafts(const int* am, int dr_lane, int b, int gamma, int vocab,
+                                            int32_t* __restrict__ accepted_len, int32_t* __restrict__ out_tokens,
+                                            int32_t* __restrict__ row_argmax, int32_t* err_word) {
+  const int lane = threadIdx.x & 31;
+  const int rows = gamma + 1;
+  if (row_argmax)
+    for (int r = lane; r < rows; r += 32) row_argmax[static_cast<size_t>(b) * rows + r] = am[r];
+  bool in_range = true, match = false;
+  if (lane < gamma) {
+    in_range = dr_lane >= 0 && dr_lane < vocab;
+    match = in_range && dr_lane == am[lane];
+  }
+  const unsigned bad = __ballot_sync(0xffffffffu, !in_range);
+  const unsigned miss = __ballot_sync(0xffffffffu, lane < gamma && !match);
+  const int a = miss ? (__ffs(miss) - 1) : gamma;
+  if (lane == 0) {
+    if (bad) raise_error(err_word, SIMSD_EW_DRAFT);
+    accepted_len[b] = a;
+  }
+  int32_t* ot = out_tokens + static_cast<size_t>(b) * rows;
+  for (int r = lane; r < rows; r += 32) ot[r] = r < a ? dr_lane : (r == a ? am[a] : -1);
+}
+
+// UNROLL 16-byte loads are in flight per thread: 8 in general, 16 when the
+// grid leaves SMs idle (then each CTA has the SM to itself).
+template <int UNROLL>
+__global__ void __launch_bounds__(kAcceptThreads) accept_kernel(const float* __restrict__ logits,
+                                                                const int32_t* __restrict__ draft, int gamma,
+                                                                int vocab, int vec4, int32_t* __restrict__ accepted_len,
+                                                                int32_t* __restrict__ out_tokens,
+                                                                int32_t* __restrict__ row_argmax, int32_t* err_word,
+                                                                uint32_t extra_arrivals, unsigned long long wait_ns) {
+  __shared__ unsigned long long best[kMaxRows];
+  __shared__ unsigned long long gath[kMaxCluster][kMaxRows];  // CTA 0: every CTA's keys
+  __shared__ __align__(8) unsigned long long gbar;              // CTA 0: one arrival per CTA
+  __shared__ int am[kMaxRows];
+  cg::cluster_group cluster = cg::this_cluster();
+  const int c = static_cast<int>(cluster.block_rank());
+  const int CL = static_cast<int>(cluster.num_blocks());
+  const int b = blockIdx.x / CL;
+  const int rows = gamma + 1;
+  const int tid = threadIdx.x;
+  for (int r = tid; r < rows; r += kAcceptThreads) best[r] = 0ull;
+  if (c == 0 && tid == 0) {
+    mbar_init(smem_u32(&gbar), static_cast<uint32_t>(CL) + extra_arrivals);
+    fence_mbar_init();
+  }
+  // CTA 0's barrier must be initialised before any CTA arrives on it: every
+  // thread arrives here and waits just before its first remote write
+  cluster_arrive_relaxed();
+  pdl_wait();
+  // the drafts are needed only at the end; their load is issued now
+  const int dr_lane = (c == 0 && tid < gamma) ? draft[static_cast<size_t>(b) * gamma + tid] : 0;
+  __syncthreads();
+
+  // This CTA owns one contiguous span of the sequence's [rows][vocab] block
+  // (in 16-byte units when rows are 16-byte aligned).
+  scan_span<UNROLL>(logits + static_cast<size_t>(b) * rows * vocab, rows, vocab, vec4, c, CL, best);
   // the next kernel may be scheduled once the stream of logits is done
   // (earlier, its waiting CTAs would sit beside this one's)
   pdl_launch_next();
@@ -195,26 +232,57 @@ __global__ void __launch_bounds__(kAcceptThreads) accept_kernel(const float* __r
   for (int r = lane; r < rows; r += 32) {
     unsigned long long k = 0ull;
     for (int p = 0; p < CL; ++p) k = gath[p][r] > k ? gath[p][r] : k;
-    const int idx = static_cast<int>(~static_cast<uint32_t>(k & 0xFFFFFFFFull));
-    am[r] = idx;
-    if (row_argmax) row_argmax[static_cast<size_t>(b) * rows + r] = idx;
+    am[r] = static_cast<int>(~static_cast<uint32_t>(k & 0xFFFFFFFFull));
   }
   __syncwarp();
-  // drafts in tau order; lane r checks draft r (gamma <= 32)
-  bool in_range = true, match = false;
-  if (lane < gamma) {
-    in_range = dr_lane >= 0 && dr_lane < vocab;
-    match = in_range && dr_lane == am[lane];
+  walk_drafts(am, dr_lane, b, gamma, vocab, accepted_len, out_tokens, row_argmax, err_word);
+}
+
+
+// Few sequences: the block of each sequence is split over `parts` CTAs that
+// need not be resident together (no cluster).  Each writes its 64-bit key
+// per row to keys[b][part][row]; accept_merge_kernel then takes the maximum
+// per row and walks the drafts.
+__global__ void __launch_bounds__(kAcceptThreads) accept_part_kernel(const float* __restrict__ logits, int gamma,
+                                                                     int vocab, int vec4, int parts,
+                                                                     unsigned long long* __restrict__ keys) {
+  __shared__ unsigned long long best[kMaxRows];
+  const int b = blockIdx.x / parts, c = blockIdx.x - b * parts;
+  const int rows = gamma + 1;
+  for (int r = threadIdx.x; r < rows; r += kAcceptThreads) best[r] = 0ull;
+  pdl_wait();
+  __syncthreads();
+  scan_span<8>(logits + static_cast<size_t>(b) * rows * vocab, rows, vocab, vec4, c, parts, best);
+  __syncthreads();
+  for (int r = threadIdx.x; r < rows; r += kAcceptThreads)
+    keys[(static_cast<size_t>(b) * parts + c) * rows + r] = best[r];
+  pdl_launch_next();
+}
+
+// One warp per sequence: the maximum key of every row over the parts, then
+// the walk.
+__global__ void __launch_bounds__(32) accept_merge_kernel(const unsigned long long* __restrict__ keys, int parts,
+                                                          const int32_t* __restrict__ draft, int gamma, int vocab,
+                                                          int32_t* __restrict__ accepted_len,
+                                                          int32_t* __restrict__ out_tokens,
+                                                          int32_t* __restrict__ row_argmax, int32_t* err_word) {
+  __shared__ int am[kMaxRows];
+  const int b = blockIdx.x, lane = threadIdx.x;
+  const int rows = gamma + 1;
+  pdl_wait();
+  const int dr_lane = lane < gamma ? draft[static_cast<size_t>(b) * gamma + lane] : 0;
+  for (int r = lane; r < rows; r += 32) {
+    unsigned long long k = 0ull;
+    const unsigned long long* kr = keys + static_cast<size_t>(b) * parts * rows + r;
+    for (int p = 0; p < parts; ++p) {
+      const unsigned long long v = kr[static_cast<size_t>(p) * rows];
+      k = v > k ? v : k;
+    }
+    am[r] = static_cast<int>(~static_cast<uint32_t>(k & 0xFFFFFFFFull));
   }
-  const unsigned bad = __ballot_sync(0xffffffffu, !in_range);
-  const unsigned miss = __ballot_sync(0xffffffffu, lane < gamma && !match);
-  const int a = miss ? (__ffs(miss) - 1) : gamma;
-  if (lane == 0) {
-    if (bad) raise_error(err_word, SIMSD_EW_DRAFT);
-    accepted_len[b] = a;
-  }
-  int32_t* ot = out_tokens + static_cast<size_t>(b) * rows;
-  for (int r = lane; r < rows; r += 32) ot[r] = r < a ? dr_lane : (r == a ? am[a] : -1);
+  __syncwarp();
+  pdl_launch_next();
+  walk_drafts(am, dr_lane, b, gamma, vocab, accepted_len, out_tokens, row_argmax, err_word);
 }
 
 namespace {
@@ -263,6 +331,41 @@ cudaError_t cluster_capacity(const ClusterCapacity** out) {
 }
 
 }  // namespace
+
+int accept_parts(int Bt, int gamma, int vocab, int num_sms) {
+  // few sequences only: one 16-CTA cluster each leaves SMs idle
+  if (static_cast<long long>(Bt) * kMaxCluster > num_sms) return 0;
+  // and at least 6 MiB of logits per sequence: below that the cluster's 16
+  // CTAs stream it about as fast as the split, which pays a second launch
+  // (measured: 3 MB per sequence 13 us either way, 15 us cluster against
+  // 17 us split at 8 sequences; 10 MB 23 against 18 us)
+  if (static_cast<long long>(gamma + 1) * vocab * 4 < (6LL << 20)) return 0;
+  // about 8 units of 16 bytes per thread of a part, at most two parts per SM
+  const long long units = static_cast<long long>(gamma + 1) * ((vocab + 3) / 4);
+  const long long by_work = units / (8LL * kAcceptThreads);
+  const long long by_sms = (2LL * num_sms + Bt - 1) / Bt;
+  const long long parts = std::min(by_work, by_sms);
+  return parts > kMaxCluster ? static_cast<int>(parts) : 0;
+}
+
+size_t accept_workspace_bytes(int Bt, int gamma, int vocab, int num_sms) {
+  const int parts = accept_parts(Bt, gamma, vocab, num_sms);
+  return parts ? static_cast<size_t>(Bt) * parts * (gamma + 1) * sizeof(unsigned long long) : 0;
+}
+
+cudaError_t launch_accept_parts(const float* logits, const int32_t* draft, int Bt, int gamma, int vocab,
+                                int32_t* accepted_len, int32_t* out_tokens, int32_t* row_argmax, void* workspace,
+                                int32_t* err_word, int num_sms, cudaStream_t stream) {
+  const int parts = accept_parts(Bt, gamma, vocab, num_sms);
+  const int vec4 = (vocab % 4 == 0) && ((reinterpret_cast<uintptr_t>(logits) & 15u) == 0);
+  auto* keys = static_cast<unsigned long long*>(workspace);
+  cudaError_t e = launch_overlapped(accept_part_kernel, dim3(static_cast<unsigned>(Bt) * parts), dim3(kAcceptThreads),
+                                    0, stream, 1u, logits, gamma, vocab, vec4, parts, keys);
+  if (e != cudaSuccess) return e;
+  return launch_overlapped(accept_merge_kernel, dim3(static_cast<unsigned>(Bt)), dim3(32), 0, stream, 1u,
+                           static_cast<const unsigned long long*>(keys), parts, draft, gamma, vocab, accepted_len,
+                           out_tokens, row_argmax, err_word);
+}
 
 cudaError_t launch_accept(const float* logits, const int32_t* draft, int Bt, int gamma, int vocab,
                           int32_t* accepted_len, int32_t* out_tokens, int32_t* row_argmax, int32_t* err_word,

@@ -285,8 +285,13 @@ int simsd_verify_attention_noalloc(int dtype, const void* q, const void* k_new, 
                                softmax_scale, out, nullptr, 0, true, simsd::WaitFault{}, err_word, stream);
 }
 
-int simsd_accept(const float* logits, const int32_t* draft, int Bt, int gamma, int vocab, int32_t* accepted_len,
-                 int32_t* out_tokens, int32_t* row_argmax, int32_t* err_word, void* stream) {
+namespace {
+
+// Greedy acceptance: the cluster kernel, or with a workspace (ws_ok) the
+// split over many CTAs when the shape takes it.
+int accept_impl(const float* logits, const int32_t* draft, int Bt, int gamma, int vocab, int32_t* accepted_len,
+                int32_t* out_tokens, int32_t* row_argmax, bool ws_ok, void* workspace, size_t workspace_bytes,
+                int32_t* err_word, void* stream) {
   // an armed wait expiry is consumed by this call whatever its outcome
   const simsd::WaitFault fault = take_armed(SIMSD_DEBUG_WAIT_ACCEPT);
   if (Bt < 0) return arg_fail("Bt < 0");
@@ -297,11 +302,43 @@ int simsd_accept(const float* logits, const int32_t* draft, int Bt, int gamma, i
   DeviceInfo info;
   int rc = require_sm103(&info);
   if (rc != SIMSD_OK) return rc;
-  cudaError_t e = simsd::launch_accept(logits, draft, Bt, gamma, vocab, accepted_len, out_tokens, row_argmax,
-                                       err_word, info.num_sms, as_stream(stream), fault);
-  if (e == cudaErrorNotSupported && fault.extra)
-    return unsupported("a planted wait expiry needs one CTA per sequence (a batch too large for clusters)");
+  const size_t need = ws_ok ? simsd::accept_workspace_bytes(Bt, gamma, vocab, info.num_sms) : 0;
+  cudaError_t e;
+  if (need > 0) {
+    if (!workspace || workspace_bytes < need) return arg_fail("workspace smaller than simsd_accept_workspace_bytes()");
+    if ((reinterpret_cast<uintptr_t>(workspace) & 7u) != 0) return arg_fail("workspace not 8-byte aligned");
+    if (fault.extra) return unsupported("a planted wait expiry needs the cluster kernel (this path has no wait)");
+    e = simsd::launch_accept_parts(logits, draft, Bt, gamma, vocab, accepted_len, out_tokens, row_argmax, workspace,
+                                   err_word, info.num_sms, as_stream(stream));
+  } else {
+    e = simsd::launch_accept(logits, draft, Bt, gamma, vocab, accepted_len, out_tokens, row_argmax, err_word,
+                             info.num_sms, as_stream(stream), fault);
+    if (e == cudaErrorNotSupported && fault.extra)
+      return unsupported("a planted wait expiry needs one CTA per sequence (a batch too large for clusters)");
+  }
   return e == cudaSuccess ? SIMSD_OK : cuda_fail(e, "accept launch");
+}
+
+}  // namespace
+
+int simsd_accept(const float* logits, const int32_t* draft, int Bt, int gamma, int vocab, int32_t* accepted_len,
+                 int32_t* out_tokens, int32_t* row_argmax, int32_t* err_word, void* stream) {
+  return accept_impl(logits, draft, Bt, gamma, vocab, accepted_len, out_tokens, row_argmax, false, nullptr, 0,
+                     err_word, stream);
+}
+
+size_t simsd_accept_workspace_bytes(int Bt, int gamma, int vocab) {
+  if (Bt <= 0 || gamma < 1 || gamma > 32 || vocab < 1 || vocab > (1 << 28)) return 0;
+  DeviceInfo info;
+  if (require_sm103(&info) != SIMSD_OK) return 0;
+  return simsd::accept_workspace_bytes(Bt, gamma, vocab, info.num_sms);
+}
+
+int simsd_accept_ws(const float* logits, const int32_t* draft, int Bt, int gamma, int vocab, int32_t* accepted_len,
+                    int32_t* out_tokens, int32_t* row_argmax, void* workspace, size_t workspace_bytes,
+                    int32_t* err_word, void* stream) {
+  return accept_impl(logits, draft, Bt, gamma, vocab, accepted_len, out_tokens, row_argmax, true, workspace,
+                     workspace_bytes, err_word, stream);
 }
 
 int simsd_accept_sampled(const float* target_logits, const float* draft_logits, const int32_t* draft,

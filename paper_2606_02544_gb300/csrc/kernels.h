@@ -34,6 +34,15 @@ cudaError_t launch_accept(const float* logits, const int32_t* draft, int Bt, int
                           int32_t* accepted_len, int32_t* out_tokens, int32_t* row_argmax, int32_t* err_word,
                           int num_sms, cudaStream_t stream, const WaitFault& fault = WaitFault{});
 
+// Few sequences with a caller workspace: each sequence's logits split over
+// accept_parts() CTAs (0: the shape takes the cluster kernel), their
+// per-row keys merged by a second launch.
+int accept_parts(int Bt, int gamma, int vocab, int num_sms);
+size_t accept_workspace_bytes(int Bt, int gamma, int vocab, int num_sms);
+cudaError_t launch_accept_parts(const float* logits, const int32_t* draft, int Bt, int gamma, int vocab,
+                                int32_t* accepted_len, int32_t* out_tokens, int32_t* row_argmax, void* workspace,
+                                int32_t* err_word, int num_sms, cudaStream_t stream);
+
 cudaError_t launch_accept_sampled(const float* target_logits, const float* draft_logits, const int32_t* draft,
                                   const float* u_accept, const float* u_sample, float temperature, int Bt,
                                   int gamma, int vocab, int32_t* accepted_len, int32_t* out_tokens,

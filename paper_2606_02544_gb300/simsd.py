@@ -25,7 +25,8 @@ EW_STEP_MAP, EW_PREFIX_LEN, EW_PAGE, EW_DRAFT, EW_TIMEOUT, EW_ACCEPT_LEN = 1, 2,
 STEP_UNDRAFTED, STEP_DECODED = -1, -2
 
 EXPORTED = ("simsd_build_mask", "simsd_verify_workspace_bytes", "simsd_verify_attention",
-            "simsd_verify_attention_noalloc", "simsd_accept", "simsd_accept_sampled", "simsd_kv_commit",
+            "simsd_verify_attention_noalloc", "simsd_accept", "simsd_accept_workspace_bytes", "simsd_accept_ws",
+            "simsd_accept_sampled", "simsd_kv_commit",
             "simsd_check_error", "simsd_debug_expire_next_wait",
             "simsd_last_error", "simsd_version")
 DEBUG_WAIT_ATTENTION, DEBUG_WAIT_ACCEPT = 1, 2
@@ -59,6 +60,9 @@ def load_library(path: str = LIB_PATH):
             lib.simsd_verify_attention_noalloc.argtypes = [I, P, P, P, P, P, I, P, I, I, P, P, P, P, F, I, I, I, I,
                                                            I, F, P, P, P]
             lib.simsd_accept.argtypes = [P, P, I, I, I, P, P, P, P, P]
+            lib.simsd_accept_workspace_bytes.argtypes = [I, I, I]
+            lib.simsd_accept_workspace_bytes.restype = Z
+            lib.simsd_accept_ws.argtypes = [P, P, I, I, I, P, P, P, P, Z, P, P]
             lib.simsd_accept_sampled.argtypes = [P, P, P, P, P, F, I, I, I, P, P, P, P]
             lib.simsd_kv_commit.argtypes = [I, P, P, I, P, P, P, F, P, P, P, I, P, I, I, P, I, I, I, I, P, P]
             lib.simsd_check_error.argtypes = [P, P, P]
@@ -149,6 +153,21 @@ def simsd_accept(logits, draft, accepted_len, out_tokens, row_argmax=None, err_w
     rc = load_library().simsd_accept(_p(logits), _p(draft), Bt, rows - 1, V, _p(accepted_len), _p(out_tokens),
                                      _p(row_argmax), _p(err_word), _stream(stream))
     _check(rc, "simsd_accept")
+
+
+def simsd_accept_workspace_bytes(Bt, gamma, vocab) -> int:
+    return int(load_library().simsd_accept_workspace_bytes(Bt, gamma, vocab))
+
+
+def simsd_accept_ws(logits, draft, accepted_len, out_tokens, workspace=None, row_argmax=None, err_word=None,
+                    stream=None):
+    """simsd_accept with a caller workspace (uint8 device tensor of
+    simsd_accept_workspace_bytes() bytes, or None when that is 0)."""
+    Bt, rows, V = logits.shape
+    nbytes = workspace.numel() * workspace.element_size() if workspace is not None else 0
+    rc = load_library().simsd_accept_ws(_p(logits), _p(draft), Bt, rows - 1, V, _p(accepted_len), _p(out_tokens),
+                                        _p(row_argmax), _p(workspace), nbytes, _p(err_word), _stream(stream))
+    _check(rc, "simsd_accept_ws")
 
 
 def simsd_accept_sampled(target_logits, draft_logits, draft, u_accept, u_sample, accepted_len, out_tokens,

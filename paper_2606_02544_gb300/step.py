@@ -5,7 +5,7 @@ A step (Sec. 3.2, one target verification forward per speculative step):
   2. simsd_verify_attention, once per layer (the masked attention; with
      ``rope_theta`` the un-rotated q / k_new are rotated at the RoPE-copy
      positions inside the kernel, Sec. 3.1)
-  3. simsd_accept          greedy longest-prefix acceptance (Eq. (2), T=0)
+  3. simsd_accept_ws       greedy longest-prefix acceptance (Eq. (2), T=0)
   4. simsd_kv_commit       append the accepted drafts' K/V, advance n_b
 All four run on one stream and are captured into one CUDA graph, so the
 step needs no host round trip.  PyTorch only allocates the buffers.
@@ -46,6 +46,10 @@ class VerifyStep:
         ws = simsd.simsd_verify_workspace_bytes(dt, w.Bt, w.gamma, w.Hq, w.Hkv, w.d, si.block_table.shape[1],
                                                 w.page_size)
         self.workspace = torch.empty(max(ws, 16), dtype=torch.uint8, device=dev) if ws > 0 else None
+        # the acceptance splits a small batch's logits over more CTAs when a
+        # workspace is given (0 bytes: the scratch-free cluster kernel)
+        aws = simsd.simsd_accept_workspace_bytes(w.Bt, w.gamma, si.logits.shape[-1]) if si.logits is not None else 0
+        self.accept_workspace = torch.empty(aws, dtype=torch.uint8, device=dev) if aws > 0 else None
         self.accepted_len = torch.empty(w.Bt, **i32)
         self.out_tokens = torch.empty(w.Bt, w.gamma + 1, **i32)
         self.row_argmax = torch.empty(w.Bt, w.gamma + 1, **i32)
@@ -77,8 +81,8 @@ class VerifyStep:
         self.run_attention()
         if attn_events is not None:
             attn_events[1].record()
-        simsd.simsd_accept(si.logits, si.draft, self.accepted_len, self.out_tokens, self.row_argmax,
-                           err_word=self.err)
+        simsd.simsd_accept_ws(si.logits, si.draft, self.accepted_len, self.out_tokens, self.accept_workspace,
+                              row_argmax=self.row_argmax, err_word=self.err)
         simsd.simsd_kv_commit(si.k_new, si.v_new, self.tau, self.section, self.accepted_len, si.k_cache,
                               si.v_cache, si.block_table, self.n, err_word=self.err, rope_pos=rope,
                               rope_theta=self.rope_theta)
@@ -97,7 +101,9 @@ class VerifyStep:
     def launches_per_step(self) -> int:
         """Kernels of this library launched by one step."""
         combine = 1 if self.workspace is not None else 0
-        return 1 + self.L * (1 + combine) + 1 + 1   # mask, attention (+ combine) per layer, accept, commit
+        accept = 2 if self.accept_workspace is not None else 1
+        # mask, attention (+ combine) per layer, accept (parts + merge), commit
+        return 1 + self.L * (1 + combine) + accept + 1
 
     def capture(self, time_attention: bool = True):
         """Captures one step into a CUDA graph (with event-record nodes
