@@ -269,6 +269,29 @@ SIMSD_API int simsd_accept_sampled(const float* target_logits, const float* draf
                                    void* stream);
 
 /*
+ * simsd_accept_sampled_workspace_bytes / simsd_accept_sampled_ws -- the same
+ * stochastic acceptance with a caller workspace.  For few sequences (at most
+ * num_SMs / 16) holding at least 6 MiB of logits each (target and draft
+ * rows), the log-sum-exp pass over every row is split over more CTAs than one
+ * cluster per sequence holds: a first launch writes per-row (max, sum) pairs
+ * of each part to the workspace, which the cluster of each sequence merges
+ * before it forms alpha_r and draws the token as simsd_accept_sampled does.
+ * The workspace bytes are 0 for other shapes (then the call is
+ * simsd_accept_sampled).  The pairs are merged in another order than the
+ * cluster kernel's, so probabilities can differ in the last fp32 bits (the
+ * same rounding as between any two summation orders).
+ *   workspace  device memory of at least the returned bytes, 8-byte
+ *              aligned, owned by the caller; no initial value needed.
+ * A workspace smaller than needed returns SIMSD_ERR_INVALID_ARG before any
+ * launch.  Two calls that share a workspace must not overlap on the GPU.
+ */
+SIMSD_API size_t simsd_accept_sampled_workspace_bytes(int Bt, int gamma, int vocab);
+SIMSD_API int simsd_accept_sampled_ws(const float* target_logits, const float* draft_logits, const int32_t* draft,
+                                      const float* u_accept, const float* u_sample, float temperature, int Bt,
+                                      int gamma, int vocab, int32_t* accepted_len, int32_t* out_tokens,
+                                      void* workspace, size_t workspace_bytes, int32_t* err_word, void* stream);
+
+/*
  * simsd_kv_commit -- append the accepted drafts' K/V to the paged cache of
  * every layer (Sec. 3.2: accepted tokens are committed; Sec. 3.3: the cache
  * is reused by later steps).

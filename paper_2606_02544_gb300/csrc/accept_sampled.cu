@@ -24,6 +24,7 @@
 #include <cooperative_groups.h>
 #include <cuda_runtime.h>
 
+#include <algorithm>
 #include <cfloat>
 #include <mutex>
 
@@ -108,6 +109,122 @@ __device__ __forceinline__ float4 load_unit(const float* rp, int col) {
   }
 }
 
+// Phase 1 of one CTA: the running (m, s) of z = x log2(e) / T over span c
+// of CL equal spans of the sequence's rows (target rows 0..gamma, then
+// draft rows), merged per warp into part[warp][row].
+template <bool VEC, int UNROLL>
+__device__ __forceinline__ void phase1_span(const float* __restrict__ tgt, const float* __restrict__ drf, int b,
+                                            int gamma, int vocab, float zscale, int c, int CL,
+                                            float2 (*part)[kSampMaxRows]) {
+  const int rows = 2 * gamma + 1;
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  const unsigned full = 0xffffffffu;
+  const int W = VEC ? (vocab >> 2) : vocab;  // units per row
+  const int Wp = (W + 31) & ~31;             // padded: a warp never straddles two rows
+  const int G = rows * (Wp >> 5);            // groups of 32 units
+  const int per = (G + CL - 1) / CL;
+  const int f0 = 32 * min(G, c * per), f1 = 32 * min(G, c * per + per);
+  constexpr int kStep = kSampThreads;
+  int f = f0 + tid;
+  int row = f / Wp;
+  int col = f - row * Wp;
+  const float* rp = row_ptr(tgt, drf, b, gamma, vocab, min(row, rows - 1));
+  int cur = row;
+  float m = kEmpty, s = 0.f;
+  // merges the warp's lanes (all on row `cur`) into its slot
+  auto flush = [&]() {
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) {
+      const float m2 = __shfl_xor_sync(full, m, o), s2 = __shfl_xor_sync(full, s, o);
+      ms_merge(m, s, m2, s2);
+    }
+    if (lane == 0) {
+      float2 p = part[warp][cur];
+      ms_merge(p.x, p.y, m, s);
+      part[warp][cur] = p;
+    }
+  };
+  auto advance = [&](int by) {
+    col += by;
+    if (col >= Wp) {
+      do {
+        col -= Wp;
+        ++row;
+      } while (col >= Wp);
+      rp = row_ptr(tgt, drf, b, gamma, vocab, min(row, rows - 1));
+    }
+  };
+  // Loads of H units.  f0, f1, Wp and the f and col of a warp's first lane
+  // are multiples of 32, so every test here is the same for the 32 lanes
+  // of a warp.  vr[u] is the unit's row, -1 past the span.
+  constexpr int H = UNROLL == 16 ? 8 : UNROLL;
+  auto fetch = [&](float4(&v)[H], int(&vr)[H]) {
+    if (f - lane + kStep * (H - 1) < f1 && col - lane + kStep * (H - 1) + 31 < W) {
+      // the common case: every unit valid, on one row, inside the row
+#pragma unroll
+      for (int u = 0; u < H; ++u) {
+        v[u] = load_unit<VEC>(rp, col + u * kStep);
+        vr[u] = row;
+      }
+      advance(kStep * H);
+    } else {
+#pragma unroll
+      for (int u = 0; u < H; ++u) {
+        vr[u] = -1;
+        if (f + u * kStep < f1) {
+          vr[u] = row;
+          v[u] = col < W ? load_unit<VEC>(rp, col) : make_float4(-INFINITY, -INFINITY, -INFINITY, -INFINITY);
+        }
+        advance(kStep);
+      }
+    }
+    f += kStep * H;
+  };
+  auto consume = [&](const float4(&v)[H], const int(&vr)[H]) {
+#pragma unroll
+    for (int u = 0; u < H; ++u) {
+      if (vr[u] < 0) break;
+      if (vr[u] != cur) {
+        flush();
+        cur = vr[u];
+        m = kEmpty;
+        s = 0.f;
+      }
+      const float mz = fmaxf(fmaxf(v[u].x, v[u].y), fmaxf(v[u].z, v[u].w)) * zscale;
+      if (mz > m) {
+        s *= ex2(m - mz);
+        m = mz;
+      }
+      const float nm = -m;
+      s += ex2(fmaf(v[u].x, zscale, nm)) + ex2(fmaf(v[u].y, zscale, nm)) + ex2(fmaf(v[u].z, zscale, nm)) +
+           ex2(fmaf(v[u].w, zscale, nm));
+    }
+  };
+  if constexpr (UNROLL == 16) {
+    // one CTA per SM: two batches of 8, the next one's loads in flight
+    // while the current one is summed
+    float4 va[H], vb[H];
+    int ra[H], rb[H];
+    fetch(va, ra);
+    while (ra[0] >= 0) {
+      fetch(vb, rb);
+      consume(va, ra);
+      if (rb[0] < 0) break;
+      fetch(va, ra);
+      consume(vb, rb);
+    }
+  } else {
+    float4 v[H];
+    int vr[H];
+    for (;;) {
+      fetch(v, vr);
+      if (vr[0] < 0) break;
+      consume(v, vr);
+    }
+  }
+  if (f0 + 32 * warp < f1) flush();
+}
+
 // Units in flight per thread in phase 1: UNROLL 8 with two CTAs per SM;
 // UNROLL 16 when the grid has at most one CTA per SM (small batches), where
 // the CTA's bytes in flight set its bandwidth: two batches of 8, one loading
@@ -116,7 +233,9 @@ template <bool VEC, int UNROLL>
 __global__ void __launch_bounds__(kSampThreads, UNROLL == 8 ? 2 : 1) accept_sampled_kernel(
     const float* __restrict__ tgt, const float* __restrict__ drf, const int32_t* __restrict__ draft,
     const float* __restrict__ u_accept, const float* __restrict__ u_sample, float zscale, int gamma, int vocab,
-    int32_t* __restrict__ accepted_len, int32_t* __restrict__ out_tokens, int32_t* err_word) {
+    int32_t* __restrict__ accepted_len, int32_t* __restrict__ out_tokens, int32_t* err_word,
+    const float2* __restrict__ pre, int pre_parts) {
+  // pre: null, or the (m, s) partials of samp_part_kernel [Bt][pre_parts][rows]
   __shared__ float2 part[kSampWarps][kSampMaxRows];  // per warp (m, s) of each row
   __shared__ float2 cta_ms[kSampMaxRows];            // this CTA's (m, s) of each row
   __shared__ float row_m[kSampMaxRows], row_s[kSampMaxRows];
@@ -156,120 +275,36 @@ __global__ void __launch_bounds__(kSampThreads, UNROLL == 8 ? 2 : 1) accept_samp
   __syncthreads();
 
   // ---- phase 1: per-row (m, s) over this CTA's span of warp-aligned units
-  {
-    const int W = VEC ? (vocab >> 2) : vocab;  // units per row
-    const int Wp = (W + 31) & ~31;             // padded: a warp never straddles two rows
-    const int G = rows * (Wp >> 5);            // groups of 32 units
-    const int per = (G + CL - 1) / CL;
-    const int f0 = 32 * min(G, c * per), f1 = 32 * min(G, c * per + per);
-    constexpr int kStep = kSampThreads;
-    int f = f0 + tid;
-    int row = f / Wp;
-    int col = f - row * Wp;
-    const float* rp = row_ptr(tgt, drf, b, gamma, vocab, min(row, rows - 1));
-    int cur = row;
-    float m = kEmpty, s = 0.f;
-    // merges the warp's lanes (all on row `cur`) into its slot
-    auto flush = [&]() {
+  // (or, with partials from samp_part_kernel, none here)
+  if (pre == nullptr) phase1_span<VEC, UNROLL>(tgt, drf, b, gamma, vocab, zscale, c, CL, part);
+  // the next kernel may be scheduled once the logits have streamed through
+  pdl_launch_next();
+  __syncthreads();
+  if (pre == nullptr) {
+    for (int r = tid; r < rows; r += kSampThreads) {
+      float m = kEmpty, s = 0.f;
+#pragma unroll
+      for (int w = 0; w < kSampWarps; ++w) ms_merge(m, s, part[w][r].x, part[w][r].y);
+      cta_ms[r] = make_float2(m, s);
+    }
+  } else {
+    // this CTA merges its share of the parts: warp w takes rows w, w+16, ...
+    // and its lanes the parts p0 + lane, p0 + lane + 32, ...
+    const int per = (pre_parts + CL - 1) / CL;
+    const int p0 = min(pre_parts, c * per), p1 = min(pre_parts, p0 + per);
+    for (int r = warp; r < rows; r += kSampWarps) {
+      float m = kEmpty, s = 0.f;
+      for (int q = p0 + lane; q < p1; q += 32) {
+        const float2 v = pre[(static_cast<size_t>(b) * pre_parts + q) * rows + r];
+        ms_merge(m, s, v.x, v.y);
+      }
 #pragma unroll
       for (int o = 16; o > 0; o >>= 1) {
         const float m2 = __shfl_xor_sync(full, m, o), s2 = __shfl_xor_sync(full, s, o);
         ms_merge(m, s, m2, s2);
       }
-      if (lane == 0) {
-        float2 p = part[warp][cur];
-        ms_merge(p.x, p.y, m, s);
-        part[warp][cur] = p;
-      }
-    };
-    auto advance = [&](int by) {
-      col += by;
-      if (col >= Wp) {
-        do {
-          col -= Wp;
-          ++row;
-        } while (col >= Wp);
-        rp = row_ptr(tgt, drf, b, gamma, vocab, min(row, rows - 1));
-      }
-    };
-    // Loads of H units.  f0, f1, Wp and the f and col of a warp's first lane
-    // are multiples of 32, so every test here is the same for the 32 lanes
-    // of a warp.  vr[u] is the unit's row, -1 past the span.
-    constexpr int H = UNROLL == 16 ? 8 : UNROLL;
-    auto fetch = [&](float4(&v)[H], int(&vr)[H]) {
-      if (f - lane + kStep * (H - 1) < f1 && col - lane + kStep * (H - 1) + 31 < W) {
-        // the common case: every unit valid, on one row, inside the row
-#pragma unroll
-        for (int u = 0; u < H; ++u) {
-          v[u] = load_unit<VEC>(rp, col + u * kStep);
-          vr[u] = row;
-        }
-        advance(kStep * H);
-      } else {
-#pragma unroll
-        for (int u = 0; u < H; ++u) {
-          vr[u] = -1;
-          if (f + u * kStep < f1) {
-            vr[u] = row;
-            v[u] = col < W ? load_unit<VEC>(rp, col) : make_float4(-INFINITY, -INFINITY, -INFINITY, -INFINITY);
-          }
-          advance(kStep);
-        }
-      }
-      f += kStep * H;
-    };
-    auto consume = [&](const float4(&v)[H], const int(&vr)[H]) {
-#pragma unroll
-      for (int u = 0; u < H; ++u) {
-        if (vr[u] < 0) break;
-        if (vr[u] != cur) {
-          flush();
-          cur = vr[u];
-          m = kEmpty;
-          s = 0.f;
-        }
-        const float mz = fmaxf(fmaxf(v[u].x, v[u].y), fmaxf(v[u].z, v[u].w)) * zscale;
-        if (mz > m) {
-          s *= ex2(m - mz);
-          m = mz;
-        }
-        const float nm = -m;
-        s += ex2(fmaf(v[u].x, zscale, nm)) + ex2(fmaf(v[u].y, zscale, nm)) + ex2(fmaf(v[u].z, zscale, nm)) +
-             ex2(fmaf(v[u].w, zscale, nm));
-      }
-    };
-    if constexpr (UNROLL == 16) {
-      // one CTA per SM: two batches of 8, the next one's loads in flight
-      // while the current one is summed
-      float4 va[H], vb[H];
-      int ra[H], rb[H];
-      fetch(va, ra);
-      while (ra[0] >= 0) {
-        fetch(vb, rb);
-        consume(va, ra);
-        if (rb[0] < 0) break;
-        fetch(va, ra);
-        consume(vb, rb);
-      }
-    } else {
-      float4 v[H];
-      int vr[H];
-      for (;;) {
-        fetch(v, vr);
-        if (vr[0] < 0) break;
-        consume(v, vr);
-      }
+      if (lane == 0) cta_ms[r] = make_float2(m, s);
     }
-    if (f0 + 32 * warp < f1) flush();
-  }
-  // the next kernel may be scheduled once the logits have streamed through
-  pdl_launch_next();
-  __syncthreads();
-  for (int r = tid; r < rows; r += kSampThreads) {
-    float m = kEmpty, s = 0.f;
-#pragma unroll
-    for (int w = 0; w < kSampWarps; ++w) ms_merge(m, s, part[w][r].x, part[w][r].y);
-    cta_ms[r] = make_float2(m, s);
   }
   cluster.sync();
 
@@ -523,6 +558,35 @@ __global__ void __launch_bounds__(kSampThreads, UNROLL == 8 ? 2 : 1) accept_samp
   cluster.sync();  // peers stay resident until every remote access is done
 }
 
+// Few sequences: phase 1 of each sequence split over `parts` CTAs that need
+// not be resident together; each merges its warps' pairs and writes the
+// (m, s) of every row to pre[b][part][row] (rows outside its span get the
+// empty pair).  accept_sampled_kernel then merges these instead of
+// streaming the logits itself.
+template <bool VEC>
+__global__ void __launch_bounds__(kSampThreads, 2) samp_part_kernel(const float* __restrict__ tgt,
+                                                                    const float* __restrict__ drf, float zscale,
+                                                                    int gamma, int vocab, int parts,
+                                                                    float2* __restrict__ pre) {
+  __shared__ float2 part[kSampWarps][kSampMaxRows];
+  const int b = blockIdx.x / parts, c = blockIdx.x - b * parts;
+  const int rows = 2 * gamma + 1;
+  const int tid = threadIdx.x;
+  for (int i = tid; i < kSampWarps * kSampMaxRows; i += kSampThreads)
+    part[i / kSampMaxRows][i % kSampMaxRows] = make_float2(kEmpty, 0.f);
+  pdl_wait();
+  __syncthreads();
+  phase1_span<VEC, 8>(tgt, drf, b, gamma, vocab, zscale, c, parts, part);
+  __syncthreads();
+  for (int r = tid; r < rows; r += kSampThreads) {
+    float m = kEmpty, s = 0.f;
+#pragma unroll
+    for (int w = 0; w < kSampWarps; ++w) ms_merge(m, s, part[w][r].x, part[w][r].y);
+    pre[(static_cast<size_t>(b) * parts + c) * rows + r] = make_float2(m, s);
+  }
+  pdl_launch_next();
+}
+
 struct SampCapacity {
   bool ready = false;
   int resident8[kSampMaxCluster + 1] = {};   // clusters resident at once, UNROLL 8
@@ -582,17 +646,34 @@ cudaError_t samp_capacity(const SampCapacity** out) {
 template <bool VEC, int UNROLL>
 cudaError_t launch_samp(dim3 grid, unsigned CL, cudaStream_t stream, const float* tl, const float* dl,
                         const int32_t* draft, const float* ua, const float* us, float zscale, int gamma, int vocab,
-                        int32_t* accepted_len, int32_t* out_tokens, int32_t* err_word) {
+                        int32_t* accepted_len, int32_t* out_tokens, int32_t* err_word, const float2* pre,
+                        int pre_parts) {
   return launch_overlapped(accept_sampled_kernel<VEC, UNROLL>, grid, dim3(kSampThreads), 0, stream, CL, tl, dl,
-                           draft, ua, us, zscale, gamma, vocab, accepted_len, out_tokens, err_word);
+                           draft, ua, us, zscale, gamma, vocab, accepted_len, out_tokens, err_word, pre, pre_parts);
 }
 
 }  // namespace
 
+int samp_parts(int Bt, int gamma, int vocab, int num_sms) {
+  // as for greedy acceptance: few sequences, each with at least 6 MiB of
+  // logits (target and draft rows), about 8 units of 16 bytes per thread
+  if (static_cast<long long>(Bt) * kSampMaxCluster > num_sms) return 0;
+  const long long rows = 2LL * gamma + 1;
+  if (rows * vocab * 4 < (6LL << 20)) return 0;
+  const long long units = rows * ((vocab + 3) / 4);
+  const long long parts = std::min(units / (8LL * kSampThreads), (2LL * num_sms + Bt - 1) / Bt);
+  return parts > kSampMaxCluster ? static_cast<int>(parts) : 0;
+}
+
+size_t samp_workspace_bytes(int Bt, int gamma, int vocab, int num_sms) {
+  const int parts = samp_parts(Bt, gamma, vocab, num_sms);
+  return parts ? static_cast<size_t>(Bt) * parts * (2 * gamma + 1) * sizeof(float2) : 0;
+}
+
 cudaError_t launch_accept_sampled(const float* target_logits, const float* draft_logits, const int32_t* draft,
                                   const float* u_accept, const float* u_sample, float temperature, int Bt,
                                   int gamma, int vocab, int32_t* accepted_len, int32_t* out_tokens,
-                                  int32_t* err_word, cudaStream_t stream) {
+                                  int32_t* err_word, cudaStream_t stream, void* workspace, int num_sms) {
   const SampCapacity* cap = nullptr;
   cudaError_t e = samp_capacity(&cap);
   if (e != cudaSuccess) return e;
@@ -610,15 +691,26 @@ cudaError_t launch_accept_sampled(const float* target_logits, const float* draft
   const dim3 grid(static_cast<unsigned>(Bt) * CL);
   const float zscale = kLog2e / temperature;
   const unsigned ucl = static_cast<unsigned>(CL);
+  // with a workspace and few sequences, phase 1 runs in samp_part_kernel
+  const int parts = workspace ? samp_parts(Bt, gamma, vocab, num_sms) : 0;
+  float2* pre = parts ? static_cast<float2*>(workspace) : nullptr;
+  if (parts) {
+    const dim3 pgrid(static_cast<unsigned>(Bt) * parts);
+    e = vec4 ? launch_overlapped(samp_part_kernel<true>, pgrid, dim3(kSampThreads), 0, stream, 1u, target_logits,
+                                 draft_logits, zscale, gamma, vocab, parts, pre)
+             : launch_overlapped(samp_part_kernel<false>, pgrid, dim3(kSampThreads), 0, stream, 1u, target_logits,
+                                 draft_logits, zscale, gamma, vocab, parts, pre);
+    if (e != cudaSuccess) return e;
+  }
   if (vec4)
     return deep ? launch_samp<true, 16>(grid, ucl, stream, target_logits, draft_logits, draft, u_accept, u_sample,
-                                        zscale, gamma, vocab, accepted_len, out_tokens, err_word)
+                                        zscale, gamma, vocab, accepted_len, out_tokens, err_word, pre, parts)
                 : launch_samp<true, 8>(grid, ucl, stream, target_logits, draft_logits, draft, u_accept, u_sample,
-                                       zscale, gamma, vocab, accepted_len, out_tokens, err_word);
+                                       zscale, gamma, vocab, accepted_len, out_tokens, err_word, pre, parts);
   return deep ? launch_samp<false, 16>(grid, ucl, stream, target_logits, draft_logits, draft, u_accept, u_sample,
-                                       zscale, gamma, vocab, accepted_len, out_tokens, err_word)
+                                       zscale, gamma, vocab, accepted_len, out_tokens, err_word, pre, parts)
               : launch_samp<false, 8>(grid, ucl, stream, target_logits, draft_logits, draft, u_accept, u_sample,
-                                      zscale, gamma, vocab, accepted_len, out_tokens, err_word);
+                                      zscale, gamma, vocab, accepted_len, out_tokens, err_word, pre, parts);
 }
 
 }  // namespace simsd

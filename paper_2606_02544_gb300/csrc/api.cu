@@ -341,9 +341,12 @@ int simsd_accept_ws(const float* logits, const int32_t* draft, int Bt, int gamma
                      workspace_bytes, err_word, stream);
 }
 
-int simsd_accept_sampled(const float* target_logits, const float* draft_logits, const int32_t* draft,
-                         const float* u_accept, const float* u_sample, float temperature, int Bt, int gamma,
-                         int vocab, int32_t* accepted_len, int32_t* out_tokens, int32_t* err_word, void* stream) {
+namespace {
+
+int accept_sampled_impl(const float* target_logits, const float* draft_logits, const int32_t* draft,
+                        const float* u_accept, const float* u_sample, float temperature, int Bt, int gamma, int vocab,
+                        int32_t* accepted_len, int32_t* out_tokens, bool ws_ok, void* workspace,
+                        size_t workspace_bytes, int32_t* err_word, void* stream) {
   if (Bt < 0) return arg_fail("Bt < 0");
   if (gamma < 1 || gamma > 32) return arg_fail("gamma must be in [1, 32]");
   if (vocab < 1 || vocab > (1 << 24)) return arg_fail("vocab must be in [1, 2^24]");
@@ -354,10 +357,40 @@ int simsd_accept_sampled(const float* target_logits, const float* draft_logits, 
   DeviceInfo info;
   int rc = require_sm103(&info);
   if (rc != SIMSD_OK) return rc;
+  const size_t need = ws_ok ? simsd::samp_workspace_bytes(Bt, gamma, vocab, info.num_sms) : 0;
+  if (need > 0) {
+    if (!workspace || workspace_bytes < need)
+      return arg_fail("workspace smaller than simsd_accept_sampled_workspace_bytes()");
+    if ((reinterpret_cast<uintptr_t>(workspace) & 7u) != 0) return arg_fail("workspace not 8-byte aligned");
+  }
   cudaError_t e = simsd::launch_accept_sampled(target_logits, draft_logits, draft, u_accept, u_sample, temperature,
                                                Bt, gamma, vocab, accepted_len, out_tokens, err_word,
-                                               as_stream(stream));
+                                               as_stream(stream), need > 0 ? workspace : nullptr, info.num_sms);
   return e == cudaSuccess ? SIMSD_OK : cuda_fail(e, "accept_sampled launch");
+}
+
+}  // namespace
+
+int simsd_accept_sampled(const float* target_logits, const float* draft_logits, const int32_t* draft,
+                         const float* u_accept, const float* u_sample, float temperature, int Bt, int gamma,
+                         int vocab, int32_t* accepted_len, int32_t* out_tokens, int32_t* err_word, void* stream) {
+  return accept_sampled_impl(target_logits, draft_logits, draft, u_accept, u_sample, temperature, Bt, gamma, vocab,
+                             accepted_len, out_tokens, false, nullptr, 0, err_word, stream);
+}
+
+size_t simsd_accept_sampled_workspace_bytes(int Bt, int gamma, int vocab) {
+  if (Bt <= 0 || gamma < 1 || gamma > 32 || vocab < 1 || vocab > (1 << 24)) return 0;
+  DeviceInfo info;
+  if (require_sm103(&info) != SIMSD_OK) return 0;
+  return simsd::samp_workspace_bytes(Bt, gamma, vocab, info.num_sms);
+}
+
+int simsd_accept_sampled_ws(const float* target_logits, const float* draft_logits, const int32_t* draft,
+                            const float* u_accept, const float* u_sample, float temperature, int Bt, int gamma,
+                            int vocab, int32_t* accepted_len, int32_t* out_tokens, void* workspace,
+                            size_t workspace_bytes, int32_t* err_word, void* stream) {
+  return accept_sampled_impl(target_logits, draft_logits, draft, u_accept, u_sample, temperature, Bt, gamma, vocab,
+                             accepted_len, out_tokens, true, workspace, workspace_bytes, err_word, stream);
 }
 
 int simsd_kv_commit(int dtype, const void* k_new, const void* v_new, int L, const int32_t* tau,

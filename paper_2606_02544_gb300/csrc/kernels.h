@@ -43,10 +43,14 @@ cudaError_t launch_accept_parts(const float* logits, const int32_t* draft, int B
                                 int32_t* accepted_len, int32_t* out_tokens, int32_t* row_argmax, void* workspace,
                                 int32_t* err_word, int num_sms, cudaStream_t stream);
 
+// workspace (may be null): with samp_workspace_bytes() > 0 bytes, phase 1
+// of few sequences is split over many CTAs (samp_part_kernel) first.
+int samp_parts(int Bt, int gamma, int vocab, int num_sms);
+size_t samp_workspace_bytes(int Bt, int gamma, int vocab, int num_sms);
 cudaError_t launch_accept_sampled(const float* target_logits, const float* draft_logits, const int32_t* draft,
                                   const float* u_accept, const float* u_sample, float temperature, int Bt,
                                   int gamma, int vocab, int32_t* accepted_len, int32_t* out_tokens,
-                                  int32_t* err_word, cudaStream_t stream);
+                                  int32_t* err_word, cudaStream_t stream, void* workspace, int num_sms);
 
 cudaError_t launch_kv_commit(int elem_bytes, const void* k_new, const void* v_new, int L, const int32_t* tau,
                              const uint8_t* section, const int32_t* accepted_len, void* k_cache, void* v_cache,

@@ -26,7 +26,8 @@ STEP_UNDRAFTED, STEP_DECODED = -1, -2
 
 EXPORTED = ("simsd_build_mask", "simsd_verify_workspace_bytes", "simsd_verify_attention",
             "simsd_verify_attention_noalloc", "simsd_accept", "simsd_accept_workspace_bytes", "simsd_accept_ws",
-            "simsd_accept_sampled", "simsd_kv_commit",
+            "simsd_accept_sampled", "simsd_accept_sampled_workspace_bytes", "simsd_accept_sampled_ws",
+            "simsd_kv_commit",
             "simsd_check_error", "simsd_debug_expire_next_wait",
             "simsd_last_error", "simsd_version")
 DEBUG_WAIT_ATTENTION, DEBUG_WAIT_ACCEPT = 1, 2
@@ -64,6 +65,9 @@ def load_library(path: str = LIB_PATH):
             lib.simsd_accept_workspace_bytes.restype = Z
             lib.simsd_accept_ws.argtypes = [P, P, I, I, I, P, P, P, P, Z, P, P]
             lib.simsd_accept_sampled.argtypes = [P, P, P, P, P, F, I, I, I, P, P, P, P]
+            lib.simsd_accept_sampled_workspace_bytes.argtypes = [I, I, I]
+            lib.simsd_accept_sampled_workspace_bytes.restype = Z
+            lib.simsd_accept_sampled_ws.argtypes = [P, P, P, P, P, F, I, I, I, P, P, P, Z, P, P]
             lib.simsd_kv_commit.argtypes = [I, P, P, I, P, P, P, F, P, P, P, I, P, I, I, P, I, I, I, I, P, P]
             lib.simsd_check_error.argtypes = [P, P, P]
             lib.simsd_debug_expire_next_wait.argtypes = [I, ctypes.c_uint]
@@ -209,3 +213,20 @@ def simsd_check_error(err_word, stream=None):
     if rc not in (SIMSD_OK, SIMSD_ERR_DEVICE):
         _check(rc, "simsd_check_error")
     return int(w.value)
+
+
+def simsd_accept_sampled_workspace_bytes(Bt, gamma, vocab) -> int:
+    return int(load_library().simsd_accept_sampled_workspace_bytes(Bt, gamma, vocab))
+
+
+def simsd_accept_sampled_ws(target_logits, draft_logits, draft, u_accept, u_sample, accepted_len, out_tokens,
+                            workspace=None, temperature=1.0, err_word=None, stream=None):
+    """simsd_accept_sampled with a caller workspace (uint8 device tensor of
+    simsd_accept_sampled_workspace_bytes() bytes, or None when that is 0)."""
+    Bt, rows, V = target_logits.shape
+    nbytes = workspace.numel() * workspace.element_size() if workspace is not None else 0
+    rc = load_library().simsd_accept_sampled_ws(_p(target_logits), _p(draft_logits), _p(draft), _p(u_accept),
+                                                _p(u_sample), float(temperature), Bt, rows - 1, V, _p(accepted_len),
+                                                _p(out_tokens), _p(workspace), nbytes, _p(err_word),
+                                                _stream(stream))
+    _check(rc, "simsd_accept_sampled_ws")
