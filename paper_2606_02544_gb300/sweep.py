@@ -109,10 +109,13 @@ def run_point(w: inputs.Workload, steps: int, peak: float) -> dict:
 
 
 def run_sampled_point(Bt: int, gamma: int, vocab: int, steps: int, peak: float) -> dict:
-    """Times simsd_accept_sampled alone (Sec. 3.2, Eq. (2)): one CUDA graph
-    of `steps` launches, L2 flushed before each when the logits fit in 4x L2,
-    every launch timed by events inside the graph."""
+    """Times simsd_accept_sampled_ws alone (Sec. 3.2, Eq. (2); few long
+    sequences split their log-sum-exp pass over many CTAs): one CUDA graph of
+    `steps` calls, L2 flushed before each when the logits fit in 4x L2, every
+    call timed by events inside the graph."""
     si = inputs.make_sampled_inputs(Bt, gamma, vocab, seed=Bt * 100 + gamma, device="cuda")
+    ws = simsd.simsd_accept_sampled_workspace_bytes(Bt, gamma, vocab)
+    work = torch.empty(ws, dtype=torch.uint8, device="cuda") if ws else None
     a = torch.empty(Bt, dtype=torch.int32, device="cuda")
     ot = torch.empty(Bt, gamma + 1, dtype=torch.int32, device="cuda")
     err = torch.zeros(1, dtype=torch.int32, device="cuda")
@@ -122,8 +125,8 @@ def run_sampled_point(Bt: int, gamma: int, vocab: int, steps: int, peak: float) 
     ev = [[torch.cuda.Event(enable_timing=True, external=True) for _ in range(2)] for _ in range(steps)]
 
     def call():
-        simsd.simsd_accept_sampled(si.target_logits, si.draft_logits, si.draft, si.u_accept, si.u_sample, a, ot,
-                                   temperature=si.temperature, err_word=err)
+        simsd.simsd_accept_sampled_ws(si.target_logits, si.draft_logits, si.draft, si.u_accept, si.u_sample, a, ot,
+                                      work, temperature=si.temperature, err_word=err)
 
     stream = torch.cuda.Stream()
     stream.wait_stream(torch.cuda.current_stream())
@@ -149,7 +152,8 @@ def run_sampled_point(Bt: int, gamma: int, vocab: int, steps: int, peak: float) 
     assert simsd.simsd_check_error(err) == 0
     t = statistics.median(ts)
     gbs = nbytes / (t * 1e-3) / 1e9
-    row = {"kernel": "accept_sampled", "Bt": Bt, "gamma": gamma, "vocab": vocab, "us": round(t * 1e3, 2),
+    row = {"kernel": "accept_sampled" + ("+parts" if ws else ""), "Bt": Bt, "gamma": gamma, "vocab": vocab,
+           "us": round(t * 1e3, 2),
            "algorithmic_bytes": nbytes, "gbs": round(gbs, 1), "frac": round(gbs / peak, 4),
            "l2": "flushed" if need_flush else "larger than L2"}
     del g, si, flush
@@ -208,9 +212,11 @@ def main(argv=None):
                 rows.append(row)
         if args.out:
             with open(args.out, "w") as f:
-                f.write(f"| Bt | gamma | us | GB/s (rows read once) | of {peak:.0f} GB/s |\n|---|---|---|---|---|\n")
+                f.write(f"| Bt | gamma | path | us | GB/s (rows read once) | of {peak:.0f} GB/s |\n"
+                        "|---|---|---|---|---|---|\n")
                 for r in rows:
-                    f.write(f"| {r['Bt']} | {r['gamma']} | {r['us']:.1f} | {r['gbs']:.0f} | "
+                    path = "parts + cluster" if r["kernel"].endswith("+parts") else "cluster"
+                    f.write(f"| {r['Bt']} | {r['gamma']} | {path} | {r['us']:.1f} | {r['gbs']:.0f} | "
                             f"{100 * r['frac']:.1f}% |\n")
         return
     for w in points(bts, ns, gs, ps, args):
