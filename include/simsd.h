@@ -272,7 +272,8 @@ SIMSD_API int simsd_accept_sampled(const float* target_logits, const float* draf
  * simsd_accept_sampled_workspace_bytes / simsd_accept_sampled_ws -- the same
  * stochastic acceptance with a caller workspace.  For few sequences (at most
  * num_SMs / 16) holding at least 6 MiB of logits each (target and draft
- * rows), the log-sum-exp pass over every row is split over more CTAs than one
+ * rows; 12 MiB when there are more than num_SMs / 32 sequences), the
+ * log-sum-exp pass over every row is split over more CTAs than one
  * cluster per sequence holds: a first launch writes per-row (max, sum) pairs
  * of each part to the workspace, which the cluster of each sequence merges
  * before it forms alpha_r and draws the token as simsd_accept_sampled does.

@@ -27,21 +27,23 @@ def _gpu_ws(si):
 
 
 @pytest.mark.parametrize("Bt,gamma,V,T,eta", [
-    (1, 8, 151936, 1.0, 0.5), (1, 32, 151936, 1.0, 0.3), (3, 16, 151936, 0.7, 0.5), (8, 8, 151936, 1.0, 0.4),
-    (9, 5, 151936, 1.3, 0.5), (2, 16, 151935, 1.0, 0.5),
+    (1, 8, 151936, 1.0, 0.5), (1, 32, 151936, 1.0, 0.3), (3, 16, 151936, 0.7, 0.5), (8, 16, 151936, 1.0, 0.4),
+    (9, 12, 151936, 1.3, 0.5), (2, 16, 151935, 1.0, 0.5),
 ])
 def test_split_matches_oracle(monkeypatch, Bt, gamma, V, T, eta):
-    # at most SMs / 16 sequences with at least 6 MiB of logits each: split
+    # at most SMs / 16 sequences with at least 6 MiB of logits each (12 MiB
+    # past SMs / 32 sequences): split
     assert simsd.simsd_accept_sampled_workspace_bytes(Bt, gamma, V) > 0
     si = inputs.make_sampled_inputs(Bt, gamma, V, seed=Bt * 31 + gamma, eta=eta, temperature=T, device="cuda")
     monkeypatch.setattr(base, "_gpu", _gpu_ws)
     base._compare(si)
 
 
-@pytest.mark.parametrize("Bt,gamma,V", [(8, 4, 151936), (16, 8, 151936), (1, 4, 1024)])
+@pytest.mark.parametrize("Bt,gamma,V", [(8, 4, 151936), (8, 8, 151936), (16, 8, 151936), (1, 4, 1024)])
 def test_no_split_is_the_cluster_kernel(monkeypatch, Bt, gamma, V):
-    # under 6 MiB a sequence, or more sequences than SMs / 16: no workspace,
-    # the same bits as simsd_accept_sampled
+    # under 6 MiB a sequence (12 MiB past SMs / 32 sequences), or more
+    # sequences than SMs / 16: no workspace, the same bits as
+    # simsd_accept_sampled
     assert simsd.simsd_accept_sampled_workspace_bytes(Bt, gamma, V) == 0
     si = inputs.make_sampled_inputs(Bt, gamma, V, seed=Bt + gamma, device="cuda")
     got = _gpu_ws(si)
