@@ -37,6 +37,11 @@ __global__ void __launch_bounds__(kF32Warps * 32) attention_f32_kernel(const __g
 
   const int n = a.prefix_len[b];
   const uint8_t si = a.section[static_cast<size_t>(b) * S + s];
+  const int ti = a.tau[static_cast<size_t>(b) * S + s];
+  // the page id of this lane's key in the warp's first chunk, loaded beside
+  // n (entries past the prefix are read but not used)
+  const int pi0 = (32 * wib + lane) / a.page_size;
+  const int pg0 = pi0 < a.max_pages ? a.block_table[static_cast<size_t>(b) * a.max_pages + pi0] : -1;
   if (wib == 0) {
     bool ok = n >= 0 && static_cast<long long>(n) <= static_cast<long long>(a.max_pages) * a.page_size;
     if (!ok && lane == 0 && s == 0 && h == 0) raise_error(a.err_word, SIMSD_EW_PREFIX_LEN);
@@ -60,7 +65,6 @@ __global__ void __launch_bounds__(kF32Warps * 32) attention_f32_kernel(const __g
     for (int c = threadIdx.x; c < d; c += blockDim.x) o[c] = 0.f;
     return;
   }
-  const int ti = a.tau[static_cast<size_t>(b) * S + s];
   if (a.rope_pos) {
     const int pos = a.rope_pos[static_cast<size_t>(b) * S + s];
     for (int i = threadIdx.x; i < d / 2; i += blockDim.x) {
@@ -83,7 +87,7 @@ __global__ void __launch_bounds__(kF32Warps * 32) attention_f32_kernel(const __g
     long long voff = -1;
     bool from_cache = false;
     if (j < n) {
-      const int pg = a.block_table[static_cast<size_t>(b) * a.max_pages + j / a.page_size];
+      const int pg = base == 32 * wib ? pg0 : a.block_table[static_cast<size_t>(b) * a.max_pages + j / a.page_size];
       voff = ((static_cast<long long>(pg) * a.Hkv + kvh) * a.page_size + (j % a.page_size)) * d;
       kr = a.k_cache + voff;
       from_cache = true;
@@ -145,14 +149,17 @@ __global__ void __launch_bounds__(kF32Warps * 32) attention_f32_kernel(const __g
     l = l * corr + ps;
 #pragma unroll
     for (int c = 0; c < DPL; ++c) acc[c] *= corr;
-    // P.V of the chunk, 8 keys at a time so that their V loads overlap
+    // P.V of the chunk, kRound keys at a time so that their V loads are in
+    // flight together (read cold, each round costs a DRAM round trip): all 32
+    // at d = 64, 8 at d = 128 (more would spill); the FMAs run in key order
+    constexpr int kRound = DPL <= 2 ? 32 : 8;
     const float* vrow = kr ? (from_cache ? a.v_cache : a.v_new) + voff : a.v_new;
 #pragma unroll 1
-    for (int j0 = 0; j0 < 32; j0 += 8) {
-      float vv[8][DPL], pj[8];
-      bool use[8];
+    for (int j0 = 0; j0 < 32; j0 += kRound) {
+      float vv[kRound][DPL], pj[kRound];
+      bool use[kRound];
 #pragma unroll
-      for (int u = 0; u < 8; ++u) {
+      for (int u = 0; u < kRound; ++u) {
         const float* vr = reinterpret_cast<const float*>(
             __shfl_sync(0xffffffffu, reinterpret_cast<uintptr_t>(vrow), j0 + u));
         pj[u] = __shfl_sync(0xffffffffu, pr, j0 + u);
@@ -161,7 +168,7 @@ __global__ void __launch_bounds__(kF32Warps * 32) attention_f32_kernel(const __g
         for (int c = 0; c < DPL; ++c) vv[u][c] = use[u] ? __ldg(vr + lane + 32 * c) : 0.f;
       }
 #pragma unroll
-      for (int u = 0; u < 8; ++u)
+      for (int u = 0; u < kRound; ++u)
 #pragma unroll
         for (int c = 0; c < DPL; ++c) acc[c] = use[u] ? fmaf(pj[u], vv[u][c], acc[c]) : acc[c];
     }
