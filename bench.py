@@ -54,27 +54,37 @@ def _peaks():
         return 6800.0, 1900.0, "fallback"
 
 
-def _kernel_sha():
+# the sources each stored traffic figure depends on: a kernel's own file and
+# the headers it includes
+TRAFFIC_SOURCES = {
+    "attention": ("attention_tc.cu", "ptx.cuh", "common.cuh"),
+    "accept": ("accept.cu", "ptx.cuh", "common.cuh"),
+    "attention_tc256": ("attention_tc256.cu", "ptx.cuh", "common.cuh"),
+}
+
+
+def _kernel_sha(kernel):
     h = hashlib.sha256()
-    for fn in ("attention_tc.cu", "attention_tc256.cu", "ptx.cuh", "common.cuh", "accept.cu"):
+    for fn in TRAFFIC_SOURCES[kernel]:
         with open(os.path.join(ROOT, "paper_2606_02544_gb300", "csrc", fn), "rb") as f:
             h.update(f.read())
     return h.hexdigest()[:16]
 
 
 TRAFFIC_SOURCE = ("stored: profiles/traffic.json (ncu dram__bytes_read.sum + dram__bytes_write.sum per launch), "
-                  "used only while the kernel sources hash to the value recorded there")
+                  "used only while the kernel's sources hash to the value recorded there")
 
 
 def _traffic(workload, kernel):
     """DRAM bytes per launch from the committed ncu summary, if it was taken
-    on the current kernel sources; else None."""
+    on the kernel's current sources; else None."""
     try:
         with open(os.path.join(ROOT, "profiles", "traffic.json")) as f:
             d = json.load(f)
-        if d.get("kernel_sha") != _kernel_sha():
+        entry = d.get(kernel, {})
+        if entry.get("sha") != _kernel_sha(kernel):
             return None
-        return d.get(kernel, {}).get(workload)
+        return entry.get(workload)
     except Exception:
         return None
 
