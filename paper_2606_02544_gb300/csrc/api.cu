@@ -163,6 +163,11 @@ int verify_attention_impl(int dtype, const void* q, const void* k_new, const voi
   if (!simsd::plan_attention_tc(Bt, gamma, Hq, Hkv, max_pages, page_size, info.num_sms, &plan))
     return unsupported("query rows per KV head: need 2*gamma*Hq/Hkv <= 128 or 128 % (Hq/Hkv) == 0");
   if (static_scratch) {
+    if (plan.streamk && plan.ws_bytes > simsd::noalloc_scratch_capacity()) {
+      // the whole-unit walk needs no scratch
+      plan.streamk = 0;
+      plan.ws_bytes = 0;
+    }
     if (plan.ws_bytes > simsd::noalloc_scratch_capacity()) {
       std::snprintf(g_last_error, sizeof(g_last_error),
                     "unsupported: these sizes need %zu bytes of scratch, more than the %zu-byte static array; "

@@ -972,11 +972,12 @@ bool plan_attention_tc(int Bt, int gamma, int Hq, int Hkv, int max_pages, int pa
     // the combine kernel merges
     pl.kind = 1;
     pl.nsplit = ns256;
+    pl.streamk = ns256 == 1 ? tc256_streamk(Bt, Hkv, max_tiles, num_sms) : 0;
     pl.sort = 0;
     pl.fuse = 0;
     pl.slots = num_sms;
     pl.ws_bytes = ns256 > 1 ? static_cast<size_t>(Bt) * Hkv * pl.rb * ns256 * pl.rows_blk * (kD + 2) * sizeof(float)
-                            : 0;
+                            : (pl.streamk ? tc256_streamk_bytes(num_sms) : 0);
     *plan = pl;
     return true;
   }

@@ -10,11 +10,20 @@
 // tensor pipe must stay busy while the softmax runs, so S is double-buffered
 // per row block: the MMAs of tile i+1 run while the softmax works on tile i.
 //
-// The kernel is persistent: one CTA per SM (512 TMEM columns, ~197 KB of
-// shared memory) walks units blockIdx.x, blockIdx.x + gridDim.x, ... in
-// longest-prefix-first order.  Tensor memory, barriers and the K/V ring
-// carry over from unit to unit; the producer loads the next unit's Q and
-// tiles while the softmax warps finish the previous one.
+// The kernel is persistent: one CTA per SM (512 TMEM columns, ~227 KB of
+// shared memory) walks pieces of units.  Tensor memory, barriers and the
+// K/V ring carry over from piece to piece; the producer loads the next
+// piece's Q and tiles while the softmax warps finish the previous one.  Two
+// walks:
+//   ranges: units (or, with fewer units than SMs, equal key-tile ranges of
+//     every unit) blockIdx.x, blockIdx.x + gridDim.x, ... in
+//     longest-prefix-first order;
+//   stream-K: the key tiles of all units, end to end, cut into gridDim.x
+//     runs of equal length; a CTA takes the pieces of the units its run
+//     overlaps.  Every SM then streams the same number of tiles, where whole
+//     units would leave some SMs with one unit more than others (256 units
+//     on 152 SMs: 104 take two, 48 one).  A unit cut by run boundaries
+//     leaves partial results that streamk_combine_kernel merges.
 //
 // Warp roles (512 threads):
 //   warps 0-3  softmax of row block A, warps 4-7 of row block B; thread i of
@@ -71,6 +80,7 @@ constexpr int kSlotBytes = 4 * kHalfBytes;   // K0 K1 V0 V1
 constexpr int kQHalfBytes = kRows * 128;     // 128 rows x 64 bf16
 constexpr int kQBlockBytes = 2 * kQHalfBytes;
 constexpr int kMaxSort = 256;                // sequences ranked by prefix length (longest first)
+constexpr int kMaxStreamK = kMaxSort - 1;    // stream-K: tile offsets of Bt + 1 sequences in `order`
 constexpr float kRescaleThreshold = 8.0f;    // log2 units: rescale when the max grows by > 2^8
 static_assert(kTile == 64, "the softmax reductions are written out for 64 keys");
 
@@ -87,8 +97,10 @@ struct Tc256Params {
   int units;   // Bt * Hkv
   int nsplit;  // key-tile ranges per unit (work items = units * nsplit)
   int items;
-  float* ws;   // nsplit > 1: partial O, (m, l) of each row block and range (the combine's layout)
-  int sort;    // rank sequences by prefix length (Bt <= kMaxSort)
+  int streamk;  // 1: equal runs of the global key-tile sequence per CTA (Bt <= kMaxStreamK)
+  int ctas;     // grid size (stream-K partial slots: 2 per CTA)
+  float* ws;    // partial O, (m, l) of split units (layouts at partial_entry)
+  int sort;     // rank sequences by prefix length (Bt <= kMaxSort)
   float scale_log2;
   unsigned long long wait_ns;
   uint32_t extra_p;  // planted extra arrivals on bar_p (a test of the bounded waits)
@@ -111,7 +123,7 @@ struct alignas(1024) Smem256 {
   int bad[2];           // per unit parity: a needed page id is out of range
   int32_t tau[2][64];   // per unit parity: slot labels of the unit's sequence
   uint8_t sect[2][64];
-  int32_t order[kMaxSort];
+  int32_t order[kMaxSort];  // ranking, or (stream-K) tile offsets of the sequences
 };
 
 constexpr size_t smem_bytes() { return sizeof(Smem256) + 1024; }
@@ -147,6 +159,16 @@ __device__ __forceinline__ void rope_chunk_pair(uint4* pa, uint4* pb, int pos, i
   *pb = make_uint4(wb[0], wb[1], wb[2], wb[3]);
 }
 
+// Tiles of a unit of a sequence with prefix length n: ceil(n / 64) + 1 (tile
+// 0: the new slots); stream-K counts one for a length out of range (a piece
+// that only zeroes the unit's rows).
+__device__ __forceinline__ bool prefix_bad(const Tc256Params& p, int n) {
+  return n < 0 || static_cast<long long>(n) > static_cast<long long>(p.max_pages) * p.page_size;
+}
+__device__ __forceinline__ int streamk_tiles(const Tc256Params& p, int n) {
+  return prefix_bad(p, n) ? 1 : (n + kTile - 1) / kTile + 1;
+}
+
 // The work item at position U of the walk: key-tile range `split` of the
 // unit (sequence b, KV head), sequences longest prefix first when ranked.
 // A unit has T = ceil(n / 64) + 1 tiles (tile 0: the new slots, 1..: the
@@ -155,6 +177,10 @@ __device__ __forceinline__ void rope_chunk_pair(uint4* pa, uint4* pb, int pos, i
 struct Unit {
   int b, kvh, n, split, t0, tiles;
   bool n_bad;
+  bool lead;  // the piece that raises the unit's error bits (range 0, or the one with tile 0)
+  bool part;  // writes partial results instead of the output
+  int slot;   // stream-K: 0 for the piece at the start of the CTA's run, else 1
+  bool last;  // the CTA's last piece
 };
 
 __device__ __forceinline__ Unit unit_at(const Tc256Params& p, const Smem256& sm, int U) {
@@ -165,7 +191,7 @@ __device__ __forceinline__ Unit unit_at(const Tc256Params& p, const Smem256& sm,
   u.kvh = unit - rank * p.Hkv;
   u.b = p.sort ? sm.order[rank] : rank;
   u.n = p.prefix_len[u.b];
-  u.n_bad = u.n < 0 || static_cast<long long>(u.n) > static_cast<long long>(p.max_pages) * p.page_size;
+  u.n_bad = prefix_bad(p, u.n);
   // T < 2^25 and split < 64: the products fit 32 bits
   const unsigned T = u.n_bad ? 0u : static_cast<unsigned>((u.n + kTile - 1) / kTile + 1);
   const unsigned ns = static_cast<unsigned>(p.nsplit), sp = static_cast<unsigned>(u.split);
@@ -174,18 +200,147 @@ __device__ __forceinline__ Unit unit_at(const Tc256Params& p, const Smem256& sm,
   return u;
 }
 
-// Partial results of a split unit, in the layout the combine kernel reads:
-// O (unnormalised, fp32) [units * 2 * nsplit][128][d], then (m, l)
-// [units * 2 * nsplit][128][2]; entry ((b Hkv + kvh) 2 + x) nsplit + split,
-// row `row` of block x.  m is the row's reference maximum in log2 units.
+// cum[b] = key tiles of the units of sequences 0 .. b-1 (Hkv units each),
+// cum[Bt] = all of them (below 2^30, as the planner checks).  Called by
+// every thread of the block; Bt <= 255.
+__device__ void streamk_offsets(const Tc256Params& p, int32_t* cum) {
+  for (int b = threadIdx.x; b < p.Bt; b += blockDim.x) cum[b + 1] = p.Hkv * streamk_tiles(p, p.prefix_len[b]);
+  __syncthreads();
+  if (threadIdx.x < 32) {
+    // lane l scans entries 8l + 1 .. 8l + 8
+    const int lane = threadIdx.x;
+    int v[8], sum = 0;
+#pragma unroll
+    for (int j = 0; j < 8; ++j) {
+      const int i = 8 * lane + j + 1;
+      v[j] = i <= p.Bt ? cum[i] : 0;
+      sum += v[j];
+    }
+    int inc = sum;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+      const int y = __shfl_up_sync(0xffffffffu, inc, o);
+      if (lane >= o) inc += y;
+    }
+    int run = inc - sum;
+#pragma unroll
+    for (int j = 0; j < 8; ++j) {
+      const int i = 8 * lane + j + 1;
+      run += v[j];
+      if (i <= p.Bt) cum[i] = run;
+    }
+    if (lane == 0) cum[0] = 0;
+  }
+  __syncthreads();
+}
+
+// The sequence whose units hold global tile G: cum[b] <= G < cum[b + 1]
+// (every sequence holds at least Hkv tiles, so b is unique).
+__device__ __forceinline__ int streamk_seq(const int32_t* cum, int Bt, int G) {
+  int lo = 0, hi = Bt - 1;
+  while (lo < hi) {
+    const int mid = (lo + hi + 1) >> 1;
+    if (cum[mid] <= G)
+      lo = mid;
+    else
+      hi = mid - 1;
+  }
+  return lo;
+}
+
+// A CTA's walk: the next item of the ranges walk, or the next tile of its
+// stream-K run [R0, R1).  The run is walked from H, the first unit start in
+// it, to R1, and then [R0, H): the piece cut at the run's start comes last,
+// so that both pieces of a unit cut by a boundary are written near the end
+// of the launch (and stay in L2 for the merge).
+struct Walk {
+  int U;  // ranges: the next item; stream-K: the phase (0: [H, R1), 1: [R0, H))
+  int G, R0, R1, H;
+};
+
+__device__ __forceinline__ Walk walk_begin(const Tc256Params& p, const Smem256& sm) {
+  Walk w;
+  w.U = blockIdx.x;
+  w.G = w.R0 = w.R1 = w.H = 0;
+  if (p.streamk) {
+    w.U = 0;
+    const int total = sm.order[p.Bt];
+    const int W = (total + static_cast<int>(gridDim.x) - 1) / static_cast<int>(gridDim.x);
+    w.R0 = static_cast<int>(min(static_cast<long long>(total), static_cast<long long>(blockIdx.x) * W));
+    w.R1 = min(total, w.R0 + W);
+    w.H = w.R0;
+    if (w.R0 < w.R1) {
+      const int b = streamk_seq(sm.order, p.Bt, w.R0);
+      const int T = streamk_tiles(p, p.prefix_len[b]);
+      const int t = (w.R0 - sm.order[b]) % T;
+      if (t > 0) w.H = min(w.R1, w.R0 - t + T);
+    }
+    w.G = w.H;
+  }
+  return w;
+}
+
+// The CTA's next piece; false when its walk is done.  Every role walks the
+// same pieces in the same order.
+__device__ __forceinline__ bool walk_next(const Tc256Params& p, const Smem256& sm, Walk& w, Unit& u) {
+  if (!p.streamk) {
+    if (w.U >= p.items) return false;
+    u = unit_at(p, sm, w.U);
+    w.U += gridDim.x;
+    u.lead = u.split == 0;
+    u.part = p.nsplit > 1;
+    u.slot = 0;
+    u.last = w.U >= p.items;
+    return true;
+  }
+  if (w.U == 0 && w.G >= w.R1) {
+    w.U = 1;  // then the piece cut at the run's start
+    w.G = w.R0;
+  }
+  if (w.U == 1 && w.G >= w.H) return false;
+  const int end = w.U == 0 ? w.R1 : w.H;
+  const int b = streamk_seq(sm.order, p.Bt, w.G);
+  u.b = b;
+  u.n = p.prefix_len[b];
+  u.n_bad = prefix_bad(p, u.n);
+  const int T = u.n_bad ? 1 : (u.n + kTile - 1) / kTile + 1;
+  const int off = w.G - sm.order[b];
+  u.kvh = off / T;
+  u.t0 = off - u.kvh * T;
+  const int take = min(T - u.t0, end - w.G);
+  u.split = 0;
+  u.tiles = u.n_bad ? 0 : take;
+  u.lead = u.t0 == 0;
+  u.part = take < T;
+  u.slot = w.G == w.R0 ? 0 : 1;
+  w.G += take;
+  u.last = w.U == 1 ? w.G >= w.H : (w.G >= w.R1 && w.H == w.R0);
+  return true;
+}
+
+// Partial results of a split unit: O (unnormalised, fp32) [entries][128][d],
+// then (m, l) [entries][128][2], row `row` of block x; m is the row's
+// reference maximum in log2 units.  Ranges walk (the combine kernel's
+// layout): entries = units * 2 * nsplit, entry ((b Hkv + kvh) 2 + x) nsplit
+// + split.  Stream-K: entries = ctas * 4, entry (cta * 2 + slot) * 2 + x.
+__device__ __forceinline__ size_t partial_entries(const Tc256Params& p) {
+  return p.streamk ? static_cast<size_t>(p.ctas) * 4 : static_cast<size_t>(p.units) * 2 * p.nsplit;
+}
+__device__ __forceinline__ size_t partial_entry(const Tc256Params& p, const Unit& u, int x) {
+  if (p.streamk) return (static_cast<size_t>(blockIdx.x) * 2 + u.slot) * 2 + x;
+  return ((static_cast<size_t>(u.b) * p.Hkv + u.kvh) * 2 + x) * p.nsplit + u.split;
+}
 __device__ __forceinline__ float* partial_o(const Tc256Params& p, const Unit& u, int x, int row) {
-  const size_t e = ((static_cast<size_t>(u.b) * p.Hkv + u.kvh) * 2 + x) * p.nsplit + u.split;
-  return p.ws + (e * kRows + row) * kD;
+  return p.ws + (partial_entry(p, u, x) * kRows + row) * kD;
 }
 __device__ __forceinline__ float* partial_ml(const Tc256Params& p, const Unit& u, int x, int row) {
-  const size_t e = ((static_cast<size_t>(u.b) * p.Hkv + u.kvh) * 2 + x) * p.nsplit + u.split;
-  const size_t entries = static_cast<size_t>(p.units) * 2 * p.nsplit;
-  return p.ws + entries * kRows * kD + (e * kRows + row) * 2;
+  return p.ws + partial_entries(p) * kRows * kD + (partial_entry(p, u, x) * kRows + row) * 2;
+}
+// Stream-K: after the partials, one record per run boundary c (int4): the
+// unit that boundary c is the first to cut (b Hkv + kvh, or -1), the CTAs
+// c0 .. c1 holding its pieces and the slot of CTA c0's piece.
+__device__ __forceinline__ int4* streamk_records(const Tc256Params& p) {
+  return reinterpret_cast<int4*>(p.ws + partial_entries(p) * kRows * (kD + 2));
 }
 
 __global__ void __launch_bounds__(kThreads, 1)
@@ -251,14 +406,11 @@ __global__ void __launch_bounds__(kThreads, 1)
     // the staging area is overwritten by TMA later
     fence_proxy_async_smem();
   }
+  if (p.streamk) streamk_offsets(p, sm.order);
   tc_fence_before();
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem = sm.tmem_base;
-  const int first_unit = blockIdx.x, step = gridDim.x;
-
-  // the last unit this CTA takes (for the dependent-launch trigger)
-  const int last_unit = first_unit + ((p.items - 1 - first_unit) / step) * step;
 
   // Register split (setmaxnreg, per warpgroup): the two softmax warpgroups
   // take 200 registers a thread, the two control warpgroups give theirs
@@ -272,10 +424,11 @@ __global__ void __launch_bounds__(kThreads, 1)
       // refills a slot's half as soon as that half is released, so K runs
       // ahead of V (K is consumed a softmax earlier than V)
       const int kv = warp == kWarpProducer ? 0 : 1;
-      uint32_t g = 0, jq = 0;  // tiles and units (with tiles) issued so far
+      uint32_t g = 0, jq = 0;  // tiles and pieces (with tiles) issued so far
       bool ok = true;
-      for (int U = first_unit; ok && U < p.items; U += step) {
-        const Unit u = unit_at(p, sm, U);
+      Walk w = walk_begin(p, sm);
+      Unit u;
+      while (ok && walk_next(p, sm, w, u)) {
         if (u.tiles == 0) continue;
         if (kv == 0) {
           if (lane == 0 && jq > 0 && !mbar_wait(smem_u32(&sm.bar_qfree), (jq - 1) & 1, abort_flag, p.wait_ns))
@@ -389,8 +542,9 @@ __global__ void __launch_bounds__(kThreads, 1)
         const uint32_t ocol = tmem + kColO + 128u * x;
         uint32_t g = 0, jq = 0;
         bool ok = true;
-        for (int U = first_unit; ok && U < p.items; U += step) {
-          const Unit u = unit_at(p, sm, U);
+        Walk w = walk_begin(p, sm);
+        Unit u;
+        while (ok && walk_next(p, sm, w, u)) {
           if (u.tiles == 0) continue;
           ++jq;
           const uint32_t g0 = g, g_end = g + u.tiles;
@@ -460,9 +614,10 @@ __global__ void __launch_bounds__(kThreads, 1)
     const uint32_t o_tmem = lane_tmem + kColO + 128u * x;
     uint32_t g = 0, jq = 0, mu = 0;
     bool ok = true;
-    for (int U = first_unit; U < p.items; U += step, ++mu) {
-      const Unit u = unit_at(p, sm, U);
-      const int par = mu & 1;  // metadata buffer of this unit
+    Walk w = walk_begin(p, sm);
+    Unit u;
+    for (; walk_next(p, sm, w, u); ++mu) {
+      const int par = mu & 1;  // metadata buffer of this piece
       // every softmax thread is done with the previous unit: its flag
       // (the other buffer) is cleared for the next one
       asm volatile("bar.sync 1, 256;" ::: "memory");
@@ -472,7 +627,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         sm.sect[par][tid] = p.section[static_cast<size_t>(u.b) * p.S + tid];
       }
       if (u.n_bad) {
-        if (tid == 0 && u.kvh == 0 && u.split == 0) raise_error(p.err_word, SIMSD_EW_PREFIX_LEN);
+        if (tid == 0 && u.kvh == 0 && u.lead) raise_error(p.err_word, SIMSD_EW_PREFIX_LEN);
       } else {
         const int npages = (u.n + p.page_size - 1) / p.page_size;
         const int32_t* bt = p.block_table + static_cast<size_t>(u.b) * p.max_pages;
@@ -483,7 +638,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
         if (bad) {
           atomicOr(&sm.bad[par], 1);
-          if (u.kvh == 0 && u.split == 0) raise_error(p.err_word, SIMSD_EW_PAGE);
+          if (u.kvh == 0 && u.lead) raise_error(p.err_word, SIMSD_EW_PAGE);
         }
       }
       asm volatile("bar.sync 1, 256;" ::: "memory");
@@ -654,7 +809,7 @@ __global__ void __launch_bounds__(kThreads, 1)
           __syncwarp();
           if (lane == 0) mbar_arrive(smem_u32(&sm.bar_p[x][buf]));
         }
-        if (U == last_unit) pdl_launch_next();
+        if (u.last) pdl_launch_next();
         // ---- epilogue: O of the unit's last PV, scaled by 1/l.  The S of
         // the last tile implies that the PV two tiles back has completed,
         // not the one just before, so the PVs of the last two tiles are
@@ -675,7 +830,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         const int h = u.kvh * p.g + hl;
         __nv_bfloat16* orow = p.out + ((static_cast<size_t>(u.b) * p.S + (row_exists ? s : 0)) * p.Hq + h) * kD;
         // a split unit leaves its partial O (fp32) and (m, l) to the combine
-        const bool part = p.nsplit > 1;
+        const bool part = u.part;
         float* wo = part ? partial_o(p, u, x, row) : nullptr;
 #pragma unroll 1
         for (int ch = 0; ch < kD / 32; ++ch) {
@@ -715,10 +870,10 @@ __global__ void __launch_bounds__(kThreads, 1)
         __syncwarp();
         if (lane == 0) mbar_arrive(smem_u32(&sm.bar_ofree[x]));
         g += u.tiles;
-      } else if (p.nsplit > 1) {
+      } else if (u.part) {
         // an empty tile range (or a prefix length out of range): an empty
         // partial, which the combine skips
-        if (U == last_unit) pdl_launch_next();
+        if (u.last) pdl_launch_next();
         if (row_exists) {
           float4* dst = reinterpret_cast<float4*>(partial_o(p, u, x, row));
 #pragma unroll 4
@@ -729,7 +884,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
       } else {
         // a prefix length out of range: this unit's rows are zero
-        if (U == last_unit) pdl_launch_next();
+        if (u.last) pdl_launch_next();
         if (row_exists) {
           const int h = u.kvh * p.g + hl;
           uint4* dst = reinterpret_cast<uint4*>(p.out + ((static_cast<size_t>(u.b) * p.S + s) * p.Hq + h) * kD);
@@ -747,6 +902,143 @@ __global__ void __launch_bounds__(kThreads, 1)
     tc_fence_after();
     tmem_dealloc(tmem, kTmemCols);
   }
+  // stream-K: the record of run boundary blockIdx.x for the merge (written
+  // last, so that it is still in L2 when the merge reads it)
+  if (p.streamk && tid == 0 && blockIdx.x > 0) {
+    int4 rec = make_int4(-1, 0, 0, 0);
+    const int total = sm.order[p.Bt];
+    const int W = (total + static_cast<int>(gridDim.x) - 1) / static_cast<int>(gridDim.x);
+    const long long G = static_cast<long long>(blockIdx.x) * W;
+    if (G < total) {
+      const int b = streamk_seq(sm.order, p.Bt, static_cast<int>(G));
+      const int T = streamk_tiles(p, p.prefix_len[b]);
+      const int off = static_cast<int>(G) - sm.order[b];
+      const int kvh = off / T, t = off - kvh * T;
+      const int start = static_cast<int>(G) - t, c0 = start / W;
+      if (t > 0 && c0 + 1 == static_cast<int>(blockIdx.x))
+        rec = make_int4(b * p.Hkv + kvh, c0, (start + T - 1) / W, start != c0 * W ? 1 : 0);
+    }
+    streamk_records(p)[blockIdx.x] = rec;
+  }
+}
+
+// Stream-K merge.  Blocks (c - 1, x, z) take run boundary c, row block x,
+// rows 16z .. 16z + 15 (four per warp, lanes over the head dimension).  The
+// boundary's record names the unit it is the first to cut and its pieces:
+// those of CTAs c0 .. c1 (CTA c0's in the record's slot, the others' in
+// slot 0).  Per row: O = sum_i 2^(m_i - M) O_i / sum_i 2^(m_i - M) l_i, M =
+// max m_i over the pieces that saw a key (l_i > 0); none gives a zero row.
+// A unit cut once (two pieces, the usual case) is merged from loads that
+// are all issued together; more pieces take the general loop.
+constexpr int kMergeRows = 4;  // rows per warp
+__global__ void __launch_bounds__(128) streamk_combine_kernel(const __grid_constant__ Tc256Params p) {
+  pdl_wait();
+  const int c = static_cast<int>(blockIdx.x) + 1, x = static_cast<int>(blockIdx.y);
+  const int4 rec = streamk_records(p)[c];
+  if (rec.x >= 0) {
+    const unsigned full = 0xffffffffu;
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    const int b = rec.x / p.Hkv, kvh = rec.x - b * p.Hkv, c0 = rec.y, np = rec.z - rec.y + 1;
+    const int row0 = static_cast<int>(blockIdx.z) * 16 + warp * kMergeRows;
+    const size_t entries = static_cast<size_t>(p.ctas) * 4;
+    const float2* wml = reinterpret_cast<const float2*>(p.ws + entries * kRows * kD);
+    auto entry = [&](int j) { return (static_cast<size_t>(c0 + j) * 2 + (j == 0 ? rec.w : 0)) * 2 + x; };
+    float M[kMergeRows], L[kMergeRows];
+    float4 acc[kMergeRows];
+#pragma unroll
+    for (int k = 0; k < kMergeRows; ++k) {
+      M[k] = -INFINITY;
+      L[k] = 0.f;
+      acc[k] = make_float4(0.f, 0.f, 0.f, 0.f);
+    }
+    if (np == 2) {
+      const size_t e0 = entry(0), e1 = entry(1);
+      const float4* o0 = reinterpret_cast<const float4*>(p.ws + (e0 * kRows + row0) * kD);
+      const float4* o1 = reinterpret_cast<const float4*>(p.ws + (e1 * kRows + row0) * kD);
+      float4 va[kMergeRows], vb[kMergeRows];
+      float2 ma[kMergeRows], mb[kMergeRows];
+#pragma unroll
+      for (int k = 0; k < kMergeRows; ++k) {
+        va[k] = o0[k * (kD / 4) + lane];
+        vb[k] = o1[k * (kD / 4) + lane];
+        ma[k] = wml[e0 * kRows + row0 + k];
+        mb[k] = wml[e1 * kRows + row0 + k];
+      }
+#pragma unroll
+      for (int k = 0; k < kMergeRows; ++k) {
+        const bool ha = ma[k].y > 0.f, hb = mb[k].y > 0.f;
+        M[k] = fmaxf(ha ? ma[k].x : -INFINITY, hb ? mb[k].x : -INFINITY);
+        const float wa = ha ? exp2f(ma[k].x - M[k]) : 0.f, wb = hb ? exp2f(mb[k].x - M[k]) : 0.f;
+        L[k] = fmaf(wa, ma[k].y, wb * mb[k].y);
+        acc[k] = make_float4(fmaf(wa, va[k].x, wb * vb[k].x), fmaf(wa, va[k].y, wb * vb[k].y),
+                             fmaf(wa, va[k].z, wb * vb[k].z), fmaf(wa, va[k].w, wb * vb[k].w));
+      }
+    } else {
+      // lane j of a chunk of 32 pieces holds piece j0 + j
+      for (int j0 = 0; j0 < np; j0 += 32) {
+        if (j0 + lane < np) {
+          const size_t e = entry(j0 + lane);
+#pragma unroll
+          for (int k = 0; k < kMergeRows; ++k) {
+            const float2 ml = wml[e * kRows + row0 + k];
+            if (ml.y > 0.f) M[k] = fmaxf(M[k], ml.x);
+          }
+        }
+      }
+#pragma unroll
+      for (int k = 0; k < kMergeRows; ++k)
+#pragma unroll
+        for (int o = 16; o > 0; o >>= 1) M[k] = fmaxf(M[k], __shfl_xor_sync(full, M[k], o));
+      for (int j0 = 0; j0 < np; j0 += 32) {
+        float wj[kMergeRows];
+#pragma unroll
+        for (int k = 0; k < kMergeRows; ++k) wj[k] = 0.f;
+        if (j0 + lane < np) {
+          const size_t e = entry(j0 + lane);
+#pragma unroll
+          for (int k = 0; k < kMergeRows; ++k) {
+            const float2 ml = wml[e * kRows + row0 + k];
+            if (ml.y > 0.f && M[k] != -INFINITY) {
+              wj[k] = exp2f(ml.x - M[k]);
+              L[k] = fmaf(wj[k], ml.y, L[k]);
+            }
+          }
+        }
+        const int cnt = min(32, np - j0);
+        for (int i = 0; i < cnt; ++i) {
+          const float4* o = reinterpret_cast<const float4*>(p.ws + (entry(j0 + i) * kRows + row0) * kD);
+          float4 v[kMergeRows];
+#pragma unroll
+          for (int k = 0; k < kMergeRows; ++k) v[k] = o[k * (kD / 4) + lane];
+#pragma unroll
+          for (int k = 0; k < kMergeRows; ++k) {
+            const float w = __shfl_sync(full, wj[k], i);
+            acc[k].x = fmaf(w, v[k].x, acc[k].x);
+            acc[k].y = fmaf(w, v[k].y, acc[k].y);
+            acc[k].z = fmaf(w, v[k].z, acc[k].z);
+            acc[k].w = fmaf(w, v[k].w, acc[k].w);
+          }
+        }
+      }
+#pragma unroll
+      for (int k = 0; k < kMergeRows; ++k)
+#pragma unroll
+        for (int o = 16; o > 0; o >>= 1) L[k] += __shfl_xor_sync(full, L[k], o);
+    }
+#pragma unroll
+    for (int k = 0; k < kMergeRows; ++k) {
+      const int row = row0 + k, s = x * p.s_blk + row / p.g;
+      if (s < p.S) {
+        const float inv = L[k] > 0.f ? 1.f / L[k] : 0.f;
+        const int h = kvh * p.g + row % p.g;
+        uint2 w2;
+        w2.x = pack_bf16x2(acc[k].x * inv, acc[k].y * inv);
+        w2.y = pack_bf16x2(acc[k].z * inv, acc[k].w * inv);
+        reinterpret_cast<uint2*>(p.out + ((static_cast<size_t>(b) * p.S + s) * p.Hq + h) * kD)[lane] = w2;
+      }
+    }
+  }
+  pdl_launch_next();
 }
 
 }  // namespace
@@ -776,6 +1068,22 @@ int tc256_splits(int Bt, int Hkv, int rb, long long max_tiles, int num_sms) {
     }
   }
   return static_cast<int>(best);
+}
+
+int tc256_streamk(int Bt, int Hkv, long long max_tiles, int num_sms) {
+  const long long units = static_cast<long long>(Bt) * Hkv;
+  if (units < num_sms || Bt > kMaxStreamK || units * max_tiles >= (1ll << 30)) return 0;
+  // whole units leave the CTAs with ceil(units / SMs) or one fewer; stream-K
+  // pays (a merge launch, ~1 piece more per CTA) when the busiest CTAs hold
+  // at least 10% more than the mean
+  const long long per_cta = (units + num_sms - 1) / num_sms;
+  return per_cta * num_sms * 10 >= units * 11 ? 1 : 0;
+}
+
+size_t tc256_streamk_bytes(int num_sms) {
+  // two partial pieces per CTA, two row blocks each: O and (m, l) of 128
+  // rows; then a 16-byte record per run boundary
+  return static_cast<size_t>(num_sms) * (4 * kRows * (kD + 2) * sizeof(float) + sizeof(int4));
 }
 
 cudaError_t launch_attention_tc256(const AttnTcArgs& a, const AttnTcPlan& pl, EncodeTiledFn encode,
@@ -826,8 +1134,9 @@ cudaError_t launch_attention_tc256(const AttnTcArgs& a, const AttnTcPlan& pl, En
   p.units = a.Bt * a.Hkv;
   p.nsplit = pl.nsplit;
   p.items = p.units * pl.nsplit;
+  p.streamk = pl.streamk;
   p.ws = static_cast<float*>(a.workspace);
-  p.sort = a.Bt <= kMaxSort ? 1 : 0;
+  p.sort = (!pl.streamk && a.Bt <= kMaxSort) ? 1 : 0;
   p.scale_log2 = a.scale * 1.4426950408889634f;
   p.wait_ns = a.fault.wait_ns ? a.fault.wait_ns : kWaitLimitNs;
   p.extra_p = a.fault.extra;
@@ -838,10 +1147,16 @@ cudaError_t launch_attention_tc256(const AttnTcArgs& a, const AttnTcPlan& pl, En
     if (e != cudaSuccess) return e;
     attr_done = true;
   }
-  const int grid = std::min(p.items, pl.num_sms);
+  const int grid = pl.streamk ? pl.num_sms : std::min(p.items, pl.num_sms);
+  p.ctas = grid;
   cudaError_t e = launch_overlapped(attention_tc256_kernel, dim3(static_cast<unsigned>(grid)), dim3(kThreads),
                                     smem_bytes(), stream, 1u, tq, tkn, tvn, tkc, tvc, p);
-  if (e != cudaSuccess || pl.nsplit == 1) return e;
+  if (e != cudaSuccess) return e;
+  if (pl.streamk)
+    return grid > 1 ? launch_overlapped(streamk_combine_kernel, dim3(static_cast<unsigned>(grid - 1), 2u, kRows / 16),
+                                        dim3(128), 0, stream, 1u, p)
+                    : cudaSuccess;
+  if (pl.nsplit == 1) return e;
   return launch_attention_combine(a, pl, stream);
 }
 

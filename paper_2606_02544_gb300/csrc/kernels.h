@@ -81,6 +81,7 @@ struct AttnTcPlan {
   int slots;        // CTAs resident at once (SMs x CTAs per SM)
   int fuse;         // 2..8 splits merge in place (cluster per unit), no workspace
   int kind;         // 0: one row block per CTA; 1: 256-row units, one persistent CTA per SM
+  int streamk;      // kind 1: equal runs of the key tiles of all units per CTA, cut units merged after
   int num_sms;
   size_t ws_bytes;  // workspace bytes for the split partials (0 if nsplit == 1)
 };
@@ -117,6 +118,11 @@ bool make_bf16_map(EncodeTiledFn encode, CUtensorMap* m, const void* base, int r
 // blocks, or fewer units than SMs with under 16 key tiles each), else the
 // key-tile ranges per unit (1 when there are at least as many units as SMs).
 int tc256_splits(int Bt, int Hkv, int rb, long long max_tiles, int num_sms);
+// 1 when the kernel walks stream-K runs (at least as many units as SMs, the
+// whole-unit walk uneven by at least 10%, Bt <= 255); its partial workspace
+// is tc256_streamk_bytes.
+int tc256_streamk(int Bt, int Hkv, long long max_tiles, int num_sms);
+size_t tc256_streamk_bytes(int num_sms);
 cudaError_t launch_attention_tc256(const AttnTcArgs& a, const AttnTcPlan& pl, EncodeTiledFn encode,
                                    cudaStream_t stream);
 // Merge of split partials (workspace layout of the plan) into the output.

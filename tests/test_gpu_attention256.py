@@ -5,12 +5,17 @@ tests/_gpu.py.
 The kernel serves units of 129..256 query rows per KV head (32 drafts with
 32/8 heads, 16 drafts with 64/8 heads, 20 drafts with 32/8 heads, where the
 second block is partly empty).  With fewer units than SMs each unit's key
-tiles are split into ranges whose partials the combine kernel merges.
+tiles are split into ranges whose partials the combine kernel merges; with
+more, when whole units would load the CTAs unevenly, every CTA takes an
+equal run of the key tiles of all units (stream-K) and the units cut by run
+boundaries are merged by a second launch.
 Cases: ragged prefixes across tile and page edges, every page size, random
 step maps, padding, undrafted and decoded positions, RoPE applied in the
 kernel (both position rules), NaN-poisoned unused cache rows, more
 sequences than the ranking handles, split units (small batches, ranges with
-no tile, the new-slot tile in range 0 only), and the error paths.
+no tile, the new-slot tile in range 0 only), stream-K runs (units cut once
+or across many CTAs, prefix lengths out of range inside a run), and the
+error paths.
 """
 import numpy as np
 import pytest
@@ -50,6 +55,18 @@ def _splits(si):
     return min(cost, key=lambda ns: (cost[ns], ns))
 
 
+def _streamk(si):
+    # at least one unit per SM, at most 255 sequences, and whole units would
+    # give the busiest CTAs at least 10% more than the mean
+    w = si.w
+    sms = torch.cuda.get_device_properties(0).multi_processor_count
+    units = w.Bt * w.Hkv
+    max_tiles = (si.block_table.shape[1] * w.page_size + 63) // 64 + 1
+    if units < sms or w.Bt > 255 or units * max_tiles >= 1 << 30:
+        return False
+    return -(-units // sms) * sms * 10 >= units * 11
+
+
 def _check(si, seqs=None, rope=None):
     assert _uses_tc256(si)
     if rope is None:
@@ -64,10 +81,10 @@ def _check(si, seqs=None, rope=None):
             pos = (n + torch.arange(si.w.S, device=n.device)[None]).to(torch.int32).contiguous()
         out, word, ws = gpu_attention(si, mask=(tau, sect), rope_pos=pos, rope_theta=theta)
         ref = oracle_attention(si, seqs=seqs, rope_theta=theta, rope_mode=mode)
-    # a workspace when the units are split, none when the kernel takes
-    # them whole
+    # a workspace when the units are split or walked in stream-K runs, none
+    # when the kernel takes them whole
     ns = _splits(si)
-    assert (ns > 1 and ws > 0) or (ns == 1 and ws == 0) or ns == 0
+    assert (ns > 1 and ws > 0) or (ns == 1 and (ws > 0) == _streamk(si)) or ns == 0
     assert word == ref.err
     got = out if seqs is None else out[torch.as_tensor(seqs, device=out.device)]
     assert_attention_close(got, ref)
@@ -102,9 +119,47 @@ def test_many_units_per_cta_and_long_prefixes():
 
 
 def test_more_sequences_than_ranked():
-    # beyond 256 sequences the walk keeps the batch order
+    # beyond 256 sequences the walk keeps the batch order (whole units)
     si = inputs.make_step_inputs(_w(300, prefix=(0, 300), seed=4), device="cuda")
+    assert not _streamk(si)
     _check(si, seqs=[0, 150, 299])
+
+
+def test_whole_units_one_per_sm():
+    # 19 x 8 = 152 units: one per SM, the whole-unit walk
+    si = inputs.make_step_inputs(_w(19, prefix=(200, 1500), seed=13), device="cuda", random_step_map=True,
+                                 poison_unused_rows=True)
+    assert _splits(si) == 1 and not _streamk(si)
+    _check(si, seqs=[0, 9, 18])
+
+
+@pytest.mark.parametrize("Bt,lens", [
+    (20, [9000] + [10] * 19),                            # the long units span many CTAs each
+    (20, [0, 64, 65, 4000, 1] * 4),                      # ragged; runs start inside and between units
+    (24, [3000, 0, 2500, 0, 700, 129] * 4),
+    (40, list(range(0, 4000, 100))),
+])
+def test_streamk_runs(Bt, lens):
+    si = inputs.make_step_inputs(_w(Bt, prefix=(0, max(lens)), seed=Bt + len(set(lens))), device="cuda",
+                                 prefix_override=np.array(lens), random_step_map=True, poison_unused_rows=True)
+    assert _streamk(si)
+    _check(si, seqs=sorted({0, 1, 3, Bt // 2, Bt - 1}))
+
+
+def test_streamk_bad_prefix_inside_runs():
+    # prefix lengths out of range and a bad page inside runs that cut units
+    si = inputs.make_step_inputs(_w(22, prefix=(2000, 3000), seed=14), device="cuda", random_step_map=True)
+    n = si.prefix_len.clone()
+    n[3] = si.block_table.shape[1] * si.w.page_size + 1
+    n[10] = -1
+    si.prefix_len = n
+    bt = si.block_table.clone()
+    bt[7, 5] = si.num_pages
+    si.block_table = bt
+    assert _streamk(si)
+    out, word = _check(si, seqs=[2, 3, 4, 7, 10, 11])
+    assert word & simsd.EW_PREFIX_LEN and word & simsd.EW_PAGE
+    assert (out[[3, 7, 10]].float() == 0).all()
 
 
 @pytest.mark.parametrize("n_draft", [None, 0])
