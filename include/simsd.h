@@ -112,11 +112,12 @@ SIMSD_API int simsd_build_mask(const int32_t* step_map, const int32_t* prefix_le
  * needs for these sizes on the current device: partial results of units
  * whose prefix is split over several CTAs (0 when nothing is split).
  * max_pages*page_size bounds every prefix length.  Shapes with 129..256
- * query rows per KV head (for example 32 drafts with 32/8 heads), at most
- * 255 sequences and at least one unit (sequence, KV head) per SM, whose
- * units would load the SMs unevenly (the busiest SM 10% above the mean),
- * give every CTA an equal share of all key tiles and need about 266 KB per
- * SM (40 MB on 152 SMs).
+ * query rows per KV head (for example 32 drafts with 32/8 heads) and at
+ * most 255 sequences whose units (sequence, KV head) would load the SMs
+ * unevenly (with at least one unit per SM: the busiest SM 10% above the
+ * mean; with fewer: when equal shares cost less than equal ranges of every
+ * unit) give every CTA an equal share of all key tiles and need about
+ * 266 KB per SM (40 MB on 152 SMs).
  */
 SIMSD_API size_t simsd_verify_workspace_bytes(int dtype, int Bt, int gamma, int Hq, int Hkv, int d, int max_pages,
                                     int page_size);
@@ -184,9 +185,10 @@ SIMSD_API int simsd_verify_attention(int dtype, const void* q, const void* k_new
  *     kept, a cudaDeviceReset between calls is not supported.
  *   - Where simsd_verify_attention would give every CTA an equal share of
  *     all key tiles (scratch beyond 12 MiB), this entry point keeps units
- *     whole instead: no scratch, and results that may differ from
- *     simsd_verify_attention's in the last bits (another order of summation).
- *   - Other sizes whose scratch would exceed 12 MiB are rejected with
+ *     whole or splits them into equal ranges as it would without that
+ *     option; results may differ from simsd_verify_attention's in the last
+ *     bits (another order of summation).
+ *   - Sizes whose scratch would exceed 12 MiB are rejected with
  *     SIMSD_ERR_UNSUPPORTED (see simsd_last_error); use
  *     simsd_verify_attention with a caller workspace for those.
  *   - All calls share the one array: calls that overlap on the GPU (on

@@ -160,14 +160,10 @@ int verify_attention_impl(int dtype, const void* q, const void* k_new, const voi
     return unsupported("page pool too large for 32-bit TMA row coordinates");
   if (static_cast<long long>(Bt) * 2 * gamma * Hq >= (1ll << 31)) return unsupported("too many query rows");
   simsd::AttnTcPlan plan;
-  if (!simsd::plan_attention_tc(Bt, gamma, Hq, Hkv, max_pages, page_size, info.num_sms, &plan))
+  if (!simsd::plan_attention_tc(Bt, gamma, Hq, Hkv, max_pages, page_size, info.num_sms, &plan, !static_scratch))
     return unsupported("query rows per KV head: need 2*gamma*Hq/Hkv <= 128 or 128 % (Hq/Hkv) == 0");
   if (static_scratch) {
-    if (plan.streamk && plan.ws_bytes > simsd::noalloc_scratch_capacity()) {
-      // the whole-unit walk needs no scratch
-      plan.streamk = 0;
-      plan.ws_bytes = 0;
-    }
+    // (stream-K runs are not used here: their partials would outgrow the array)
     if (plan.ws_bytes > simsd::noalloc_scratch_capacity()) {
       std::snprintf(g_last_error, sizeof(g_last_error),
                     "unsupported: these sizes need %zu bytes of scratch, more than the %zu-byte static array; "

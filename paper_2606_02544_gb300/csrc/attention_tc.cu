@@ -950,7 +950,7 @@ bool make_bf16_map(EncodeTiledFn encode, CUtensorMap* m, const void* base, int r
 }
 
 bool plan_attention_tc(int Bt, int gamma, int Hq, int Hkv, int max_pages, int page_size, int num_sms,
-                       AttnTcPlan* plan) {
+                       AttnTcPlan* plan, bool allow_streamk) {
   const int S = 2 * gamma, g = Hq / Hkv;
   const int R = g * S;
   AttnTcPlan pl{};
@@ -971,13 +971,15 @@ bool plan_attention_tc(int Bt, int gamma, int Hq, int Hkv, int max_pages, int pa
     // than SMs each unit's key tiles are split into ranges whose partials
     // the combine kernel merges
     pl.kind = 1;
-    pl.nsplit = ns256;
-    pl.streamk = ns256 == 1 ? tc256_streamk(Bt, Hkv, max_tiles, num_sms) : 0;
+    pl.streamk = allow_streamk ? tc256_streamk(Bt, Hkv, max_tiles, ns256, num_sms) : 0;
+    pl.nsplit = pl.streamk ? 1 : ns256;
     pl.sort = 0;
     pl.fuse = 0;
     pl.slots = num_sms;
-    pl.ws_bytes = ns256 > 1 ? static_cast<size_t>(Bt) * Hkv * pl.rb * ns256 * pl.rows_blk * (kD + 2) * sizeof(float)
-                            : (pl.streamk ? tc256_streamk_bytes(num_sms) : 0);
+    pl.ws_bytes = pl.streamk ? tc256_streamk_bytes(num_sms)
+                  : pl.nsplit > 1
+                      ? static_cast<size_t>(Bt) * Hkv * pl.rb * pl.nsplit * pl.rows_blk * (kD + 2) * sizeof(float)
+                      : 0;
     *plan = pl;
     return true;
   }

@@ -1070,14 +1070,22 @@ int tc256_splits(int Bt, int Hkv, int rb, long long max_tiles, int num_sms) {
   return static_cast<int>(best);
 }
 
-int tc256_streamk(int Bt, int Hkv, long long max_tiles, int num_sms) {
+int tc256_streamk(int Bt, int Hkv, long long max_tiles, int nsplit, int num_sms) {
   const long long units = static_cast<long long>(Bt) * Hkv;
-  if (units < num_sms || Bt > kMaxStreamK || units * max_tiles >= (1ll << 30)) return 0;
-  // whole units leave the CTAs with ceil(units / SMs) or one fewer; stream-K
-  // pays (a merge launch, ~1 piece more per CTA) when the busiest CTAs hold
-  // at least 10% more than the mean
-  const long long per_cta = (units + num_sms - 1) / num_sms;
-  return per_cta * num_sms * 10 >= units * 11 ? 1 : 0;
+  if (nsplit < 1 || Bt > kMaxStreamK || units * max_tiles >= (1ll << 30)) return 0;
+  if (units >= num_sms) {
+    // whole units leave the CTAs with ceil(units / SMs) or one fewer;
+    // stream-K pays (a merge launch, ~1 piece more per CTA) when the
+    // busiest CTAs hold at least 10% more than the mean
+    const long long per_cta = (units + num_sms - 1) / num_sms;
+    return per_cta * num_sms * 10 >= units * 11 ? 1 : 0;
+  }
+  // fewer units than SMs: the ranges' cost (tc256_splits) against equal runs
+  // plus about three items (the pieces at both ends of a run, the merge)
+  const long long kItemCost = 14;
+  const long long ranges = (units * nsplit + num_sms - 1) / num_sms * ((max_tiles + nsplit - 1) / nsplit + kItemCost);
+  const long long runs = (units * max_tiles + num_sms - 1) / num_sms + 3 * kItemCost;
+  return runs < ranges ? 1 : 0;
 }
 
 size_t tc256_streamk_bytes(int num_sms) {

@@ -86,8 +86,9 @@ struct AttnTcPlan {
   size_t ws_bytes;  // workspace bytes for the split partials (0 if nsplit == 1)
 };
 // Returns false if the shape is not supported by the tensor-core kernel.
+// allow_streamk = false keeps the 256-row kernel on whole units or ranges.
 bool plan_attention_tc(int Bt, int gamma, int Hq, int Hkv, int max_pages, int page_size, int num_sms,
-                       AttnTcPlan* plan);
+                       AttnTcPlan* plan, bool allow_streamk = true);
 
 struct AttnTcArgs {
   const void *q, *k_new, *v_new, *k_cache, *v_cache;
@@ -118,10 +119,11 @@ bool make_bf16_map(EncodeTiledFn encode, CUtensorMap* m, const void* base, int r
 // blocks, or fewer units than SMs with under 16 key tiles each), else the
 // key-tile ranges per unit (1 when there are at least as many units as SMs).
 int tc256_splits(int Bt, int Hkv, int rb, long long max_tiles, int num_sms);
-// 1 when the kernel walks stream-K runs (at least as many units as SMs, the
-// whole-unit walk uneven by at least 10%, Bt <= 255); its partial workspace
-// is tc256_streamk_bytes.
-int tc256_streamk(int Bt, int Hkv, long long max_tiles, int num_sms);
+// 1 when the kernel walks stream-K runs instead of the nsplit ranges that
+// tc256_splits chose (Bt <= 255; with at least as many units as SMs when
+// the whole-unit walk is uneven by at least 10%, with fewer when the cost
+// model favours equal runs); its partial workspace is tc256_streamk_bytes.
+int tc256_streamk(int Bt, int Hkv, long long max_tiles, int nsplit, int num_sms);
 size_t tc256_streamk_bytes(int num_sms);
 cudaError_t launch_attention_tc256(const AttnTcArgs& a, const AttnTcPlan& pl, EncodeTiledFn encode,
                                    cudaStream_t stream);

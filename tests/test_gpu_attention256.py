@@ -56,15 +56,20 @@ def _splits(si):
 
 
 def _streamk(si):
-    # at least one unit per SM, at most 255 sequences, and whole units would
-    # give the busiest CTAs at least 10% more than the mean
+    # at most 255 sequences; with at least one unit per SM when whole units
+    # would give the busiest CTAs at least 10% more than the mean, with fewer
+    # when equal runs plus three items cost less than the chosen ranges
     w = si.w
     sms = torch.cuda.get_device_properties(0).multi_processor_count
     units = w.Bt * w.Hkv
     max_tiles = (si.block_table.shape[1] * w.page_size + 63) // 64 + 1
-    if units < sms or w.Bt > 255 or units * max_tiles >= 1 << 30:
+    ns = _splits(si)
+    if ns < 1 or w.Bt > 255 or units * max_tiles >= 1 << 30:
         return False
-    return -(-units // sms) * sms * 10 >= units * 11
+    if units >= sms:
+        return -(-units // sms) * sms * 10 >= units * 11
+    ranges = -(-units * ns // sms) * (-(-max_tiles // ns) + 14)
+    return -(-units * max_tiles // sms) + 3 * 14 < ranges
 
 
 def _check(si, seqs=None, rope=None):
@@ -144,6 +149,22 @@ def test_streamk_runs(Bt, lens):
                                  prefix_override=np.array(lens), random_step_map=True, poison_unused_rows=True)
     assert _streamk(si)
     _check(si, seqs=sorted({0, 1, 3, Bt // 2, Bt - 1}))
+
+
+def test_streamk_small_batch_long_prefixes():
+    # 8 x 8 units of ~460 tiles, fewer than SMs: equal runs of ~200 tiles
+    # (units spanning three CTAs) cost less than two ranges a unit, which
+    # leave 24 of 152 SMs idle
+    si = inputs.make_step_inputs(_w(8, prefix=(28000, 30000), seed=15), device="cuda", random_step_map=True)
+    assert _splits(si) > 1 and _streamk(si)
+    _check(si, seqs=[0, 7])
+
+
+def test_split_units_keep_ranges():
+    # the split tests above run the ranges walk, not stream-K
+    for Bt, prefix, P in [(1, (3000, 3000), 64), (8, (1500, 2000), 64), (12, (2000, 6000), 64), (2, (1000, 1100), 8)]:
+        si = inputs.make_step_inputs(_w(Bt, prefix=prefix, P=P, seed=1), device="cuda")
+        assert _splits(si) > 1 and not _streamk(si)
 
 
 def test_streamk_bad_prefix_inside_runs():

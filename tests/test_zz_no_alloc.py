@@ -6,7 +6,11 @@ not stall on the allocator, or code running where allocation is not
 allowed).  Both entry points run the same kernels on the same plan and
 differ only in where the split partials live (the library's static array
 instead of caller memory), so their outputs must be bit-identical, on
-consecutive calls that share the static array.  This file is collected
+consecutive calls that share the static array.  The one exception: where
+simsd_verify_attention gives every CTA an equal share of all key tiles
+(stream-K, whose partials would not fit the array), the no-alloc entry
+point keeps the plan it had without that option; both are checked against
+the oracle there.  This file is collected
 last, so that a run that stops at the first failure has run every other
 test first.
 """
@@ -73,6 +77,22 @@ def test_noalloc_fp32_and_unsplit_shapes():
         want, _ = _regular(si, tau, sect)
         got = _noalloc(si, tau, sect)
         assert torch.equal(got, want)
+
+
+def test_noalloc_keeps_whole_units_where_streamk_runs():
+    # 20 sequences of 32 drafts: simsd_verify_attention walks stream-K runs
+    # (40 MB of partials); the no-alloc entry point keeps the units whole,
+    # no scratch: another order of summation, both within the bars
+    from tests._gpu import assert_attention_close, oracle_attention
+    w = inputs.Workload("na5", "bf16", 20, 32, 8, 128, 32, (100, 900), 1, 64, 0.5, 1 / np.sqrt(128), 1.0, 25)
+    si = inputs.make_step_inputs(w, device="cuda", random_step_map=True, with_logits=False)
+    tau, sect, _, _, _ = gpu_mask(si, mask_bits=False)
+    want, ws = _regular(si, tau, sect)
+    assert ws > NOALLOC_SCRATCH_BYTES
+    got = _noalloc(si, tau, sect)
+    ref = oracle_attention(si, seqs=[0, 9, 19])
+    for out in (want, got):
+        assert_attention_close(out[torch.as_tensor([0, 9, 19], device=out.device)], ref)
 
 
 def test_noalloc_rejects_sizes_beyond_the_static_scratch():
