@@ -241,8 +241,10 @@ __global__ void __launch_bounds__(kAcceptThreads) accept_kernel(const float* __r
 
 // Few sequences: the block of each sequence is split over `parts` CTAs that
 // need not be resident together (no cluster).  Each writes its 64-bit key
-// per row to keys[b][part][row]; accept_merge_kernel then takes the maximum
-// per row and walks the drafts.
+// per row to keys[b][row][part]; accept_merge_kernel then takes the maximum
+// per row and walks the drafts.  The merge launch is let in as soon as this
+// grid has started, so that its launch latency hides behind the streaming
+// (its blocks, one per sequence, only wait for this grid to complete).
 __global__ void __launch_bounds__(kAcceptThreads) accept_part_kernel(const float* __restrict__ logits, int gamma,
                                                                      int vocab, int vec4, int parts,
                                                                      unsigned long long* __restrict__ keys) {
@@ -251,38 +253,49 @@ __global__ void __launch_bounds__(kAcceptThreads) accept_part_kernel(const float
   const int rows = gamma + 1;
   for (int r = threadIdx.x; r < rows; r += kAcceptThreads) best[r] = 0ull;
   pdl_wait();
+  pdl_launch_next();
   __syncthreads();
   scan_span<8>(logits + static_cast<size_t>(b) * rows * vocab, rows, vocab, vec4, c, parts, best);
   __syncthreads();
   for (int r = threadIdx.x; r < rows; r += kAcceptThreads)
-    keys[(static_cast<size_t>(b) * parts + c) * rows + r] = best[r];
-  pdl_launch_next();
+    keys[(static_cast<size_t>(b) * rows + r) * parts + c] = best[r];
 }
 
-// One warp per sequence: the maximum key of every row over the parts, then
-// the walk.
-__global__ void __launch_bounds__(32) accept_merge_kernel(const unsigned long long* __restrict__ keys, int parts,
-                                                          const int32_t* __restrict__ draft, int gamma, int vocab,
-                                                          int32_t* __restrict__ accepted_len,
-                                                          int32_t* __restrict__ out_tokens,
-                                                          int32_t* __restrict__ row_argmax, int32_t* err_word) {
+// One block per sequence: warp w takes rows w, w + 32 (the maximum key over
+// the parts, lanes over the parts: coalesced loads of keys[b][row][part],
+// all of a lane's issued together), then warp 0 walks the drafts.
+constexpr int kMergeThreads = 1024;
+__global__ void __launch_bounds__(kMergeThreads) accept_merge_kernel(const unsigned long long* __restrict__ keys,
+                                                                     int parts, const int32_t* __restrict__ draft,
+                                                                     int gamma, int vocab,
+                                                                     int32_t* __restrict__ accepted_len,
+                                                                     int32_t* __restrict__ out_tokens,
+                                                                     int32_t* __restrict__ row_argmax,
+                                                                     int32_t* err_word) {
   __shared__ int am[kMaxRows];
-  const int b = blockIdx.x, lane = threadIdx.x;
+  const int b = blockIdx.x, lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
   const int rows = gamma + 1;
+  const unsigned full = 0xffffffffu;
   pdl_wait();
-  const int dr_lane = lane < gamma ? draft[static_cast<size_t>(b) * gamma + lane] : 0;
-  for (int r = lane; r < rows; r += 32) {
+  const int dr_lane = (warp == 0 && lane < gamma) ? draft[static_cast<size_t>(b) * gamma + lane] : 0;
+  for (int r = warp; r < rows; r += kMergeThreads / 32) {
+    const unsigned long long* kr = keys + (static_cast<size_t>(b) * rows + r) * parts;
     unsigned long long k = 0ull;
-    const unsigned long long* kr = keys + static_cast<size_t>(b) * parts * rows + r;
-    for (int p = 0; p < parts; ++p) {
-      const unsigned long long v = kr[static_cast<size_t>(p) * rows];
+#pragma unroll 4
+    for (int p = lane; p < parts; p += 32) {
+      const unsigned long long v = kr[p];
       k = v > k ? v : k;
     }
-    am[r] = static_cast<int>(~static_cast<uint32_t>(k & 0xFFFFFFFFull));
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) {
+      const unsigned long long v = __shfl_xor_sync(full, k, o);
+      k = v > k ? v : k;
+    }
+    if (lane == 0) am[r] = static_cast<int>(~static_cast<uint32_t>(k & 0xFFFFFFFFull));
   }
-  __syncwarp();
+  __syncthreads();
   pdl_launch_next();
-  walk_drafts(am, dr_lane, b, gamma, vocab, accepted_len, out_tokens, row_argmax, err_word);
+  if (warp == 0) walk_drafts(am, dr_lane, b, gamma, vocab, accepted_len, out_tokens, row_argmax, err_word);
 }
 
 namespace {
@@ -362,7 +375,7 @@ cudaError_t launch_accept_parts(const float* logits, const int32_t* draft, int B
   cudaError_t e = launch_overlapped(accept_part_kernel, dim3(static_cast<unsigned>(Bt) * parts), dim3(kAcceptThreads),
                                     0, stream, 1u, logits, gamma, vocab, vec4, parts, keys);
   if (e != cudaSuccess) return e;
-  return launch_overlapped(accept_merge_kernel, dim3(static_cast<unsigned>(Bt)), dim3(32), 0, stream, 1u,
+  return launch_overlapped(accept_merge_kernel, dim3(static_cast<unsigned>(Bt)), dim3(kMergeThreads), 0, stream, 1u,
                            static_cast<const unsigned long long*>(keys), parts, draft, gamma, vocab, accepted_len,
                            out_tokens, row_argmax, err_word);
 }
