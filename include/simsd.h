@@ -283,12 +283,15 @@ SIMSD_API int simsd_accept_sampled(const float* target_logits, const float* draf
 /*
  * simsd_accept_sampled_workspace_bytes / simsd_accept_sampled_ws -- the same
  * stochastic acceptance with a caller workspace.  For few sequences (at most
- * num_SMs / 16) holding at least 6 MiB of logits each (target and draft
- * rows; 12 MiB when there are more than num_SMs / 32 sequences), the
- * log-sum-exp pass over every row is split over more CTAs than one
- * cluster per sequence holds: a first launch writes per-row (max, sum) pairs
- * of each part to the workspace, which the cluster of each sequence merges
- * before it forms alpha_r and draws the token as simsd_accept_sampled does.
+ * num_SMs / 16) holding at least 3 MiB of logits each (target and draft
+ * rows), the log-sum-exp pass over every row is split over more CTAs than
+ * one cluster per sequence holds: a first launch writes per-row (max, sum)
+ * pairs of each part to the workspace; a second, over spans of row a,
+ * merges them, forms alpha_r, sums the residual weights of its span and
+ * lets the last CTA of each sequence draw the token by the same inverse CDF
+ * as simsd_accept_sampled (per-sequence arrival counts in the workspace,
+ * reset by the first launch of every call, so the workspace need not start
+ * zeroed).
  * The workspace bytes are 0 for other shapes (then the call is
  * simsd_accept_sampled).  The pairs are merged in another order than the
  * cluster kernel's, so probabilities can differ in the last fp32 bits (the

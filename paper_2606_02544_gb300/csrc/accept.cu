@@ -356,7 +356,7 @@ int accept_parts(int Bt, int gamma, int vocab, int num_sms) {
   // about 8 units of 16 bytes per thread of a part, at most two parts per SM
   const long long units = static_cast<long long>(gamma + 1) * ((vocab + 3) / 4);
   const long long by_work = units / (8LL * kAcceptThreads);
-  const long long by_sms = (2LL * num_sms + Bt - 1) / Bt;
+  const long long by_sms = 2LL * num_sms / Bt;  // one wave of two CTAs per SM
   const long long parts = std::min(by_work, by_sms);
   return parts > kMaxCluster ? static_cast<int>(parts) : 0;
 }

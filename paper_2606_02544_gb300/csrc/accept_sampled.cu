@@ -21,6 +21,12 @@
 // the CTA whose range holds it; there the warp whose part holds it finds the
 // macro-step by a scan of the kept sums and walks only that one.  Row a is read a second time (2 of the
 // 2*gamma+1 rows); no global scratch memory is used.
+//
+// Few sequences with a caller workspace: phase 1 is split over many CTAs
+// that need not be resident together (samp_part_kernel, per-part (m, s) of
+// every row), then samp_resid_kernel, one CTA per (sequence, part), merges
+// the (m, s), takes a, sums its span of row a and lets the last CTA of the
+// sequence draw the token: no cluster and no CTA waiting for another.
 #include <cooperative_groups.h>
 #include <cuda_runtime.h>
 
@@ -107,6 +113,40 @@ __device__ __forceinline__ float4 load_unit(const float* rp, int col) {
   } else {
     return make_float4(__ldg(rp + col), -INFINITY, -INFINITY, -INFINITY);
   }
+}
+
+// The accepted length of sequence b (one warp, lane r taking draft r): with
+// the rows' base-2 log-sum-exp (m, s) in row_m / row_s and the drafts' own
+// logits zt / zd, draft r is accepted iff u_r < alpha_r = min(1,
+// p_theta(x_r) / p_phi(x_r)); a is the first rejection (gamma when there is
+// none).  A draft token out of range is rejected and flagged.  With `write`
+// set, lane 0 stores a and the lanes the tokens of every position but a
+// (accepted drafts, then -1).
+__device__ __forceinline__ int accept_walk(int b, int gamma, int vocab, float zscale, const float* row_m,
+                                           const float* row_s, float zt, float zd, float ua, bool bad,
+                                           const int32_t* __restrict__ draft, int32_t* __restrict__ accepted_len,
+                                           int32_t* __restrict__ out_tokens, int32_t* err_word, bool write) {
+  const int lane = threadIdx.x & 31;
+  const unsigned full = 0xffffffffu;
+  bool acc = false;
+  if (lane < gamma && !bad) {
+    // log2 of p_theta(x) / p_phi(x)
+    const int rd = gamma + 1 + lane;
+    const float lr = (zt * zscale - row_m[lane] - log2f(row_s[lane])) - (zd * zscale - row_m[rd] - log2f(row_s[rd]));
+    const float alpha = lr >= 0.f ? 1.f : exp2f(lr);
+    acc = ua < alpha;
+  }
+  const unsigned rej = __ballot_sync(full, lane < gamma && !acc);
+  const int a = rej ? __ffs(rej) - 1 : gamma;
+  if (write) {
+    if (__any_sync(full, bad) && lane == 0) raise_error(err_word, SIMSD_EW_DRAFT);
+    if (lane == 0) accepted_len[b] = a;
+    int32_t* ot = out_tokens + static_cast<size_t>(b) * (gamma + 1);
+    for (int r = lane; r <= gamma; r += 32)
+      if (r != a) ot[r] = r < a ? draft[static_cast<size_t>(b) * gamma + r] : -1;
+  }
+  (void)vocab;
+  return a;
 }
 
 // Phase 1 of one CTA: the running (m, s) of z = x log2(e) / T over span c
@@ -233,9 +273,7 @@ template <bool VEC, int UNROLL>
 __global__ void __launch_bounds__(kSampThreads, UNROLL == 8 ? 2 : 1) accept_sampled_kernel(
     const float* __restrict__ tgt, const float* __restrict__ drf, const int32_t* __restrict__ draft,
     const float* __restrict__ u_accept, const float* __restrict__ u_sample, float zscale, int gamma, int vocab,
-    int32_t* __restrict__ accepted_len, int32_t* __restrict__ out_tokens, int32_t* err_word,
-    const float2* __restrict__ pre, int pre_parts) {
-  // pre: null, or the (m, s) partials of samp_part_kernel [Bt][pre_parts][rows]
+    int32_t* __restrict__ accepted_len, int32_t* __restrict__ out_tokens, int32_t* err_word) {
   __shared__ float2 part[kSampWarps][kSampMaxRows];  // per warp (m, s) of each row
   __shared__ float2 cta_ms[kSampMaxRows];            // this CTA's (m, s) of each row
   __shared__ float row_m[kSampMaxRows], row_s[kSampMaxRows];
@@ -275,36 +313,15 @@ __global__ void __launch_bounds__(kSampThreads, UNROLL == 8 ? 2 : 1) accept_samp
   __syncthreads();
 
   // ---- phase 1: per-row (m, s) over this CTA's span of warp-aligned units
-  // (or, with partials from samp_part_kernel, none here)
-  if (pre == nullptr) phase1_span<VEC, UNROLL>(tgt, drf, b, gamma, vocab, zscale, c, CL, part);
+  phase1_span<VEC, UNROLL>(tgt, drf, b, gamma, vocab, zscale, c, CL, part);
   // the next kernel may be scheduled once the logits have streamed through
   pdl_launch_next();
   __syncthreads();
-  if (pre == nullptr) {
-    for (int r = tid; r < rows; r += kSampThreads) {
-      float m = kEmpty, s = 0.f;
+  for (int r = tid; r < rows; r += kSampThreads) {
+    float m = kEmpty, s = 0.f;
 #pragma unroll
-      for (int w = 0; w < kSampWarps; ++w) ms_merge(m, s, part[w][r].x, part[w][r].y);
-      cta_ms[r] = make_float2(m, s);
-    }
-  } else {
-    // this CTA merges its share of the parts: warp w takes rows w, w+16, ...
-    // and its lanes the parts p0 + lane, p0 + lane + 32, ...
-    const int per = (pre_parts + CL - 1) / CL;
-    const int p0 = min(pre_parts, c * per), p1 = min(pre_parts, p0 + per);
-    for (int r = warp; r < rows; r += kSampWarps) {
-      float m = kEmpty, s = 0.f;
-      for (int q = p0 + lane; q < p1; q += 32) {
-        const float2 v = pre[(static_cast<size_t>(b) * pre_parts + q) * rows + r];
-        ms_merge(m, s, v.x, v.y);
-      }
-#pragma unroll
-      for (int o = 16; o > 0; o >>= 1) {
-        const float m2 = __shfl_xor_sync(full, m, o), s2 = __shfl_xor_sync(full, s, o);
-        ms_merge(m, s, m2, s2);
-      }
-      if (lane == 0) cta_ms[r] = make_float2(m, s);
-    }
+    for (int w = 0; w < kSampWarps; ++w) ms_merge(m, s, part[w][r].x, part[w][r].y);
+    cta_ms[r] = make_float2(m, s);
   }
   cluster.sync();
 
@@ -338,22 +355,10 @@ __global__ void __launch_bounds__(kSampThreads, UNROLL == 8 ? 2 : 1) accept_samp
     if (warp == 0) {
       cp_async_wait_all();
       __syncwarp();
-      bool acc = false;
-      if (lane < gamma && !bad) {
-        // log2 of p_theta(x) / p_phi(x)
-        const int rd = gamma + 1 + lane;
-        const float lr = (zt_sh[lane] * zscale - row_m[lane] - log2f(row_s[lane])) -
-                         (zd_sh[lane] * zscale - row_m[rd] - log2f(row_s[rd]));
-        const float alpha = lr >= 0.f ? 1.f : exp2f(lr);
-        acc = ua_sh[lane] < alpha;
-      }
-      const unsigned rej = __ballot_sync(full, lane < gamma && !acc);
-      if (__any_sync(full, bad) && lane == 0) raise_error(err_word, SIMSD_EW_DRAFT);
-      const int a = rej ? __ffs(rej) - 1 : gamma;
-      if (lane == 0) accepted_len[b] = a;
-      int32_t* ot = out_tokens + static_cast<size_t>(b) * (gamma + 1);
-      for (int r = lane; r <= gamma; r += 32)
-        if (r != a) ot[r] = r < a ? draft[static_cast<size_t>(b) * gamma + r] : -1;
+      const bool lb = lane < gamma;
+      const int a = accept_walk(b, gamma, vocab, zscale, row_m, row_s, lb ? zt_sh[lane] : 0.f,
+                                lb ? zd_sh[lane] : 0.f, lb ? ua_sh[lane] : 0.f, bad, draft, accepted_len, out_tokens,
+                                err_word, true);
       // a and the merged (m, s) of the rows phase 2 needs, to every CTA
       if (lane < CL) {
         const int rd = gamma + 1 + a;
@@ -567,7 +572,8 @@ template <bool VEC>
 __global__ void __launch_bounds__(kSampThreads, 2) samp_part_kernel(const float* __restrict__ tgt,
                                                                     const float* __restrict__ drf, float zscale,
                                                                     int gamma, int vocab, int parts,
-                                                                    float2* __restrict__ pre) {
+                                                                    float2* __restrict__ pre,
+                                                                    unsigned* __restrict__ arrivals) {
   __shared__ float2 part[kSampWarps][kSampMaxRows];
   const int b = blockIdx.x / parts, c = blockIdx.x - b * parts;
   const int rows = 2 * gamma + 1;
@@ -575,6 +581,8 @@ __global__ void __launch_bounds__(kSampThreads, 2) samp_part_kernel(const float*
   for (int i = tid; i < kSampWarps * kSampMaxRows; i += kSampThreads)
     part[i / kSampMaxRows][i % kSampMaxRows] = make_float2(kEmpty, 0.f);
   pdl_wait();
+  // the arrival count samp_resid_kernel uses for this sequence starts at 0
+  if (c == 0 && tid == 0) arrivals[b] = 0u;
   __syncthreads();
   phase1_span<VEC, 8>(tgt, drf, b, gamma, vocab, zscale, c, parts, part);
   __syncthreads();
@@ -585,6 +593,262 @@ __global__ void __launch_bounds__(kSampThreads, 2) samp_part_kernel(const float*
     pre[(static_cast<size_t>(b) * parts + c) * rows + r] = make_float2(m, s);
   }
   pdl_launch_next();
+}
+
+// Row a's weights at one unit of 4 columns (1 in the scalar layout, the
+// other three 0): p_theta = 2^(z_t - m_t) / s_t and the residual
+// max(0, p_theta - p_phi) (p_theta again when there is no draft row).
+struct RowW {
+  const float* trow;
+  const float* drow;
+  float zscale, nmt, it, nmd, id;
+  bool resid;
+};
+struct UnitW {
+  float4 t, r;
+};
+template <bool VEC>
+__device__ __forceinline__ UnitW unit_weights(const RowW& w, int u) {
+  const float4 xt = load_unit_cached<VEC>(w.trow, u);
+  UnitW o;
+  o.t = make_float4(ex2(fmaf(xt.x, w.zscale, w.nmt)) * w.it, ex2(fmaf(xt.y, w.zscale, w.nmt)) * w.it,
+                    ex2(fmaf(xt.z, w.zscale, w.nmt)) * w.it, ex2(fmaf(xt.w, w.zscale, w.nmt)) * w.it);
+  if (w.resid) {
+    const float4 xd = load_unit_cached<VEC>(w.drow, u);
+    o.r = make_float4(fmaxf(0.f, o.t.x - ex2(fmaf(xd.x, w.zscale, w.nmd)) * w.id),
+                      fmaxf(0.f, o.t.y - ex2(fmaf(xd.y, w.zscale, w.nmd)) * w.id),
+                      fmaxf(0.f, o.t.z - ex2(fmaf(xd.z, w.zscale, w.nmd)) * w.id),
+                      fmaxf(0.f, o.t.w - ex2(fmaf(xd.w, w.zscale, w.nmd)) * w.id));
+  } else {
+    o.r = o.t;
+  }
+  return o;
+}
+
+// Sum of a value over the CTA (every thread gets it).
+__device__ __forceinline__ float cta_sum(float v, float* red) {
+  const unsigned full = 0xffffffffu;
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(full, v, o);
+  __syncthreads();
+  if (lane == 0) red[warp] = v;
+  __syncthreads();
+  float t = 0.f;
+#pragma unroll
+  for (int w = 0; w < kSampWarps; ++w) t += red[w];
+  return t;
+}
+
+// Few sequences, after samp_part_kernel: one CTA per (sequence b, span c of
+// row a; rparts spans).  Every CTA merges the parts' (m, s) of every row
+// (eight loads a lane in flight) and takes the accepted
+// length a itself (part 0 stores the outputs); then it sums the weights of
+// its span c of row a's units, both the residual max(0, p_theta -
+// p_phi) and p_theta (the fallback when the residual is empty), and
+// counts itself in.  The last CTA of the sequence to arrive draws the token
+// by inverse CDF with u_sample: the spans in order of the vocabulary give
+// the one that holds the threshold (the first of positive weight whose end
+// passes it, else, by rounding, the last of positive weight), and a scan of
+// that span the token (the first of positive weight whose cumulative weight
+// passes it, else the last of positive weight).  No CTA waits for another.
+template <bool VEC>
+__global__ void __launch_bounds__(kSampThreads, 2) samp_resid_kernel(
+    const float* __restrict__ tgt, const float* __restrict__ drf, const int32_t* __restrict__ draft,
+    const float* __restrict__ u_accept, const float* __restrict__ u_sample, float zscale, int gamma, int vocab,
+    int32_t* __restrict__ accepted_len, int32_t* __restrict__ out_tokens, int32_t* err_word,
+    const float2* __restrict__ pre, int parts, int rparts, float2* __restrict__ sums,
+    unsigned* __restrict__ arrivals) {
+  __shared__ float row_m[kSampMaxRows], row_s[kSampMaxRows];
+  __shared__ float red[kSampWarps], red2[kSampWarps];
+  __shared__ int a_sh, last_sh, tok_sh, pos_sh;
+  __shared__ float thr_sh, base_sh;
+  __shared__ int owner_sh, mode_sh;  // mode: 0 residual, 1 p_theta, -1 no positive weight
+  const int b = blockIdx.x / rparts, c = blockIdx.x - b * rparts;
+  const int rows = 2 * gamma + 1;
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  const unsigned full = 0xffffffffu;
+  pdl_wait();
+  float zt = 0.f, zd = 0.f, ua = 0.f;
+  bool bad = false;
+  if (warp == 0 && lane < gamma) {
+    const int x = draft[static_cast<size_t>(b) * gamma + lane];
+    ua = u_accept[static_cast<size_t>(b) * gamma + lane];
+    bad = x < 0 || x >= vocab;
+    if (!bad) {
+      zt = __ldg(tgt + (static_cast<size_t>(b) * (gamma + 1) + lane) * vocab + x);
+      zd = __ldg(drf + (static_cast<size_t>(b) * gamma + lane) * vocab + x);
+    }
+  }
+  // the rows' (m, s): warp w merges rows w, w + 16, ..., lanes over the parts
+  for (int r = warp; r < rows; r += kSampWarps) {
+    float m = kEmpty, sm = 0.f;
+    for (int q0 = 0; q0 < parts; q0 += 32 * 8) {
+      float2 v[8];
+#pragma unroll
+      for (int j = 0; j < 8; ++j) {
+        const int q = q0 + 32 * j + lane;
+        v[j] = q < parts ? pre[(static_cast<size_t>(b) * parts + q) * rows + r] : make_float2(kEmpty, 0.f);
+      }
+#pragma unroll
+      for (int j = 0; j < 8; ++j) ms_merge(m, sm, v[j].x, v[j].y);
+    }
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) {
+      const float m2 = __shfl_xor_sync(full, m, o), s2 = __shfl_xor_sync(full, sm, o);
+      ms_merge(m, sm, m2, s2);
+    }
+    if (lane == 0) {
+      row_m[r] = m;
+      row_s[r] = sm;
+    }
+  }
+  __syncthreads();
+  if (warp == 0) {
+    const int a = accept_walk(b, gamma, vocab, zscale, row_m, row_s, zt, zd, ua, bad, draft, accepted_len,
+                              out_tokens, err_word, c == 0);
+    if (lane == 0) a_sh = a;
+  }
+  __syncthreads();
+  // ---- the weights of row a over this part's span of units
+  const int a = a_sh;
+  const bool resid = a < gamma;
+  const float* trow = tgt + (static_cast<size_t>(b) * (gamma + 1) + a) * vocab;
+  const float* drow = resid ? drf + (static_cast<size_t>(b) * gamma + a) * vocab : trow;
+  const float nmt = -row_m[a], it = 1.f / row_s[a];
+  const float nmd = resid ? -row_m[gamma + 1 + a] : 0.f, id = resid ? 1.f / row_s[gamma + 1 + a] : 0.f;
+  const int W = VEC ? (vocab >> 2) : vocab;
+  const int per = (W + rparts - 1) / rparts;
+  const RowW rw{trow, drow, zscale, nmt, it, nmd, id, resid};
+  {
+    const int u0 = min(W, c * per), u1 = min(W, u0 + per);
+    float st = 0.f, sr = 0.f;
+    for (int u = u0 + tid; u < u1; u += kSampThreads) {
+      const UnitW w = unit_weights<VEC>(rw, u);
+      st += (w.t.x + w.t.y) + (w.t.z + w.t.w);
+      sr += (w.r.x + w.r.y) + (w.r.z + w.r.w);
+    }
+    st = cta_sum(st, red);
+    sr = cta_sum(sr, red2);
+    if (tid == 0) {
+      sums[static_cast<size_t>(b) * rparts + c] = make_float2(sr, st);
+      __threadfence();
+      last_sh = atomicAdd(arrivals + b, 1u) == static_cast<unsigned>(rparts - 1);
+    }
+  }
+  pdl_launch_next();
+  __syncthreads();
+  if (!last_sh) return;
+  __threadfence();
+  // ---- the last CTA of the sequence: which span holds the threshold
+  if (warp == 0) {
+    // the other CTAs' sums, read past L1 (they were written by other SMs)
+    const volatile float* vs = reinterpret_cast<const volatile float*>(sums + static_cast<size_t>(b) * rparts);
+    float tr = 0.f, tt = 0.f;
+    for (int q = lane; q < rparts; q += 32) {
+      tr += vs[2 * q];
+      tt += vs[2 * q + 1];
+    }
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) {
+      tr += __shfl_xor_sync(full, tr, o);
+      tt += __shfl_xor_sync(full, tt, o);
+    }
+    // an empty residual (p_theta = p_phi to fp32 precision) cannot reject:
+    // the draw falls back to p_theta
+    int mode = (resid && tr > kResidFloor) || (!resid && tr > 0.f) ? 0 : (tt > 0.f ? 1 : -1);
+    const float total = mode == 0 ? tr : tt;
+    const float thr = u_sample[b] * total;
+    int owner = -1, last_pos = -1;
+    float base = 0.f, last_base = 0.f, run = 0.f;
+    for (int q0 = 0; q0 < rparts && mode >= 0 && owner < 0; q0 += 32) {
+      const int q = q0 + lane;
+      const float wq = q < rparts ? vs[2 * q + (mode == 0 ? 0 : 1)] : 0.f;
+      float incl = wq;
+#pragma unroll
+      for (int o = 1; o < 32; o <<= 1) {
+        const float y = __shfl_up_sync(full, incl, o);
+        if (lane >= o) incl += y;
+      }
+      incl += run;
+      const unsigned hold = __ballot_sync(full, wq > 0.f && thr < incl);
+      const unsigned pos = __ballot_sync(full, wq > 0.f);
+      if (hold) {
+        const int l = __ffs(hold) - 1;
+        owner = q0 + l;
+        base = __shfl_sync(full, incl - wq, l);
+      } else if (pos) {
+        const int l = 31 - __clz(pos);
+        last_pos = q0 + l;
+        last_base = __shfl_sync(full, incl - wq, l);
+      }
+      run = __shfl_sync(full, incl, 31);
+    }
+    if (owner < 0 && mode >= 0) {
+      owner = last_pos;
+      base = last_base;
+    }
+    if (lane == 0) {
+      mode_sh = owner < 0 ? -1 : mode;
+      owner_sh = owner;
+      thr_sh = thr;
+      base_sh = base;
+      tok_sh = 0x7fffffff;
+      pos_sh = -1;
+    }
+  }
+  __syncthreads();
+  const int mode = mode_sh;
+  if (mode < 0) {
+    if (tid == 0) out_tokens[static_cast<size_t>(b) * (gamma + 1) + a] = -1;
+    return;
+  }
+  // ---- the owner span: thread t takes k consecutive units, a scan over the
+  // threads, then each thread walks its own units in order
+  const int u0 = min(W, owner_sh * per), u1 = min(W, u0 + per);
+  const int k = (u1 - u0 + kSampThreads - 1) / kSampThreads;
+  const int t0 = min(u1, u0 + tid * k), t1 = min(u1, t0 + k);
+  float mine = 0.f;
+  for (int u = t0; u < t1; ++u) {
+    const UnitW uw = unit_weights<VEC>(rw, u);
+    const float4 w = mode == 0 ? uw.r : uw.t;
+    mine += (w.x + w.y) + (w.z + w.w);
+  }
+  // exclusive scan of the threads' sums (in thread order = vocabulary order)
+  float incl = mine;
+#pragma unroll
+  for (int o = 1; o < 32; o <<= 1) {
+    const float y = __shfl_up_sync(full, incl, o);
+    if (lane >= o) incl += y;
+  }
+  if (lane == 31) red[warp] = incl;
+  __syncthreads();
+  float before = 0.f;
+  for (int w = 0; w < warp; ++w) before += red[w];
+  float cum = base_sh + before + incl - mine;
+  const float thr = thr_sh;
+  int hit = -1, lastp = -1;
+  // one column: its weight, then the cumulative weight past it
+  auto step = [&](float w, int col) {
+    if (w > 0.f) {
+      if (hit < 0 && cum + w > thr) hit = col;
+      lastp = col;
+    }
+    cum += w;
+  };
+  for (int u = t0; u < t1 && hit < 0; ++u) {
+    const UnitW uw = unit_weights<VEC>(rw, u);
+    const float4 w = mode == 0 ? uw.r : uw.t;
+    const int col = VEC ? 4 * u : u;  // (the scalar layout's other three weights are 0)
+    step(w.x, col);
+    step(w.y, col + 1);
+    step(w.z, col + 2);
+    step(w.w, col + 3);
+  }
+  if (hit >= 0) atomicMin(&tok_sh, hit);
+  if (lastp >= 0) atomicMax(&pos_sh, lastp);
+  __syncthreads();
+  if (tid == 0) out_tokens[static_cast<size_t>(b) * (gamma + 1) + a] = tok_sh != 0x7fffffff ? tok_sh : pos_sh;
 }
 
 struct SampCapacity {
@@ -646,10 +910,9 @@ cudaError_t samp_capacity(const SampCapacity** out) {
 template <bool VEC, int UNROLL>
 cudaError_t launch_samp(dim3 grid, unsigned CL, cudaStream_t stream, const float* tl, const float* dl,
                         const int32_t* draft, const float* ua, const float* us, float zscale, int gamma, int vocab,
-                        int32_t* accepted_len, int32_t* out_tokens, int32_t* err_word, const float2* pre,
-                        int pre_parts) {
+                        int32_t* accepted_len, int32_t* out_tokens, int32_t* err_word) {
   return launch_overlapped(accept_sampled_kernel<VEC, UNROLL>, grid, dim3(kSampThreads), 0, stream, CL, tl, dl,
-                           draft, ua, us, zscale, gamma, vocab, accepted_len, out_tokens, err_word, pre, pre_parts);
+                           draft, ua, us, zscale, gamma, vocab, accepted_len, out_tokens, err_word);
 }
 
 }  // namespace
@@ -659,25 +922,65 @@ int samp_parts(int Bt, int gamma, int vocab, int num_sms) {
   // logits (target and draft rows), about 8 units of 16 bytes per thread
   if (static_cast<long long>(Bt) * kSampMaxCluster > num_sms) return 0;
   const long long rows = 2LL * gamma + 1;
-  // when the clusters alone already cover over half the SMs the extra launch
-  // pays only for larger blocks (8 sequences: 10 MB each 35.2 us in clusters
-  // against 37.1 us split, 20 MB 52.0 against 47.5 us)
-  const long long min_bytes = static_cast<long long>(Bt) * kSampMaxCluster * 2 > num_sms ? (12LL << 20) : (6LL << 20);
-  if (rows * vocab * 4 < min_bytes) return 0;
+  // at least 3 MiB of logits a sequence (measured with the current second
+  // launch, L2 flushed: 1 x 9 rows 23.2 -> 19.6 us, 8 x 17 rows 37.5 -> 34.4
+  // us; 4 x 9 rows even)
+  if (rows * vocab * 4 < (3LL << 20)) return 0;
   const long long units = rows * ((vocab + 3) / 4);
-  const long long parts = std::min(units / (8LL * kSampThreads), (2LL * num_sms + Bt - 1) / Bt);
+  // at most two CTAs per SM in all: one wave
+  const long long parts = std::min(units / (8LL * kSampThreads), 2LL * num_sms / Bt);
   return parts > kSampMaxCluster ? static_cast<int>(parts) : 0;
 }
 
+// Spans of row a in samp_resid_kernel: about 1024 units (16 KB of each of
+// the two rows) a CTA, at most the parts of phase 1.
+int samp_resid_parts(int parts, int vocab) {
+  const int units = (vocab + 3) / 4;
+  return std::max(1, std::min(parts, (units + 1023) / 1024));
+}
+
+// Workspace of the split path: the parts' (m, s) [Bt][parts][rows] (float2),
+// the spans' weight sums of row a [Bt][rparts <= parts] (float2: residual,
+// p_theta), then an arrival count per sequence (uint32).
 size_t samp_workspace_bytes(int Bt, int gamma, int vocab, int num_sms) {
   const int parts = samp_parts(Bt, gamma, vocab, num_sms);
-  return parts ? static_cast<size_t>(Bt) * parts * (2 * gamma + 1) * sizeof(float2) : 0;
+  if (!parts) return 0;
+  const size_t n = static_cast<size_t>(Bt) * parts;
+  return n * (2 * gamma + 1) * sizeof(float2) + n * sizeof(float2) + ((static_cast<size_t>(Bt) * 4 + 7) & ~size_t{7});
 }
 
 cudaError_t launch_accept_sampled(const float* target_logits, const float* draft_logits, const int32_t* draft,
                                   const float* u_accept, const float* u_sample, float temperature, int Bt,
                                   int gamma, int vocab, int32_t* accepted_len, int32_t* out_tokens,
                                   int32_t* err_word, cudaStream_t stream, void* workspace, int num_sms) {
+  const bool vec4 = (vocab % 4 == 0) && ((reinterpret_cast<uintptr_t>(target_logits) & 15u) == 0) &&
+                    ((reinterpret_cast<uintptr_t>(draft_logits) & 15u) == 0);
+  const float zscale = kLog2e / temperature;
+  // with a workspace and few sequences: the log-sum-exp pass split over many
+  // CTAs (samp_part_kernel), then samp_resid_kernel over the same CTAs
+  const int parts = workspace ? samp_parts(Bt, gamma, vocab, num_sms) : 0;
+  if (parts) {
+    const size_t n = static_cast<size_t>(Bt) * parts;
+    float2* pre = static_cast<float2*>(workspace);
+    float2* sums = pre + n * (2 * gamma + 1);
+    unsigned* arrivals = reinterpret_cast<unsigned*>(sums + n);
+    const dim3 pgrid(static_cast<unsigned>(n));
+    const int rparts = samp_resid_parts(parts, vocab);
+    const dim3 rgrid(static_cast<unsigned>(Bt) * rparts);
+    cudaError_t e = vec4 ? launch_overlapped(samp_part_kernel<true>, pgrid, dim3(kSampThreads), 0, stream, 1u,
+                                             target_logits, draft_logits, zscale, gamma, vocab, parts, pre, arrivals)
+                         : launch_overlapped(samp_part_kernel<false>, pgrid, dim3(kSampThreads), 0, stream, 1u,
+                                             target_logits, draft_logits, zscale, gamma, vocab, parts, pre, arrivals);
+    if (e != cudaSuccess) return e;
+    return vec4 ? launch_overlapped(samp_resid_kernel<true>, rgrid, dim3(kSampThreads), 0, stream, 1u, target_logits,
+                                    draft_logits, draft, u_accept, u_sample, zscale, gamma, vocab, accepted_len,
+                                    out_tokens, err_word, static_cast<const float2*>(pre), parts, rparts, sums,
+                                    arrivals)
+                : launch_overlapped(samp_resid_kernel<false>, rgrid, dim3(kSampThreads), 0, stream, 1u,
+                                    target_logits, draft_logits, draft, u_accept, u_sample, zscale, gamma, vocab,
+                                    accepted_len, out_tokens, err_word, static_cast<const float2*>(pre), parts, rparts,
+                                    sums, arrivals);
+  }
   const SampCapacity* cap = nullptr;
   cudaError_t e = samp_capacity(&cap);
   if (e != cudaSuccess) return e;
@@ -690,31 +993,17 @@ cudaError_t launch_accept_sampled(const float* target_logits, const float* draft
       break;
     }
   const bool deep = cap->resident16[CL] >= Bt;
-  const bool vec4 = (vocab % 4 == 0) && ((reinterpret_cast<uintptr_t>(target_logits) & 15u) == 0) &&
-                    ((reinterpret_cast<uintptr_t>(draft_logits) & 15u) == 0);
   const dim3 grid(static_cast<unsigned>(Bt) * CL);
-  const float zscale = kLog2e / temperature;
   const unsigned ucl = static_cast<unsigned>(CL);
-  // with a workspace and few sequences, phase 1 runs in samp_part_kernel
-  const int parts = workspace ? samp_parts(Bt, gamma, vocab, num_sms) : 0;
-  float2* pre = parts ? static_cast<float2*>(workspace) : nullptr;
-  if (parts) {
-    const dim3 pgrid(static_cast<unsigned>(Bt) * parts);
-    e = vec4 ? launch_overlapped(samp_part_kernel<true>, pgrid, dim3(kSampThreads), 0, stream, 1u, target_logits,
-                                 draft_logits, zscale, gamma, vocab, parts, pre)
-             : launch_overlapped(samp_part_kernel<false>, pgrid, dim3(kSampThreads), 0, stream, 1u, target_logits,
-                                 draft_logits, zscale, gamma, vocab, parts, pre);
-    if (e != cudaSuccess) return e;
-  }
   if (vec4)
     return deep ? launch_samp<true, 16>(grid, ucl, stream, target_logits, draft_logits, draft, u_accept, u_sample,
-                                        zscale, gamma, vocab, accepted_len, out_tokens, err_word, pre, parts)
+                                        zscale, gamma, vocab, accepted_len, out_tokens, err_word)
                 : launch_samp<true, 8>(grid, ucl, stream, target_logits, draft_logits, draft, u_accept, u_sample,
-                                       zscale, gamma, vocab, accepted_len, out_tokens, err_word, pre, parts);
+                                       zscale, gamma, vocab, accepted_len, out_tokens, err_word);
   return deep ? launch_samp<false, 16>(grid, ucl, stream, target_logits, draft_logits, draft, u_accept, u_sample,
-                                       zscale, gamma, vocab, accepted_len, out_tokens, err_word, pre, parts)
+                                       zscale, gamma, vocab, accepted_len, out_tokens, err_word)
               : launch_samp<false, 8>(grid, ucl, stream, target_logits, draft_logits, draft, u_accept, u_sample,
-                                      zscale, gamma, vocab, accepted_len, out_tokens, err_word, pre, parts);
+                                      zscale, gamma, vocab, accepted_len, out_tokens, err_word);
 }
 
 }  // namespace simsd

@@ -215,7 +215,7 @@ def main(argv=None):
                 f.write(f"| Bt | gamma | path | us | GB/s (rows read once) | of {peak:.0f} GB/s |\n"
                         "|---|---|---|---|---|---|\n")
                 for r in rows:
-                    path = "parts + cluster" if r["kernel"].endswith("+parts") else "cluster"
+                    path = "parts + spans" if r["kernel"].endswith("+parts") else "cluster"
                     f.write(f"| {r['Bt']} | {r['gamma']} | {path} | {r['us']:.1f} | {r['gbs']:.0f} | "
                             f"{100 * r['frac']:.1f}% |\n")
         return
