@@ -348,11 +348,12 @@ cudaError_t cluster_capacity(const ClusterCapacity** out) {
 int accept_parts(int Bt, int gamma, int vocab, int num_sms) {
   // few sequences only: one 16-CTA cluster each leaves SMs idle
   if (static_cast<long long>(Bt) * kMaxCluster > num_sms) return 0;
-  // and at least 6 MiB of logits per sequence: below that the cluster's 16
+  // and at least 4 MiB of logits per sequence: below that the cluster's 16
   // CTAs stream it about as fast as the split, which pays a second launch
-  // (measured: 3 MB per sequence 13 us either way, 15 us cluster against
-  // 17 us split at 8 sequences; 10 MB 23 against 18 us)
-  if (static_cast<long long>(gamma + 1) * vocab * 4 < (6LL << 20)) return 0;
+  // (measured, L2 flushed: 3 MB per sequence 15.0 us cluster against 15.5
+  // us split at 8 sequences; 5.5 MB 21.2 against 18.1 us, 10 MB 23.2
+  // against 14.0 us at one sequence)
+  if (static_cast<long long>(gamma + 1) * vocab * 4 < (4LL << 20)) return 0;
   // about 8 units of 16 bytes per thread of a part, at most two parts per SM
   const long long units = static_cast<long long>(gamma + 1) * ((vocab + 3) / 4);
   const long long by_work = units / (8LL * kAcceptThreads);

@@ -41,9 +41,10 @@ def _run_ws(logits, draft, expect_split=None):
 
 
 @pytest.mark.parametrize("Bt,gamma,V", [(1, 16, 151936), (1, 32, 151936), (2, 16, 151936), (5, 16, 151936),
-                                        (9, 12, 151936), (2, 16, 151935), (3, 32, 50001)])
+                                        (9, 12, 151936), (2, 16, 151935), (3, 32, 50001), (8, 8, 151936),
+                                        (4, 8, 151936)])
 def test_split_bit_exact(Bt, gamma, V):
-    # few sequences with at least 6 MiB of logits each: the logits of each
+    # few sequences with at least 4 MiB of logits each: the logits of each
     # split over many CTAs; an odd vocabulary streams scalars
     logits, draft = _accept_case(Bt, gamma, V, seed=Bt * 100 + gamma + V % 7)
     _run_ws(logits, draft, expect_split=True)
@@ -52,7 +53,7 @@ def test_split_bit_exact(Bt, gamma, V):
 @pytest.mark.parametrize("Bt,gamma,V", [(64, 16, 151936), (10, 16, 151936), (8, 4, 151936), (1, 4, 151936),
                                         (2, 4, 1024), (1, 1, 64)])
 def test_no_split_keeps_the_cluster_kernel(Bt, gamma, V):
-    # more sequences than SMs / 16, or under 6 MiB of logits a sequence: no
+    # more sequences than SMs / 16, or under 4 MiB of logits a sequence: no
     # workspace, the cluster kernel, same results
     logits, draft = _accept_case(Bt, gamma, V, seed=7 + Bt)
     _run_ws(logits, draft, expect_split=False)
