@@ -194,11 +194,11 @@ def attention_check(got, ref):
           "rms_rel": float(np.sqrt(np.nanmean(diff * diff)) / rms_r) if rms_r > 0 else 0.0,
           "max_abs_r": float(np.max(np.abs(r))) if r.size else 0.0}
     if ref.dtype == "f32":
-        st["north_star_ok"] = finite and st["max_abs"] <= F32_ATOL
-        st["bound_ok"] = st["north_star_ok"]
+        st["tolerance_ok"] = finite and st["max_abs"] <= F32_ATOL
+        st["bound_ok"] = st["tolerance_ok"]
         st["max_ratio"] = st["max_abs"] / F32_ATOL
     else:
-        st["north_star_ok"] = finite and bool((diff <= BF16_ATOL + BF16_RTOL * np.abs(r)).all())
+        st["tolerance_ok"] = finite and bool((diff <= BF16_ATOL + BF16_RTOL * np.abs(r)).all())
         mag = ref.absv + np.abs(r)
         tol = mag * (U_BF16 * (1 + 2.0 ** -7) + math.expm1(2 * ref.delta) + (ref.tiles + 70) * 2.0 ** -23) + 1e-12
         ratio = diff / tol
@@ -206,7 +206,7 @@ def attention_check(got, ref):
         st["max_ratio"] = float(np.nanmax(ratio)) if r.size else 0.0
         st["bound_median"] = float(np.median(tol)) if r.size else 0.0
         st["out_of_bound"] = int((~(ratio <= 1.0)).sum())
-    st["ok"] = st["north_star_ok"] and st["bound_ok"]
+    st["ok"] = st["tolerance_ok"] and st["bound_ok"]
     return st
 
 
@@ -214,6 +214,6 @@ def assert_attention_close(got, ref):
     st = attention_check(got, ref)
     PARITY_LOG.append((os.environ.get("PYTEST_CURRENT_TEST", "?").split(" ")[0], st))
     assert st["finite"], "non-finite output"
-    assert st["north_star_ok"], f"outside the stated tolerance: {st}"
+    assert st["tolerance_ok"], f"outside the stated tolerance: {st}"
     assert st["bound_ok"], f"outside the derived bf16 bound: {st}"
     return st["max_abs"]

@@ -44,7 +44,7 @@ def _case(name, seqs=None, layers=None):
 def test_zero_output_fails(name, seqs, layers):
     _, got, ref = _case(name, seqs, layers)
     st = attention_check(torch.zeros_like(got), ref)
-    assert st["north_star_ok"], "the stated tolerance alone accepts zeros at this size"
+    assert st["tolerance_ok"], "the stated tolerance alone accepts zeros at this size"
     assert not st["bound_ok"] and st["out_of_bound"] > 0.5 * st["elements"], st
 
 
