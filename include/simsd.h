@@ -114,10 +114,9 @@ SIMSD_API int simsd_build_mask(const int32_t* step_map, const int32_t* prefix_le
  * max_pages*page_size bounds every prefix length.  Shapes with 129..256
  * query rows per KV head (for example 32 drafts with 32/8 heads) and at
  * most 255 sequences whose units (sequence, KV head) would load the SMs
- * unevenly (with at least one unit per SM: the busiest SM 10% above the
- * mean; with fewer: when equal shares cost less than equal ranges of every
- * unit) give every CTA an equal share of all key tiles and need about
- * 266 KB per SM (40 MB on 152 SMs).
+ * unevenly enough that equal shares pay for their extra pieces and merge
+ * (long prefixes: a cost model in key tiles) give every CTA an equal share
+ * of all key tiles and need about 266 KB per SM (40 MB on 152 SMs).
  */
 SIMSD_API size_t simsd_verify_workspace_bytes(int dtype, int Bt, int gamma, int Hq, int Hkv, int d, int max_pages,
                                     int page_size);

@@ -119,10 +119,10 @@ bool make_bf16_map(EncodeTiledFn encode, CUtensorMap* m, const void* base, int r
 // blocks, or fewer units than SMs with under 16 key tiles each), else the
 // key-tile ranges per unit (1 when there are at least as many units as SMs).
 int tc256_splits(int Bt, int Hkv, int rb, long long max_tiles, int num_sms);
-// 1 when the kernel walks stream-K runs instead of the nsplit ranges that
-// tc256_splits chose (Bt <= 255; with at least as many units as SMs when
-// the whole-unit walk is uneven by at least 10%, with fewer when the cost
-// model favours equal runs); its partial workspace is tc256_streamk_bytes.
+// 1 when the kernel walks stream-K runs instead of the nsplit ranges (or
+// whole units) that tc256_splits chose: Bt <= 255 and a cost model in key
+// tiles favours equal runs by at least 3%; its partial workspace is
+// tc256_streamk_bytes.
 int tc256_streamk(int Bt, int Hkv, long long max_tiles, int nsplit, int num_sms);
 size_t tc256_streamk_bytes(int num_sms);
 cudaError_t launch_attention_tc256(const AttnTcArgs& a, const AttnTcPlan& pl, EncodeTiledFn encode,

@@ -56,20 +56,20 @@ def _splits(si):
 
 
 def _streamk(si):
-    # at most 255 sequences; with at least one unit per SM when whole units
-    # would give the busiest CTAs at least 10% more than the mean, with fewer
-    # when equal runs plus three items cost less than the chosen ranges
+    # at most 255 sequences, and equal runs of all key tiles cost at least 3%
+    # less than the ranges (or whole units): per CTA, items of their tiles
+    # plus 14 each; a run of W tiles overlaps ceil(W / T) + 1 units, plus 10
+    # for the merge launch
     w = si.w
     sms = torch.cuda.get_device_properties(0).multi_processor_count
     units = w.Bt * w.Hkv
-    max_tiles = (si.block_table.shape[1] * w.page_size + 63) // 64 + 1
+    T = (si.block_table.shape[1] * w.page_size + 63) // 64 + 1
     ns = _splits(si)
-    if ns < 1 or w.Bt > 255 or units * max_tiles >= 1 << 30:
+    if ns < 1 or w.Bt > 255 or units * T >= 1 << 30:
         return False
-    if units >= sms:
-        return -(-units // sms) * sms * 10 >= units * 11
-    ranges = -(-units * ns // sms) * (-(-max_tiles // ns) + 14)
-    return -(-units * max_tiles // sms) + 3 * 14 < ranges
+    ranges = -(-units * ns // sms) * (-(-T // ns) + 14)
+    W = -(-units * T // sms)
+    return (W + (-(-W // T) + 1) * 14 + 10) * 100 < ranges * 97
 
 
 def _check(si, seqs=None, rope=None):
@@ -138,24 +138,48 @@ def test_whole_units_one_per_sm():
     _check(si, seqs=[0, 9, 18])
 
 
-@pytest.mark.parametrize("Bt,lens", [
-    (20, [9000] + [10] * 19),                            # the long units span many CTAs each
-    (20, [0, 64, 65, 4000, 1] * 4),                      # ragged; runs start inside and between units
-    (24, [3000, 0, 2500, 0, 700, 129] * 4),
-    (40, list(range(0, 4000, 100))),
+@pytest.mark.parametrize("Bt,lens,P", [
+    (20, [9000] + [10] * 19, 64),                        # the long units span many CTAs each
+    (20, [9000] + [10] * 19, 16),
+    (20, [0, 64, 65, 4000, 1] * 4, 64),                  # ragged; runs start inside and between units
+    (20, [0, 64, 65, 4000, 1] * 4, 256),
+    (24, [3000, 0, 2500, 0, 700, 129] * 4, 64),
+    (40, list(range(0, 4000, 100)), 32),
 ])
-def test_streamk_runs(Bt, lens):
-    si = inputs.make_step_inputs(_w(Bt, prefix=(0, max(lens)), seed=Bt + len(set(lens))), device="cuda",
+def test_streamk_runs(Bt, lens, P):
+    si = inputs.make_step_inputs(_w(Bt, prefix=(0, max(lens)), P=P, seed=Bt + len(set(lens)) + P), device="cuda",
                                  prefix_override=np.array(lens), random_step_map=True, poison_unused_rows=True)
     assert _streamk(si)
     _check(si, seqs=sorted({0, 1, 3, Bt // 2, Bt - 1}))
 
 
+@pytest.mark.parametrize("mode", [1, 2])
+def test_streamk_rope(mode):
+    si = inputs.make_step_inputs(_w(20, prefix=(2000, 3000), seed=40 + mode), device="cuda", random_step_map=True)
+    assert _streamk(si)
+    _check(si, seqs=[0, 10, 19], rope=(1e6, mode))
+
+
+def test_streamk_deterministic():
+    si = inputs.make_step_inputs(_w(24, prefix=(1500, 4000), seed=16), device="cuda", random_step_map=True)
+    assert _streamk(si)
+    a, _, _ = gpu_attention(si)
+    b, _, _ = gpu_attention(si)
+    assert torch.equal(a, b)
+
+
+def test_short_units_stay_whole():
+    # 20 sequences of at most 700 keys (12 tiles): the pieces and the merge
+    # of equal runs would cost more than the uneven whole units
+    si = inputs.make_step_inputs(_w(20, prefix=(0, 700), seed=17), device="cuda")
+    assert _splits(si) == 1 and not _streamk(si)
+
+
 def test_streamk_small_batch_long_prefixes():
-    # 8 x 8 units of ~460 tiles, fewer than SMs: equal runs of ~200 tiles
-    # (units spanning three CTAs) cost less than two ranges a unit, which
-    # leave 24 of 152 SMs idle
-    si = inputs.make_step_inputs(_w(8, prefix=(28000, 30000), seed=15), device="cuda", random_step_map=True)
+    # 8 x 8 units of ~510 tiles, fewer than SMs: equal runs of ~216 tiles
+    # (units spanning three CTAs) cost less than seven ranges a unit in three
+    # waves of items (measured 262 -> 244 us at 32768 keys)
+    si = inputs.make_step_inputs(_w(8, prefix=(32000, 32768), seed=15), device="cuda", random_step_map=True)
     assert _splits(si) > 1 and _streamk(si)
     _check(si, seqs=[0, 7])
 

@@ -21,21 +21,21 @@ pytestmark = pytest.mark.gpu
 
 
 @pytest.mark.parametrize("Bt,Hq,gamma,prefix", [(40, 16, 4, (100, 300)), (20, 32, 32, (100, 300)),
-                                               (2, 32, 32, (1500, 2000))])
+                                               (20, 32, 32, (3000, 4000)), (2, 32, 32, (1500, 2000))])
 def test_attention_wait_runs_out_and_the_context_stays_usable(Bt, Hq, gamma, prefix):
     # 40 sequences x 8 KV heads of 16 rows: 320 unsplit units in two waves
     # of the one-row-block kernel; 20 x 8 units of 256 rows: the persistent
-    # two-row-block kernel in stream-K runs, then its merge (each block's PV
-    # issuer waits for P that the planted count never completes); 2 x 8
-    # units of 256 rows: the same kernel with key-tile ranges, then the
-    # combine kernel
+    # two-row-block kernel on whole short units, or in stream-K runs of long
+    # ones, then their merge (each block's PV issuer waits for P that the
+    # planted count never completes); 2 x 8 units of 256 rows: the same
+    # kernel with key-tile ranges, then the combine kernel
     w = inputs.Workload("we", "bf16", Bt, Hq, 8, 128, gamma, prefix, 1, 64, 0.5, 1 / np.sqrt(128), 1.0, 31)
     si = inputs.make_step_inputs(w, device="cuda", random_step_map=True, with_logits=False)
     tau, sect, _, _, merr = gpu_mask(si, mask_bits=False)
     assert simsd.simsd_check_error(merr) == 0
     before, word, ws = gpu_attention(si, mask=(tau, sect))
     # a workspace for the ranges and the stream-K partials of the 256-row units
-    assert word == 0 and (ws > 0) == (gamma == 32)
+    assert word == 0 and (ws > 0) == (gamma == 32 and (Bt == 2 or prefix[0] >= 3000))
     simsd.simsd_debug_expire_next_wait(simsd.DEBUG_WAIT_ATTENTION, 200)
     out = torch.full_like(si.q[0], float("nan"))
     err = torch.zeros(1, dtype=torch.int32, device="cuda")

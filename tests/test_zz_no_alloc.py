@@ -84,7 +84,7 @@ def test_noalloc_keeps_whole_units_where_streamk_runs():
     # (40 MB of partials); the no-alloc entry point keeps the units whole,
     # no scratch: another order of summation, both within the bars
     from tests._gpu import assert_attention_close, oracle_attention
-    w = inputs.Workload("na5", "bf16", 20, 32, 8, 128, 32, (100, 900), 1, 64, 0.5, 1 / np.sqrt(128), 1.0, 25)
+    w = inputs.Workload("na5", "bf16", 20, 32, 8, 128, 32, (3000, 4000), 1, 64, 0.5, 1 / np.sqrt(128), 1.0, 25)
     si = inputs.make_step_inputs(w, device="cuda", random_step_map=True, with_logits=False)
     tau, sect, _, _, _ = gpu_mask(si, mask_bits=False)
     want, ws = _regular(si, tau, sect)
