@@ -341,6 +341,32 @@ SIMSD_API int simsd_kv_commit(int dtype, const void* k_new, const void* v_new, i
 SIMSD_API int simsd_check_error(const int32_t* err_word, int32_t* host_word, void* stream);
 
 /*
+ * simsd_plan_attention -- the work decomposition simsd_verify_attention
+ * takes for these sizes on a GPU with num_sms SMs (a diagnostic for host
+ * code and tests; the paper has no counterpart).  Pure host arithmetic: no
+ * device is touched, so it works without a GPU.
+ *   plan[5]   int32, written: [0] kernel (0 bf16 one row block per CTA,
+ *             1 bf16 256-row units, 2 fp32 CUDA cores); [1] key-tile
+ *             ranges per unit (1: whole units); [2] 1 when the 256-row
+ *             kernel walks stream-K runs; [3] query rows per row block;
+ *             [4] 1 when 2..8 ranges merge in a cluster (no workspace).
+ *   ws_bytes  written: the workspace simsd_verify_attention needs on such a
+ *             device (what simsd_verify_workspace_bytes returns there).
+ * Bt = 0 is accepted (an empty batch: no workspace).  Returns SIMSD_OK,
+ * SIMSD_ERR_INVALID_ARG (null outputs, num_sms < 1, sizes out of range) or
+ * SIMSD_ERR_UNSUPPORTED (a shape the kernels do not take).
+ *
+ * simsd_plan_accept -- the same for simsd_accept_ws (sampled = 0) and
+ * simsd_accept_sampled_ws (sampled = 1): *parts CTAs per sequence for the
+ * streaming pass (0: the cluster kernel, no workspace) and *ws_bytes of
+ * workspace.  Returns SIMSD_OK or SIMSD_ERR_INVALID_ARG.
+ */
+SIMSD_API int simsd_plan_attention(int dtype, int Bt, int gamma, int Hq, int Hkv, int d, int max_pages,
+                                   int page_size, int num_sms, int32_t* plan, size_t* ws_bytes);
+SIMSD_API int simsd_plan_accept(int sampled, int Bt, int gamma, int vocab, int num_sms, int32_t* parts,
+                                size_t* ws_bytes);
+
+/*
  * simsd_debug_expire_next_wait -- test hook for failure detection; the paper
  * has no counterpart.  Arms the next bf16 simsd_verify_attention
  * (which = SIMSD_DEBUG_WAIT_ATTENTION) or simsd_accept

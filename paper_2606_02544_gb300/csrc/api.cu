@@ -386,6 +386,48 @@ size_t simsd_accept_sampled_workspace_bytes(int Bt, int gamma, int vocab) {
   return simsd::samp_workspace_bytes(Bt, gamma, vocab, info.num_sms);
 }
 
+int simsd_plan_attention(int dtype, int Bt, int gamma, int Hq, int Hkv, int d, int max_pages, int page_size,
+                         int num_sms, int32_t* plan, size_t* ws_bytes) {
+  if (!plan || !ws_bytes || num_sms < 1) return arg_fail("null output or num_sms < 1");
+  if (Bt < 0 || gamma < 1 || gamma > 32 || Hq <= 0 || Hkv <= 0 || Hq % Hkv != 0 || max_pages < 0 ||
+      page_size <= 0)
+    return arg_fail("sizes out of range");
+  for (int i = 0; i < 5; ++i) plan[i] = 0;
+  *ws_bytes = 0;
+  if (dtype == SIMSD_F32) {
+    if (d != 64 && d != 128) return unsupported("fp32 path needs d = 64 or 128");
+    plan[0] = 2;
+    plan[1] = 1;
+    plan[3] = 2 * gamma * (Hq / Hkv);
+    return SIMSD_OK;
+  }
+  if (dtype != SIMSD_BF16) return unsupported("dtype");
+  if (d != 128) return unsupported("bf16 path needs d = 128");
+  simsd::AttnTcPlan pl;
+  if (!simsd::plan_attention_tc(Bt > 0 ? Bt : 1, gamma, Hq, Hkv, max_pages, page_size, num_sms, &pl))
+    return unsupported("query rows per KV head: need 2*gamma*Hq/Hkv <= 128 or 128 % (Hq/Hkv) == 0");
+  plan[0] = pl.kind;
+  plan[1] = pl.nsplit;
+  plan[2] = pl.streamk;
+  plan[3] = pl.rows_blk;
+  plan[4] = pl.fuse;
+  *ws_bytes = Bt > 0 ? pl.ws_bytes : 0;
+  return SIMSD_OK;
+}
+
+int simsd_plan_accept(int sampled, int Bt, int gamma, int vocab, int num_sms, int32_t* parts, size_t* ws_bytes) {
+  if (!parts || !ws_bytes || num_sms < 1) return arg_fail("null output or num_sms < 1");
+  if (Bt < 0 || gamma < 1 || gamma > 32 || vocab < 1 || vocab > (sampled ? (1 << 24) : (1 << 28)))
+    return arg_fail("sizes out of range");
+  *parts = 0;
+  *ws_bytes = 0;
+  if (Bt == 0) return SIMSD_OK;
+  *parts = sampled ? simsd::samp_parts(Bt, gamma, vocab, num_sms) : simsd::accept_parts(Bt, gamma, vocab, num_sms);
+  *ws_bytes = sampled ? simsd::samp_workspace_bytes(Bt, gamma, vocab, num_sms)
+                      : simsd::accept_workspace_bytes(Bt, gamma, vocab, num_sms);
+  return SIMSD_OK;
+}
+
 int simsd_accept_sampled_ws(const float* target_logits, const float* draft_logits, const int32_t* draft,
                             const float* u_accept, const float* u_sample, float temperature, int Bt, int gamma,
                             int vocab, int32_t* accepted_len, int32_t* out_tokens, void* workspace,

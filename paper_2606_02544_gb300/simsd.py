@@ -27,7 +27,7 @@ STEP_UNDRAFTED, STEP_DECODED = -1, -2
 EXPORTED = ("simsd_build_mask", "simsd_verify_workspace_bytes", "simsd_verify_attention",
             "simsd_verify_attention_noalloc", "simsd_accept", "simsd_accept_workspace_bytes", "simsd_accept_ws",
             "simsd_accept_sampled", "simsd_accept_sampled_workspace_bytes", "simsd_accept_sampled_ws",
-            "simsd_kv_commit",
+            "simsd_kv_commit", "simsd_plan_attention", "simsd_plan_accept",
             "simsd_check_error", "simsd_debug_expire_next_wait",
             "simsd_last_error", "simsd_version")
 DEBUG_WAIT_ATTENTION, DEBUG_WAIT_ACCEPT = 1, 2
@@ -71,10 +71,13 @@ def load_library(path: str = LIB_PATH):
             lib.simsd_kv_commit.argtypes = [I, P, P, I, P, P, P, F, P, P, P, I, P, I, I, P, I, I, I, I, P, P]
             lib.simsd_check_error.argtypes = [P, P, P]
             lib.simsd_debug_expire_next_wait.argtypes = [I, ctypes.c_uint]
+            lib.simsd_plan_attention.argtypes = [I, I, I, I, I, I, I, I, I, P, P]
+            lib.simsd_plan_accept.argtypes = [I, I, I, I, I, P, P]
             lib.simsd_last_error.restype = ctypes.c_char_p
             for name in ("simsd_build_mask", "simsd_verify_attention", "simsd_verify_attention_noalloc",
                          "simsd_accept", "simsd_accept_sampled", "simsd_kv_commit", "simsd_check_error",
-                         "simsd_debug_expire_next_wait", "simsd_version"):
+                         "simsd_debug_expire_next_wait", "simsd_version", "simsd_plan_attention",
+                         "simsd_plan_accept"):
                 getattr(lib, name).restype = ctypes.c_int
             _lib = lib
     return _lib
@@ -105,6 +108,32 @@ def _dtype_code(t):
 
 def simsd_version() -> int:
     return load_library().simsd_version()
+
+
+def simsd_plan_attention(dtype, Bt, gamma, Hq, Hkv, d, max_pages, page_size, num_sms):
+    """The plan simsd_verify_attention takes on a GPU with num_sms SMs (no
+    device needed): dict of kernel, nsplit, streamk, rows_blk, fuse and
+    ws_bytes."""
+    plan = (ctypes.c_int32 * 5)()
+    ws = ctypes.c_size_t(0)
+    rc = load_library().simsd_plan_attention(dtype, Bt, gamma, Hq, Hkv, d, max_pages, page_size, num_sms,
+                                             ctypes.cast(plan, ctypes.c_void_p), ctypes.cast(ctypes.pointer(ws),
+                                                                                            ctypes.c_void_p))
+    _check(rc, "simsd_plan_attention")
+    return {"kernel": plan[0], "nsplit": plan[1], "streamk": plan[2], "rows_blk": plan[3], "fuse": plan[4],
+            "ws_bytes": ws.value}
+
+
+def simsd_plan_accept(sampled, Bt, gamma, vocab, num_sms):
+    """(parts, ws_bytes) of simsd_accept_ws (sampled False) or
+    simsd_accept_sampled_ws (True) on a GPU with num_sms SMs."""
+    parts = ctypes.c_int32(0)
+    ws = ctypes.c_size_t(0)
+    rc = load_library().simsd_plan_accept(int(bool(sampled)), Bt, gamma, vocab, num_sms,
+                                          ctypes.cast(ctypes.pointer(parts), ctypes.c_void_p),
+                                          ctypes.cast(ctypes.pointer(ws), ctypes.c_void_p))
+    _check(rc, "simsd_plan_accept")
+    return parts.value, ws.value
 
 
 def simsd_build_mask(step_map, prefix_len, gamma, tau, section, rope_pos, mask_bits=None, err_word=None,

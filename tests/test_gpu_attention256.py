@@ -22,6 +22,7 @@ import pytest
 import torch
 
 from paper_2606_02544_gb300 import inputs, simsd
+from tests import _plan
 from tests._gpu import assert_attention_close, gpu_attention, gpu_mask, oracle_attention
 
 pytestmark = pytest.mark.gpu
@@ -40,36 +41,20 @@ def _uses_tc256(si):
 
 
 def _splits(si):
-    # key-tile ranges per unit: one with at least one unit per SM, else the
-    # count (at least two tiles a range) that minimises the items a CTA
-    # walks times their tiles plus a fixed 14
+    # key-tile ranges per unit as the planner chooses them (tests/_plan.py):
+    # 1 with at least one unit per SM, 0 when the one-row-block kernel takes
+    # the shape
     w = si.w
     sms = torch.cuda.get_device_properties(0).multi_processor_count
-    units = w.Bt * w.Hkv
-    if units >= sms:
-        return 1
-    max_tiles = (si.block_table.shape[1] * w.page_size + 63) // 64 + 1
-    if max_tiles < 16:
-        return 0  # the one-row-block kernel takes short units
-    cost = {ns: -(-units * ns // sms) * (-(-max_tiles // ns) + 14) for ns in range(1, min(64, max(1, max_tiles // 2)) + 1)}
-    return min(cost, key=lambda ns: (cost[ns], ns))
+    return _plan.tc256_splits(w.Bt, w.Hkv, 2, _plan.max_tiles(si.block_table.shape[1], w.page_size), sms)
 
 
 def _streamk(si):
-    # at most 255 sequences, and equal runs of all key tiles cost at least 3%
-    # less than the ranges (or whole units): per CTA, items of their tiles
-    # plus 14 each; a run of W tiles overlaps ceil(W / T) + 1 units, plus 10
-    # for the merge launch
+    # equal runs of all key tiles instead of those ranges (tests/_plan.py)
     w = si.w
     sms = torch.cuda.get_device_properties(0).multi_processor_count
-    units = w.Bt * w.Hkv
-    T = (si.block_table.shape[1] * w.page_size + 63) // 64 + 1
-    ns = _splits(si)
-    if ns < 1 or w.Bt > 255 or units * T >= 1 << 30:
-        return False
-    ranges = -(-units * ns // sms) * (-(-T // ns) + 14)
-    W = -(-units * T // sms)
-    return (W + (-(-W // T) + 1) * 14 + 10) * 100 < ranges * 97
+    T = _plan.max_tiles(si.block_table.shape[1], w.page_size)
+    return _plan.tc256_streamk(w.Bt, w.Hkv, T, _splits(si), sms)
 
 
 def _check(si, seqs=None, rope=None):
