@@ -232,7 +232,7 @@ RopeTable make_rope_table(double theta, int d) {
 
 extern "C" {
 
-int simsd_version(void) { return 1 * 10000 + 0 * 100 + 0; }
+int simsd_version(void) { return 1 * 10000 + 1 * 100 + 0; }
 
 const char* simsd_last_error(void) { return g_last_error; }
 

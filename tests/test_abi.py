@@ -37,7 +37,7 @@ def test_every_declared_symbol_is_exported(lib):
 
 
 def test_host_validation_without_gpu(lib):
-    assert lib.simsd_version() == 10000
+    assert lib.simsd_version() == 10100
     P = ctypes.c_void_p
     one = ctypes.c_void_p(16)
     # gamma outside [1, 32]
