@@ -920,17 +920,24 @@ __global__ void __launch_bounds__(128) combine_kernel(const __grid_constant__ Tc
   pdl_launch_next();
 }
 
+// The kernels' shared-memory attributes, set once per device (function
+// attributes apply to the current device only).
 cudaError_t ensure_smem_attr() {
-  static bool done = false;
-  if (done) return cudaSuccess;
+  static std::mutex mu;
+  static bool done[64] = {};
+  int dev = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) return e;
+  if (dev < 0 || dev >= 64) return cudaErrorInvalidDevice;
+  std::lock_guard<std::mutex> lk(mu);
+  if (done[dev]) return cudaSuccess;
   for (auto kern : {attention_tc_kernel<false>, attention_tc_kernel<true>}) {
-    cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                         static_cast<int>(smem_bytes()));
+    e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(smem_bytes()));
     if (e != cudaSuccess) return e;
     e = cudaFuncSetAttribute(kern, cudaFuncAttributePreferredSharedMemoryCarveout, cudaSharedmemCarveoutMaxShared);
     if (e != cudaSuccess) return e;
   }
-  done = true;
+  done[dev] = true;
   return cudaSuccess;
 }
 

@@ -54,6 +54,7 @@
 #include <cuda_runtime.h>
 
 #include <algorithm>
+#include <mutex>
 
 #include "common.cuh"
 #include "kernels.h"
@@ -1149,12 +1150,22 @@ cudaError_t launch_attention_tc256(const AttnTcArgs& a, const AttnTcPlan& pl, En
   p.scale_log2 = a.scale * 1.4426950408889634f;
   p.wait_ns = a.fault.wait_ns ? a.fault.wait_ns : kWaitLimitNs;
   p.extra_p = a.fault.extra;
-  static bool attr_done = false;
-  if (!attr_done) {
-    cudaError_t e = cudaFuncSetAttribute(attention_tc256_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                         static_cast<int>(smem_bytes()));
+  {
+    // the shared-memory attribute, once per device (function attributes
+    // apply to the current device only)
+    static std::mutex mu;
+    static bool done[64] = {};
+    int dev = 0;
+    cudaError_t e = cudaGetDevice(&dev);
     if (e != cudaSuccess) return e;
-    attr_done = true;
+    if (dev < 0 || dev >= 64) return cudaErrorInvalidDevice;
+    std::lock_guard<std::mutex> lk(mu);
+    if (!done[dev]) {
+      e = cudaFuncSetAttribute(attention_tc256_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                               static_cast<int>(smem_bytes()));
+      if (e != cudaSuccess) return e;
+      done[dev] = true;
+    }
   }
   const int grid = pl.streamk ? pl.num_sms : std::min(p.items, pl.num_sms);
   p.ctas = grid;
