@@ -176,6 +176,14 @@ def test_split_units_keep_ranges():
         assert _splits(si) > 1 and not _streamk(si)
 
 
+def test_streamk_largest_batch():
+    # 255 sequences, the most stream-K takes: the tile offsets of all of them
+    # fill the CTA's 256-entry table; ~16k-key prefixes (17 GB of cache)
+    si = inputs.make_step_inputs(_w(255, prefix=(15000, 16000), seed=18), device="cuda", random_step_map=True)
+    assert _streamk(si)
+    _check(si, seqs=[0, 127, 254])
+
+
 def test_streamk_bad_prefix_inside_runs():
     # prefix lengths out of range and a bad page inside runs that cut units
     si = inputs.make_step_inputs(_w(22, prefix=(2000, 3000), seed=14), device="cuda", random_step_map=True)
