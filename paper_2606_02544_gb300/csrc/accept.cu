@@ -261,10 +261,15 @@ __global__ void __launch_bounds__(kAcceptThreads) accept_part_kernel(const float
     keys[(static_cast<size_t>(b) * rows + r) * parts + c] = best[r];
 }
 
-// One block per sequence: warp w takes rows w, w + 32 (the maximum key over
-// the parts, lanes over the parts: coalesced loads of keys[b][row][part],
-// all of a lane's issued together), then warp 0 walks the drafts.
+// One block per sequence: warp w takes rows w and w + 32 (the maximum key
+// over the parts, lanes over the parts: coalesced loads of
+// keys[b][row][part]), then warp 0 walks the drafts.  A lane's keys of both
+// rows, up to kMergePer each (the parts of a one-wave grid on up to 160
+// SMs), are loaded before any is compared, so that a warp waits for one
+// round trip however many rows and parts it has; more parts take further
+// rounds.
 constexpr int kMergeThreads = 1024;
+constexpr int kMergePer = 10;
 __global__ void __launch_bounds__(kMergeThreads) accept_merge_kernel(const unsigned long long* __restrict__ keys,
                                                                      int parts, const int32_t* __restrict__ draft,
                                                                      int gamma, int vocab,
@@ -278,21 +283,34 @@ __global__ void __launch_bounds__(kMergeThreads) accept_merge_kernel(const unsig
   const unsigned full = 0xffffffffu;
   pdl_wait();
   const int dr_lane = (warp == 0 && lane < gamma) ? draft[static_cast<size_t>(b) * gamma + lane] : 0;
-  for (int r = warp; r < rows; r += kMergeThreads / 32) {
-    const unsigned long long* kr = keys + (static_cast<size_t>(b) * rows + r) * parts;
-    unsigned long long k = 0ull;
-#pragma unroll 4
-    for (int p = lane; p < parts; p += 32) {
-      const unsigned long long v = kr[p];
-      k = v > k ? v : k;
+  static_assert(kMaxRows <= 2 * (kMergeThreads / 32), "two rows a warp at most");
+  const int r0 = warp, r1 = warp + kMergeThreads / 32;
+  const bool has0 = r0 < rows, has1 = r1 < rows;
+  const unsigned long long* k0 = keys + (static_cast<size_t>(b) * rows + (has0 ? r0 : 0)) * parts;
+  const unsigned long long* k1 = keys + (static_cast<size_t>(b) * rows + (has1 ? r1 : 0)) * parts;
+  unsigned long long m0 = 0ull, m1 = 0ull;
+  for (int p0 = 0; has0 && p0 < parts; p0 += 32 * kMergePer) {
+    unsigned long long v0[kMergePer], v1[kMergePer];
+#pragma unroll
+    for (int j = 0; j < kMergePer; ++j) {
+      const int p = p0 + 32 * j + lane;
+      v0[j] = p < parts ? k0[p] : 0ull;
+      v1[j] = has1 && p < parts ? k1[p] : 0ull;
     }
 #pragma unroll
-    for (int o = 16; o > 0; o >>= 1) {
-      const unsigned long long v = __shfl_xor_sync(full, k, o);
-      k = v > k ? v : k;
+    for (int j = 0; j < kMergePer; ++j) {
+      m0 = v0[j] > m0 ? v0[j] : m0;
+      m1 = v1[j] > m1 ? v1[j] : m1;
     }
-    if (lane == 0) am[r] = static_cast<int>(~static_cast<uint32_t>(k & 0xFFFFFFFFull));
   }
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) {
+    const unsigned long long u0 = __shfl_xor_sync(full, m0, o), u1 = __shfl_xor_sync(full, m1, o);
+    m0 = u0 > m0 ? u0 : m0;
+    m1 = u1 > m1 ? u1 : m1;
+  }
+  if (lane == 0 && has0) am[r0] = static_cast<int>(~static_cast<uint32_t>(m0 & 0xFFFFFFFFull));
+  if (lane == 0 && has1) am[r1] = static_cast<int>(~static_cast<uint32_t>(m1 & 0xFFFFFFFFull));
   __syncthreads();
   pdl_launch_next();
   if (warp == 0) walk_drafts(am, dr_lane, b, gamma, vocab, accepted_len, out_tokens, row_argmax, err_word);
