@@ -680,27 +680,50 @@ __global__ void __launch_bounds__(kSampThreads, 2) samp_resid_kernel(
       zd = __ldg(drf + (static_cast<size_t>(b) * gamma + lane) * vocab + x);
     }
   }
-  // the rows' (m, s): warp w merges rows w, w + 16, ..., lanes over the parts
-  for (int r = warp; r < rows; r += kSampWarps) {
-    float m = kEmpty, sm = 0.f;
-    for (int q0 = 0; q0 < parts; q0 += 32 * 8) {
-      float2 v[8];
+  // the rows' (m, s): warp w merges rows w, w + 16, ... (at most
+  // kRowsPerWarp), lanes over the parts.  samp_part_kernel cut the rows'
+  // groups of 32 units into parts of `per` groups, so row r's pair is
+  // non-empty only in parts r*Wg/per .. ((r+1)*Wg - 1)/per (the others hold
+  // the empty pair, which a merge leaves unchanged); a lane loads one pair
+  // of each of the warp's rows per round, all before any is merged
+  {
+    constexpr int kRowsPerWarp = (kSampMaxRows + kSampWarps - 1) / kSampWarps;
+    const int Wg = ((VEC ? (vocab >> 2) : vocab) + 31) >> 5;  // groups per row
+    const int per = (rows * Wg + parts - 1) / parts;
+    float m[kRowsPerWarp], sm[kRowsPerWarp];
+    int q_lo[kRowsPerWarp], q_n[kRowsPerWarp];
+    int most = 0;
 #pragma unroll
-      for (int j = 0; j < 8; ++j) {
-        const int q = q0 + 32 * j + lane;
-        v[j] = q < parts ? pre[(static_cast<size_t>(b) * parts + q) * rows + r] : make_float2(kEmpty, 0.f);
+    for (int i = 0; i < kRowsPerWarp; ++i) {
+      const int r = warp + kSampWarps * i;
+      m[i] = kEmpty;
+      sm[i] = 0.f;
+      q_lo[i] = r < rows ? r * Wg / per : 0;
+      q_n[i] = r < rows ? min(parts - 1, ((r + 1) * Wg - 1) / per) - q_lo[i] + 1 : 0;
+      most = max(most, q_n[i]);
+    }
+    for (int k0 = 0; k0 < most; k0 += 32) {
+      float2 v[kRowsPerWarp];
+#pragma unroll
+      for (int i = 0; i < kRowsPerWarp; ++i) {
+        const int k = k0 + lane, r = warp + kSampWarps * i;
+        v[i] = k < q_n[i] ? pre[(static_cast<size_t>(b) * parts + q_lo[i] + k) * rows + r] : make_float2(kEmpty, 0.f);
       }
 #pragma unroll
-      for (int j = 0; j < 8; ++j) ms_merge(m, sm, v[j].x, v[j].y);
+      for (int i = 0; i < kRowsPerWarp; ++i) ms_merge(m[i], sm[i], v[i].x, v[i].y);
     }
 #pragma unroll
-    for (int o = 16; o > 0; o >>= 1) {
-      const float m2 = __shfl_xor_sync(full, m, o), s2 = __shfl_xor_sync(full, sm, o);
-      ms_merge(m, sm, m2, s2);
-    }
-    if (lane == 0) {
-      row_m[r] = m;
-      row_s[r] = sm;
+    for (int i = 0; i < kRowsPerWarp; ++i) {
+      const int r = warp + kSampWarps * i;
+#pragma unroll
+      for (int o = 16; o > 0; o >>= 1) {
+        const float m2 = __shfl_xor_sync(full, m[i], o), s2 = __shfl_xor_sync(full, sm[i], o);
+        ms_merge(m[i], sm[i], m2, s2);
+      }
+      if (lane == 0 && r < rows) {
+        row_m[r] = m[i];
+        row_s[r] = sm[i];
+      }
     }
   }
   __syncthreads();
