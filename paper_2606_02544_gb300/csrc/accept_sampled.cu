@@ -642,7 +642,7 @@ __device__ __forceinline__ float cta_sum(float v, float* red) {
 
 // Few sequences, after samp_part_kernel: one CTA per (sequence b, span c of
 // row a; rparts spans).  Every CTA merges the parts' (m, s) of every row
-// (eight loads a lane in flight) and takes the accepted
+// (over the parts whose spans overlap the row) and takes the accepted
 // length a itself (part 0 stores the outputs); then it sums the weights of
 // its span c of row a's units, both the residual max(0, p_theta -
 // p_phi) and p_theta (the fallback when the residual is empty), and
