@@ -710,17 +710,19 @@ __global__ void __launch_bounds__(kSampThreads, 2) samp_resid_kernel(
         v[i] = k < q_n[i] ? pre[(static_cast<size_t>(b) * parts + q_lo[i] + k) * rows + r] : make_float2(kEmpty, 0.f);
       }
 #pragma unroll
-      for (int i = 0; i < kRowsPerWarp; ++i) ms_merge(m[i], sm[i], v[i].x, v[i].y);
+      for (int i = 0; i < kRowsPerWarp; ++i)
+        if (warp + kSampWarps * i < rows) ms_merge(m[i], sm[i], v[i].x, v[i].y);
     }
 #pragma unroll
     for (int i = 0; i < kRowsPerWarp; ++i) {
       const int r = warp + kSampWarps * i;
+      if (r >= rows) continue;  // (the same for the whole warp)
 #pragma unroll
       for (int o = 16; o > 0; o >>= 1) {
         const float m2 = __shfl_xor_sync(full, m[i], o), s2 = __shfl_xor_sync(full, sm[i], o);
         ms_merge(m[i], sm[i], m2, s2);
       }
-      if (lane == 0 && r < rows) {
+      if (lane == 0) {
         row_m[r] = m[i];
         row_s[r] = sm[i];
       }
