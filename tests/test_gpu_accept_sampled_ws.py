@@ -1,6 +1,7 @@
 """GPU parity of simsd_accept_sampled_ws: stochastic acceptance with a caller
 workspace, where the log-sum-exp pass of a small batch is split over many
-CTAs (per-part (max, sum) pairs merged by each sequence's cluster).  The
+CTAs (per-part (max, sum) pairs, merged by a second launch over spans of
+row a whose last CTA per sequence draws the token).  The
 comparison with the oracle is the one of tests/test_gpu_accept_sampled.py:
 identical results wherever the oracle's own numbers put every decision
 outside the fp32 band, a valid choice inside it."""
@@ -31,6 +32,9 @@ def _gpu_ws(si):
     (1, 8, 151936, 1.0, 0.5), (1, 32, 151936, 1.0, 0.3), (3, 16, 151936, 0.7, 0.5), (8, 16, 151936, 1.0, 0.4),
     (9, 12, 151936, 1.3, 0.5), (2, 16, 151935, 1.0, 0.5), (8, 4, 151936, 1.0, 0.5), (8, 8, 151936, 0.8, 0.6),
     (1, 2, 262144, 1.0, 0.5), (5, 1, 400000, 1.0, 0.5),
+    # 3 rows over 192 parts: each row's pairs span ~64 parts, more than a
+    # warp's lanes take in one round
+    (1, 1, 1048576, 1.0, 0.5),
 ])
 def test_split_matches_oracle(monkeypatch, Bt, gamma, V, T, eta):
     # at most SMs / 16 sequences with at least 3 MiB of logits each: split
