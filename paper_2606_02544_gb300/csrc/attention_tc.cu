@@ -855,6 +855,7 @@ __global__ void __maxnreg__(kMaxRegs)
 // O = sum_i 2^(m_i - M) O_i / sum_i 2^(m_i - M) l_i.  One warp per row; the
 // lanes take the splits' (m, l) in parallel, then sum the partial O rows with
 // lanes over the head dimension (independent loads, several in flight).
+constexpr int kCombineBatch = 16;
 __global__ void __launch_bounds__(128) combine_kernel(const __grid_constant__ TcParams p) {
   pdl_wait();
   const int lane = threadIdx.x & 31;
@@ -895,14 +896,25 @@ __global__ void __launch_bounds__(128) combine_kernel(const __grid_constant__ Tc
         }
       }
       const int cnt = min(32, p.nsplit - c0);
-#pragma unroll 4
-      for (int j = 0; j < cnt; ++j) {
-        const float w = __shfl_sync(full, wj, j);
-        const float4 o = reinterpret_cast<const float4*>(p.ws + ((e0 + c0 + j) * p.rows_blk + row) * kD)[lane];
-        acc.x = fmaf(w, o.x, acc.x);
-        acc.y = fmaf(w, o.y, acc.y);
-        acc.z = fmaf(w, o.z, acc.z);
-        acc.w = fmaf(w, o.w, acc.w);
+      // the partials of kCombineBatch splits are loaded before any is
+      // added (one round trip per batch; the sum keeps the split order)
+      const float4* ob = reinterpret_cast<const float4*>(p.ws + ((e0 + c0) * p.rows_blk + row) * kD) + lane;
+      const size_t split4 = static_cast<size_t>(p.rows_blk) * (kD / 4);  // float4s from one split to the next
+      for (int j0 = 0; j0 < cnt; j0 += kCombineBatch) {
+        float4 o[kCombineBatch];
+#pragma unroll
+        for (int j = 0; j < kCombineBatch; ++j)
+          o[j] = j0 + j < cnt ? ob[(j0 + j) * split4] : make_float4(0.f, 0.f, 0.f, 0.f);
+#pragma unroll
+        for (int j = 0; j < kCombineBatch; ++j) {
+          if (j0 + j < cnt) {  // (the same for the whole warp)
+            const float w = __shfl_sync(full, wj, j0 + j);
+            acc.x = fmaf(w, o[j].x, acc.x);
+            acc.y = fmaf(w, o[j].y, acc.y);
+            acc.z = fmaf(w, o[j].z, acc.z);
+            acc.w = fmaf(w, o[j].w, acc.w);
+          }
+        }
       }
     }
   }
