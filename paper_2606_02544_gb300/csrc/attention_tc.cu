@@ -855,7 +855,9 @@ __global__ void __maxnreg__(kMaxRegs)
 // O = sum_i 2^(m_i - M) O_i / sum_i 2^(m_i - M) l_i.  One warp per row; the
 // lanes take the splits' (m, l) in parallel, then sum the partial O rows with
 // lanes over the head dimension (independent loads, several in flight).
-constexpr int kCombineBatch = 16;
+// kBatch: splits whose partials a lane loads before adding any (see
+// launch_combine for the choice)
+template <int kBatch>
 __global__ void __launch_bounds__(128) combine_kernel(const __grid_constant__ TcParams p) {
   pdl_wait();
   const int lane = threadIdx.x & 31;
@@ -896,17 +898,17 @@ __global__ void __launch_bounds__(128) combine_kernel(const __grid_constant__ Tc
         }
       }
       const int cnt = min(32, p.nsplit - c0);
-      // the partials of kCombineBatch splits are loaded before any is
-      // added (one round trip per batch; the sum keeps the split order)
+      // the partials of kBatch splits are loaded before any is added (one
+      // round trip per batch; the sum keeps the split order)
       const float4* ob = reinterpret_cast<const float4*>(p.ws + ((e0 + c0) * p.rows_blk + row) * kD) + lane;
       const size_t split4 = static_cast<size_t>(p.rows_blk) * (kD / 4);  // float4s from one split to the next
-      for (int j0 = 0; j0 < cnt; j0 += kCombineBatch) {
-        float4 o[kCombineBatch];
+      for (int j0 = 0; j0 < cnt; j0 += kBatch) {
+        float4 o[kBatch];
 #pragma unroll
-        for (int j = 0; j < kCombineBatch; ++j)
+        for (int j = 0; j < kBatch; ++j)
           o[j] = j0 + j < cnt ? ob[(j0 + j) * split4] : make_float4(0.f, 0.f, 0.f, 0.f);
 #pragma unroll
-        for (int j = 0; j < kCombineBatch; ++j) {
+        for (int j = 0; j < kBatch; ++j) {
           if (j0 + j < cnt) {  // (the same for the whole warp)
             const float w = __shfl_sync(full, wj, j0 + j);
             acc.x = fmaf(w, o[j].x, acc.x);
@@ -1025,6 +1027,18 @@ bool plan_attention_tc(int Bt, int gamma, int Hq, int Hkv, int max_pages, int pa
   return true;
 }
 
+// The combine launch, a warp per row.  With many splits a row (a small
+// batch) a lane loads 16 splits' partials at once: 128 registers, four
+// blocks per SM, which pays while the grid fits in one wave of those.
+// Otherwise four at a time (about 56 registers): a large grid merging a
+// few splits a row needs its blocks resident more than wide loads.
+cudaError_t launch_combine(const TcParams& p, long long warps, int num_sms, cudaStream_t stream) {
+  const long long blocks = (warps + 3) / 4;
+  const bool wide = p.nsplit > 4 && blocks <= 4LL * num_sms;
+  return wide ? launch_overlapped(combine_kernel<16>, dim3(static_cast<unsigned>(blocks)), dim3(128), 0, stream, 1, p)
+              : launch_overlapped(combine_kernel<4>, dim3(static_cast<unsigned>(blocks)), dim3(128), 0, stream, 1, p);
+}
+
 cudaError_t launch_attention_combine(const AttnTcArgs& a, const AttnTcPlan& pl, cudaStream_t stream) {
   TcParams p{};
   p.out = static_cast<__nv_bfloat16*>(a.out);
@@ -1040,7 +1054,7 @@ cudaError_t launch_attention_combine(const AttnTcArgs& a, const AttnTcPlan& pl, 
   p.s_blk = pl.s_blk;
   p.nsplit = pl.nsplit;
   const long long warps = static_cast<long long>(a.Bt) * a.Hkv * pl.rb * pl.rows_blk;
-  return launch_overlapped(combine_kernel, dim3(static_cast<unsigned>((warps + 3) / 4)), dim3(128), 0, stream, 1, p);
+  return launch_combine(p, warps, pl.num_sms, stream);
 }
 
 cudaError_t launch_attention_tc(const AttnTcArgs& a, const AttnTcPlan& pl, EncodeTiledFn encode,
@@ -1114,7 +1128,7 @@ cudaError_t launch_attention_tc(const AttnTcArgs& a, const AttnTcPlan& pl, Encod
                                               dim3(kThreads), smem_bytes(), stream, 1u, tq, tkn, tvn, tkc, tvc, p);
   if (e != cudaSuccess || pl.nsplit == 1 || pl.fuse) return e;
   const long long warps = static_cast<long long>(a.Bt) * a.Hkv * pl.rb * pl.rows_blk;
-  return launch_overlapped(combine_kernel, dim3(static_cast<unsigned>((warps + 3) / 4)), dim3(128), 0, stream, 1, p);
+  return launch_combine(p, warps, pl.num_sms, stream);
 }
 
 size_t noalloc_scratch_capacity() { return sizeof(g_noalloc_scratch); }
